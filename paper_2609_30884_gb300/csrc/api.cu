@@ -1,0 +1,879 @@
+// C ABI of the bounded-recomputation library: argument validation, workspace
+// planning and the per-layer launch sequence (see include/crf.h).
+//
+// Executable restart (Section 4.2): for each layer l of the union of the
+// requests' windows, the rows of every request whose window covers l form one
+// activation matrix, and the layer runs as
+//   rmsnorm -> [LoRA down] -> QKV GEMM (+LoRA up, bias, RoPE, q out, K/V to pages)
+//   -> causal GQA attention over the pages -> [LoRA down] -> O GEMM (+residual)
+//   -> rmsnorm -> [LoRA down] -> gate|up GEMM (+SwiGLU) -> [LoRA down] -> down GEMM (+residual)
+// Then the last prefix row of each request that asks for it continues through
+// layers e..N-1 against the historical cache (first-step state, Section S2.1).
+#include "../../include/crf.h"
+#include "common.cuh"
+#include "kernels.h"
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <set>
+#include <string>
+#include <vector>
+
+using namespace crf;
+
+struct crf_ctx {
+  int device;
+  int num_sms;
+  int* status_dev;
+};
+
+namespace {
+
+thread_local std::string g_err;
+
+crf_status fail(crf_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return st;
+}
+
+#define CRF_CUDA(expr)                                                                  \
+  do {                                                                                  \
+    cudaError_t _e = (expr);                                                            \
+    if (_e != cudaSuccess)                                                              \
+      return fail(CRF_ECUDA, "%s failed: %s (%s:%d)", #expr, cudaGetErrorString(_e), __FILE__, \
+                  __LINE__);                                                            \
+  } while (0)
+
+inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+struct Dims {
+  int N, h, hq, hkv, d, f, V, qd, kvd;
+  float eps;
+  double theta;
+  bool bias;
+};
+
+Dims dims_of(const crf_model_dims& m) {
+  Dims d;
+  d.N = m.n_layers;
+  d.h = m.hidden;
+  d.hq = m.n_q_heads;
+  d.hkv = m.n_kv_heads;
+  d.d = m.head_dim;
+  d.f = m.ffn;
+  d.V = m.vocab;
+  d.qd = m.n_q_heads * m.head_dim;
+  d.kvd = m.n_kv_heads * m.head_dim;
+  d.eps = m.rms_eps;
+  d.theta = m.rope_theta;
+  d.bias = m.qkv_bias != 0;
+  return d;
+}
+
+void module_shape(const Dims& d, int m, int& out, int& in) {
+  switch (m) {
+    case CRF_MOD_Q: out = d.qd; in = d.h; break;
+    case CRF_MOD_K:
+    case CRF_MOD_V: out = d.kvd; in = d.h; break;
+    case CRF_MOD_O: out = d.h; in = d.qd; break;
+    case CRF_MOD_GATE:
+    case CRF_MOD_UP: out = d.f; in = d.h; break;
+    default: out = d.h; in = d.f; break;
+  }
+}
+
+crf_status check_dims(const crf_model_dims& m) {
+  if (m.n_layers < 1 || m.hidden < 1 || m.n_q_heads < 1 || m.n_kv_heads < 1 || m.ffn < 1 ||
+      m.vocab < 1)
+    return fail(CRF_EINVAL, "model dims must be positive");
+  if (m.head_dim != 64 && m.head_dim != 128)
+    return fail(CRF_EUNSUPPORTED, "head_dim %d unsupported (64 or 128)", m.head_dim);
+  if (m.n_q_heads % m.n_kv_heads != 0)
+    return fail(CRF_ESHAPE, "n_q_heads %d not a multiple of n_kv_heads %d", m.n_q_heads,
+                m.n_kv_heads);
+  if (m.hidden % 64 != 0 || m.ffn % 8 != 0)
+    return fail(CRF_EUNSUPPORTED, "hidden must be a multiple of 64 and ffn of 8");
+  if (!(m.rms_eps >= 0.f) || !(m.rope_theta > 0.f))
+    return fail(CRF_EINVAL, "rms_eps must be >= 0 and rope_theta > 0");
+  return CRF_OK;
+}
+
+crf_status check_lora(const crf_lora_dims& l) {
+  if (l.rank != 8 && l.rank != 16) return fail(CRF_EUNSUPPORTED, "LoRA rank %d unsupported (8 or 16)", l.rank);
+  if (!std::isfinite(l.alpha)) return fail(CRF_EINVAL, "LoRA alpha must be finite");
+  if (l.module_mask & ~0x7Fu) return fail(CRF_EINVAL, "module_mask has bits beyond the 7 modules");
+  return CRF_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// ---------------------------------------------------------------- workspace plan
+struct Plan {
+  int M = 0;          // max batched rows over layers
+  int max_n = 0;
+  int dec_rows = 0;   // requests asking for the first-step state
+  int splits = 1;
+  size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_rope;
+  size_t off_dx0, off_dec;  // decode: bf16 starting rows, fp32 scratch
+  size_t dec_bytes;
+  size_t total;
+};
+
+int dec_splits(int max_n) { return std::max(1, std::min(64, (max_n + 511) / 512)); }
+
+Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
+  Plan p;
+  for (int l = 0; l < D.N; ++l) {
+    int m = 0;
+    for (int i = 0; i < n_req; ++i)
+      if (reqs[i].s <= l && l < reqs[i].e) m += reqs[i].n_tokens;
+    p.M = std::max(p.M, m);
+  }
+  for (int i = 0; i < n_req; ++i) {
+    p.max_n = std::max(p.max_n, reqs[i].n_tokens);
+    if (reqs[i].final_hidden_out) ++p.dec_rows;
+  }
+  const size_t M = static_cast<size_t>(p.M);
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = align256(o + bytes);
+    return at;
+  };
+  p.off_g0 = take(M * D.h * 2);
+  p.off_g1 = take(M * D.h * 2);
+  p.off_x1 = take(M * D.h * 2);
+  p.off_xn = take(M * D.h * 2);
+  p.off_q = take(M * D.qd * 2);
+  p.off_o = take(M * D.qd * 2);
+  p.off_mlp = take(M * D.f * 2);
+  p.off_xa = take(M * 64 * 2);
+  p.off_rope = take(static_cast<size_t>(p.max_n) * (D.d / 2) * sizeof(float2));
+  p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
+  p.splits = dec_splits(p.max_n);
+  // decode scratch, fp32: x, xn, x1, q, k, v, o, xa, gu, m, part
+  const size_t dec = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + kRankPad + 3 * D.f) * 4 +
+                     static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
+  p.dec_bytes = align256(dec);
+  p.off_dec = take(p.dec_rows ? p.dec_bytes : 0);
+  p.total = o;
+  return p;
+}
+
+// ---------------------------------------------------------------- request checks
+crf_status check_model_layers(const crf_model* model, int l0, int l1, const Dims& D) {
+  for (int l = l0; l < l1; ++l) {
+    const crf_layer_weights& w = model->layers[l];
+    for (int m = 0; m < CRF_NUM_MODULES; ++m)
+      if (!w.W[m] || !aligned16(w.W[m])) return fail(CRF_EINVAL, "layer %d weight %d null or misaligned", l, m);
+    if (!w.ln1 || !w.ln2) return fail(CRF_EINVAL, "layer %d norm gain is null", l);
+    if (D.bias)
+      for (int j = 0; j < 3; ++j)
+        if (!w.bias[j]) return fail(CRF_EINVAL, "layer %d qkv bias %d is null", l, j);
+  }
+  return CRF_OK;
+}
+
+crf_status check_adapter_layers(const crf_adapter* a, int l0, int l1) {
+  for (int l = l0; l < l1; ++l)
+    for (int m = 0; m < CRF_NUM_MODULES; ++m) {
+      if (!(a->dims.module_mask & (1u << m))) continue;
+      const void* A = a->A[l * 7 + m];
+      const void* B = a->B[l * 7 + m];
+      if (!A || !B || !aligned16(A) || !aligned16(B))
+        return fail(CRF_EINVAL, "adapter layer %d module %d factor null or misaligned", l, m);
+    }
+  return CRF_OK;
+}
+
+// ---------------------------------------------------------------- one layer
+struct LayerCtx {
+  const Dims* D;
+  const crf_ctx* ctx;
+  const crf_model* model;
+  const crf_adapter* ad;
+  const crf_kv_pool* pool;
+  cudaStream_t st;
+  uint8_t* ws;
+  const Plan* plan;
+  float scale;
+};
+
+bool adapted(const crf_adapter* a, int m) { return (a->dims.module_mask >> m) & 1u; }
+
+// LoRA down product of `X` for the listed modules into XA (16 columns per module).
+cudaError_t lora_down(const LayerCtx& c, int l, const void* X, int M, int K, const int* mods, int nm,
+                      __nv_bfloat16* XA) {
+  GemmDesc g;
+  std::memset(&g, 0, sizeof(g));
+  g.A = X;
+  g.M = M;
+  g.K = K;
+  g.lda = K;
+  g.ngroups = 1;
+  g.nseg = nm;
+  for (int s = 0; s < nm; ++s) {
+    g.B[s] = c.ad->A[l * 7 + mods[s]];
+    g.B_rows[s] = c.ad->dims.rank;
+    g.ldb[s] = K;
+  }
+  g.group_cols[0] = nm * kRankPad;
+  g.epi = kEpiScaleBf16;
+  g.scale = c.scale;
+  g.out = XA;
+  g.ldo = 64;
+  g.status = c.ctx->status_dev;
+  return launch_gemm(g, nm * kRankPad, c.ctx->num_sms, c.st);
+}
+
+crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_bfloat16* X_out,
+                     int M, const ReqTable& rt) {
+  const Dims& D = *c.D;
+  const crf_layer_weights& w = c.model->layers[l];
+  const Plan& p = *c.plan;
+  uint8_t* ws = c.ws;
+  auto* X1 = reinterpret_cast<__nv_bfloat16*>(ws + p.off_x1);
+  auto* XN = reinterpret_cast<__nv_bfloat16*>(ws + p.off_xn);
+  auto* Q = reinterpret_cast<__nv_bfloat16*>(ws + p.off_q);
+  auto* O = reinterpret_cast<__nv_bfloat16*>(ws + p.off_o);
+  auto* MLP = reinterpret_cast<__nv_bfloat16*>(ws + p.off_mlp);
+  auto* XA = reinterpret_cast<__nv_bfloat16*>(ws + p.off_xa);
+  auto* rope = reinterpret_cast<const float2*>(ws + p.off_rope);
+  const int rank = c.ad->dims.rank;
+
+  // 1. RMSNorm before attention
+  CRF_CUDA(launch_rmsnorm(X_in, static_cast<const __nv_bfloat16*>(w.ln1), XN, M, D.h, D.eps, c.st));
+
+  // 2-3. q/k/v projections (+ LoRA, bias, RoPE; K/V into the pages of layer l)
+  {
+    int mods[3], nm = 0;
+    for (int m = 0; m < 3; ++m)
+      if (adapted(c.ad, m)) mods[nm++] = m;
+    if (nm) CRF_CUDA(lora_down(c, l, XN, M, D.h, mods, nm, XA));
+    GemmDesc g;
+    std::memset(&g, 0, sizeof(g));
+    g.A = XN;
+    g.M = M;
+    g.K = D.h;
+    g.lda = D.h;
+    g.ngroups = 3;
+    g.nseg = 1;
+    const int rows[3] = {D.qd, D.kvd, D.kvd};
+    int xa = 0;
+    for (int m = 0; m < 3; ++m) {
+      g.B[m] = w.W[m];
+      g.B_rows[m] = rows[m];
+      g.ldb[m] = D.h;
+      g.group_cols[m] = rows[m];
+      if (adapted(c.ad, m)) {
+        g.BL[m] = c.ad->B[l * 7 + m];
+        g.lora_on[m][0] = 1;
+        g.xa_col[m][0] = xa;
+        xa += kRankPad;
+      }
+      g.bias[m] = D.bias ? w.bias[m] : nullptr;
+    }
+    g.XA = XA;
+    g.ldxa = 64;
+    g.rank = rank;
+    g.epi = kEpiQkv;
+    g.rope = rope;
+    g.head_dim = D.d;
+    g.n_kv_heads = D.hkv;
+    g.qbuf = Q;
+    g.ldq = D.qd;
+    g.kpages = c.pool->k_pages[l];
+    g.vpages = c.pool->v_pages[l];
+    g.req = rt;
+    g.status = c.ctx->status_dev;
+    CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
+  }
+
+  // 4. causal GQA attention over the pages of layer l
+  {
+    AttnDesc a;
+    a.q = Q;
+    a.ldq = D.qd;
+    a.kpages = static_cast<const __nv_bfloat16*>(c.pool->k_pages[l]);
+    a.vpages = static_cast<const __nv_bfloat16*>(c.pool->v_pages[l]);
+    a.out = O;
+    a.ldo = D.qd;
+    a.n_q_heads = D.hq;
+    a.n_kv_heads = D.hkv;
+    a.head_dim = D.d;
+    a.req = rt;
+    a.status = c.ctx->status_dev;
+    CRF_CUDA(launch_attention(a, c.ctx->num_sms, c.st));
+  }
+
+  // 5-6. output projection + residual: X1 = X_in + O W_o^T (+ LoRA)
+  auto proj_resid = [&](int m, const void* A, int K, const void* resid, void* out) -> cudaError_t {
+    const bool lo = adapted(c.ad, m);
+    if (lo) {
+      const int mods[1] = {m};
+      cudaError_t e = lora_down(c, l, A, M, K, mods, 1, XA);
+      if (e != cudaSuccess) return e;
+    }
+    GemmDesc g;
+    std::memset(&g, 0, sizeof(g));
+    g.A = A;
+    g.M = M;
+    g.K = K;
+    g.lda = K;
+    g.ngroups = 1;
+    g.nseg = 1;
+    g.B[0] = w.W[m];
+    g.B_rows[0] = D.h;
+    g.ldb[0] = K;
+    g.group_cols[0] = D.h;
+    if (lo) {
+      g.XA = XA;
+      g.ldxa = 64;
+      g.BL[0] = c.ad->B[l * 7 + m];
+      g.rank = rank;
+      g.lora_on[0][0] = 1;
+      g.xa_col[0][0] = 0;
+    }
+    g.epi = kEpiResid;
+    g.out = out;
+    g.ldo = D.h;
+    g.resid = resid;
+    g.ld_resid = D.h;
+    g.status = c.ctx->status_dev;
+    return launch_gemm(g, 256, c.ctx->num_sms, c.st);
+  };
+  CRF_CUDA(proj_resid(CRF_MOD_O, O, D.qd, X_in, X1));
+
+  // 7. RMSNorm before the MLP
+  CRF_CUDA(launch_rmsnorm(X1, static_cast<const __nv_bfloat16*>(w.ln2), XN, M, D.h, D.eps, c.st));
+
+  // 8-9. gate|up projections with SwiGLU epilogue
+  {
+    int mods[2], nm = 0;
+    for (int m = CRF_MOD_GATE; m <= CRF_MOD_UP; ++m)
+      if (adapted(c.ad, m)) mods[nm++] = m;
+    if (nm) CRF_CUDA(lora_down(c, l, XN, M, D.h, mods, nm, XA));
+    GemmDesc g;
+    std::memset(&g, 0, sizeof(g));
+    g.A = XN;
+    g.M = M;
+    g.K = D.h;
+    g.lda = D.h;
+    g.ngroups = 1;
+    g.nseg = 2;
+    int xa = 0;
+    for (int s = 0; s < 2; ++s) {
+      const int m = CRF_MOD_GATE + s;
+      g.B[s] = w.W[m];
+      g.B_rows[s] = D.f;
+      g.ldb[s] = D.h;
+      if (adapted(c.ad, m)) {
+        g.BL[s] = c.ad->B[l * 7 + m];
+        g.lora_on[0][s] = 1;
+        g.xa_col[0][s] = xa;
+        xa += kRankPad;
+      }
+    }
+    g.group_cols[0] = D.f;
+    g.XA = XA;
+    g.ldxa = 64;
+    g.rank = rank;
+    g.epi = kEpiSwiGLU;
+    g.out = MLP;
+    g.ldo = D.f;
+    g.status = c.ctx->status_dev;
+    CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
+  }
+
+  // 10-11. down projection + residual: X_out = X1 + MLP W_d^T (+ LoRA)
+  CRF_CUDA(proj_resid(CRF_MOD_DOWN, MLP, D.f, X1, X_out));
+  return CRF_OK;
+}
+
+// ---------------------------------------------------------------- decode row
+// Carry one row (fp32) through layers [l0, N) at position `pos`, reading each
+// layer's cached K/V at positions < pos from the pages.
+crf_status decode_row(const LayerCtx& c, int l0, const __nv_bfloat16* start_row, int pos,
+                      const int32_t* page_table, void* out_bf16) {
+  const Dims& D = *c.D;
+  const Plan& p = *c.plan;
+  float* base = reinterpret_cast<float*>(c.ws + p.off_dec);
+  float* x = base;
+  float* xn = x + D.h;
+  float* x1 = xn + D.h;
+  float* q = x1 + D.h;
+  float* o = q + D.qd;
+  float* k = o + D.qd;
+  float* v = k + D.kvd;
+  float* xa = v + D.kvd;
+  float* gu = xa + kRankPad;
+  float* m = gu + 2 * D.f;
+  float* part = m + D.f;
+  const int rank = c.ad->dims.rank;
+  CRF_CUDA(launch_bf16_to_f32(start_row, x, D.h, c.st));
+  auto proj = [&](int l, int mod, const float* in, int in_dim, int out_dim, const void* bias,
+                  const float* resid, float* y) -> cudaError_t {
+    GemvDesc g{};
+    g.W = static_cast<const __nv_bfloat16*>(c.model->layers[l].W[mod]);
+    g.out_dim = out_dim;
+    g.in_dim = in_dim;
+    g.x = in;
+    g.rows = 1;
+    g.bias = static_cast<const __nv_bfloat16*>(bias);
+    if (adapted(c.ad, mod)) {
+      cudaError_t e = launch_lora_down_rows(static_cast<const __nv_bfloat16*>(c.ad->A[l * 7 + mod]),
+                                            rank, in_dim, in, 1, c.scale, xa, c.st);
+      if (e != cudaSuccess) return e;
+      g.BL = static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + mod]);
+      g.xa = xa;
+      g.rank = rank;
+    }
+    g.resid = resid;
+    g.y = y;
+    return launch_gemv(g, c.st);
+  };
+  for (int l = l0; l < D.N; ++l) {
+    const crf_layer_weights& w = c.model->layers[l];
+    CRF_CUDA(launch_rmsnorm_f32(x, static_cast<const __nv_bfloat16*>(w.ln1), xn, 1, D.h, D.eps, c.st));
+    CRF_CUDA(proj(l, CRF_MOD_Q, xn, D.h, D.qd, D.bias ? w.bias[0] : nullptr, nullptr, q));
+    CRF_CUDA(proj(l, CRF_MOD_K, xn, D.h, D.kvd, D.bias ? w.bias[1] : nullptr, nullptr, k));
+    CRF_CUDA(proj(l, CRF_MOD_V, xn, D.h, D.kvd, D.bias ? w.bias[2] : nullptr, nullptr, v));
+    CRF_CUDA(launch_rope_rows(q, 1, D.hq, D.d, pos, D.theta, c.st));
+    CRF_CUDA(launch_rope_rows(k, 1, D.hkv, D.d, pos, D.theta, c.st));
+    DecodeAttnDesc a;
+    std::memset(&a, 0, sizeof(a));
+    a.q = q;
+    a.k_self = k;
+    a.v_self = v;
+    a.kpages = static_cast<const __nv_bfloat16*>(c.pool->k_pages[l]);
+    a.vpages = static_cast<const __nv_bfloat16*>(c.pool->v_pages[l]);
+    a.page_table[0] = page_table;
+    a.pos[0] = pos;
+    a.out = o;
+    a.part = part;
+    a.rows = 1;
+    a.n_q_heads = D.hq;
+    a.n_kv_heads = D.hkv;
+    a.head_dim = D.d;
+    a.splits = p.splits;
+    a.max_pos = pos;
+    CRF_CUDA(launch_decode_attention(a, c.st));
+    CRF_CUDA(proj(l, CRF_MOD_O, o, D.qd, D.h, nullptr, x, x1));
+    CRF_CUDA(launch_rmsnorm_f32(x1, static_cast<const __nv_bfloat16*>(w.ln2), xn, 1, D.h, D.eps, c.st));
+    CRF_CUDA(proj(l, CRF_MOD_GATE, xn, D.h, D.f, nullptr, nullptr, gu));
+    CRF_CUDA(proj(l, CRF_MOD_UP, xn, D.h, D.f, nullptr, nullptr, gu + D.f));
+    CRF_CUDA(launch_swiglu_f32(gu, m, 1, D.f, c.st));
+    CRF_CUDA(proj(l, CRF_MOD_DOWN, m, D.f, D.h, nullptr, x1, x));
+  }
+  CRF_CUDA(launch_f32_to_bf16(x, static_cast<__nv_bfloat16*>(out_bf16), D.h, c.st));
+  return CRF_OK;
+}
+
+crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const crf_adapter* cur,
+                             const crf_kv_pool* pool, const crf_request* reqs, int n_req,
+                             const Dims& D, cudaStream_t st) {
+  if (n_req < 1 || n_req > CRF_MAX_REQUESTS)
+    return fail(CRF_EINVAL, "n_req %d outside [1, %d]", n_req, CRF_MAX_REQUESTS);
+  if (!pool || !pool->k_pages || !pool->v_pages || pool->num_pages < 1)
+    return fail(CRF_EINVAL, "kv pool missing");
+  std::vector<char> seen(static_cast<size_t>(pool->num_pages), 0);
+  for (int i = 0; i < n_req; ++i) {
+    const crf_request& r = reqs[i];
+    if (r.n_tokens < 1) return fail(CRF_EINVAL, "request %d: n_tokens must be >= 1", i);
+    if (r.s < 0 || r.s > r.e || r.e > D.N)
+      return fail(CRF_EINVAL, "request %d: window [%d,%d) outside [0,%d]", i, r.s, r.e, D.N);
+    if (r.s == r.e && !r.final_hidden_out)
+      return fail(CRF_EINVAL, "request %d: empty window without final_hidden_out", i);
+    if (!r.page_table) return fail(CRF_EINVAL, "request %d: page_table is null", i);
+    if (r.s == 0 && !r.tokens) return fail(CRF_EINVAL, "request %d: tokens required when s == 0", i);
+    if (r.s > 0 && !r.hidden_in) return fail(CRF_EINVAL, "request %d: hidden_in required when s > 0", i);
+    if (r.s == 0 && !model->embed) return fail(CRF_EINVAL, "model embedding is null");
+    if (r.hidden_in && !aligned16(r.hidden_in)) return fail(CRF_EINVAL, "request %d: hidden_in misaligned", i);
+    if (r.hidden_out)
+      for (int j = 0; j < r.e - r.s; ++j)
+        if (!r.hidden_out[j] || !aligned16(r.hidden_out[j]))
+          return fail(CRF_EINVAL, "request %d: hidden_out[%d] null or misaligned", i, j);
+    const int l_end = r.final_hidden_out ? D.N : r.e;
+    crf_status s = check_model_layers(model, r.s, l_end, D);
+    if (s != CRF_OK) return s;
+    s = check_adapter_layers(cur, r.s, l_end);
+    if (s != CRF_OK) return s;
+    for (int l = r.s; l < l_end; ++l)
+      if (!pool->k_pages[l] || !pool->v_pages[l] || !aligned16(pool->k_pages[l]) ||
+          !aligned16(pool->v_pages[l]))
+        return fail(CRF_EINVAL, "kv pool layer %d null or misaligned", l);
+    // page ids: in range and not shared between requests
+    const int np = (r.n_tokens + kPage - 1) / kPage;
+    std::vector<int32_t> pt(np);
+    CRF_CUDA(cudaMemcpyAsync(pt.data(), r.page_table, np * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+    CRF_CUDA(cudaStreamSynchronize(st));
+    for (int j = 0; j < np; ++j) {
+      if (pt[j] < 0 || pt[j] >= pool->num_pages)
+        return fail(CRF_EINVAL, "request %d: page id %d out of range [0,%d)", i, pt[j], pool->num_pages);
+      if (seen[pt[j]]) return fail(CRF_EINVAL, "request %d: page %d used twice", i, pt[j]);
+      seen[pt[j]] = 1;
+    }
+  }
+  (void)ctx;
+  return CRF_OK;
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+extern "C" {
+
+const char* crf_last_error(void) { return g_err.c_str(); }
+
+crf_status crf_create(crf_ctx** out, int device) {
+  if (!out) return fail(CRF_EINVAL, "out is null");
+  *out = nullptr;
+  int count = 0;
+  CRF_CUDA(cudaGetDeviceCount(&count));
+  if (device < 0 || device >= count) return fail(CRF_EINVAL, "device %d out of range", device);
+  CRF_CUDA(cudaSetDevice(device));
+  cudaDeviceProp prop;
+  CRF_CUDA(cudaGetDeviceProperties(&prop, device));
+  if (prop.major != 10 || prop.minor != 3)
+    return fail(CRF_EUNSUPPORTED, "device is sm_%d%d; this library is built for sm_103a", prop.major,
+                prop.minor);
+  crf_ctx* c = new crf_ctx;
+  c->device = device;
+  c->num_sms = prop.multiProcessorCount;
+  c->status_dev = nullptr;
+  cudaError_t e = cudaMalloc(&c->status_dev, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemset(c->status_dev, 0, sizeof(int));
+  if (e != cudaSuccess) {
+    if (c->status_dev) cudaFree(c->status_dev);
+    delete c;
+    return fail(CRF_ECUDA, "status word: %s", cudaGetErrorString(e));
+  }
+  *out = c;
+  return CRF_OK;
+}
+
+crf_status crf_destroy(crf_ctx* ctx) {
+  if (!ctx) return fail(CRF_EINVAL, "ctx is null");
+  cudaFree(ctx->status_dev);
+  delete ctx;
+  return CRF_OK;
+}
+
+crf_status crf_check(crf_ctx* ctx, void* stream) {
+  if (!ctx) return fail(CRF_EINVAL, "ctx is null");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CRF_CUDA(cudaStreamSynchronize(st));
+  int status = 0;
+  CRF_CUDA(cudaMemcpy(&status, ctx->status_dev, sizeof(int), cudaMemcpyDeviceToHost));
+  if (status) {
+    CRF_CUDA(cudaMemset(ctx->status_dev, 0, sizeof(int)));
+    return fail(CRF_ETIMEOUT, "a kernel abandoned a bounded wait (status 0x%x)", status);
+  }
+  return CRF_OK;
+}
+
+crf_status crf_workspace_size(crf_ctx* ctx, const crf_model* model, const crf_lora_dims* lora,
+                              const crf_request* reqs, int n_req, size_t* bytes) {
+  if (!ctx || !model || !lora || !reqs || !bytes) return fail(CRF_EINVAL, "null argument");
+  crf_status s = check_dims(model->dims);
+  if (s != CRF_OK) return s;
+  s = check_lora(*lora);
+  if (s != CRF_OK) return s;
+  if (n_req < 1 || n_req > CRF_MAX_REQUESTS) return fail(CRF_EINVAL, "n_req out of range");
+  const Dims D = dims_of(model->dims);
+  for (int i = 0; i < n_req; ++i)
+    if (reqs[i].n_tokens < 1 || reqs[i].s < 0 || reqs[i].s > reqs[i].e || reqs[i].e > D.N)
+      return fail(CRF_EINVAL, "request %d malformed", i);
+  *bytes = make_plan(D, reqs, n_req).total;
+  return CRF_OK;
+}
+
+crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_adapter* cur,
+                                const crf_kv_pool* pool, const crf_request* reqs, int n_req,
+                                void* workspace, size_t ws_bytes, void* stream) {
+  if (!ctx || !model || !cur || !pool || !reqs) return fail(CRF_EINVAL, "null argument");
+  if (!model->layers) return fail(CRF_EINVAL, "model layers missing");
+  if (!cur->A || !cur->B) return fail(CRF_EINVAL, "adapter tables missing");
+  crf_status s = check_dims(model->dims);
+  if (s != CRF_OK) return s;
+  s = check_lora(cur->dims);
+  if (s != CRF_OK) return s;
+  CRF_CUDA(cudaSetDevice(ctx->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const Dims D = dims_of(model->dims);
+  s = validate_requests(ctx, model, cur, pool, reqs, n_req, D, st);
+  if (s != CRF_OK) return s;
+  const Plan plan = make_plan(D, reqs, n_req);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return fail(CRF_EINVAL, "workspace null or not 256-byte aligned");
+  if (ws_bytes < plan.total)
+    return fail(CRF_ENOMEM, "workspace %zu bytes, %zu needed", ws_bytes, plan.total);
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  LayerCtx c;
+  c.D = &D;
+  c.ctx = ctx;
+  c.model = model;
+  c.ad = cur;
+  c.pool = pool;
+  c.st = st;
+  c.ws = ws;
+  c.plan = &plan;
+  c.scale = cur->dims.alpha / cur->dims.rank;
+
+  CRF_CUDA(launch_rope_table(reinterpret_cast<float2*>(ws + plan.off_rope), plan.max_n, D.d, D.theta, st));
+
+  __nv_bfloat16* G[2] = {reinterpret_cast<__nv_bfloat16*>(ws + plan.off_g0),
+                         reinterpret_cast<__nv_bfloat16*>(ws + plan.off_g1)};
+  auto* dx0 = reinterpret_cast<__nv_bfloat16*>(ws + plan.off_dx0);
+  const size_t row_bytes = static_cast<size_t>(D.h) * 2;
+  std::vector<const __nv_bfloat16*> curp(n_req, nullptr);  // current hidden rows per request
+  for (int i = 0; i < n_req; ++i)
+    if (reqs[i].s > 0) curp[i] = static_cast<const __nv_bfloat16*>(reqs[i].hidden_in);
+
+  int lmin = D.N, lmax = 0;
+  for (int i = 0; i < n_req; ++i)
+    if (reqs[i].s < reqs[i].e) {
+      lmin = std::min(lmin, reqs[i].s);
+      lmax = std::max(lmax, reqs[i].e);
+    }
+  for (int l = lmin; l < lmax; ++l) {
+    std::vector<int> act;
+    for (int i = 0; i < n_req; ++i)
+      if (reqs[i].s <= l && l < reqs[i].e) act.push_back(i);
+    if (act.empty()) continue;
+    ReqTable rt;
+    std::memset(&rt, 0, sizeof(rt));
+    int M = 0;
+    for (int i : act) {
+      rt.row0[rt.n] = M;
+      rt.len[rt.n] = reqs[i].n_tokens;
+      rt.page_table[rt.n] = reqs[i].page_table;
+      ++rt.n;
+      M += reqs[i].n_tokens;
+    }
+    const bool single = act.size() == 1;
+    const int i0 = act[0];
+    // input rows
+    const __nv_bfloat16* X_in = nullptr;
+    int in_buf = -1;
+    if (single && curp[i0] && !(reqs[i0].s == l && l == 0)) {
+      X_in = curp[i0];
+    } else {
+      // in place already?
+      for (int b = 0; b < 2 && !X_in; ++b) {
+        bool all = true;
+        for (int k = 0; k < rt.n; ++k)
+          all &= curp[act[k]] == G[b] + static_cast<size_t>(rt.row0[k]) * D.h;
+        if (all) {
+          X_in = G[b];
+          in_buf = b;
+        }
+      }
+      if (!X_in) {
+        // gather into the buffer not holding any current rows
+        int b = 0;
+        for (int k = 0; k < rt.n; ++k) {
+          const auto* cp = curp[act[k]];
+          if (cp >= G[0] && cp < G[0] + static_cast<size_t>(plan.M) * D.h) b = 1;
+        }
+        for (int k = 0; k < rt.n; ++k) {
+          const int i = act[k];
+          __nv_bfloat16* dst = G[b] + static_cast<size_t>(rt.row0[k]) * D.h;
+          if (reqs[i].s == l && l == 0) {
+            CRF_CUDA(launch_embed(static_cast<const __nv_bfloat16*>(model->embed), reqs[i].tokens, dst,
+                                  reqs[i].n_tokens, D.h, st));
+          } else {
+            CRF_CUDA(cudaMemcpyAsync(dst, curp[i], reqs[i].n_tokens * row_bytes,
+                                     cudaMemcpyDeviceToDevice, st));
+          }
+        }
+        X_in = G[b];
+        in_buf = b;
+      }
+    }
+    // output rows
+    __nv_bfloat16* X_out;
+    if (single && reqs[i0].hidden_out) {
+      X_out = static_cast<__nv_bfloat16*>(reqs[i0].hidden_out[l - reqs[i0].s]);
+    } else {
+      int b = in_buf >= 0 ? 1 - in_buf : 0;
+      X_out = G[b];
+    }
+    s = run_layer(c, l, X_in, X_out, M, rt);
+    if (s != CRF_OK) return s;
+    for (int k = 0; k < rt.n; ++k) {
+      const int i = act[k];
+      curp[i] = X_out + static_cast<size_t>(rt.row0[k]) * D.h;
+      if (!single && reqs[i].hidden_out)
+        CRF_CUDA(cudaMemcpyAsync(reqs[i].hidden_out[l - reqs[i].s], curp[i],
+                                 reqs[i].n_tokens * row_bytes, cudaMemcpyDeviceToDevice, st));
+      if (l == reqs[i].e - 1 && reqs[i].final_hidden_out)
+        CRF_CUDA(cudaMemcpyAsync(dx0 + static_cast<size_t>(i) * D.h,
+                                 curp[i] + static_cast<size_t>(reqs[i].n_tokens - 1) * D.h, row_bytes,
+                                 cudaMemcpyDeviceToDevice, st));
+    }
+  }
+
+  // first-step state: the last prefix row through layers e..N-1 on the historical cache
+  for (int i = 0; i < n_req; ++i) {
+    const crf_request& r = reqs[i];
+    if (!r.final_hidden_out) continue;
+    const __nv_bfloat16* start = dx0 + static_cast<size_t>(i) * D.h;
+    if (r.s == r.e) {
+      if (r.s == 0) {
+        CRF_CUDA(launch_embed(static_cast<const __nv_bfloat16*>(model->embed), r.tokens + (r.n_tokens - 1),
+                              dx0 + static_cast<size_t>(i) * D.h, 1, D.h, st));
+      } else {
+        CRF_CUDA(cudaMemcpyAsync(dx0 + static_cast<size_t>(i) * D.h,
+                                 static_cast<const __nv_bfloat16*>(r.hidden_in) +
+                                     static_cast<size_t>(r.n_tokens - 1) * D.h,
+                                 row_bytes, cudaMemcpyDeviceToDevice, st));
+      }
+    }
+    if (r.e == D.N) {
+      CRF_CUDA(cudaMemcpyAsync(r.final_hidden_out, start, row_bytes, cudaMemcpyDeviceToDevice, st));
+    } else {
+      s = decode_row(c, r.e, start, r.n_tokens - 1, r.page_table, r.final_hidden_out);
+      if (s != CRF_OK) return s;
+    }
+  }
+  CRF_CUDA(cudaGetLastError());
+  return CRF_OK;
+}
+
+// ---------------------------------------------------------------- drift
+static int drift_blocks_per_side(const crf_ctx* ctx, int n_items) {
+  const int want = (4 * ctx->num_sms + 2 * n_items - 1) / std::max(1, 2 * n_items);
+  return std::max(1, std::min(16, want));
+}
+
+crf_status crf_drift_workspace_size(crf_ctx* ctx, const crf_model_dims* dims,
+                                    const crf_lora_dims* lora, size_t* bytes) {
+  if (!ctx || !dims || !lora || !bytes) return fail(CRF_EINVAL, "null argument");
+  crf_status s = check_lora(*lora);
+  if (s != CRF_OK) return s;
+  int nm = 0;
+  for (int m = 0; m < 7; ++m) nm += (lora->module_mask >> m) & 1;
+  const int items = dims->n_layers * nm;
+  const int bps = drift_blocks_per_side(ctx, std::max(1, items));
+  const size_t r2 = 2 * lora->rank;
+  *bytes = align256(static_cast<size_t>(items) * 2 * bps * r2 * r2 * sizeof(float));
+  return CRF_OK;
+}
+
+crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter* cur,
+                     const crf_adapter* const* anchors, float* out_sq, void* workspace,
+                     size_t ws_bytes, void* stream) {
+  if (!ctx || !dims || !cur || !anchors || !out_sq) return fail(CRF_EINVAL, "null argument");
+  if (dims->n_layers < 1) return fail(CRF_EINVAL, "n_layers must be positive");
+  crf_status s = check_lora(cur->dims);
+  if (s != CRF_OK) return s;
+  if (!cur->A || !cur->B) return fail(CRF_EINVAL, "adapter tables missing");
+  const Dims D = dims_of(*dims);
+  std::vector<DriftItem> items;
+  for (int l = 0; l < D.N; ++l) {
+    const crf_adapter* an = anchors[l];
+    if (!an || !an->A || !an->B) return fail(CRF_EINVAL, "anchor %d missing", l);
+    if (an->dims.rank != cur->dims.rank || an->dims.module_mask != cur->dims.module_mask)
+      return fail(CRF_ESHAPE, "anchor %d has different LoRA dims", l);
+    for (int m = 0; m < 7; ++m) {
+      if (!adapted(cur, m)) continue;
+      DriftItem it;
+      it.A0 = static_cast<const __nv_bfloat16*>(an->A[l * 7 + m]);
+      it.B0 = static_cast<const __nv_bfloat16*>(an->B[l * 7 + m]);
+      it.A1 = static_cast<const __nv_bfloat16*>(cur->A[l * 7 + m]);
+      it.B1 = static_cast<const __nv_bfloat16*>(cur->B[l * 7 + m]);
+      if (!it.A0 || !it.B0 || !it.A1 || !it.B1)
+        return fail(CRF_EINVAL, "layer %d module %d factor is null", l, m);
+      module_shape(D, m, it.out_dim, it.in_dim);
+      it.out_index = l * 7 + m;
+      items.push_back(it);
+    }
+  }
+  size_t need = 0;
+  s = crf_drift_workspace_size(ctx, dims, &cur->dims, &need);
+  if (s != CRF_OK) return s;
+  if (!workspace || ws_bytes < need) return fail(CRF_ENOMEM, "drift workspace %zu < %zu", ws_bytes, need);
+  CRF_CUDA(cudaSetDevice(ctx->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CRF_CUDA(cudaMemsetAsync(out_sq, 0, static_cast<size_t>(D.N) * 7 * 2 * sizeof(float), st));
+  if (items.empty()) return CRF_OK;
+  const int bps = drift_blocks_per_side(ctx, static_cast<int>(items.size()));
+  CRF_CUDA(launch_drift(items.data(), static_cast<int>(items.size()), cur->dims.rank,
+                        static_cast<float*>(workspace), bps, out_sq, st));
+  return CRF_OK;
+}
+
+// ---------------------------------------------------------------- KL
+static int kl_splits(const crf_ctx* ctx, int n_rows, int vocab) {
+  const int want = (2 * ctx->num_sms + n_rows - 1) / std::max(1, n_rows);
+  return std::max(1, std::min(want, (vocab + 1023) / 1024));
+}
+
+crf_status crf_kl_workspace_size(crf_ctx* ctx, int n_rows, int vocab, int hidden, size_t* bytes) {
+  if (!ctx || !bytes || n_rows < 1 || vocab < 1 || hidden < 0)
+    return fail(CRF_EINVAL, "bad argument");
+  const int sp = kl_splits(ctx, n_rows, vocab);
+  size_t o = align256(static_cast<size_t>(n_rows) * sp * 5 * sizeof(float));
+  if (hidden > 0) {
+    o += align256(static_cast<size_t>(2 * n_rows) * hidden * sizeof(float)) * 2;
+    o += align256(static_cast<size_t>(2 * n_rows) * vocab * sizeof(float));
+  }
+  *bytes = o;
+  return CRF_OK;
+}
+
+crf_status crf_kl(crf_ctx* ctx, const crf_model* model, const void* ref, const void* cur,
+                  int n_rows, int vocab, float* out_kl, float* logits_out, void* workspace,
+                  size_t ws_bytes, void* stream) {
+  if (!ctx || !ref || !cur || !out_kl) return fail(CRF_EINVAL, "null argument");
+  if (n_rows < 1 || vocab < 1) return fail(CRF_EINVAL, "n_rows and vocab must be positive");
+  const int hidden = model ? model->dims.hidden : 0;
+  if (model) {
+    if (model->dims.vocab != vocab) return fail(CRF_ESHAPE, "vocab %d != model vocab %d", vocab, model->dims.vocab);
+    if (!model->lm_head || !model->final_norm) return fail(CRF_EINVAL, "model LM head or final norm is null");
+    if (hidden < 1 || hidden % 8) return fail(CRF_EUNSUPPORTED, "hidden must be a positive multiple of 8");
+  }
+  size_t need = 0;
+  crf_status s = crf_kl_workspace_size(ctx, n_rows, vocab, hidden, &need);
+  if (s != CRF_OK) return s;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255) || ws_bytes < need)
+    return fail(CRF_ENOMEM, "KL workspace null, misaligned or %zu < %zu", ws_bytes, need);
+  CRF_CUDA(cudaSetDevice(ctx->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const int sp = kl_splits(ctx, n_rows, vocab);
+  float* part = reinterpret_cast<float*>(ws);
+  size_t o = align256(static_cast<size_t>(n_rows) * sp * 5 * sizeof(float));
+  const float* zr = static_cast<const float*>(ref);
+  const float* zc = static_cast<const float*>(cur);
+  if (model) {
+    float* hf = reinterpret_cast<float*>(ws + o);
+    o += align256(static_cast<size_t>(2 * n_rows) * hidden * sizeof(float));
+    float* hn = reinterpret_cast<float*>(ws + o);
+    o += align256(static_cast<size_t>(2 * n_rows) * hidden * sizeof(float));
+    float* logits = logits_out ? logits_out : reinterpret_cast<float*>(ws + o);
+    CRF_CUDA(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(ref), hf, n_rows * hidden, st));
+    CRF_CUDA(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(cur), hf + static_cast<size_t>(n_rows) * hidden,
+                                n_rows * hidden, st));
+    CRF_CUDA(launch_rmsnorm_f32(hf, static_cast<const __nv_bfloat16*>(model->final_norm), hn, 2 * n_rows,
+                                hidden, model->dims.rms_eps, st));
+    CRF_CUDA(launch_lm_head(static_cast<const __nv_bfloat16*>(model->lm_head), hn, 2 * n_rows, vocab,
+                            hidden, logits, st));
+    zr = logits;
+    zc = logits + static_cast<size_t>(n_rows) * vocab;
+  }
+  CRF_CUDA(launch_kl(zr, zc, n_rows, vocab, out_kl, part, sp, st));
+  return CRF_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,152 @@
+// Internal launcher interface between the C ABI layer (api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace crf {
+
+constexpr int kMaxReq = 32;   // equals CRF_MAX_REQUESTS
+constexpr int kPage = 16;
+constexpr int kRankPad = 16;  // LoRA rank padded to one K=16 MMA step
+
+// Rows of a batched activation matrix that belong to each request.
+struct ReqTable {
+  int n;
+  int row0[kMaxReq];
+  int len[kMaxReq];
+  const int32_t* page_table[kMaxReq];
+};
+
+enum EpiKind : int {
+  kEpiScaleBf16 = 0,  // out = bf16(acc * scale)                        (LoRA down product)
+  kEpiQkv = 1,        // +bias, RoPE(q,k); q -> qbuf, k/v -> KV pages    (Eq. S3)
+  kEpiResid = 2,      // out = bf16(resid + acc)                         (o / down projection)
+  kEpiSwiGLU = 3      // out = bf16(silu(gate) * up), tile = [gate | up]  (MLP)
+};
+
+// Host description of one GEMM  D[M, cols] = A[M, K] * B[cols, K]^T (+ LoRA ext) -> epilogue.
+// Column space: `ngroups` groups laid side by side, each with its own weight
+// matrix (plain mode, nseg == 1), or one group whose tiles stack `nseg` equal
+// row segments of different matrices (paired / stacked mode, ngroups == 1).
+struct GemmDesc {
+  const void* A;
+  int M, K, lda;
+  int ngroups, nseg;
+  const void* B[3];       // map index g + s
+  int B_rows[3];          // rows of each B matrix
+  int ldb[3];
+  int group_cols[3];      // valid output columns per group (plain) / per segment (stacked)
+  // LoRA extension: D += XA[:, xa_col] * BL^T (K = 16); XA already scaled by alpha/r
+  const void* XA;
+  int ldxa;
+  const void* BL[3];
+  int rank;
+  int lora_on[3][3];
+  int xa_col[3][3];
+  // epilogue
+  int epi;
+  float scale;
+  void* out;
+  int ldo;
+  const void* resid;
+  int ld_resid;
+  const void* bias[3];
+  const float2* rope;     // [positions][head_dim/2] (cos, sin)
+  int head_dim, n_kv_heads;
+  void* qbuf;
+  int ldq;
+  void* kpages;
+  void* vpages;
+  ReqTable req;
+  int* status;
+};
+
+// Launch the tcgen05 GEMM. bn: 256 or 128 for projections; 16/32/48 for LoRA down.
+cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream);
+
+// ------------------------------------------------------------------ other kernels
+cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double theta,
+                              cudaStream_t stream);
+cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bfloat16* y,
+                           int rows, int hidden, float eps, cudaStream_t stream);
+cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv_bfloat16* out,
+                         int n, int hidden, cudaStream_t stream);
+
+// Causal GQA prefill attention over the paged cache of the current layer.
+struct AttnDesc {
+  const __nv_bfloat16* q;  // [rows, Hq*d] post-RoPE
+  int ldq;
+  const __nv_bfloat16* kpages;  // [P][Hkv][16][d]
+  const __nv_bfloat16* vpages;
+  __nv_bfloat16* out;      // [rows, Hq*d]
+  int ldo;
+  int n_q_heads, n_kv_heads, head_dim;
+  ReqTable req;
+  int* status;
+};
+cudaError_t launch_attention(const AttnDesc& d, int num_sms, cudaStream_t stream);
+
+// Small-M decode path (the last prefix row through the layers after the window).
+// y[r, j] = sum_i W[j, i] x[r, i] (+ bias[j]) (+ sum_k BL[j, k] xa[r, k]) (+ resid[r, j])
+struct GemvDesc {
+  const __nv_bfloat16* W;
+  int out_dim, in_dim;
+  const float* x;          // [rows, in_dim] fp32
+  int rows;
+  const __nv_bfloat16* bias;
+  const __nv_bfloat16* BL; // [out_dim, rank] or null
+  const float* xa;         // [rows, rank] fp32 already scaled by alpha/r
+  int rank;
+  const float* resid;      // [rows, out_dim] fp32 or null
+  float* y;                // [rows, out_dim] fp32
+};
+cudaError_t launch_gemv(const GemvDesc& d, cudaStream_t stream);
+// xa[r, k] = scale * sum_i A[k, i] x[r, i]
+cudaError_t launch_lora_down_rows(const __nv_bfloat16* A, int rank, int in_dim, const float* x,
+                                  int rows, float scale, float* xa, cudaStream_t stream);
+cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y, int rows,
+                               int hidden, float eps, cudaStream_t stream);
+// Single-query attention of `rows` decode rows (one per request) over pages [0, pos) plus own k/v.
+struct DecodeAttnDesc {
+  const float* q;          // [rows, Hq*d] fp32 post-RoPE
+  const float* k_self;     // [rows, Hkv*d]
+  const float* v_self;
+  const __nv_bfloat16* kpages;
+  const __nv_bfloat16* vpages;
+  const int32_t* page_table[kMaxReq];  // per decode row
+  int pos[kMaxReq];        // position of the decode row (= number of cached keys before it)
+  float* out;              // [rows, Hq*d]
+  float* part;             // scratch [rows, Hq, splits, d + 2]
+  int rows, n_q_heads, n_kv_heads, head_dim, splits, max_pos;
+};
+cudaError_t launch_decode_attention(const DecodeAttnDesc& d, cudaStream_t stream);
+cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, int pos,
+                             double theta, cudaStream_t stream);
+cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream);
+cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream);
+cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStream_t stream);
+cudaError_t launch_gather_rows_f32(const __nv_bfloat16* src, const int64_t* row_index, float* dst,
+                                   int rows, int hidden, cudaStream_t stream);
+
+// LM head + KL: logits [2*rows, V] (ref rows first) from final-normed hidden rows.
+cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,
+                           float* logits, cudaStream_t stream);
+// KL per row from fp32 logits; part: scratch [rows][splits][4].
+cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab, float* out,
+                      float* part, int splits, cudaStream_t stream);
+
+// Drift: per (layer, module) squared norms; see crf_drift.
+struct DriftItem {
+  const __nv_bfloat16* A0; const __nv_bfloat16* B0;
+  const __nv_bfloat16* A1; const __nv_bfloat16* B1;
+  int in_dim, out_dim;
+  int out_index;           // layer * 7 + module
+};
+cudaError_t launch_drift(const DriftItem* items_dev, int n_items, int rank, float* grams,
+                         int blocks_per_side, float* out_sq, cudaStream_t stream);
+
+}  // namespace crf

@@ -1,0 +1,559 @@
+// Memory-bound kernels: RMSNorm, embedding gather, RoPE angle table, the
+// small-M decode path (GEMV with fused LoRA, RoPE on rows, SwiGLU), the LM
+// head, the first-step KL reduction (Section S2.1) and the rank-factored
+// adapter drift (Eq. 8).
+#include "common.cuh"
+#include "kernels.h"
+
+#include <cfloat>
+
+namespace crf {
+
+namespace {
+
+// ------------------------------------------------------------------ RoPE table
+// table[p][i] = (cos, sin)(p * theta^(-2i/d)), angle formed in fp64.
+__global__ void rope_table_kernel(float2* table, int n_pos, int half, double theta, int d) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= n_pos * half) return;
+  const int p = idx / half, i = idx % half;
+  // angle p * theta^(-2i/d) in fp64, reduced to turns in [0, 1), then fp32 sincospi
+  const double inv_freq = pow(theta, -2.0 * i / d);
+  double turns = static_cast<double>(p) * inv_freq * 0.15915494309189535;  // 1 / (2 pi)
+  turns -= floor(turns);
+  float s, c;
+  sincospif(static_cast<float>(2.0 * turns), &s, &c);
+  table[idx] = make_float2(c, s);
+}
+
+// ------------------------------------------------------------------ RMSNorm
+// One warp per row: y = x * rsqrt(mean(x^2) + eps) * g, fp32 math, bf16 out.
+__global__ void rmsnorm_kernel(const __nv_bfloat16* __restrict__ x,
+                               const __nv_bfloat16* __restrict__ g, __nv_bfloat16* __restrict__ y,
+                               int rows, int hidden, float eps) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= rows) return;
+  const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)warp * hidden);
+  const uint4* gr = reinterpret_cast<const uint4*>(g);
+  uint4* yr = reinterpret_cast<uint4*>(y + (size_t)warp * hidden);
+  const int nv = hidden / 8;
+  float ss = 0.f;
+  for (int i = lane; i < nv; i += 32) {
+    const uint4 u = xr[i];
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float a = bf16_lo(w[j]), b = bf16_hi(w[j]);
+      ss += a * a + b * b;
+    }
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / hidden + eps);
+  for (int i = lane; i < nv; i += 32) {
+    const uint4 u = xr[i];
+    const uint4 gv = gr[i];
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      o[j] = pack_bf16(bf16_lo(w[j]) * inv * bf16_lo(gw[j]), bf16_hi(w[j]) * inv * bf16_hi(gw[j]));
+    yr[i] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+__global__ void rmsnorm_f32_kernel(const float* __restrict__ x, const __nv_bfloat16* __restrict__ g,
+                                   float* __restrict__ y, int rows, int hidden, float eps) {
+  const int row = blockIdx.x;
+  __shared__ float red[32];
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < hidden; i += blockDim.x) {
+    const float v = x[(size_t)row * hidden + i];
+    ss += v * v;
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  const float inv = rsqrtf(red[0] / hidden + eps);
+  for (int i = threadIdx.x; i < hidden; i += blockDim.x)
+    y[(size_t)row * hidden + i] = x[(size_t)row * hidden + i] * inv * __bfloat162float(g[i]);
+}
+
+// ------------------------------------------------------------------ embedding
+__global__ void embed_kernel(const __nv_bfloat16* __restrict__ e, const int32_t* __restrict__ tok,
+                             __nv_bfloat16* __restrict__ out, int n, int hidden) {
+  const int nv = hidden / 8;
+  const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (size_t)n * nv) return;
+  const int t = static_cast<int>(idx / nv), c = static_cast<int>(idx % nv);
+  reinterpret_cast<uint4*>(out + (size_t)t * hidden)[c] =
+      reinterpret_cast<const uint4*>(e + (size_t)tok[t] * hidden)[c];
+}
+
+// ------------------------------------------------------------------ decode-path GEMV
+// Block of 8 warps; warp w computes output j = blockIdx.x * 8 + w for every row.
+// x is staged through shared memory in K chunks.
+constexpr int kGemvWarps = 8;
+constexpr int kGemvChunk = 1024;
+constexpr int kGemvMaxRows = 8;
+
+__global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const GemvDesc d) {
+  __shared__ float xs[kGemvMaxRows * kGemvChunk];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = blockIdx.x * kGemvWarps + warp;
+  const int r0 = blockIdx.y * kGemvMaxRows;
+  const int nr = min(kGemvMaxRows, d.rows - r0);
+  float acc[kGemvMaxRows];
+#pragma unroll
+  for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = 0.f;
+  for (int k0 = 0; k0 < d.in_dim; k0 += kGemvChunk) {
+    const int kc = min(kGemvChunk, d.in_dim - k0);
+    __syncthreads();
+    for (int i = threadIdx.x; i < nr * kc; i += blockDim.x) {
+      const int r = i / kc, c = i % kc;
+      xs[r * kGemvChunk + c] = d.x[(size_t)(r0 + r) * d.in_dim + k0 + c];
+    }
+    __syncthreads();
+    if (j < d.out_dim) {
+      const __nv_bfloat16* wr = d.W + (size_t)j * d.in_dim + k0;
+      for (int c = lane * 8; c < kc; c += 256) {
+        const uint4 u = *reinterpret_cast<const uint4*>(wr + c);
+        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+        float wf[8];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          wf[2 * q] = bf16_lo(wv[q]);
+          wf[2 * q + 1] = bf16_hi(wv[q]);
+        }
+#pragma unroll
+        for (int r = 0; r < kGemvMaxRows; ++r) {
+          if (r < nr) {
+            const float* xr = xs + r * kGemvChunk + c;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) acc[r] += wf[q] * xr[q];
+          }
+        }
+      }
+    }
+  }
+  if (j >= d.out_dim) return;
+#pragma unroll
+  for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = warp_sum(acc[r]);
+  if (lane < nr) {
+    const int r = lane;
+    float v = 0.f;
+#pragma unroll
+    for (int q = 0; q < kGemvMaxRows; ++q)
+      if (q == r) v = acc[q];
+    if (d.bias) v += __bfloat162float(d.bias[j]);
+    if (d.BL) {
+      for (int k = 0; k < d.rank; ++k)
+        v += __bfloat162float(d.BL[(size_t)j * d.rank + k]) * d.xa[(size_t)(r0 + r) * d.rank + k];
+    }
+    if (d.resid) v += d.resid[(size_t)(r0 + r) * d.out_dim + j];
+    d.y[(size_t)(r0 + r) * d.out_dim + j] = v;
+  }
+}
+
+// xa[r, k] = scale * <A[k, :], x[r, :]>, one warp per (r, k).
+__global__ void lora_down_rows_kernel(const __nv_bfloat16* __restrict__ A, int rank, int in_dim,
+                                      const float* __restrict__ x, int rows, float scale,
+                                      float* __restrict__ xa) {
+  const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w >= rows * rank) return;
+  const int r = w / rank, k = w % rank;
+  float s = 0.f;
+  for (int i = lane; i < in_dim; i += 32)
+    s += __bfloat162float(A[(size_t)k * in_dim + i]) * x[(size_t)r * in_dim + i];
+  s = warp_sum(s);
+  if (lane == 0) xa[(size_t)r * rank + k] = s * scale;
+}
+
+// Rotate-half RoPE on fp32 rows x [rows, heads, d] at positions pos[r], angle in fp64.
+__global__ void rope_rows_kernel(float* x, int rows, int heads, int d, int pos, double theta) {
+  const int half = d / 2;
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * heads * half) return;
+  const int i = idx % half;
+  const int h = (idx / half) % heads;
+  const int r = idx / (half * heads);
+  double turns = static_cast<double>(pos) * pow(theta, -2.0 * i / d) * 0.15915494309189535;
+  turns -= floor(turns);
+  float s, c;
+  sincospif(static_cast<float>(2.0 * turns), &s, &c);
+  float* base = x + ((size_t)r * heads + h) * d;
+  const float x1 = base[i], x2 = base[i + half];
+  base[i] = x1 * c - x2 * s;
+  base[i + half] = x2 * c + x1 * s;
+}
+
+// gu [rows, 2, ffn] (gate then up) -> m [rows, ffn]
+__global__ void swiglu_f32_kernel(const float* gu, float* m, int rows, int ffn) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * ffn) return;
+  const int r = idx / ffn, j = idx % ffn;
+  const float g = gu[(size_t)r * 2 * ffn + j], u = gu[(size_t)r * 2 * ffn + ffn + j];
+  m[idx] = g / (1.f + __expf(-g)) * u;
+}
+
+__global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) y[i] = __float2bfloat16_rn(x[i]);
+}
+__global__ void bf16_to_f32_kernel(const __nv_bfloat16* x, float* y, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) y[i] = __bfloat162float(x[i]);
+}
+__global__ void gather_rows_f32_kernel(const __nv_bfloat16* src, const int64_t* row_index, float* dst,
+                                       int rows, int hidden) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * hidden) return;
+  const int r = idx / hidden, c = idx % hidden;
+  dst[idx] = __bfloat162float(src[row_index[r] * hidden + c]);
+}
+
+// ------------------------------------------------------------------ KL
+// Per (row, split): online (max, sum e^(z* - m), sum e^(z* - m)(z* - z)) for the
+// reference and (max, sum e^(z - m)) for the current logits.
+constexpr int kKlThreads = 256;
+
+__global__ void __launch_bounds__(kKlThreads) kl_partial_kernel(const float* __restrict__ zr,
+                                                                const float* __restrict__ zc,
+                                                                int vocab, int splits,
+                                                                float* __restrict__ part) {
+  const int row = blockIdx.y, sp = blockIdx.x;
+  const int per = (vocab + splits - 1) / splits;
+  const int v0 = sp * per, v1 = min(vocab, v0 + per);
+  const float* a = zr + (size_t)row * vocab;
+  const float* b = zc + (size_t)row * vocab;
+  float mr = -FLT_MAX, sr = 0.f, dr = 0.f, mc = -FLT_MAX, sc = 0.f;
+  for (int i = v0 + threadIdx.x; i < v1; i += kKlThreads) {
+    const float x = a[i], y = b[i];
+    if (x > mr) {
+      const float f = __expf(mr - x);
+      sr *= f;
+      dr *= f;
+      mr = x;
+    }
+    const float e = __expf(x - mr);
+    sr += e;
+    dr += e * (x - y);
+    if (y > mc) {
+      sc *= __expf(mc - y);
+      mc = y;
+    }
+    sc += __expf(y - mc);
+  }
+  // block combine
+  __shared__ float s_mr[kKlThreads], s_sr[kKlThreads], s_dr[kKlThreads], s_mc[kKlThreads],
+      s_sc[kKlThreads];
+  s_mr[threadIdx.x] = mr;
+  s_sr[threadIdx.x] = sr;
+  s_dr[threadIdx.x] = dr;
+  s_mc[threadIdx.x] = mc;
+  s_sc[threadIdx.x] = sc;
+  __syncthreads();
+  for (int off = kKlThreads / 2; off > 0; off >>= 1) {
+    if (threadIdx.x < off) {
+      const int o = threadIdx.x + off;
+      const float M = fmaxf(s_mr[threadIdx.x], s_mr[o]);
+      const float f1 = s_mr[threadIdx.x] == -FLT_MAX ? 0.f : __expf(s_mr[threadIdx.x] - M);
+      const float f2 = s_mr[o] == -FLT_MAX ? 0.f : __expf(s_mr[o] - M);
+      s_sr[threadIdx.x] = s_sr[threadIdx.x] * f1 + s_sr[o] * f2;
+      s_dr[threadIdx.x] = s_dr[threadIdx.x] * f1 + s_dr[o] * f2;
+      s_mr[threadIdx.x] = M;
+      const float Mc = fmaxf(s_mc[threadIdx.x], s_mc[o]);
+      const float g1 = s_mc[threadIdx.x] == -FLT_MAX ? 0.f : __expf(s_mc[threadIdx.x] - Mc);
+      const float g2 = s_mc[o] == -FLT_MAX ? 0.f : __expf(s_mc[o] - Mc);
+      s_sc[threadIdx.x] = s_sc[threadIdx.x] * g1 + s_sc[o] * g2;
+      s_mc[threadIdx.x] = Mc;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    float* p = part + ((size_t)row * splits + sp) * 5;
+    p[0] = s_mr[0];
+    p[1] = s_sr[0];
+    p[2] = s_dr[0];
+    p[3] = s_mc[0];
+    p[4] = s_sc[0];
+  }
+}
+
+// KL = D/S* + (M + log S) - (M* + log S*)  combining the splits of one row (fp64).
+__global__ void kl_final_kernel(const float* part, int splits, float* out, int rows) {
+  const int row = blockIdx.x * blockDim.x + threadIdx.x;
+  if (row >= rows) return;
+  const float* p = part + (size_t)row * splits * 5;
+  double Mr = -1e300, Mc = -1e300;
+  for (int s = 0; s < splits; ++s) {
+    Mr = fmax(Mr, (double)p[s * 5 + 0]);
+    Mc = fmax(Mc, (double)p[s * 5 + 3]);
+  }
+  double Sr = 0, Dr = 0, Sc = 0;
+  for (int s = 0; s < splits; ++s) {
+    const double fr = exp((double)p[s * 5 + 0] - Mr);
+    Sr += fr * p[s * 5 + 1];
+    Dr += fr * p[s * 5 + 2];
+    Sc += exp((double)p[s * 5 + 3] - Mc) * p[s * 5 + 4];
+  }
+  out[row] = static_cast<float>(Dr / Sr + (Mc + log(Sc)) - (Mr + log(Sr)));
+}
+
+// ------------------------------------------------------------------ drift
+// Partial 2r x 2r Grams over a chunk of the long dimension, for one side of one
+// (layer, module) item. Side 0 (B): vector per output row o is
+// (B1[o,:] - B0[o,:], B0[o,:]); side 1 (A): vector per input column c is
+// (A1[:,c], A1[:,c] - A0[:,c]).
+constexpr int kDriftRows = 128;
+constexpr int kMaxDriftItems = 224;
+
+struct DriftBatch {
+  DriftItem items[kMaxDriftItems];
+  int n_items;
+};
+
+template <int R2>
+__global__ void __launch_bounds__(256) drift_partial_kernel(const __grid_constant__ DriftBatch batch,
+                                                            int blocks_per_side, float* grams) {
+  constexpr int R = R2 / 2;
+  const int item = blockIdx.z, side = blockIdx.y, blk = blockIdx.x;
+  const DriftItem& it = batch.items[item];
+  const int L = side == 0 ? it.out_dim : it.in_dim;
+  const int per = (L + blocks_per_side - 1) / blocks_per_side;
+  const int l0 = blk * per, l1 = min(L, l0 + per);
+  __shared__ float vec[kDriftRows][R2 + 1];
+  constexpr int T = R2 / 4;  // 4x4 tiles per dimension
+  // thread layout: group = tid / (T*T) splits the rows of each chunk
+  constexpr int TILES = T * T;
+  constexpr int GROUPS = 256 / TILES;
+  const int tid = threadIdx.x;
+  const int grp = tid / TILES, tt = tid % TILES;
+  const int ti = tt / T, tj = tt % T;
+  float acc[4][4];
+#pragma unroll
+  for (int a = 0; a < 4; ++a)
+#pragma unroll
+    for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
+  for (int c0 = l0; c0 < l1; c0 += kDriftRows) {
+    const int cn = min(kDriftRows, l1 - c0);
+    __syncthreads();
+    for (int i = tid; i < cn * R; i += 256) {
+      if (side == 0) {
+        const int rr = i / R, k = i % R;
+        const size_t off = (size_t)(c0 + rr) * R + k;
+        const float b0 = __bfloat162float(it.B0[off]), b1 = __bfloat162float(it.B1[off]);
+        vec[rr][k] = b1 - b0;
+        vec[rr][R + k] = b0;
+      } else {
+        const int k = i / cn, rr = i % cn;  // coalesced along the input dimension
+        const size_t off = (size_t)k * it.in_dim + c0 + rr;
+        const float a0 = __bfloat162float(it.A0[off]), a1 = __bfloat162float(it.A1[off]);
+        vec[rr][k] = a1;
+        vec[rr][R + k] = a1 - a0;
+      }
+    }
+    __syncthreads();
+    for (int rr = grp; rr < cn; rr += GROUPS) {
+      float x[4], y[4];
+#pragma unroll
+      for (int a = 0; a < 4; ++a) {
+        x[a] = vec[rr][ti * 4 + a];
+        y[a] = vec[rr][tj * 4 + a];
+      }
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] += x[a] * y[b];
+    }
+  }
+  // reduce the groups through shared memory (reuse vec as [GROUPS][R2*R2] is too big; do it in steps)
+  __shared__ float red[R2 * R2];
+  for (int gg = 0; gg < GROUPS; ++gg) {
+    __syncthreads();
+    if (grp == gg) {
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          float& dst = red[(ti * 4 + a) * R2 + tj * 4 + b];
+          dst = (gg == 0 ? 0.f : dst) + acc[a][b];
+        }
+    }
+  }
+  __syncthreads();
+  float* out = grams + (((size_t)item * 2 + side) * blocks_per_side + blk) * R2 * R2;
+  for (int i = tid; i < R2 * R2; i += 256) out[i] = red[i];
+}
+
+template <int R2>
+__global__ void __launch_bounds__(256) drift_final_kernel(const __grid_constant__ DriftBatch batch,
+                                                          int blocks_per_side, const float* grams,
+                                                          float* out_sq) {
+  constexpr int R = R2 / 2;
+  const int item = blockIdx.x;
+  __shared__ float gb[R2 * R2], ga[R2 * R2];
+  for (int i = threadIdx.x; i < R2 * R2; i += 256) {
+    float sb = 0.f, sa = 0.f;
+    for (int b = 0; b < blocks_per_side; ++b) {
+      sb += grams[(((size_t)item * 2 + 0) * blocks_per_side + b) * R2 * R2 + i];
+      sa += grams[(((size_t)item * 2 + 1) * blocks_per_side + b) * R2 * R2 + i];
+    }
+    gb[i] = sb;
+    ga[i] = sa;
+  }
+  __syncthreads();
+  // trace(Gb Ga) = sum_ij Gb[i,j] Ga[j,i]
+  float t = 0.f;
+  for (int i = threadIdx.x; i < R2 * R2; i += 256) {
+    const int a = i / R2, b = i % R2;
+    t += gb[i] * ga[b * R2 + a];
+  }
+  __shared__ float red[8];
+  t = warp_sum(t);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = t;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float tot = 0.f;
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    float par = 0.f;
+    for (int k = 0; k < R; ++k) par += gb[k * R2 + k] + ga[(R + k) * R2 + R + k];
+    out_sq[batch.items[item].out_index * 2 + 0] = tot;
+    out_sq[batch.items[item].out_index * 2 + 1] = par;
+  }
+}
+
+inline int cdiv(long a, long b) { return static_cast<int>((a + b - 1) / b); }
+
+}  // namespace
+
+cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double theta,
+                              cudaStream_t stream) {
+  const int half = head_dim / 2;
+  const int n = n_pos * half;
+  if (n == 0) return cudaSuccess;
+  rope_table_kernel<<<cdiv(n, 256), 256, 0, stream>>>(table, n_pos, half, theta, head_dim);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bfloat16* y,
+                           int rows, int hidden, float eps, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  rmsnorm_kernel<<<cdiv(rows, 8), 256, 0, stream>>>(x, g, y, rows, hidden, eps);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv_bfloat16* out,
+                         int n, int hidden, cudaStream_t stream) {
+  const long total = (long)n * (hidden / 8);
+  if (total == 0) return cudaSuccess;
+  embed_kernel<<<cdiv(total, 256), 256, 0, stream>>>(embed, tokens, out, n, hidden);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemv(const GemvDesc& d, cudaStream_t stream) {
+  if (d.rows == 0 || d.out_dim == 0) return cudaSuccess;
+  dim3 grid(cdiv(d.out_dim, kGemvWarps), cdiv(d.rows, kGemvMaxRows));
+  gemv_kernel<<<grid, kGemvWarps * 32, 0, stream>>>(d);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lora_down_rows(const __nv_bfloat16* A, int rank, int in_dim, const float* x,
+                                  int rows, float scale, float* xa, cudaStream_t stream) {
+  const int warps = rows * rank;
+  if (warps == 0) return cudaSuccess;
+  lora_down_rows_kernel<<<cdiv(warps, 8), 256, 0, stream>>>(A, rank, in_dim, x, rows, scale, xa);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y, int rows,
+                               int hidden, float eps, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  rmsnorm_f32_kernel<<<rows, 256, 0, stream>>>(x, g, y, rows, hidden, eps);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, int pos,
+                             double theta, cudaStream_t stream) {
+  const int n = rows * heads * head_dim / 2;
+  if (n == 0) return cudaSuccess;
+  rope_rows_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, rows, heads, head_dim, pos, theta);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream) {
+  const int n = rows * ffn;
+  if (n == 0) return cudaSuccess;
+  swiglu_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(gu, m, rows, ffn);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  f32_to_bf16_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, y, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  bf16_to_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, y, n);
+  return cudaGetLastError();
+}
+cudaError_t launch_gather_rows_f32(const __nv_bfloat16* src, const int64_t* row_index, float* dst,
+                                   int rows, int hidden, cudaStream_t stream) {
+  const int n = rows * hidden;
+  if (n == 0) return cudaSuccess;
+  gather_rows_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(src, row_index, dst, rows, hidden);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,
+                           float* logits, cudaStream_t stream) {
+  GemvDesc d{};
+  d.W = W;
+  d.out_dim = vocab;
+  d.in_dim = hidden;
+  d.x = h;
+  d.rows = rows;
+  d.y = logits;
+  return launch_gemv(d, stream);
+}
+
+cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab, float* out,
+                      float* part, int splits, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  kl_partial_kernel<<<dim3(splits, rows), kKlThreads, 0, stream>>>(zref, zcur, vocab, splits, part);
+  kl_final_kernel<<<cdiv(rows, 64), 64, 0, stream>>>(part, splits, out, rows);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, float* grams,
+                         int blocks_per_side, float* out_sq, cudaStream_t stream) {
+  for (int base = 0; base < n_items; base += kMaxDriftItems) {
+    DriftBatch b;
+    b.n_items = n_items - base < kMaxDriftItems ? n_items - base : kMaxDriftItems;
+    for (int i = 0; i < b.n_items; ++i) b.items[i] = items[base + i];
+    dim3 g1(blocks_per_side, 2, b.n_items);
+    if (rank == 16) {
+      drift_partial_kernel<32><<<g1, 256, 0, stream>>>(b, blocks_per_side, grams);
+      drift_final_kernel<32><<<b.n_items, 256, 0, stream>>>(b, blocks_per_side, grams, out_sq);
+    } else if (rank == 8) {
+      drift_partial_kernel<16><<<g1, 256, 0, stream>>>(b, blocks_per_side, grams);
+      drift_final_kernel<16><<<b.n_items, 256, 0, stream>>>(b, blocks_per_side, grams, out_sq);
+    } else {
+      return cudaErrorInvalidValue;
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace crf
