@@ -1,0 +1,455 @@
+#!/usr/bin/env python3
+"""Benchmark of bounded KV-cache recomputation on one GB300 per rank.
+
+Workload (default ``7b-16k-w4``): Qwen2.5-7B-shaped random-init bf16 decoder
+(28 layers, hidden 3584, 28/4 heads, SwiGLU 18944, vocab 152064), rank-16
+LoRA (alpha 32) on all seven projections, one 16384-token prefix whose cache
+and hidden checkpoints were built under adapter v0, current adapter v1.
+
+One step = the whole hot path once:
+  drift of v1 against every layer's anchor (28 layers x 7 modules),
+  crf_recompute_window over [14, 18) from the layer-13 checkpoint (K/V
+  rewritten into the permuted 16-token pages, checkpoints H_14..H_17
+  refreshed), the last prefix row carried through layers 18..27 against the
+  historical cache, and the first-step KL against the fresh reference.
+Metric: recomputed layer*tokens/s (4 * 16384 per step). The same JSON line
+carries ms per refresh for windows of 1/2/4 layers and the full prefill, the
+live per-kernel roofline, an end-to-end number through pinned host buffers,
+clocks, and the CPU oracle on a bounded sample.
+
+``--impl reference`` times the CPU oracle (the plain restatement of the
+method) on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "recomputed layer*tokens/s"
+UNIT = "layer*tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-i", str(self.index), "-lms", "100", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        sm = []
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+            except ValueError:
+                pass
+            for j, nm in enumerate(names):
+                if r[5 + j].lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": float(rows[0][2]) if rows[0][2].replace(".", "").isdigit() else None,
+                "samples": len(rows), "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------- workload
+def algorithmic_work(cfg, lc, n):
+    """Algorithmic FLOPs per kernel kind for one recomputed layer over n tokens (and bytes)."""
+    h, f, qd, kvd, r = cfg.hidden, cfg.ffn, cfg.n_q_heads * cfg.head_dim, cfg.n_kv_heads * cfg.head_dim, lc.rank
+    ad = lambda m: m in lc.modules
+    up = lambda m, out: 2 * n * r * out if ad(m) else 0
+    flops = {
+        "gemm_qkv_rope_paged": 2 * n * h * (qd + 2 * kvd) + up("q", qd) + up("k", kvd) + up("v", kvd),
+        "gemm_o_resid": 2 * n * qd * h + up("o", h),
+        "gemm_gateup_swiglu": 2 * n * h * 2 * f + up("gate", f) + up("up", f),
+        "gemm_down_resid": 2 * n * f * h + up("down", h),
+        # down product x A^T of every adapted module: 2 n r in_m
+        "gemm_lora_down": 2 * n * r * (h * sum(ad(m) for m in ("q", "k", "v", "gate", "up"))
+                                       + qd * ad("o") + f * ad("down")),
+        "attn_prefill_paged": 4 * cfg.n_q_heads * cfg.head_dim * n * (n + 1) // 2,
+    }
+    byts = {"rmsnorm": 2 * (2 * n * h * 2)}   # two norms, read + write bf16
+    return flops, byts
+
+
+def build_state(wl, device, ctx):
+    import torch
+    import synth
+    import paper_2609_30884_gb300 as crf
+    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed
+
+    cfg, lc = wl.model, wl.lora
+    n = wl.n_tokens[0]
+    s, e = wl.windows[0]
+    N = cfg.n_layers
+    st = {"cfg": cfg, "lc": lc, "n": n, "s": s, "e": e}
+    dm = DeviceModel(cfg, device)
+    v_old = DeviceAdapter(cfg, lc, 0, device)
+    v_cur = DeviceAdapter(cfg, lc, 1, device)
+    P = pages_needed(n)
+    pool = make_pool(cfg, P, device)
+    pt = synth.page_permutation(P, 1, device)
+    tokens = synth.token_ids(cfg, n, device=device)
+    ckpt = [torch.empty(n, cfg.hidden, dtype=torch.bfloat16, device=device) for _ in range(N)]
+    fresh_fin = torch.empty(cfg.hidden, dtype=torch.bfloat16, device=device)
+    full_req = crf.Request(pt, 0, N, tokens=tokens, hidden_out=ckpt, final_hidden_out=fresh_fin)
+    ws = ctx.workspace(dm.crf, v_cur.crf, [full_req])
+    # fresh reference (current adapter) on a scratch pool, then the stale cache (old adapter)
+    fresh_pool = make_pool(cfg, P, device)
+    ctx.recompute_window(dm.crf, v_cur.crf, fresh_pool,
+                         [crf.Request(pt, 0, N, tokens=tokens, final_hidden_out=fresh_fin)], ws)
+    torch.cuda.synchronize()
+    del fresh_pool
+    ctx.recompute_window(dm.crf, v_old.crf, pool, [crf.Request(pt, 0, N, tokens=tokens, hidden_out=ckpt)], ws)
+    ctx.check()
+    fin = torch.empty(cfg.hidden, dtype=torch.bfloat16, device=device)
+    h_in = ckpt[s - 1] if s > 0 else None
+    req = crf.Request(pt, s, e, n_tokens=n, tokens=tokens, hidden_in=h_in, hidden_out=ckpt[s:e],
+                      final_hidden_out=fin)
+    out_sq = torch.empty(N, 7, 2, dtype=torch.float32, device=device)
+    dws = ctx.drift_workspace(dm.crf.dims_c, v_cur.crf.dims_c)
+    out_kl = torch.empty(1, dtype=torch.float32, device=device)
+    kws = ctx.kl_workspace(1, cfg.vocab, cfg.hidden)
+    st.update(dm=dm, v_old=v_old, v_cur=v_cur, pool=pool, pt=pt, tokens=tokens, ckpt=ckpt,
+              fresh_fin=fresh_fin, fin=fin, req=req, ws=ws, out_sq=out_sq, dws=dws, out_kl=out_kl,
+              kws=kws, anchors=[v_old.crf] * N)
+    return st
+
+
+def run_step(ctx, st):
+    ctx.drift(st["dm"].crf.dims_c, st["v_cur"].crf, st["anchors"], st["out_sq"], st["dws"])
+    ctx.recompute_window(st["dm"].crf, st["v_cur"].crf, st["pool"], [st["req"]], st["ws"])
+    ctx.kl(st["dm"].crf, st["fresh_fin"][None], st["fin"][None], st["out_kl"], st["cfg"].vocab,
+           st["kws"])
+
+
+def time_refresh(ctx, st, s, e, reps=3):
+    """ms of crf_recompute_window alone for window [s, e) (no tail decode)."""
+    import torch
+    import paper_2609_30884_gb300 as crf
+    n = st["n"]
+    req = crf.Request(st["pt"], s, e, n_tokens=n, tokens=st["tokens"],
+                      hidden_in=st["ckpt"][s - 1] if s > 0 else None, hidden_out=st["ckpt"][s:e])
+    ctx.recompute_window(st["dm"].crf, st["v_cur"].crf, st["pool"], [req], st["ws"])
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        ctx.recompute_window(st["dm"].crf, st["v_cur"].crf, st["pool"], [req], st["ws"])
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def cpu_oracle_sample(wl, n_rows, layer=None, x=None, weights=None, adapter=None):
+    """Time the oracle on one window layer over the first n_rows tokens of the prefix."""
+    import numpy as np
+    import synth
+    from oracle import build as obuild, decoder as D
+    cfg, lc = wl.model, wl.lora
+    layer = wl.windows[0][0] if layer is None else layer
+    P = obuild.layer_params(cfg, layer, tensors=weights)
+    A = obuild.layer_adapter(cfg, lc, 1, layer, tensors=adapter)
+    if x is None:
+        x = synth.hidden_state(cfg, n_rows, "bench_restart", layer).float().numpy()
+    dims = obuild.dims_of(cfg)
+    t0 = time.perf_counter()
+    D.decoder_layer(np.asarray(x[:n_rows], np.float32), P, A, dims, np.float32, chunk=512)
+    return time.perf_counter() - t0
+
+
+def blas_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        return max((i.get("num_threads", 0) for i in threadpool_info()), default=os.cpu_count())
+    except Exception:
+        return int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1))
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import synth
+    wl = synth.workload(args.workload)
+    n_rows = args.ref_rows
+    s, _ = wl.windows[0]
+    weights = synth.layer_weights(wl.model, s)
+    adapter = synth.adapter_version(wl.model, wl.lora, 1, s)
+    import numpy as np
+    x = synth.hidden_state(wl.model, n_rows, "bench_restart", s).float().numpy()
+    for _ in range(args.warmup):
+        cpu_oracle_sample(wl, n_rows, s, x, weights, adapter)
+    times = [cpu_oracle_sample(wl, n_rows, s, x, weights, adapter) for _ in range(args.steps)]
+    ms = 1000.0 * statistics.mean(times)
+    value = n_rows / (ms / 1000.0)
+    cores = blas_threads()
+    sample = (f"oracle decoder layer {s} of {wl.name} over the first {n_rows} of "
+              f"{wl.n_tokens[0]} tokens per step (fp32 NumPy)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded counter-based generator, random-init Qwen2.5-7B shape)",
+            "config": config_of(wl),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def config_of(wl):
+    s, e = wl.windows[0]
+    return {"workload": f"{args_workload_name(wl)}: {wl.name}", "prefix_tokens": wl.n_tokens[0],
+            "window": [s, e], "layers_recomputed": e - s, "n_layers": wl.model.n_layers,
+            "lora_rank": wl.lora.rank, "lora_modules": list(wl.lora.modules),
+            "page_tokens": 16, "l2": "inputs larger than L2 (1.9 GB of window weights per step)"}
+
+
+def args_workload_name(wl):
+    import synth
+    for k, v in synth.WORKLOADS.items():
+        if v is wl:
+            return k
+    return wl.name
+
+
+# ----------------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="crf", choices=["crf", "reference"])
+    ap.add_argument("--workload", default="7b-16k-w4")
+    ap.add_argument("--cpu-rows", type=int, default=4096, help="tokens in the CPU-oracle sample")
+    ap.add_argument("--ref-rows", type=int, default=1024, help="tokens per reference-arm step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "crf":
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device(f"cuda:{local}"))
+    torch.cuda.set_device(local)
+    device = f"cuda:{local}"
+
+    from paper_2609_30884_gb300 import build as _build
+    if rank == 0 or world == 1:
+        _build.build()
+    if world > 1:
+        dist.barrier()
+    import synth
+    import paper_2609_30884_gb300 as crf
+
+    wl = synth.workload(args.workload)
+    cfg, lc = wl.model, wl.lora
+    ctx = crf.Context(local)
+    st = build_state(wl, device, ctx)
+    n, s, e = st["n"], st["s"], st["e"]
+    units = (e - s) * n
+
+    for _ in range(args.warmup):
+        run_step(ctx, st)
+    ctx.check()
+
+    # ---------------- timed region: device-resident inputs
+    clocks = ClockSampler(local)
+    clocks.start()
+    ctx.profile_enable(True, 8192)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.steps):
+        run_step(ctx, st)
+    t1.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = t0.elapsed_time(t1)
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    clk = clocks.stop()
+    ctx.check()
+    if world > 1:
+        tt = torch.tensor([elapsed_ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(tt.item())
+    ms_step = elapsed_ms / args.steps
+    value = world * units * args.steps / (elapsed_ms / 1000.0)
+
+    # ---------------- end to end: restart state from pinned host memory, KL back to host
+    h_host = st["ckpt"][s - 1].to("cpu").pin_memory() if s > 0 else None
+    kl_host = torch.empty(1, dtype=torch.float32).pin_memory()
+    stream = torch.cuda.current_stream()
+
+    def e2e_step():
+        if h_host is not None:
+            st["ckpt"][s - 1].copy_(h_host, non_blocking=True)
+        run_step(ctx, st)
+        kl_host.copy_(st["out_kl"], non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = a.elapsed_time(b)
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    h2d = (st["ckpt"][s - 1].numel() * 2 if s > 0 else 0)
+    e2e = {"value": world * units * args.steps / (e2e_ms / 1000.0), "unit": UNIT,
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4,
+           "ms_per_step": e2e_ms / args.steps, "kl_first_step": float(kl_host.item())}
+
+    # ---------------- per-kernel roofline from the live events
+    peaks, peak_src = load_peaks()
+    flops_layer, bytes_layer = algorithmic_work(cfg, lc, n)
+    layers_per_step = e - s
+    kernels = {}
+    gpu_launches = 0
+    for name, (ms, cnt) in prof.items():
+        if name == "_dropped":
+            continue
+        gpu_launches += cnt
+        entry = {"launches": cnt, "ms_total": round(ms, 4),
+                 "ms_per_step": round(ms / args.steps, 4)}
+        if name in flops_layer:
+            fl = flops_layer[name] * layers_per_step * args.steps
+            tf = fl / (ms / 1000.0) / 1e12
+            entry.update(bound="tensor", tflops=round(tf, 1),
+                         frac=round(tf / peaks["bf16_tflops"], 4))
+        if name in bytes_layer:
+            by = bytes_layer[name] * layers_per_step * args.steps
+            gbs = by / (ms / 1000.0) / 1e9
+            entry.update(bound="hbm", gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4))
+        kernels[name] = entry
+    dom = max((k for k in kernels if k in flops_layer), key=lambda k: kernels[k]["ms_total"])
+    launches_dom = kernels[dom]["launches"]
+    roofline = {"kernel": dom, "bound": "tensor", "achieved": kernels[dom]["tflops"],
+                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": kernels[dom]["frac"], "traffic": None,
+                "peak_source": f"bf16_tflops ({peak_src}, burst)",
+                "frac_of_sustained": round(kernels[dom]["tflops"] / peaks.get("bf16_tflops_sustained", 1700.0), 4),
+                "algorithmic_flops_per_launch": flops_layer[dom],
+                "launches": launches_dom}
+    gemm_names = [k for k in kernels if k.startswith("gemm_") and k in flops_layer]
+    gemm_fl = sum(flops_layer[k] for k in gemm_names) * layers_per_step * args.steps
+    gemm_ms = sum(kernels[k]["ms_total"] for k in gemm_names)
+    gemm_tf = gemm_fl / (gemm_ms / 1000.0) / 1e12 if gemm_ms else 0.0
+
+    # ---------------- window sweep (ms per 16K-prefix refresh)
+    sweep = {}
+    if not args.no_sweep:
+        for ln in (1, 2, 4):
+            sweep[f"window_{ln}"] = round(time_refresh(ctx, st, s, min(s + ln, cfg.n_layers)), 3)
+        sweep["full_prefill_28"] = round(time_refresh(ctx, st, 0, cfg.n_layers, reps=2), 3)
+        sweep["layer_tokens_per_s_full"] = round(cfg.n_layers * n / (sweep["full_prefill_28"] / 1000.0))
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded counter-based generator, random-init Qwen2.5-7B shape)",
+            "config": config_of(wl), "gpu_launches": gpu_launches, "e2e": e2e,
+            "roofline": roofline, "clocks": clk,
+            "gemm_tflops_all": round(gemm_tf, 1),
+            "gemm_frac_all": round(gemm_tf / peaks["bf16_tflops"], 4),
+            "ms_per_refresh": sweep, "kernels": kernels,
+            "step": "drift(28x7) + recompute_window[14,18) + tail decode 18..27 + KL(first step)"}
+
+    # ---------------- CPU oracle baseline (rank 0, one GPU only)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        w = {k: v.to("cpu") for k, v in st["dm"].layers[s].items()}
+        ad = {m: (a.to("cpu"), b.to("cpu")) for m, (a, b) in st["v_cur"].layers[s].items()}
+        x = st["ckpt"][s - 1][:args.cpu_rows].float().cpu().numpy() if s > 0 else None
+        secs = cpu_oracle_sample(wl, args.cpu_rows, s, x, w, ad)
+        line["cpu_baseline"] = {
+            "value": args.cpu_rows / secs, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+            "sample": (f"oracle decoder layer {s} over the first {args.cpu_rows} of {n} tokens "
+                       f"(fp32 NumPy), {secs:.1f} s")}
+    if rank == 0:
+        print(json.dumps(line))
+    ctx.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

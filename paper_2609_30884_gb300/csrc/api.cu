@@ -28,9 +28,52 @@ struct crf_ctx {
   int device;
   int num_sms;
   int* status_dev;
+  // per-launch timing (crf_profile_enable)
+  bool prof_on = false;
+  std::vector<cudaEvent_t> ev;
+  int ev_used = 0;
+  struct Rec {
+    int kind, idx, kernels;
+  };
+  std::vector<Rec> rec;
+  int dropped = 0;
 };
 
 namespace {
+
+enum ProfKind : int {
+  kPQkv, kPO, kPGateUp, kPDown, kPLoraDown, kPAttn, kPNorm, kPEmbed, kPRope, kPCopy,
+  kPDecode, kPLmHead, kPKl, kPDrift, kPNumKinds
+};
+const char* const kProfNames[kPNumKinds] = {
+    "gemm_qkv_rope_paged", "gemm_o_resid", "gemm_gateup_swiglu", "gemm_down_resid",
+    "gemm_lora_down", "attn_prefill_paged", "rmsnorm", "embed_gather", "rope_table", "row_copy",
+    "tail_decode", "lm_head", "kl_reduce", "drift_gram"};
+
+// Brackets the launches issued in its lifetime with two events on `st` when
+// profiling is on; `kernels` is how many kernels those launches are.
+struct ProfScope {
+  crf_ctx* c;
+  int kind, kernels, idx;
+  cudaStream_t st;
+  ProfScope(crf_ctx* c_, int kind_, cudaStream_t st_, int kernels_ = 1)
+      : c(c_), kind(kind_), kernels(kernels_), idx(-1), st(st_) {
+    if (!c->prof_on) return;
+    if (c->ev_used + 2 > static_cast<int>(c->ev.size())) {
+      c->dropped += kernels;
+      return;
+    }
+    idx = c->ev_used;
+    c->ev_used += 2;
+    cudaEventRecord(c->ev[idx], st);
+  }
+  ~ProfScope() {
+    if (idx >= 0) {
+      cudaEventRecord(c->ev[idx + 1], st);
+      c->rec.push_back({kind, idx, kernels});
+    }
+  }
+};
 
 thread_local std::string g_err;
 
@@ -197,7 +240,7 @@ crf_status check_adapter_layers(const crf_adapter* a, int l0, int l1) {
 // ---------------------------------------------------------------- one layer
 struct LayerCtx {
   const Dims* D;
-  const crf_ctx* ctx;
+  crf_ctx* ctx;
   const crf_model* model;
   const crf_adapter* ad;
   const crf_kv_pool* pool;
@@ -212,6 +255,7 @@ bool adapted(const crf_adapter* a, int m) { return (a->dims.module_mask >> m) & 
 // LoRA down product of `X` for the listed modules into XA (16 columns per module).
 cudaError_t lora_down(const LayerCtx& c, int l, const void* X, int M, int K, const int* mods, int nm,
                       __nv_bfloat16* XA) {
+  ProfScope ps(c.ctx, kPLoraDown, c.st);
   GemmDesc g;
   std::memset(&g, 0, sizeof(g));
   g.A = X;
@@ -250,7 +294,10 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
   const int rank = c.ad->dims.rank;
 
   // 1. RMSNorm before attention
-  CRF_CUDA(launch_rmsnorm(X_in, static_cast<const __nv_bfloat16*>(w.ln1), XN, M, D.h, D.eps, c.st));
+  {
+    ProfScope ps(c.ctx, kPNorm, c.st);
+    CRF_CUDA(launch_rmsnorm(X_in, static_cast<const __nv_bfloat16*>(w.ln1), XN, M, D.h, D.eps, c.st));
+  }
 
   // 2-3. q/k/v projections (+ LoRA, bias, RoPE; K/V into the pages of layer l)
   {
@@ -294,6 +341,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.vpages = c.pool->v_pages[l];
     g.req = rt;
     g.status = c.ctx->status_dev;
+    ProfScope ps(c.ctx, kPQkv, c.st);
     CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
   }
 
@@ -311,6 +359,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     a.head_dim = D.d;
     a.req = rt;
     a.status = c.ctx->status_dev;
+    ProfScope ps(c.ctx, kPAttn, c.st);
     CRF_CUDA(launch_attention(a, c.ctx->num_sms, c.st));
   }
 
@@ -348,12 +397,16 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.resid = resid;
     g.ld_resid = D.h;
     g.status = c.ctx->status_dev;
+    ProfScope ps(c.ctx, m == CRF_MOD_O ? kPO : kPDown, c.st);
     return launch_gemm(g, 256, c.ctx->num_sms, c.st);
   };
   CRF_CUDA(proj_resid(CRF_MOD_O, O, D.qd, X_in, X1));
 
   // 7. RMSNorm before the MLP
-  CRF_CUDA(launch_rmsnorm(X1, static_cast<const __nv_bfloat16*>(w.ln2), XN, M, D.h, D.eps, c.st));
+  {
+    ProfScope ps(c.ctx, kPNorm, c.st);
+    CRF_CUDA(launch_rmsnorm(X1, static_cast<const __nv_bfloat16*>(w.ln2), XN, M, D.h, D.eps, c.st));
+  }
 
   // 8-9. gate|up projections with SwiGLU epilogue
   {
@@ -390,6 +443,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.out = MLP;
     g.ldo = D.f;
     g.status = c.ctx->status_dev;
+    ProfScope ps(c.ctx, kPGateUp, c.st);
     CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
   }
 
@@ -404,6 +458,10 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
 crf_status decode_row(const LayerCtx& c, int l0, const __nv_bfloat16* start_row, int pos,
                       const int32_t* page_table, void* out_bf16) {
   const Dims& D = *c.D;
+  int n_adapted = 0;
+  for (int m = 0; m < 7; ++m) n_adapted += adapted(c.ad, m) ? 1 : 0;
+  // per layer: 2 norms, 7 GEMVs, adapted LoRA downs, 2 RoPE, 2 attention, 1 SwiGLU; + 2 converts
+  ProfScope ps(c.ctx, kPDecode, c.st, (D.N - l0) * (14 + n_adapted) + 2);
   const Plan& p = *c.plan;
   float* base = reinterpret_cast<float*>(c.ws + p.off_dec);
   float* x = base;
@@ -562,6 +620,7 @@ crf_status crf_create(crf_ctx** out, int device) {
 
 crf_status crf_destroy(crf_ctx* ctx) {
   if (!ctx) return fail(CRF_EINVAL, "ctx is null");
+  for (cudaEvent_t e : ctx->ev) cudaEventDestroy(e);
   cudaFree(ctx->status_dev);
   delete ctx;
   return CRF_OK;
@@ -629,7 +688,10 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
   c.plan = &plan;
   c.scale = cur->dims.alpha / cur->dims.rank;
 
-  CRF_CUDA(launch_rope_table(reinterpret_cast<float2*>(ws + plan.off_rope), plan.max_n, D.d, D.theta, st));
+  {
+    ProfScope ps(ctx, kPRope, st);
+    CRF_CUDA(launch_rope_table(reinterpret_cast<float2*>(ws + plan.off_rope), plan.max_n, D.d, D.theta, st));
+  }
 
   __nv_bfloat16* G[2] = {reinterpret_cast<__nv_bfloat16*>(ws + plan.off_g0),
                          reinterpret_cast<__nv_bfloat16*>(ws + plan.off_g1)};
@@ -689,9 +751,11 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
           const int i = act[k];
           __nv_bfloat16* dst = G[b] + static_cast<size_t>(rt.row0[k]) * D.h;
           if (reqs[i].s == l && l == 0) {
+            ProfScope ps(ctx, kPEmbed, st);
             CRF_CUDA(launch_embed(static_cast<const __nv_bfloat16*>(model->embed), reqs[i].tokens, dst,
                                   reqs[i].n_tokens, D.h, st));
           } else {
+            ProfScope ps(ctx, kPCopy, st, 0);
             CRF_CUDA(cudaMemcpyAsync(dst, curp[i], reqs[i].n_tokens * row_bytes,
                                      cudaMemcpyDeviceToDevice, st));
           }
@@ -712,6 +776,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
     if (s != CRF_OK) return s;
     for (int k = 0; k < rt.n; ++k) {
       const int i = act[k];
+      ProfScope ps(ctx, kPCopy, st, 0);
       curp[i] = X_out + static_cast<size_t>(rt.row0[k]) * D.h;
       if (!single && reqs[i].hidden_out)
         CRF_CUDA(cudaMemcpyAsync(reqs[i].hidden_out[l - reqs[i].s], curp[i],
@@ -729,6 +794,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
     if (!r.final_hidden_out) continue;
     const __nv_bfloat16* start = dx0 + static_cast<size_t>(i) * D.h;
     if (r.s == r.e) {
+      ProfScope ps(ctx, r.s == 0 ? kPEmbed : kPCopy, st, r.s == 0 ? 1 : 0);
       if (r.s == 0) {
         CRF_CUDA(launch_embed(static_cast<const __nv_bfloat16*>(model->embed), r.tokens + (r.n_tokens - 1),
                               dx0 + static_cast<size_t>(i) * D.h, 1, D.h, st));
@@ -740,6 +806,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
       }
     }
     if (r.e == D.N) {
+      ProfScope ps(ctx, kPCopy, st, 0);
       CRF_CUDA(cudaMemcpyAsync(r.final_hidden_out, start, row_bytes, cudaMemcpyDeviceToDevice, st));
     } else {
       s = decode_row(c, r.e, start, r.n_tokens - 1, r.page_table, r.final_hidden_out);
@@ -808,6 +875,7 @@ crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter
   CRF_CUDA(cudaMemsetAsync(out_sq, 0, static_cast<size_t>(D.N) * 7 * 2 * sizeof(float), st));
   if (items.empty()) return CRF_OK;
   const int bps = drift_blocks_per_side(ctx, static_cast<int>(items.size()));
+  ProfScope ps(ctx, kPDrift, st, 2 * ((static_cast<int>(items.size()) + 223) / 224));
   CRF_CUDA(launch_drift(items.data(), static_cast<int>(items.size()), cur->dims.rank,
                         static_cast<float*>(workspace), bps, out_sq, st));
   return CRF_OK;
@@ -862,6 +930,7 @@ crf_status crf_kl(crf_ctx* ctx, const crf_model* model, const void* ref, const v
     float* hn = reinterpret_cast<float*>(ws + o);
     o += align256(static_cast<size_t>(2 * n_rows) * hidden * sizeof(float));
     float* logits = logits_out ? logits_out : reinterpret_cast<float*>(ws + o);
+    ProfScope ps(ctx, kPLmHead, st, 4);
     CRF_CUDA(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(ref), hf, n_rows * hidden, st));
     CRF_CUDA(launch_bf16_to_f32(static_cast<const __nv_bfloat16*>(cur), hf + static_cast<size_t>(n_rows) * hidden,
                                 n_rows * hidden, st));
@@ -872,7 +941,60 @@ crf_status crf_kl(crf_ctx* ctx, const crf_model* model, const void* ref, const v
     zr = logits;
     zc = logits + static_cast<size_t>(n_rows) * vocab;
   }
-  CRF_CUDA(launch_kl(zr, zc, n_rows, vocab, out_kl, part, sp, st));
+  {
+    ProfScope ps(ctx, kPKl, st, 2);
+    CRF_CUDA(launch_kl(zr, zc, n_rows, vocab, out_kl, part, sp, st));
+  }
+  return CRF_OK;
+}
+
+// ---------------------------------------------------------------- profiling
+crf_status crf_profile_enable(crf_ctx* ctx, int on, int max_launches) {
+  if (!ctx) return fail(CRF_EINVAL, "ctx is null");
+  if (on && max_launches < 1) return fail(CRF_EINVAL, "max_launches must be positive");
+  CRF_CUDA(cudaSetDevice(ctx->device));
+  if (on) {
+    const size_t want = static_cast<size_t>(2) * max_launches;
+    while (ctx->ev.size() < want) {
+      cudaEvent_t e;
+      CRF_CUDA(cudaEventCreate(&e));
+      ctx->ev.push_back(e);
+    }
+  }
+  ctx->prof_on = on != 0;
+  ctx->ev_used = 0;
+  ctx->rec.clear();
+  ctx->dropped = 0;
+  return CRF_OK;
+}
+
+crf_status crf_profile_read(crf_ctx* ctx, int max_kinds, char* names, double* total_ms,
+                            int* launches, int* n_kinds, int* dropped) {
+  if (!ctx || !names || !total_ms || !launches || !n_kinds) return fail(CRF_EINVAL, "null argument");
+  double ms[kPNumKinds] = {0};
+  int cnt[kPNumKinds] = {0};
+  bool seen[kPNumKinds] = {false};
+  for (const auto& r : ctx->rec) {
+    CRF_CUDA(cudaEventSynchronize(ctx->ev[r.idx + 1]));
+    float t = 0.f;
+    CRF_CUDA(cudaEventElapsedTime(&t, ctx->ev[r.idx], ctx->ev[r.idx + 1]));
+    ms[r.kind] += t;
+    cnt[r.kind] += r.kernels;
+    seen[r.kind] = true;
+  }
+  int k = 0;
+  for (int i = 0; i < kPNumKinds && k < max_kinds; ++i) {
+    if (!seen[i]) continue;
+    std::snprintf(names + 32 * k, 32, "%s", kProfNames[i]);
+    total_ms[k] = ms[i];
+    launches[k] = cnt[i];
+    ++k;
+  }
+  *n_kinds = k;
+  if (dropped) *dropped = ctx->dropped;
+  ctx->ev_used = 0;
+  ctx->rec.clear();
+  ctx->dropped = 0;
   return CRF_OK;
 }
 
