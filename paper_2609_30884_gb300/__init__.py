@@ -29,7 +29,8 @@ from .abi import CrfError
 
 MODULES = ("q", "k", "v", "o", "gate", "up", "down")
 
-__all__ = ["Context", "Model", "Adapter", "KVPool", "Request", "CrfError", "MODULES", "abi"]
+__all__ = ["Context", "Model", "Adapter", "KVPool", "Request", "CrfError", "MODULES", "abi",
+           "kl_logits_noalloc"]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -216,3 +217,16 @@ class Context:
             out[name] = (ms[i], cnt[i])
         out["_dropped"] = (0.0, dropped.value)
         return out
+
+
+def kl_logits_noalloc(device: int, z_ref: torch.Tensor, z_cur: torch.Tensor, out_kl: torch.Tensor,
+                      stream=None) -> None:
+    """crf_kl_logits_noalloc: KL(softmax(z_ref) || softmax(z_cur)) per row with no workspace.
+
+    For callers that cannot allocate device memory at call time; the library's fixed device
+    scratch serves every call, so calls must not overlap on the GPU.
+    """
+    lib = abi.load()
+    abi.check(lib.crf_kl_logits_noalloc(device, z_ref.data_ptr(), z_cur.data_ptr(),
+                                        int(z_ref.shape[0]), int(z_ref.shape[1]),
+                                        out_kl.data_ptr(), _stream(stream)))

@@ -22,7 +22,8 @@ MAX_REQUESTS = 32
 # Every symbol include/crf.h declares.
 EXPORTS = ("crf_create", "crf_destroy", "crf_last_error", "crf_check", "crf_workspace_size",
            "crf_recompute_window", "crf_drift_workspace_size", "crf_drift",
-           "crf_kl_workspace_size", "crf_kl", "crf_profile_enable", "crf_profile_read")
+           "crf_kl_workspace_size", "crf_kl", "crf_kl_logits_noalloc", "crf_profile_enable",
+           "crf_profile_read")
 
 
 class ModelDims(ctypes.Structure):
@@ -87,6 +88,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                        c_size_t, P], c_int),
         "crf_kl_workspace_size": ([P, c_int, c_int, c_int, POINTER(c_size_t)], c_int),
         "crf_kl": ([P, POINTER(Model), P, P, c_int, c_int, P, P, P, c_size_t, P], c_int),
+        "crf_kl_logits_noalloc": ([c_int, P, P, c_int, c_int, P, P], c_int),
         "crf_profile_enable": ([P, c_int, c_int], c_int),
         "crf_profile_read": ([P, c_int, ctypes.c_char_p, POINTER(ctypes.c_double), POINTER(c_int),
                               POINTER(c_int), POINTER(c_int)], c_int),

@@ -586,6 +586,11 @@ crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const c
 
 }  // namespace
 
+namespace crf {
+// Records `msg` as this thread's crf_last_error() text (used by other translation units).
+void set_last_error(const char* msg) { g_err = msg ? msg : ""; }
+}  // namespace crf
+
 // ====================================================================== ABI
 extern "C" {
 
