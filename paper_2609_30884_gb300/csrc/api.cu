@@ -17,6 +17,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <set>
 #include <string>
@@ -28,6 +29,8 @@ struct crf_ctx {
   int device;
   int num_sms;
   int* status_dev;
+  // CRF_ATTENTION=mma selects the mma.sync prefill attention instead of tcgen05
+  bool attn_mma_sync = false;
   // per-launch timing (crf_profile_enable)
   bool prof_on = false;
   std::vector<cudaEvent_t> ev;
@@ -360,7 +363,10 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     a.req = rt;
     a.status = c.ctx->status_dev;
     ProfScope ps(c.ctx, kPAttn, c.st);
-    CRF_CUDA(launch_attention(a, c.ctx->num_sms, c.st));
+    if (c.ctx->attn_mma_sync)
+      CRF_CUDA(launch_attention(a, c.ctx->num_sms, c.st));
+    else
+      CRF_CUDA(launch_attention_tc(a, c.pool->num_pages, M, c.st));
   }
 
   // 5-6. output projection + residual: X1 = X_in + O W_o^T (+ LoRA)
@@ -611,6 +617,8 @@ crf_status crf_create(crf_ctx** out, int device) {
   crf_ctx* c = new crf_ctx;
   c->device = device;
   c->num_sms = prop.multiProcessorCount;
+  const char* attn = std::getenv("CRF_ATTENTION");
+  c->attn_mma_sync = attn && std::strcmp(attn, "mma") == 0;
   c->status_dev = nullptr;
   cudaError_t e = cudaMalloc(&c->status_dev, sizeof(int));
   if (e == cudaSuccess) e = cudaMemset(c->status_dev, 0, sizeof(int));

@@ -1,0 +1,428 @@
+// Causal grouped-query prefill attention on tcgen05, reading K/V from the
+// paged cache of the layer being recomputed.
+//
+// softmax(q k^T / sqrt(d) + causal mask) v over the whole prefix for every
+// query head; query head h reads kv head h / (Hq / Hkv). One CTA takes 128
+// query rows of two query heads that share a kv head (GQA), so every K/V tile
+// is fetched once for both. Warp roles:
+//   warp 0      TMA producer: the two Q tiles, then K and V tiles (8 pages of
+//               16 tokens each) into a 2-deep shared-memory ring
+//   warp 1      allocates TMEM and issues tcgen05.mma from one thread:
+//               S_t = Q_t K^T into TMEM, then O_t += P_t V with P_t read
+//               from TMEM (A operand) and V an MN-major shared operand
+//   warps 2-5   softmax of head 0, warps 6-9 softmax of head 1: one thread
+//               per query row; S from TMEM, online max / sum in fp32, P back
+//               into TMEM as bf16 over the S columns; O rescaled in TMEM only
+//               when the running max grows by more than 2^8
+// TMEM: S0 | S1 | O0 | O1, 128 columns each. Every wait is bounded.
+#include "common.cuh"
+#include "kernels.h"
+
+#include <algorithm>
+#include <cfloat>
+#include <cstring>
+
+namespace crf {
+
+namespace {
+
+constexpr int kM = 128;          // query rows per tile
+constexpr int kN = 128;          // keys per kv tile
+constexpr int kPagesPerTile = kN / kPage;
+constexpr int kThreadsAttn = 320;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
+
+struct AttnTcArgs {
+  CUtensorMap tmQ;  // q [rows, Hq*D], box {64, 128}
+  CUtensorMap tmK;  // K pool viewed as [pages*Hkv*16, D], box {64, 16}
+  CUtensorMap tmV;
+  __nv_bfloat16* out;
+  int ldo;
+  int n_q_heads, n_kv_heads, group, pairs;
+  int total_items;
+  ReqTable req;
+  int* status;
+};
+
+struct AttnWork {
+  int req, qt, g, h0, h1;
+};
+
+__device__ __forceinline__ bool attn_work(const AttnTcArgs& a, int idx, AttnWork& w) {
+  const int per_qt = a.n_kv_heads * a.pairs;
+  for (int i = 0; i < a.req.n; ++i) {
+    const int nqt = (a.req.len[i] + kM - 1) / kM;
+    const int items = nqt * per_qt;
+    if (idx < items) {
+      w.req = i;
+      w.qt = nqt - 1 - idx / per_qt;  // longest (latest) query tiles first
+      const int rem = idx % per_qt;
+      w.g = rem / a.pairs;
+      const int pp = rem % a.pairs;
+      w.h0 = w.g * a.group + 2 * pp;
+      w.h1 = (2 * pp + 1 < a.group) ? w.h0 + 1 : -1;
+      return true;
+    }
+    idx -= items;
+  }
+  return false;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_constant__ AttnTcArgs a) {
+  constexpr int HALVES = D / 64;
+  constexpr int Q_BYTES = kM * D * 2;
+  constexpr int KV_BYTES = kN * D * 2;
+  constexpr int HALF_ROWS_BYTES = kN * 128;  // one 64-column half of a 128-row tile
+  constexpr uint32_t TMEM_COLS = 512;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + 2 * Q_BYTES;
+  uint8_t* sV = sK + 2 * KV_BYTES;
+  __shared__ __align__(8) uint64_t q_full, o_full, drain_bar;
+  __shared__ __align__(8) uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
+  __shared__ __align__(8) uint64_t s_full[2], p_full[2];
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ volatile int abort_flag;
+
+  AttnWork w;
+  if (!attn_work(a, blockIdx.x, w)) return;
+  const int n = a.req.len[w.req];
+  const int row0 = a.req.row0[w.req];
+  const int32_t* pt = a.req.page_table[w.req];
+  const int q0 = w.qt * kM;
+  const int kv_end = min(q0 + kM, n);
+  const int J = (kv_end + kN - 1) / kN;
+  const int n_pages = (n + kPage - 1) / kPage;
+  const int ntiles = w.h1 >= 0 ? 2 : 1;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(&q_full, 1);
+    mbar_init(&o_full, 1);
+    mbar_init(&drain_bar, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&k_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+      mbar_init(&v_full[i], 1);
+      mbar_init(&v_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], 4);
+    }
+    abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_base_sh, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_sh;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      bool ok = true;
+      int armed_k[2] = {-1, -1}, armed_v[2] = {-1, -1};
+      mbar_arrive_expect_tx(&q_full, ntiles * Q_BYTES);
+      for (int t = 0; t < ntiles; ++t) {
+        const int head = t == 0 ? w.h0 : w.h1;
+        for (int h = 0; h < HALVES; ++h)
+          tma_load_2d(sQ + t * Q_BYTES + h * (kM * 128), &a.tmQ, &q_full, head * D + 64 * h,
+                      row0 + q0);
+      }
+      for (int j = 0; j < J && ok; ++j) {
+        const int st = j & 1;
+        const uint32_t ph = (j >> 1) & 1;
+        for (int kv = 0; kv < 2 && ok; ++kv) {
+          uint64_t* full = kv == 0 ? &k_full[st] : &v_full[st];
+          uint64_t* empty = kv == 0 ? &k_empty[st] : &v_empty[st];
+          if (!mbar_wait(empty, ph ^ 1, &abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full, KV_BYTES);
+          uint8_t* dst = (kv == 0 ? sK : sV) + st * KV_BYTES;
+          const CUtensorMap* map = kv == 0 ? &a.tmK : &a.tmV;
+          for (int p = 0; p < kPagesPerTile; ++p) {
+            // pages past the prefix repeat the last page: finite data, masked below
+            const int page = pt[min(j * kPagesPerTile + p, n_pages - 1)];
+            const int row = (page * a.n_kv_heads + w.g) * kPage;
+            for (int h = 0; h < HALVES; ++h)
+              tma_load_2d(dst + h * HALF_ROWS_BYTES + p * kPage * 128, map, full, 64 * h, row);
+          }
+          (kv == 0 ? armed_k : armed_v)[st] = ph;
+        }
+      }
+      if (!ok) {
+        volatile int never = 0;
+        for (int s = 0; s < 2; ++s) {
+          if (armed_k[s] >= 0) mbar_wait(&k_full[s], armed_k[s], &never, nullptr);
+          if (armed_v[s] >= 0) mbar_wait(&v_full[s], armed_v[s], &never, nullptr);
+        }
+        mbar_wait(&q_full, 0, &never, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait(&q_full, 0, &abort_flag, a.status);
+      bool issued = false;
+      const uint32_t idesc_s = idesc_bf16_f32(kM, kN);
+      const uint32_t idesc_o = idesc_bf16_f32(kM, D, false, true);
+      for (int j = 0; j < J && ok; ++j) {
+        const int st = j & 1;
+        const uint32_t ph = (j >> 1) & 1;
+        if (!mbar_wait(&k_full[st], ph, &abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kb = smem_u32(sK + st * KV_BYTES);
+        for (int t = 0; t < ntiles; ++t) {
+          const uint32_t qb = smem_u32(sQ + t * Q_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * HALF_ROWS_BYTES + (kk & 3) * 32;
+            mma_bf16_ss(tmem + t * 128, smem_desc(qb + off, 16, 1024, kSwizzle128B),
+                        smem_desc(kb + off, 16, 1024, kSwizzle128B), idesc_s, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&s_full[t]);
+        }
+        issued = true;
+        mma_commit(&k_empty[st]);
+        if (!mbar_wait(&v_full[st], ph, &abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        const uint32_t vb = smem_u32(sV + st * KV_BYTES);
+        for (int t = 0; t < ntiles && ok; ++t) {
+          if (!mbar_wait(&p_full[t], j & 1, &abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < kN / 16; ++kk) {
+            // P: 16 keys = 8 packed bf16x2 columns; V: 16 key rows = 2 KB
+            mma_bf16_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
+                        smem_desc(vb + kk * 2048, HALF_ROWS_BYTES, 1024, kSwizzle128B), idesc_o,
+                        (j > 0 || kk > 0) ? 1u : 0u);
+          }
+        }
+        if (!ok) break;
+        mma_commit(&v_empty[st]);
+      }
+      if (ok) {
+        mma_commit(&o_full);
+      } else if (issued) {
+        mma_commit(&drain_bar);
+        volatile int never = 0;
+        mbar_wait(&drain_bar, 0, &never, nullptr);
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- softmax + epilogue
+    const int t = (warp - 2) >> 2;
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;  // query row within the tile (= TMEM lane)
+    const int head = t == 0 ? w.h0 : w.h1;
+    if (head >= 0) {
+      const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+      const uint32_t tS = tmem + lane_off + t * 128;
+      const uint32_t tO = tmem + lane_off + 256 + t * 128;
+      const float sl2 = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
+      const int qrow = q0 + r;
+      float m_run = -FLT_MAX, l_run = 0.f;
+      bool ok = true;
+      for (int j = 0; j < J && ok; ++j) {
+        // warp-uniform outcome: the TMEM accesses below are warp-collective
+        ok = __all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, &abort_flag, a.status));
+        if (!ok) break;
+        tc_fence_after();
+        uint32_t sr[4][32];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+        tmem_ld_wait();
+        const int k0 = j * kN;
+        const bool last = j == J - 1;
+        float mt = -FLT_MAX;
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            float x = __uint_as_float(sr[c][i]) * sl2;
+            if (last) {
+              const int col = k0 + c * 32 + i;
+              if (col > qrow || col >= kv_end) x = -FLT_MAX;
+            }
+            sr[c][i] = __float_as_uint(x);
+            mt = fmaxf(mt, x);
+          }
+        const float m_new = fmaxf(m_run, mt);
+        const bool grow = m_new > m_run + kRescaleThreshold;
+        const float alpha = grow ? ex2_approx(m_run - m_new) : 1.0f;
+        if (j > 0 && __any_sync(0xffffffffu, grow)) {
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(tO + c * 32, o);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+            tmem_st32(tO + c * 32, o);
+          }
+          tmem_st_wait();
+        }
+        if (grow) {
+          l_run *= alpha;
+          m_run = m_new;
+        }
+        float rs = 0.f;
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float x0 = __uint_as_float(sr[2 * c + i / 16][(2 * i) % 32]);
+            const float x1 = __uint_as_float(sr[2 * c + i / 16][(2 * i + 1) % 32]);
+            const float p0 = x0 <= -FLT_MAX ? 0.f : ex2_approx(x0 - m_run);
+            const float p1 = x1 <= -FLT_MAX ? 0.f : ex2_approx(x1 - m_run);
+            rs += p0 + p1;
+            pk[i] = pack_bf16(p0, p1);
+          }
+          tmem_st32(tS + c * 32, pk);
+        }
+        tmem_st_wait();
+        l_run += rs;
+        if (last && t == 0 && kv_end - k0 < kN) {
+          // zero V rows past the prefix so that 0 * stale data cannot produce NaN
+          const int st = j & 1;
+          ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (j >> 1) & 1, &abort_flag, a.status));
+          if (ok) {
+            uint8_t* vt = sV + st * KV_BYTES;
+            const int zr0 = kv_end - k0;
+            const int chunks = (kN - zr0) * HALVES * 8;
+            for (int i = threadIdx.x - 64; i < chunks; i += 128) {
+              const int rr = zr0 + i / (HALVES * 8);
+              const int h = (i / 8) % HALVES;
+              const int ch = i % 8;
+              *reinterpret_cast<uint4*>(vt + h * HALF_ROWS_BYTES + rr * 128 + ch * 16) =
+                  make_uint4(0, 0, 0, 0);
+            }
+            fence_proxy_async_smem();
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[t]);
+      }
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&o_full, 0, &abort_flag, a.status));
+      if (ok) {
+        tc_fence_after();
+        const float inv = l_run > 0.f ? 1.0f / l_run : 0.f;
+        const bool store = qrow < n;
+        __nv_bfloat16* dst = a.out + (size_t)(row0 + qrow) * a.ldo + head * D;
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + c * 32, o);
+          tmem_ld_wait();
+          if (store) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              uint4 v;
+              v.x = pack_bf16(__uint_as_float(o[8 * i + 0]) * inv, __uint_as_float(o[8 * i + 1]) * inv);
+              v.y = pack_bf16(__uint_as_float(o[8 * i + 2]) * inv, __uint_as_float(o[8 * i + 3]) * inv);
+              v.z = pack_bf16(__uint_as_float(o[8 * i + 4]) * inv, __uint_as_float(o[8 * i + 5]) * inv);
+              v.w = pack_bf16(__uint_as_float(o[8 * i + 6]) * inv, __uint_as_float(o[8 * i + 7]) * inv);
+              reinterpret_cast<uint4*>(dst + c * 32)[i] = v;
+            }
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+bool map2d(CUtensorMap* m, const void* base, long rows, int cols, int box_rows) {
+  EncodeTiledFn fn = encode();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_tc(const AttnTcArgs& args, cudaStream_t stream) {
+  constexpr int smem = 2 * kM * D * 2 + 4 * kN * D * 2 + 1024;
+  static bool set = false;
+  if (!set) {
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    set = true;
+  }
+  attn_tc_kernel<D><<<args.total_items, kThreadsAttn, smem, stream>>>(args);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows, cudaStream_t stream) {
+  AttnTcArgs a;
+  std::memset(&a, 0, sizeof(a));
+  const int D = d.head_dim;
+  if (!map2d(&a.tmQ, d.q, total_rows, d.n_q_heads * D, kM)) return cudaErrorInvalidValue;
+  const long pool_rows = static_cast<long>(num_pages) * d.n_kv_heads * kPage;
+  if (!map2d(&a.tmK, d.kpages, pool_rows, D, kPage)) return cudaErrorInvalidValue;
+  if (!map2d(&a.tmV, d.vpages, pool_rows, D, kPage)) return cudaErrorInvalidValue;
+  a.out = d.out;
+  a.ldo = d.ldo;
+  a.n_q_heads = d.n_q_heads;
+  a.n_kv_heads = d.n_kv_heads;
+  a.group = d.n_q_heads / d.n_kv_heads;
+  a.pairs = (a.group + 1) / 2;
+  a.req = d.req;
+  a.status = d.status;
+  a.total_items = 0;
+  for (int i = 0; i < d.req.n; ++i)
+    a.total_items += ((d.req.len[i] + kM - 1) / kM) * d.n_kv_heads * a.pairs;
+  if (a.total_items == 0) return cudaSuccess;
+  if (D == 128) return launch_tc<128>(a, stream);
+  if (D == 64) return launch_tc<64>(a, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace crf

@@ -439,7 +439,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       const Tile tl = decode_tile(t, a);
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
-      if (!mbar_wait(&tfull_bar[acc], acc_phase, &abort_flag, a.status)) break;
+      // warp-uniform outcome: the TMEM loads of the epilogue are warp-collective
+      if (!__all_sync(0xffffffffu, mbar_wait(&tfull_bar[acc], acc_phase, &abort_flag, a.status)))
+        break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
       epilogue_tile<BN>(a, tl, tacc, row_in_tile);

@@ -89,6 +89,9 @@ struct AttnDesc {
   int* status;
 };
 cudaError_t launch_attention(const AttnDesc& d, int num_sms, cudaStream_t stream);
+// tcgen05 version: num_pages of the pool, total_rows of q (for the TMA maps).
+cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows,
+                                cudaStream_t stream);
 
 // Small-M decode path (the last prefix row through the layers after the window).
 // y[r, j] = sum_i W[j, i] x[r, i] (+ bias[j]) (+ sum_k BL[j, k] xa[r, k]) (+ resid[r, j])
