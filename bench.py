@@ -271,6 +271,49 @@ def args_workload_name(wl):
     return wl.name
 
 
+def run_window_only(args):
+    """One window layer (or a few) over the prefix, nothing else: the small profiling case.
+
+    Holds only the window's layer weights, one KV pool and the workspace (a few GB for the
+    7B shape), so a kernel of the window can be captured by a profiler on its own.
+    """
+    import torch
+    import synth
+    import paper_2609_30884_gb300 as crf
+    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed
+
+    wl = synth.workload(args.workload)
+    cfg, lc = wl.model, wl.lora
+    n = args.tokens or wl.n_tokens[0]
+    s, e = wl.windows[0]
+    device = "cuda:0"
+    ctx = crf.Context(0)
+    dm = DeviceModel(cfg, device, layers=range(s, e), with_head=False)
+    cur = DeviceAdapter(cfg, lc, 1, device, layers=range(s, e))
+    P = pages_needed(n)
+    pool = make_pool(cfg, P, device)
+    pt = synth.page_permutation(P, 1, device)
+    h_in = synth.hidden_state(cfg, n, device=device)
+    h_out = [torch.empty(n, cfg.hidden, dtype=torch.bfloat16, device=device) for _ in range(e - s)]
+    req = crf.Request(pt, s, e, hidden_in=h_in, hidden_out=h_out)
+    ws = ctx.workspace(dm.crf, cur.crf, [req])
+    for _ in range(args.warmup):
+        ctx.recompute_window(dm.crf, cur.crf, pool, [req], ws)
+    ctx.check()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        ctx.recompute_window(dm.crf, cur.crf, pool, [req], ws)
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    print(json.dumps({"case": "window-only", "workload": args.workload, "tokens": n,
+                      "window": [s, e], "ms_per_window": ms,
+                      "layer_tokens_per_s": (e - s) * n / (ms / 1000.0)}))
+    ctx.close()
+    return 0
+
+
 # ----------------------------------------------------------------------------- main
 def main():
     ap = argparse.ArgumentParser()
@@ -283,7 +326,12 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=1024, help="tokens per reference-arm step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--case", default="step", choices=["step", "window-only"],
+                    help="window-only: the small profiling case (window layers only)")
+    ap.add_argument("--tokens", type=int, default=0, help="prefix length for --case window-only")
     args = ap.parse_args()
+    if args.case == "window-only":
+        return run_window_only(args)
     if args.warmup < 3 and args.impl == "crf":
         args.warmup = 3
     if args.impl == "reference":

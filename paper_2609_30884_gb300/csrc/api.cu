@@ -173,7 +173,8 @@ struct Plan {
   size_t total;
 };
 
-int dec_splits(int max_n) { return std::max(1, std::min(64, (max_n + 511) / 512)); }
+// decode attention partials: one per 256-position chunk of the longest prefix
+int dec_splits(int max_n) { return std::max(1, (max_n + 255) / 256); }
 
 Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   Plan p;

@@ -263,90 +263,149 @@ __global__ void __launch_bounds__(kWarps * 32, 1) attn_prefill_kernel(const Attn
 }
 
 // ---------------------------------------------------------------- decode attention
-// One decode row per request: q [Hq*d] fp32 attends to the request's cached keys
-// at positions < pos (from the pages) plus its own fresh k/v. Split over
-// positions; partial (max, sum, acc) combined by the second kernel.
-constexpr int kDecThreads = 128;
+// One decode row per request: q [Hq*d] (fp32, rotated) attends to the request's
+// cached keys at positions < pos (from the pages) plus its own fresh k/v at pos.
+// A block takes one kv head and one chunk of 256 positions and serves every query
+// head of that kv group, so each K/V row is read once per chunk:
+//   1. thread t scores position chunk0 + t against all heads of the group,
+//   2. warp h turns head h's scores into exp(s - max) and their sum,
+//   3. warp w accumulates positions 32w..32w+31 into per-lane 4-dim slices of O,
+//      and the 8 warp partials are summed through shared memory.
+// The chunk partials (max, sum, O) are merged by decode_attn_combine.
+constexpr int kDecThreads = 256;
+constexpr int kDecChunk = 256;
+constexpr int kDecMaxGroup = 8;
 
 template <int D>
 __global__ void __launch_bounds__(kDecThreads) decode_attn_partial(const DecodeAttnDesc p) {
+  constexpr int DPL = D / 32;  // dims per lane in the PV accumulation
   const int r = blockIdx.z;
-  const int h = blockIdx.y;
-  const int split = blockIdx.x;
+  const int g = blockIdx.y;
+  const int chunk = blockIdx.x;
   const int pos = p.pos[r];
-  const int g = h / (p.n_q_heads / p.n_kv_heads);
+  const int grp = p.n_q_heads / p.n_kv_heads;
   const int32_t* pt = p.page_table[r];
-  const int total = pos + 1;  // cached keys 0..pos-1 plus self
-  const int per = (total + p.splits - 1) / p.splits;
-  const int t0 = split * per;
-  const int t1 = min(total, t0 + per);
-  __shared__ float q_s[D];
-  __shared__ float sc[kDecThreads];
-  __shared__ float red[kDecThreads / 32];
-  for (int i = threadIdx.x; i < D; i += kDecThreads) q_s[i] = p.q[(size_t)r * p.n_q_heads * D + h * D + i];
-  __syncthreads();
+  const int total = pos + 1;
+  const int t0 = chunk * kDecChunk;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __shared__ float q_s[kDecMaxGroup][D];
+  __shared__ float sc[kDecMaxGroup][kDecChunk];
+  __shared__ float stat[kDecMaxGroup][2];
+  __shared__ float red[kDecThreads / 32][kDecMaxGroup][D];
+  if (t0 >= total) return;
   const float scale = rsqrtf(static_cast<float>(D));
-  float* part = p.part + (((size_t)r * p.n_q_heads + h) * p.splits + split) * (D + 2);
-  float m = -FLT_MAX, l = 0.f;
-  // each thread accumulates acc for dims threadIdx.x (and + 128 for D > 128; D <= 128 here)
-  float acc = 0.f;
-  const int dd = threadIdx.x;
-  for (int base = t0; base < t1; base += kDecThreads) {
-    const int t = base + threadIdx.x;
-    float s = -FLT_MAX;
-    if (t < t1) {
-      float dot = 0.f;
-      if (t < pos) {
-        const __nv_bfloat16* kr =
-            p.kpages + (((size_t)pt[t / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D;
-        for (int i = 0; i < D; i += 8) {
-          const uint4 u = *reinterpret_cast<const uint4*>(kr + i);
-          const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+  for (int i = threadIdx.x; i < grp * D; i += kDecThreads)
+    q_s[i / D][i % D] = p.q[(size_t)r * p.n_q_heads * D + (g * grp + i / D) * D + i % D] * scale;
+  __syncthreads();
+  // 1. scores
+  {
+    const int t = t0 + threadIdx.x;
+    float dot[kDecMaxGroup];
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            dot += q_s[i + 2 * j] * bf16_lo(wv[j]) + q_s[i + 2 * j + 1] * bf16_hi(wv[j]);
+    for (int h = 0; h < kDecMaxGroup; ++h) dot[h] = 0.f;
+    if (t < total) {
+      if (t < pos) {
+        const uint4* kr = reinterpret_cast<const uint4*>(
+            p.kpages + (((size_t)pt[t / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D);
+#pragma unroll 4
+        for (int i = 0; i < D / 8; ++i) {
+          const uint4 u = kr[i];
+          const float k8[8] = {bf16_lo(u.x), bf16_hi(u.x), bf16_lo(u.y), bf16_hi(u.y),
+                               bf16_lo(u.z), bf16_hi(u.z), bf16_lo(u.w), bf16_hi(u.w)};
+#pragma unroll
+          for (int h = 0; h < kDecMaxGroup; ++h)
+            if (h < grp)
+#pragma unroll
+              for (int e = 0; e < 8; ++e) dot[h] += q_s[h][8 * i + e] * k8[e];
         }
       } else {
         const float* kr = p.k_self + (size_t)r * p.n_kv_heads * D + g * D;
-        for (int i = 0; i < D; ++i) dot += q_s[i] * kr[i];
-      }
-      s = dot * scale;
-    }
-    sc[threadIdx.x] = s;
-    // block max of this chunk
-    float cm = warp_max(s);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = cm;
-    __syncthreads();
-    cm = red[0];
-    for (int i = 1; i < kDecThreads / 32; ++i) cm = fmaxf(cm, red[i]);
-    const float m_new = fmaxf(m, cm);
-    const float alpha = (m == -FLT_MAX) ? 0.f : __expf(m - m_new);
-    acc *= alpha;
-    l *= alpha;
-    const int cnt = min(kDecThreads, t1 - base);
-    for (int j = 0; j < cnt; ++j) {
-      const float pj = __expf(sc[j] - m_new);
-      l += pj;
-      const int tt = base + j;
-      if (dd < D) {
-        float vv;
-        if (tt < pos) {
-          const __nv_bfloat16* vr =
-              p.vpages + (((size_t)pt[tt / kPage] * p.n_kv_heads + g) * kPage + tt % kPage) * D;
-          vv = __bfloat162float(vr[dd]);
-        } else {
-          vv = p.v_self[(size_t)r * p.n_kv_heads * D + g * D + dd];
+        for (int i = 0; i < D; ++i) {
+          const float kv = kr[i];
+#pragma unroll
+          for (int h = 0; h < kDecMaxGroup; ++h)
+            if (h < grp) dot[h] += q_s[h][i] * kv;
         }
-        acc += pj * vv;
       }
     }
-    m = m_new;
-    __syncthreads();
+#pragma unroll
+    for (int h = 0; h < kDecMaxGroup; ++h)
+      if (h < grp) sc[h][threadIdx.x] = t < total ? dot[h] : -FLT_MAX;
   }
-  if (dd < D) part[dd] = acc;
-  if (threadIdx.x == 0) {
-    part[D] = m;
-    part[D + 1] = l;
+  __syncthreads();
+  // 2. per-head max, exponentials, sum (warp h)
+  if (warp < grp) {
+    float m = -FLT_MAX;
+    for (int i = lane; i < kDecChunk; i += 32) m = fmaxf(m, sc[warp][i]);
+    m = warp_max(m);
+    float l = 0.f;
+    for (int i = lane; i < kDecChunk; i += 32) {
+      const float e = sc[warp][i] == -FLT_MAX ? 0.f : __expf(sc[warp][i] - m);
+      sc[warp][i] = e;
+      l += e;
+    }
+    l = warp_sum(l);
+    if (lane == 0) {
+      stat[warp][0] = m;
+      stat[warp][1] = l;
+    }
+  }
+  __syncthreads();
+  // 3. O partial: warp w takes positions t0 + 32w .. t0 + 32w + 31
+  float acc[kDecMaxGroup][DPL];
+#pragma unroll
+  for (int h = 0; h < kDecMaxGroup; ++h)
+#pragma unroll
+    for (int e = 0; e < DPL; ++e) acc[h][e] = 0.f;
+  const int kb = warp * 32;
+  const int kend = min(32, total - t0 - kb);
+  for (int k = 0; k < kend; ++k) {
+    const int t = t0 + kb + k;
+    float v[DPL];
+    if (t < pos) {
+      const __nv_bfloat16* vr =
+          p.vpages + (((size_t)pt[t / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D + lane * DPL;
+      if (DPL == 4) {
+        const uint2 u = *reinterpret_cast<const uint2*>(vr);
+        v[0] = bf16_lo(u.x);
+        v[1 % DPL] = bf16_hi(u.x);
+        v[2 % DPL] = bf16_lo(u.y);
+        v[3 % DPL] = bf16_hi(u.y);
+      } else {
+        const uint32_t u = *reinterpret_cast<const uint32_t*>(vr);
+        v[0] = bf16_lo(u);
+        v[1 % DPL] = bf16_hi(u);
+      }
+    } else {
+      const float* vr = p.v_self + (size_t)r * p.n_kv_heads * D + g * D + lane * DPL;
+#pragma unroll
+      for (int e = 0; e < DPL; ++e) v[e] = vr[e];
+    }
+#pragma unroll
+    for (int h = 0; h < kDecMaxGroup; ++h)
+      if (h < grp) {
+        const float ph = sc[h][kb + k];
+#pragma unroll
+        for (int e = 0; e < DPL; ++e) acc[h][e] += ph * v[e];
+      }
+  }
+#pragma unroll
+  for (int h = 0; h < kDecMaxGroup; ++h)
+    if (h < grp)
+#pragma unroll
+      for (int e = 0; e < DPL; ++e) red[warp][h][lane * DPL + e] = acc[h][e];
+  __syncthreads();
+  for (int i = threadIdx.x; i < grp * D; i += kDecThreads) {
+    const int h = i / D, d = i % D;
+    float o = 0.f;
+#pragma unroll
+    for (int w = 0; w < kDecThreads / 32; ++w) o += red[w][h][d];
+    float* part = p.part + (((size_t)r * p.n_q_heads + g * grp + h) * p.splits + chunk) * (D + 2);
+    part[d] = o;
+    if (d == 0) {
+      part[D] = stat[h][0];
+      part[D + 1] = stat[h][1];
+    }
   }
 }
 
@@ -354,14 +413,13 @@ template <int D>
 __global__ void decode_attn_combine(const DecodeAttnDesc p) {
   const int r = blockIdx.y, h = blockIdx.x;
   const int dd = threadIdx.x;
+  const int n_chunks = (p.pos[r] + 1 + kDecChunk - 1) / kDecChunk;
   const float* base = p.part + ((size_t)r * p.n_q_heads + h) * p.splits * (D + 2);
   float m = -FLT_MAX;
-  for (int s = 0; s < p.splits; ++s) m = fmaxf(m, base[s * (D + 2) + D]);
+  for (int s = 0; s < n_chunks; ++s) m = fmaxf(m, base[s * (D + 2) + D]);
   float l = 0.f, acc = 0.f;
-  for (int s = 0; s < p.splits; ++s) {
-    const float ms = base[s * (D + 2) + D];
-    if (ms == -FLT_MAX) continue;
-    const float f = __expf(ms - m);
+  for (int s = 0; s < n_chunks; ++s) {
+    const float f = __expf(base[s * (D + 2) + D] - m);
     l += f * base[s * (D + 2) + D + 1];
     if (dd < D) acc += f * base[s * (D + 2) + dd];
   }
@@ -402,7 +460,12 @@ cudaError_t launch_attention(const AttnDesc& d, int num_sms, cudaStream_t stream
 }
 
 cudaError_t launch_decode_attention(const DecodeAttnDesc& d, cudaStream_t stream) {
-  dim3 g1(d.splits, d.n_q_heads, d.rows), g2(d.n_q_heads, d.rows);
+  if (d.n_q_heads / d.n_kv_heads > kDecMaxGroup) return cudaErrorInvalidValue;
+  int max_pos = 0;
+  for (int r = 0; r < d.rows; ++r) max_pos = max(max_pos, d.pos[r]);
+  const int chunks = (max_pos + 1 + kDecChunk - 1) / kDecChunk;
+  if (chunks > d.splits) return cudaErrorInvalidValue;
+  dim3 g1(chunks, d.n_kv_heads, d.rows), g2(d.n_q_heads, d.rows);
   if (d.head_dim == 128) {
     decode_attn_partial<128><<<g1, kDecThreads, 0, stream>>>(d);
     decode_attn_combine<128><<<g2, 128, 0, stream>>>(d);

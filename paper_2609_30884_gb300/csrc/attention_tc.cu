@@ -31,6 +31,23 @@ constexpr int kN = 128;          // keys per kv tile
 constexpr int kPagesPerTile = kN / kPage;
 constexpr int kThreadsAttn = 320;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+// Number of 32-key chunks per tile (0..4) whose exponentials run on the FMA pipe
+// (exp2_fma) instead of the special-function unit, off the diagonal tile.
+constexpr int kFmaExpChunks = 0;
+
+// 2^x on the FMA pipe for x in [-125, 9]: x = n + f with n = round(x) (the 1.5 * 2^23
+// addend leaves round(x) in the low mantissa bits), f in [-1/2, 1/2]; 2^f from a cubic
+// whose coefficients were fitted here for minimax relative error on [-1/2, 1/2]
+// (Chebyshev-node start, Lawson reweighting; max relative error 7.5e-5, far below the
+// bf16 rounding of P); n is added to the exponent field.
+__device__ __forceinline__ float exp2_fma(float x) {
+  x = fmaxf(x, -125.0f);
+  const float big = 12582912.0f;
+  const float t = x + big;
+  const float f = x - (t - big);
+  const float p = fmaf(fmaf(fmaf(0.05517132f, f, 0.24261054f), f, 0.69326099f), f, 0.99992811f);
+  return __int_as_float(__float_as_int(p) + ((__float_as_int(t) - __float_as_int(big)) << 23));
+}
 
 struct AttnTcArgs {
   CUtensorMap tmQ;  // q [rows, Hq*D], box {64, 128}
@@ -170,33 +187,37 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
+    // Order: S0(0) S1(0) | PV0(j) S0(j+1) PV1(j) S1(j+1) | ... so that the softmax of one
+    // head overlaps the products of the other. tcgen05.mma of one thread execute in issue
+    // order, so S_t(j+1) overwrites the S/P columns only after PV_t(j) has read P_t(j).
     if (lane == 0) {
       bool ok = mbar_wait(&q_full, 0, &abort_flag, a.status);
       bool issued = false;
       const uint32_t idesc_s = idesc_bf16_f32(kM, kN);
       const uint32_t idesc_o = idesc_bf16_f32(kM, D, false, true);
+      auto issue_s = [&](int t, int st) {
+        const uint32_t kb = smem_u32(sK + st * KV_BYTES);
+        const uint32_t qb = smem_u32(sQ + t * Q_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * HALF_ROWS_BYTES + (kk & 3) * 32;
+          mma_bf16_ss(tmem + t * 128, smem_desc(qb + off, 16, 1024, kSwizzle128B),
+                      smem_desc(kb + off, 16, 1024, kSwizzle128B), idesc_s, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(&s_full[t]);
+      };
+      if (ok) ok = mbar_wait(&k_full[0], 0, &abort_flag, a.status);
+      if (ok) {
+        tc_fence_after();
+        for (int t = 0; t < ntiles; ++t) issue_s(t, 0);
+        mma_commit(&k_empty[0]);
+        issued = true;
+      }
       for (int j = 0; j < J && ok; ++j) {
         const int st = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        if (!mbar_wait(&k_full[st], ph, &abort_flag, a.status)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t kb = smem_u32(sK + st * KV_BYTES);
-        for (int t = 0; t < ntiles; ++t) {
-          const uint32_t qb = smem_u32(sQ + t * Q_BYTES);
-#pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * HALF_ROWS_BYTES + (kk & 3) * 32;
-            mma_bf16_ss(tmem + t * 128, smem_desc(qb + off, 16, 1024, kSwizzle128B),
-                        smem_desc(kb + off, 16, 1024, kSwizzle128B), idesc_s, kk > 0 ? 1u : 0u);
-          }
-          mma_commit(&s_full[t]);
-        }
-        issued = true;
-        mma_commit(&k_empty[st]);
-        if (!mbar_wait(&v_full[st], ph, &abort_flag, a.status)) {
+        const int nst = (j + 1) & 1;
+        const bool more = j + 1 < J;
+        if (!mbar_wait(&v_full[st], (j >> 1) & 1, &abort_flag, a.status)) {
           ok = false;
           break;
         }
@@ -214,9 +235,20 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
                         smem_desc(vb + kk * 2048, HALF_ROWS_BYTES, 1024, kSwizzle128B), idesc_o,
                         (j > 0 || kk > 0) ? 1u : 0u);
           }
+          if (more) {
+            if (t == 0) {
+              if (!mbar_wait(&k_full[nst], ((j + 1) >> 1) & 1, &abort_flag, a.status)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+            }
+            issue_s(t, nst);
+          }
         }
         if (!ok) break;
         mma_commit(&v_empty[st]);
+        if (more) mma_commit(&k_empty[nst]);
       }
       if (ok) {
         mma_commit(&o_full);
@@ -238,20 +270,21 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
       const uint32_t tO = tmem + lane_off + 256 + t * 128;
       const float sl2 = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
       const int qrow = q0 + r;
-      float m_run = -FLT_MAX, l_run = 0.f;
+      float m_run = -INFINITY, l_run = 0.f;
       bool ok = true;
       for (int j = 0; j < J && ok; ++j) {
         // warp-uniform outcome: the TMEM accesses below are warp-collective
         ok = __all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, &abort_flag, a.status));
         if (!ok) break;
         tc_fence_after();
+        const int k0 = j * kN;
+        const bool last = j == J - 1;
         uint32_t sr[4][32];
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
         tmem_ld_wait();
-        const int k0 = j * kN;
-        const bool last = j == J - 1;
-        float mt = -FLT_MAX;
+        // row max over the scaled scores; masked entries (diagonal tile only) become -inf
+        float mt = -INFINITY;
 #pragma unroll
         for (int c = 0; c < 4; ++c)
 #pragma unroll
@@ -259,14 +292,14 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
             float x = __uint_as_float(sr[c][i]) * sl2;
             if (last) {
               const int col = k0 + c * 32 + i;
-              if (col > qrow || col >= kv_end) x = -FLT_MAX;
+              if (col > qrow || col >= kv_end) x = -INFINITY;
             }
             sr[c][i] = __float_as_uint(x);
             mt = fmaxf(mt, x);
           }
-        const float m_new = fmaxf(m_run, mt);
-        const bool grow = m_new > m_run + kRescaleThreshold;
-        const float alpha = grow ? ex2_approx(m_run - m_new) : 1.0f;
+        // rescale O only when the running max grows by more than 2^8
+        const bool grow = mt > m_run + kRescaleThreshold;
+        const float alpha = grow ? ex2_approx(m_run - mt) : 1.0f;
         if (j > 0 && __any_sync(0xffffffffu, grow)) {
           for (int c = 0; c < D / 32; ++c) {
             uint32_t o[32];
@@ -280,18 +313,20 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
         }
         if (grow) {
           l_run *= alpha;
-          m_run = m_new;
+          m_run = mt;
         }
         float rs = 0.f;
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
+          // keys 64c .. 64c+63 -> packed bf16 P columns 32c .. 32c+31 (S already in registers)
           uint32_t pk[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const float x0 = __uint_as_float(sr[2 * c + i / 16][(2 * i) % 32]);
-            const float x1 = __uint_as_float(sr[2 * c + i / 16][(2 * i + 1) % 32]);
-            const float p0 = x0 <= -FLT_MAX ? 0.f : ex2_approx(x0 - m_run);
-            const float p1 = x1 <= -FLT_MAX ? 0.f : ex2_approx(x1 - m_run);
+            const float x0 = __uint_as_float(sr[2 * c + i / 16][(2 * i) % 32]) - m_run;
+            const float x1 = __uint_as_float(sr[2 * c + i / 16][(2 * i + 1) % 32]) - m_run;
+            const bool fma_pipe = !last && 2 * c + i / 16 >= 4 - kFmaExpChunks;
+            const float p0 = fma_pipe ? exp2_fma(x0) : ex2_approx(x0);
+            const float p1 = fma_pipe ? exp2_fma(x1) : ex2_approx(x1);
             rs += p0 + p1;
             pk[i] = pack_bf16(p0, p1);
           }

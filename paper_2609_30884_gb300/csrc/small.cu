@@ -6,20 +6,25 @@
 #include "kernels.h"
 
 #include <cfloat>
+#include <cmath>
 
 namespace crf {
 
 namespace {
 
 // ------------------------------------------------------------------ RoPE table
-// table[p][i] = (cos, sin)(p * theta^(-2i/d)), angle formed in fp64.
-__global__ void rope_table_kernel(float2* table, int n_pos, int half, double theta, int d) {
+// table[p][i] = (cos, sin)(p * theta^(-2i/d)): the angle in turns, p * theta^(-2i/d) / (2 pi),
+// is formed in fp64 (per-frequency factors computed on the host in fp64), reduced to [0, 1)
+// and evaluated with fp32 sincospi.
+struct RopeFreqs {
+  double turns_per_pos[64];
+};
+
+__global__ void rope_table_kernel(float2* table, int n_pos, int half, const __grid_constant__ RopeFreqs f) {
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= n_pos * half) return;
   const int p = idx / half, i = idx % half;
-  // angle p * theta^(-2i/d) in fp64, reduced to turns in [0, 1), then fp32 sincospi
-  const double inv_freq = pow(theta, -2.0 * i / d);
-  double turns = static_cast<double>(p) * inv_freq * 0.15915494309189535;  // 1 / (2 pi)
+  double turns = static_cast<double>(p) * f.turns_per_pos[i];
   turns -= floor(turns);
   float s, c;
   sincospif(static_cast<float>(2.0 * turns), &s, &c);
@@ -98,52 +103,69 @@ __global__ void embed_kernel(const __nv_bfloat16* __restrict__ e, const int32_t*
 }
 
 // ------------------------------------------------------------------ decode-path GEMV
-// Block of 8 warps; warp w computes output j = blockIdx.x * 8 + w for every row.
-// x is staged through shared memory in K chunks.
+// Warp per output j (8 per block), for up to 8 rows at once. Each lane streams 16-byte
+// pieces of the weight row, four in flight; x is read through the cache (every warp of the
+// GPU reads the same few rows).
 constexpr int kGemvWarps = 8;
-constexpr int kGemvChunk = 1024;
 constexpr int kGemvMaxRows = 8;
 
+template <int NR>
+__device__ __forceinline__ void gemv_row_block(const GemvDesc& d, int j, int r0, int lane,
+                                               float (&acc)[kGemvMaxRows]) {
+  const __nv_bfloat16* wr = d.W + (size_t)j * d.in_dim;
+  const int n8 = d.in_dim / 8;
+  int c = lane;
+  for (; c + 96 < n8; c += 128) {
+    uint4 u[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) u[q] = __ldg(reinterpret_cast<const uint4*>(wr) + c + 32 * q);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float w8[8] = {bf16_lo(u[q].x), bf16_hi(u[q].x), bf16_lo(u[q].y), bf16_hi(u[q].y),
+                           bf16_lo(u[q].z), bf16_hi(u[q].z), bf16_lo(u[q].w), bf16_hi(u[q].w)};
+      const int col = 8 * (c + 32 * q);
+#pragma unroll
+      for (int r = 0; r < NR; ++r) {
+        const float4* xr = reinterpret_cast<const float4*>(d.x + (size_t)(r0 + r) * d.in_dim + col);
+        const float4 a = __ldg(xr), b = __ldg(xr + 1);
+        acc[r] += w8[0] * a.x + w8[1] * a.y + w8[2] * a.z + w8[3] * a.w + w8[4] * b.x +
+                  w8[5] * b.y + w8[6] * b.z + w8[7] * b.w;
+      }
+    }
+  }
+  for (; c < n8; c += 32) {
+    const uint4 u = __ldg(reinterpret_cast<const uint4*>(wr) + c);
+    const float w8[8] = {bf16_lo(u.x), bf16_hi(u.x), bf16_lo(u.y), bf16_hi(u.y),
+                         bf16_lo(u.z), bf16_hi(u.z), bf16_lo(u.w), bf16_hi(u.w)};
+#pragma unroll
+    for (int r = 0; r < NR; ++r) {
+      const float4* xr = reinterpret_cast<const float4*>(d.x + (size_t)(r0 + r) * d.in_dim + 8 * c);
+      const float4 a = __ldg(xr), b = __ldg(xr + 1);
+      acc[r] += w8[0] * a.x + w8[1] * a.y + w8[2] * a.z + w8[3] * a.w + w8[4] * b.x +
+                w8[5] * b.y + w8[6] * b.z + w8[7] * b.w;
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const GemvDesc d) {
-  __shared__ float xs[kGemvMaxRows * kGemvChunk];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int j = blockIdx.x * kGemvWarps + warp;
   const int r0 = blockIdx.y * kGemvMaxRows;
   const int nr = min(kGemvMaxRows, d.rows - r0);
+  if (j >= d.out_dim) return;
   float acc[kGemvMaxRows];
 #pragma unroll
   for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = 0.f;
-  for (int k0 = 0; k0 < d.in_dim; k0 += kGemvChunk) {
-    const int kc = min(kGemvChunk, d.in_dim - k0);
-    __syncthreads();
-    for (int i = threadIdx.x; i < nr * kc; i += blockDim.x) {
-      const int r = i / kc, c = i % kc;
-      xs[r * kGemvChunk + c] = d.x[(size_t)(r0 + r) * d.in_dim + k0 + c];
-    }
-    __syncthreads();
-    if (j < d.out_dim) {
-      const __nv_bfloat16* wr = d.W + (size_t)j * d.in_dim + k0;
-      for (int c = lane * 8; c < kc; c += 256) {
-        const uint4 u = *reinterpret_cast<const uint4*>(wr + c);
-        const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
-        float wf[8];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          wf[2 * q] = bf16_lo(wv[q]);
-          wf[2 * q + 1] = bf16_hi(wv[q]);
-        }
-#pragma unroll
-        for (int r = 0; r < kGemvMaxRows; ++r) {
-          if (r < nr) {
-            const float* xr = xs + r * kGemvChunk + c;
-#pragma unroll
-            for (int q = 0; q < 8; ++q) acc[r] += wf[q] * xr[q];
-          }
-        }
-      }
-    }
+  switch (nr) {
+    case 1: gemv_row_block<1>(d, j, r0, lane, acc); break;
+    case 2: gemv_row_block<2>(d, j, r0, lane, acc); break;
+    case 3: gemv_row_block<3>(d, j, r0, lane, acc); break;
+    case 4: gemv_row_block<4>(d, j, r0, lane, acc); break;
+    case 5: gemv_row_block<5>(d, j, r0, lane, acc); break;
+    case 6: gemv_row_block<6>(d, j, r0, lane, acc); break;
+    case 7: gemv_row_block<7>(d, j, r0, lane, acc); break;
+    default: gemv_row_block<8>(d, j, r0, lane, acc); break;
   }
-  if (j >= d.out_dim) return;
 #pragma unroll
   for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = warp_sum(acc[r]);
   if (lane < nr) {
@@ -288,24 +310,30 @@ __global__ void __launch_bounds__(kKlThreads) kl_partial_kernel(const float* __r
   }
 }
 
-// KL = D/S* + (M + log S) - (M* + log S*)  combining the splits of one row (fp64).
+// KL = D/S* + (M + log S) - (M* + log S*), combining the splits of one row (warp per row).
 __global__ void kl_final_kernel(const float* part, int splits, float* out, int rows) {
-  const int row = blockIdx.x * blockDim.x + threadIdx.x;
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
   if (row >= rows) return;
   const float* p = part + (size_t)row * splits * 5;
-  double Mr = -1e300, Mc = -1e300;
-  for (int s = 0; s < splits; ++s) {
-    Mr = fmax(Mr, (double)p[s * 5 + 0]);
-    Mc = fmax(Mc, (double)p[s * 5 + 3]);
+  float Mr = -FLT_MAX, Mc = -FLT_MAX;
+  for (int s = lane; s < splits; s += 32) {
+    Mr = fmaxf(Mr, p[s * 5 + 0]);
+    Mc = fmaxf(Mc, p[s * 5 + 3]);
   }
-  double Sr = 0, Dr = 0, Sc = 0;
-  for (int s = 0; s < splits; ++s) {
-    const double fr = exp((double)p[s * 5 + 0] - Mr);
+  Mr = warp_max(Mr);
+  Mc = warp_max(Mc);
+  float Sr = 0.f, Dr = 0.f, Sc = 0.f;
+  for (int s = lane; s < splits; s += 32) {
+    const float fr = p[s * 5 + 0] == -FLT_MAX ? 0.f : __expf(p[s * 5 + 0] - Mr);
     Sr += fr * p[s * 5 + 1];
     Dr += fr * p[s * 5 + 2];
-    Sc += exp((double)p[s * 5 + 3] - Mc) * p[s * 5 + 4];
+    Sc += (p[s * 5 + 3] == -FLT_MAX ? 0.f : __expf(p[s * 5 + 3] - Mc)) * p[s * 5 + 4];
   }
-  out[row] = static_cast<float>(Dr / Sr + (Mc + log(Sc)) - (Mr + log(Sr)));
+  Sr = warp_sum(Sr);
+  Dr = warp_sum(Dr);
+  Sc = warp_sum(Sc);
+  if (lane == 0) out[row] = Dr / Sr + (Mc + logf(Sc)) - (Mr + logf(Sr));
 }
 
 // ------------------------------------------------------------------ drift
@@ -440,7 +468,11 @@ cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double the
   const int half = head_dim / 2;
   const int n = n_pos * half;
   if (n == 0) return cudaSuccess;
-  rope_table_kernel<<<cdiv(n, 256), 256, 0, stream>>>(table, n_pos, half, theta, head_dim);
+  if (half > 64) return cudaErrorInvalidValue;
+  RopeFreqs f;
+  for (int i = 0; i < half; ++i)
+    f.turns_per_pos[i] = std::pow(theta, -2.0 * i / head_dim) / (2.0 * 3.14159265358979323846);
+  rope_table_kernel<<<cdiv(n, 256), 256, 0, stream>>>(table, n_pos, half, f);
   return cudaGetLastError();
 }
 
@@ -461,6 +493,7 @@ cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv
 
 cudaError_t launch_gemv(const GemvDesc& d, cudaStream_t stream) {
   if (d.rows == 0 || d.out_dim == 0) return cudaSuccess;
+  if (d.in_dim % 8 != 0) return cudaErrorInvalidValue;
   dim3 grid(cdiv(d.out_dim, kGemvWarps), cdiv(d.rows, kGemvMaxRows));
   gemv_kernel<<<grid, kGemvWarps * 32, 0, stream>>>(d);
   return cudaGetLastError();
@@ -530,7 +563,7 @@ cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab,
                       float* part, int splits, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
   kl_partial_kernel<<<dim3(splits, rows), kKlThreads, 0, stream>>>(zref, zcur, vocab, splits, part);
-  kl_final_kernel<<<cdiv(rows, 64), 64, 0, stream>>>(part, splits, out, rows);
+  kl_final_kernel<<<cdiv(rows, 8), 256, 0, stream>>>(part, splits, out, rows);
   return cudaGetLastError();
 }
 
