@@ -307,9 +307,22 @@ def run_window_only(args):
     b.record()
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / args.steps
+    ctx.profile_enable(True, 4096)
+    for _ in range(args.steps):
+        ctx.recompute_window(dm.crf, cur.crf, pool, [req], ws)
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    flops, _ = algorithmic_work(cfg, lc, n)
+    kern = {}
+    for k, (kms, cnt) in prof.items():
+        if k == "_dropped" or cnt == 0:
+            continue
+        kern[k] = {"ms_per_window": round(kms / args.steps, 4)}
+        if k in flops:
+            kern[k]["tflops"] = round(flops[k] * (e - s) * args.steps / (kms / 1000.0) / 1e12, 1)
     print(json.dumps({"case": "window-only", "workload": args.workload, "tokens": n,
                       "window": [s, e], "ms_per_window": ms,
-                      "layer_tokens_per_s": (e - s) * n / (ms / 1000.0)}))
+                      "layer_tokens_per_s": (e - s) * n / (ms / 1000.0), "kernels": kern}))
     ctx.close()
     return 0
 

@@ -31,23 +31,6 @@ constexpr int kN = 128;          // keys per kv tile
 constexpr int kPagesPerTile = kN / kPage;
 constexpr int kThreadsAttn = 320;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
-// Number of 32-key chunks per tile (0..4) whose exponentials run on the FMA pipe
-// (exp2_fma) instead of the special-function unit, off the diagonal tile.
-constexpr int kFmaExpChunks = 0;
-
-// 2^x on the FMA pipe for x in [-125, 9]: x = n + f with n = round(x) (the 1.5 * 2^23
-// addend leaves round(x) in the low mantissa bits), f in [-1/2, 1/2]; 2^f from a cubic
-// whose coefficients were fitted here for minimax relative error on [-1/2, 1/2]
-// (Chebyshev-node start, Lawson reweighting; max relative error 7.5e-5, far below the
-// bf16 rounding of P); n is added to the exponent field.
-__device__ __forceinline__ float exp2_fma(float x) {
-  x = fmaxf(x, -125.0f);
-  const float big = 12582912.0f;
-  const float t = x + big;
-  const float f = x - (t - big);
-  const float p = fmaf(fmaf(fmaf(0.05517132f, f, 0.24261054f), f, 0.69326099f), f, 0.99992811f);
-  return __int_as_float(__float_as_int(p) + ((__float_as_int(t) - __float_as_int(big)) << 23));
-}
 
 struct AttnTcArgs {
   CUtensorMap tmQ;  // q [rows, Hq*D], box {64, 128}
@@ -83,6 +66,76 @@ __device__ __forceinline__ bool attn_work(const AttnTcArgs& a, int idx, AttnWork
     idx -= items;
   }
   return false;
+}
+
+// One query row's share of one kv tile: S row (128 raw scores) from TMEM, running max
+// and sum update, O rescaled in TMEM when the max grows by more than 2^8, and P (bf16,
+// unnormalised) written back over the S columns. MASK (diagonal tile only) sets every
+// key index above `lim` to -inf; the common off-diagonal instance has no masking code.
+template <int D, bool MASK>
+__device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, bool first, int lim,
+                                             float sl2, float& m_run, float& l_run) {
+  uint32_t sr[4][32];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+  tmem_ld_wait();
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int c = 0; c < 4; ++c)
+#pragma unroll
+    for (int i = 0; i < 32; i += 2) {
+      float x0 = __uint_as_float(sr[c][i]), x1 = __uint_as_float(sr[c][i + 1]);
+      if (MASK) {
+        if (c * 32 + i > lim) {
+          x0 = -INFINITY;
+          sr[c][i] = __float_as_uint(x0);
+        }
+        if (c * 32 + i + 1 > lim) {
+          x1 = -INFINITY;
+          sr[c][i + 1] = __float_as_uint(x1);
+        }
+      }
+      mx0 = fmaxf(mx0, x0);
+      mx1 = fmaxf(mx1, x1);
+    }
+  const float mt = fmaxf(mx0, mx1);
+  // the running max is kept in raw score units; p = 2^(s * sl2 - m_run * sl2)
+  const bool grow = (mt - m_run) * sl2 > kRescaleThreshold;
+  const float alpha = grow ? ex2_approx((m_run - mt) * sl2) : 1.0f;
+  if (!first && __any_sync(0xffffffffu, grow)) {
+#pragma unroll 1
+    for (int c = 0; c < D / 32; ++c) {
+      uint32_t o[32];
+      tmem_ld32(tO + c * 32, o);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+      tmem_st32(tO + c * 32, o);
+    }
+    tmem_st_wait();
+  }
+  if (grow) {
+    l_run *= alpha;
+    m_run = mt;
+  }
+  const float neg_m = -m_run * sl2;
+  float rs0 = 0.f, rs1 = 0.f;
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    // keys 32c .. 32c+31 -> packed bf16 P columns 16c .. 16c+15 (S already in registers)
+    uint32_t pk[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c][2 * i]), sl2, neg_m));
+      const float p1 = ex2_approx(fmaf(__uint_as_float(sr[c][2 * i + 1]), sl2, neg_m));
+      rs0 += p0;
+      rs1 += p1;
+      pk[i] = pack_bf16(p0, p1);
+    }
+    tmem_st16(tS + 16 * c, pk);
+  }
+  tmem_st_wait();
+  l_run += rs0 + rs1;
 }
 
 template <int D>
@@ -270,7 +323,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
       const uint32_t tO = tmem + lane_off + 256 + t * 128;
       const float sl2 = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
       const int qrow = q0 + r;
-      float m_run = -INFINITY, l_run = 0.f;
+      float m_run = -INFINITY, l_run = 0.f;  // running max in raw score units
       bool ok = true;
       for (int j = 0; j < J && ok; ++j) {
         // warp-uniform outcome: the TMEM accesses below are warp-collective
@@ -279,61 +332,12 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
         tc_fence_after();
         const int k0 = j * kN;
         const bool last = j == J - 1;
-        uint32_t sr[4][32];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
-        tmem_ld_wait();
-        // row max over the scaled scores; masked entries (diagonal tile only) become -inf
-        float mt = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            float x = __uint_as_float(sr[c][i]) * sl2;
-            if (last) {
-              const int col = k0 + c * 32 + i;
-              if (col > qrow || col >= kv_end) x = -INFINITY;
-            }
-            sr[c][i] = __float_as_uint(x);
-            mt = fmaxf(mt, x);
-          }
-        // rescale O only when the running max grows by more than 2^8
-        const bool grow = mt > m_run + kRescaleThreshold;
-        const float alpha = grow ? ex2_approx(m_run - mt) : 1.0f;
-        if (j > 0 && __any_sync(0xffffffffu, grow)) {
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32(tO + c * 32, o);
-            tmem_ld_wait();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-            tmem_st32(tO + c * 32, o);
-          }
-          tmem_st_wait();
+        if (last) {
+          // keys above min(query row, prefix end - 1) are masked on the diagonal tile
+          softmax_tile<D, true>(tS, tO, j == 0, min(qrow, kv_end - 1) - k0, sl2, m_run, l_run);
+        } else {
+          softmax_tile<D, false>(tS, tO, j == 0, 0, sl2, m_run, l_run);
         }
-        if (grow) {
-          l_run *= alpha;
-          m_run = mt;
-        }
-        float rs = 0.f;
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          // keys 64c .. 64c+63 -> packed bf16 P columns 32c .. 32c+31 (S already in registers)
-          uint32_t pk[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float x0 = __uint_as_float(sr[2 * c + i / 16][(2 * i) % 32]) - m_run;
-            const float x1 = __uint_as_float(sr[2 * c + i / 16][(2 * i + 1) % 32]) - m_run;
-            const bool fma_pipe = !last && 2 * c + i / 16 >= 4 - kFmaExpChunks;
-            const float p0 = fma_pipe ? exp2_fma(x0) : ex2_approx(x0);
-            const float p1 = fma_pipe ? exp2_fma(x1) : ex2_approx(x1);
-            rs += p0 + p1;
-            pk[i] = pack_bf16(p0, p1);
-          }
-          tmem_st32(tS + c * 32, pk);
-        }
-        tmem_st_wait();
-        l_run += rs;
         if (last && t == 0 && kv_end - k0 < kN) {
           // zero V rows past the prefix so that 0 * stale data cannot produce NaN
           const int st = j & 1;
