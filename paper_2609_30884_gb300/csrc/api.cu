@@ -207,7 +207,7 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
   p.splits = dec_splits(p.max_n);
   // decode scratch, fp32: x, xn, x1, q, k, v, o, xa, gu, m, part
-  const size_t dec = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + kRankPad + 3 * D.f) * 4 +
+  const size_t dec = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 3 * kRankPad + 3 * D.f) * 4 +
                      static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
   p.dec_bytes = align256(dec);
   p.off_dec = take(p.dec_rows ? p.dec_bytes : 0);
@@ -465,54 +465,80 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
 crf_status decode_row(const LayerCtx& c, int l0, const __nv_bfloat16* start_row, int pos,
                       const int32_t* page_table, void* out_bf16) {
   const Dims& D = *c.D;
-  int n_adapted = 0;
-  for (int m = 0; m < 7; ++m) n_adapted += adapted(c.ad, m) ? 1 : 0;
-  // per layer: 2 norms, 7 GEMVs, adapted LoRA downs, 2 RoPE, 2 attention, 1 SwiGLU; + 2 converts
-  ProfScope ps(c.ctx, kPDecode, c.st, (D.N - l0) * (14 + n_adapted) + 2);
+  const bool ad_qkv = adapted(c.ad, 0) || adapted(c.ad, 1) || adapted(c.ad, 2);
+  const bool ad_gu = adapted(c.ad, CRF_MOD_GATE) || adapted(c.ad, CRF_MOD_UP);
+  (void)ad_qkv;
+  (void)ad_gu;
+  const int lora_launches = adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN);
+  // per layer: 2 norm + LoRA-down launches, other LoRA downs, 4 GEMVs, 1 RoPE, 2 attention,
+  // 1 SwiGLU; + 2 converts
+  ProfScope ps(c.ctx, kPDecode, c.st, (D.N - l0) * (10 + lora_launches) + 2);
   const Plan& p = *c.plan;
   float* base = reinterpret_cast<float*>(c.ws + p.off_dec);
   float* x = base;
   float* xn = x + D.h;
   float* x1 = xn + D.h;
-  float* q = x1 + D.h;
-  float* o = q + D.qd;
-  float* k = o + D.qd;
+  float* q = x1 + D.h;  // q | k | v contiguous
+  float* k = q + D.qd;
   float* v = k + D.kvd;
-  float* xa = v + D.kvd;
-  float* gu = xa + kRankPad;
+  float* o = v + D.kvd;
+  float* xa = o + D.qd;  // three rank-padded slots
+  float* gu = xa + 3 * kRankPad;
   float* m = gu + 2 * D.f;
   float* part = m + D.f;
   const int rank = c.ad->dims.rank;
   CRF_CUDA(launch_bf16_to_f32(start_row, x, D.h, c.st));
-  auto proj = [&](int l, int mod, const float* in, int in_dim, int out_dim, const void* bias,
-                  const float* resid, float* y) -> cudaError_t {
+  // segments [mods] sharing input `in`: LoRA down products of the adapted ones, then one GEMV
+  // norm_gain: normalise `raw` into `in` inside the LoRA-down launch (replaces the RMSNorm)
+  auto proj = [&](int l, const int* mods, int nm, const float* raw, const void* norm_gain, float* in,
+                  int in_dim, float* const* ys, const int* outs, const float* resid) -> cudaError_t {
+    if (!norm_gain) in = const_cast<float*>(raw);
+    LoraDownRows ld{};
     GemvDesc g{};
-    g.W = static_cast<const __nv_bfloat16*>(c.model->layers[l].W[mod]);
-    g.out_dim = out_dim;
+    g.nseg = nm;
     g.in_dim = in_dim;
     g.x = in;
     g.rows = 1;
-    g.bias = static_cast<const __nv_bfloat16*>(bias);
-    if (adapted(c.ad, mod)) {
-      cudaError_t e = launch_lora_down_rows(static_cast<const __nv_bfloat16*>(c.ad->A[l * 7 + mod]),
-                                            rank, in_dim, in, 1, c.scale, xa, c.st);
-      if (e != cudaSuccess) return e;
-      g.BL = static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + mod]);
-      g.xa = xa;
-      g.rank = rank;
+    g.rank = rank;
+    for (int s = 0; s < nm; ++s) {
+      const int mod = mods[s];
+      GemvSeg& sg = g.seg[s];
+      sg.W = static_cast<const __nv_bfloat16*>(c.model->layers[l].W[mod]);
+      sg.out_dim = outs[s];
+      sg.bias = (mod < 3 && D.bias) ? static_cast<const __nv_bfloat16*>(c.model->layers[l].bias[mod])
+                                    : nullptr;
+      sg.y = ys[s];
+      sg.resid = resid;
+      if (adapted(c.ad, mod)) {
+        sg.BL = static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + mod]);
+        sg.xa = xa + s * kRankPad;
+        ld.A[ld.n] = static_cast<const __nv_bfloat16*>(c.ad->A[l * 7 + mod]);
+        ld.xa[ld.n] = xa + s * kRankPad;
+        ++ld.n;
+      }
     }
-    g.resid = resid;
-    g.y = y;
-    return launch_gemv(g, c.st);
+    if (ld.n || norm_gain) {
+      cudaError_t e = launch_lora_down_rows(ld, rank, in_dim, raw, 1, c.scale,
+                                            static_cast<const __nv_bfloat16*>(norm_gain), D.eps,
+                                            in, c.st);
+      if (e != cudaSuccess) return e;
+    }
+    return launch_gemv(g, c.ctx->num_sms, c.st);
   };
+  const int m_qkv[3] = {CRF_MOD_Q, CRF_MOD_K, CRF_MOD_V};
+  const int o_qkv[3] = {D.qd, D.kvd, D.kvd};
+  float* const y_qkv[3] = {q, k, v};
+  const int m_o[1] = {CRF_MOD_O}, o_o[1] = {D.h};
+  float* const y_o[1] = {x1};
+  const int m_gu[2] = {CRF_MOD_GATE, CRF_MOD_UP}, o_gu[2] = {D.f, D.f};
+  float* const y_gu[2] = {gu, gu + D.f};
+  const int m_d[1] = {CRF_MOD_DOWN}, o_d[1] = {D.h};
+  float* const y_d[1] = {x};
   for (int l = l0; l < D.N; ++l) {
     const crf_layer_weights& w = c.model->layers[l];
-    CRF_CUDA(launch_rmsnorm_f32(x, static_cast<const __nv_bfloat16*>(w.ln1), xn, 1, D.h, D.eps, c.st));
-    CRF_CUDA(proj(l, CRF_MOD_Q, xn, D.h, D.qd, D.bias ? w.bias[0] : nullptr, nullptr, q));
-    CRF_CUDA(proj(l, CRF_MOD_K, xn, D.h, D.kvd, D.bias ? w.bias[1] : nullptr, nullptr, k));
-    CRF_CUDA(proj(l, CRF_MOD_V, xn, D.h, D.kvd, D.bias ? w.bias[2] : nullptr, nullptr, v));
-    CRF_CUDA(launch_rope_rows(q, 1, D.hq, D.d, pos, D.theta, c.st));
-    CRF_CUDA(launch_rope_rows(k, 1, D.hkv, D.d, pos, D.theta, c.st));
+    CRF_CUDA(proj(l, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr));
+    // q and k heads are contiguous: one rotation launch
+    CRF_CUDA(launch_rope_rows(q, 1, D.hq + D.hkv, D.d, pos, D.theta, c.st));
     DecodeAttnDesc a;
     std::memset(&a, 0, sizeof(a));
     a.q = q;
@@ -531,12 +557,10 @@ crf_status decode_row(const LayerCtx& c, int l0, const __nv_bfloat16* start_row,
     a.splits = p.splits;
     a.max_pos = pos;
     CRF_CUDA(launch_decode_attention(a, c.st));
-    CRF_CUDA(proj(l, CRF_MOD_O, o, D.qd, D.h, nullptr, x, x1));
-    CRF_CUDA(launch_rmsnorm_f32(x1, static_cast<const __nv_bfloat16*>(w.ln2), xn, 1, D.h, D.eps, c.st));
-    CRF_CUDA(proj(l, CRF_MOD_GATE, xn, D.h, D.f, nullptr, nullptr, gu));
-    CRF_CUDA(proj(l, CRF_MOD_UP, xn, D.h, D.f, nullptr, nullptr, gu + D.f));
+    CRF_CUDA(proj(l, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x));
+    CRF_CUDA(proj(l, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr));
     CRF_CUDA(launch_swiglu_f32(gu, m, 1, D.f, c.st));
-    CRF_CUDA(proj(l, CRF_MOD_DOWN, m, D.f, D.h, nullptr, x1, x));
+    CRF_CUDA(proj(l, m_d, 1, m, nullptr, nullptr, D.f, y_d, o_d, x1));
   }
   CRF_CUDA(launch_f32_to_bf16(x, static_cast<__nv_bfloat16*>(out_bf16), D.h, c.st));
   return CRF_OK;
@@ -951,7 +975,7 @@ crf_status crf_kl(crf_ctx* ctx, const crf_model* model, const void* ref, const v
     CRF_CUDA(launch_rmsnorm_f32(hf, static_cast<const __nv_bfloat16*>(model->final_norm), hn, 2 * n_rows,
                                 hidden, model->dims.rms_eps, st));
     CRF_CUDA(launch_lm_head(static_cast<const __nv_bfloat16*>(model->lm_head), hn, 2 * n_rows, vocab,
-                            hidden, logits, st));
+                            hidden, logits, ctx->num_sms, st));
     zr = logits;
     zc = logits + static_cast<size_t>(n_rows) * vocab;
   }

@@ -292,10 +292,15 @@ __global__ void __launch_bounds__(kDecThreads) decode_attn_partial(const DecodeA
   __shared__ float sc[kDecMaxGroup][kDecChunk];
   __shared__ float stat[kDecMaxGroup][2];
   __shared__ float red[kDecThreads / 32][kDecMaxGroup][D];
+  __shared__ int page_s[kDecChunk / kPage];
   if (t0 >= total) return;
   const float scale = rsqrtf(static_cast<float>(D));
   for (int i = threadIdx.x; i < grp * D; i += kDecThreads)
     q_s[i / D][i % D] = p.q[(size_t)r * p.n_q_heads * D + (g * grp + i / D) * D + i % D] * scale;
+  if (threadIdx.x < kDecChunk / kPage) {
+    const int t = t0 + threadIdx.x * kPage;
+    page_s[threadIdx.x] = t < pos ? pt[t / kPage] : 0;
+  }
   __syncthreads();
   // 1. scores
   {
@@ -306,7 +311,7 @@ __global__ void __launch_bounds__(kDecThreads) decode_attn_partial(const DecodeA
     if (t < total) {
       if (t < pos) {
         const uint4* kr = reinterpret_cast<const uint4*>(
-            p.kpages + (((size_t)pt[t / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D);
+            p.kpages + (((size_t)page_s[threadIdx.x / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D);
 #pragma unroll 4
         for (int i = 0; i < D / 8; ++i) {
           const uint4 u = kr[i];
@@ -358,21 +363,22 @@ __global__ void __launch_bounds__(kDecThreads) decode_attn_partial(const DecodeA
 #pragma unroll
     for (int e = 0; e < DPL; ++e) acc[h][e] = 0.f;
   const int kb = warp * 32;
-  const int kend = min(32, total - t0 - kb);
+  const int kend = max(0, min(32, total - t0 - kb));
+#pragma unroll 8
   for (int k = 0; k < kend; ++k) {
     const int t = t0 + kb + k;
     float v[DPL];
     if (t < pos) {
-      const __nv_bfloat16* vr =
-          p.vpages + (((size_t)pt[t / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D + lane * DPL;
+      const __nv_bfloat16* vr = p.vpages +
+          (((size_t)page_s[(kb + k) / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D + lane * DPL;
       if (DPL == 4) {
-        const uint2 u = *reinterpret_cast<const uint2*>(vr);
+        const uint2 u = __ldg(reinterpret_cast<const uint2*>(vr));
         v[0] = bf16_lo(u.x);
         v[1 % DPL] = bf16_hi(u.x);
         v[2 % DPL] = bf16_lo(u.y);
         v[3 % DPL] = bf16_hi(u.y);
       } else {
-        const uint32_t u = *reinterpret_cast<const uint32_t*>(vr);
+        const uint32_t u = __ldg(reinterpret_cast<const uint32_t*>(vr));
         v[0] = bf16_lo(u);
         v[1 % DPL] = bf16_hi(u);
       }

@@ -94,23 +94,37 @@ cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows
                                 cudaStream_t stream);
 
 // Small-M decode path (the last prefix row through the layers after the window).
-// y[r, j] = sum_i W[j, i] x[r, i] (+ bias[j]) (+ sum_k BL[j, k] xa[r, k]) (+ resid[r, j])
-struct GemvDesc {
-  const __nv_bfloat16* W;
-  int out_dim, in_dim;
-  const float* x;          // [rows, in_dim] fp32
-  int rows;
-  const __nv_bfloat16* bias;
-  const __nv_bfloat16* BL; // [out_dim, rank] or null
-  const float* xa;         // [rows, rank] fp32 already scaled by alpha/r
-  int rank;
-  const float* resid;      // [rows, out_dim] fp32 or null
-  float* y;                // [rows, out_dim] fp32
+// Up to three row-stacked weight segments share one launch and one input x:
+// y_s[r, j] = sum_i W_s[j, i] x[r, i] (+ bias_s[j]) (+ sum_k BL_s[j, k] xa_s[r, k]) (+ resid_s[r, j])
+struct GemvSeg {
+  const __nv_bfloat16* W;  // [out_dim, in_dim]
+  int out_dim;
+  const __nv_bfloat16* bias;  // [out_dim] or null
+  const __nv_bfloat16* BL;    // [out_dim, rank] or null
+  const float* xa;            // [rows, rank] fp32, already scaled by alpha/r
+  const float* resid;         // [rows, out_dim] fp32 or null
+  float* y;                   // [rows, out_dim] fp32
 };
-cudaError_t launch_gemv(const GemvDesc& d, cudaStream_t stream);
-// xa[r, k] = scale * sum_i A[k, i] x[r, i]
-cudaError_t launch_lora_down_rows(const __nv_bfloat16* A, int rank, int in_dim, const float* x,
-                                  int rows, float scale, float* xa, cudaStream_t stream);
+struct GemvDesc {
+  GemvSeg seg[3];
+  int nseg;
+  int in_dim;
+  const float* x;  // [rows, in_dim] fp32
+  int rows;        // 1..8
+  int rank;
+};
+cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream);
+// xa_m[r, k] = scale * sum_i A_m[k, i] x[r, i] for up to three modules m sharing x
+struct LoraDownRows {
+  const __nv_bfloat16* A[3];
+  float* xa[3];
+  int n;
+};
+// With norm_gain != null, x is normalised first (rmsnorm(x) * norm_gain, eps) and the
+// normalised rows are also written to xn (so the launch replaces the separate RMSNorm).
+cudaError_t launch_lora_down_rows(const LoraDownRows& m, int rank, int in_dim, const float* x,
+                                  int rows, float scale, const __nv_bfloat16* norm_gain, float eps,
+                                  float* xn, cudaStream_t stream);
 cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y, int rows,
                                int hidden, float eps, cudaStream_t stream);
 // Single-query attention of `rows` decode rows (one per request) over pages [0, pos) plus own k/v.
@@ -137,7 +151,7 @@ cudaError_t launch_gather_rows_f32(const __nv_bfloat16* src, const int64_t* row_
 
 // LM head + KL: logits [2*rows, V] (ref rows first) from final-normed hidden rows.
 cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,
-                           float* logits, cudaStream_t stream);
+                           float* logits, int num_sms, cudaStream_t stream);
 // KL per row from fp32 logits; part: scratch [rows][splits][4].
 cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab, float* out,
                       float* part, int splits, cudaStream_t stream);

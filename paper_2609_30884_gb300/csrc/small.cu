@@ -103,100 +103,147 @@ __global__ void embed_kernel(const __nv_bfloat16* __restrict__ e, const int32_t*
 }
 
 // ------------------------------------------------------------------ decode-path GEMV
-// Warp per output j (8 per block), for up to 8 rows at once. Each lane streams 16-byte
-// pieces of the weight row, four in flight; x is read through the cache (every warp of the
-// GPU reads the same few rows).
+// A block of 8 warps takes 8/KS groups of OPW consecutive outputs of one segment; the KS
+// warps of a group split the input dimension, each lane streaming 16-byte pieces of the
+// OPW weight rows (x read through the cache and reused across the OPW rows). Partials are
+// summed in shared memory in a fixed order (deterministic), then bias, LoRA up product and
+// residual are added.
 constexpr int kGemvWarps = 8;
 constexpr int kGemvMaxRows = 8;
 
-template <int NR>
-__device__ __forceinline__ void gemv_row_block(const GemvDesc& d, int j, int r0, int lane,
-                                               float (&acc)[kGemvMaxRows]) {
-  const __nv_bfloat16* wr = d.W + (size_t)j * d.in_dim;
+struct GemvLaunch {
+  GemvDesc d;
+  int opw, ks;
+  int block0[4];  // first block of each segment
+};
+
+template <int OPW, int NR>
+__global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const __grid_constant__ GemvLaunch L) {
+  __shared__ float red[kGemvWarps][OPW][NR];
+  const GemvDesc& d = L.d;
+  const int ks = L.ks;
+  int s = 0;
+  while (s < d.nseg - 1 && static_cast<int>(blockIdx.x) >= L.block0[s + 1]) ++s;
+  const GemvSeg& sg = d.seg[s];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gl = warp / ks, kp = warp % ks;
+  const int groups_per_block = kGemvWarps / ks;
+  const int g = (static_cast<int>(blockIdx.x) - L.block0[s]) * groups_per_block + gl;
+  const int j0 = g * OPW;
   const int n8 = d.in_dim / 8;
-  int c = lane;
-  for (; c + 96 < n8; c += 128) {
-    uint4 u[4];
+  const int per = (n8 + ks - 1) / ks;
+  const int p0 = kp * per, p1 = min(n8, p0 + per);
+  float acc[OPW][NR];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) u[q] = __ldg(reinterpret_cast<const uint4*>(wr) + c + 32 * q);
+  for (int o = 0; o < OPW; ++o)
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float w8[8] = {bf16_lo(u[q].x), bf16_hi(u[q].x), bf16_lo(u[q].y), bf16_hi(u[q].y),
-                           bf16_lo(u[q].z), bf16_hi(u[q].z), bf16_lo(u[q].w), bf16_hi(u[q].w)};
-      const int col = 8 * (c + 32 * q);
+    for (int r = 0; r < NR; ++r) acc[o][r] = 0.f;
+  if (j0 < sg.out_dim) {
+    const uint4* wrow[OPW];
+#pragma unroll
+    for (int o = 0; o < OPW; ++o)
+      wrow[o] = reinterpret_cast<const uint4*>(sg.W + (size_t)min(j0 + o, sg.out_dim - 1) * d.in_dim);
+#pragma unroll 2
+    for (int c = p0 + lane; c < p1; c += 32) {
+      uint4 u[OPW];
+#pragma unroll
+      for (int o = 0; o < OPW; ++o) u[o] = __ldg(wrow[o] + c);
 #pragma unroll
       for (int r = 0; r < NR; ++r) {
-        const float4* xr = reinterpret_cast<const float4*>(d.x + (size_t)(r0 + r) * d.in_dim + col);
-        const float4 a = __ldg(xr), b = __ldg(xr + 1);
-        acc[r] += w8[0] * a.x + w8[1] * a.y + w8[2] * a.z + w8[3] * a.w + w8[4] * b.x +
-                  w8[5] * b.y + w8[6] * b.z + w8[7] * b.w;
+        if (r < d.rows) {
+          const float4* xr = reinterpret_cast<const float4*>(d.x + (size_t)r * d.in_dim) + 2 * c;
+          const float4 a = __ldg(xr), b = __ldg(xr + 1);
+#pragma unroll
+          for (int o = 0; o < OPW; ++o)
+            acc[o][r] += bf16_lo(u[o].x) * a.x + bf16_hi(u[o].x) * a.y + bf16_lo(u[o].y) * a.z +
+                         bf16_hi(u[o].y) * a.w + bf16_lo(u[o].z) * b.x + bf16_hi(u[o].z) * b.y +
+                         bf16_lo(u[o].w) * b.z + bf16_hi(u[o].w) * b.w;
+        }
       }
     }
   }
-  for (; c < n8; c += 32) {
-    const uint4 u = __ldg(reinterpret_cast<const uint4*>(wr) + c);
-    const float w8[8] = {bf16_lo(u.x), bf16_hi(u.x), bf16_lo(u.y), bf16_hi(u.y),
-                         bf16_lo(u.z), bf16_hi(u.z), bf16_lo(u.w), bf16_hi(u.w)};
+#pragma unroll
+  for (int o = 0; o < OPW; ++o)
 #pragma unroll
     for (int r = 0; r < NR; ++r) {
-      const float4* xr = reinterpret_cast<const float4*>(d.x + (size_t)(r0 + r) * d.in_dim + 8 * c);
-      const float4 a = __ldg(xr), b = __ldg(xr + 1);
-      acc[r] += w8[0] * a.x + w8[1] * a.y + w8[2] * a.z + w8[3] * a.w + w8[4] * b.x +
-                w8[5] * b.y + w8[6] * b.z + w8[7] * b.w;
+      const float v = warp_sum(acc[o][r]);
+      if (lane == 0) red[warp][o][r] = v;
     }
-  }
+  __syncthreads();
+  if (kp != 0 || lane >= OPW * NR) return;
+  const int o = lane / NR, r = lane % NR;
+  const int j = j0 + o;
+  if (j >= sg.out_dim || r >= d.rows) return;
+  float v = 0.f;
+  for (int q = 0; q < ks; ++q) v += red[gl * ks + q][o][r];
+  if (sg.bias) v += __bfloat162float(sg.bias[j]);
+  if (sg.BL)
+    for (int k = 0; k < d.rank; ++k)
+      v += __bfloat162float(sg.BL[(size_t)j * d.rank + k]) * sg.xa[(size_t)r * d.rank + k];
+  if (sg.resid) v += sg.resid[(size_t)r * sg.out_dim + j];
+  sg.y[(size_t)r * sg.out_dim + j] = v;
 }
 
-__global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const GemvDesc d) {
+// xa_m[r, k] = scale * <A_m[k, :], x_r> for up to three modules, one block per (module, row, k).
+// With a norm gain g, x_r is first replaced by rmsnorm(x_r) * g: every block computes the row's
+// mean square, and the extra blocks (one per row) also write the normalised row to xn.
+constexpr int kLdThreads = 256;
+
+__global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
+    const LoraDownRows m, int rank, int in_dim, const float* __restrict__ x, int rows, float scale,
+    const __nv_bfloat16* __restrict__ g, float eps, float* __restrict__ xn) {
+  __shared__ float red[kLdThreads / 32];
+  const int b = blockIdx.x;
+  const int n_dot = m.n * rows * rank;
+  const int r = b < n_dot ? (b / rank) % rows : b - n_dot;
+  const float* xr = x + (size_t)r * in_dim;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.x * kGemvWarps + warp;
-  const int r0 = blockIdx.y * kGemvMaxRows;
-  const int nr = min(kGemvMaxRows, d.rows - r0);
-  if (j >= d.out_dim) return;
-  float acc[kGemvMaxRows];
-#pragma unroll
-  for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = 0.f;
-  switch (nr) {
-    case 1: gemv_row_block<1>(d, j, r0, lane, acc); break;
-    case 2: gemv_row_block<2>(d, j, r0, lane, acc); break;
-    case 3: gemv_row_block<3>(d, j, r0, lane, acc); break;
-    case 4: gemv_row_block<4>(d, j, r0, lane, acc); break;
-    case 5: gemv_row_block<5>(d, j, r0, lane, acc); break;
-    case 6: gemv_row_block<6>(d, j, r0, lane, acc); break;
-    case 7: gemv_row_block<7>(d, j, r0, lane, acc); break;
-    default: gemv_row_block<8>(d, j, r0, lane, acc); break;
-  }
-#pragma unroll
-  for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = warp_sum(acc[r]);
-  if (lane < nr) {
-    const int r = lane;
-    float v = 0.f;
-#pragma unroll
-    for (int q = 0; q < kGemvMaxRows; ++q)
-      if (q == r) v = acc[q];
-    if (d.bias) v += __bfloat162float(d.bias[j]);
-    if (d.BL) {
-      for (int k = 0; k < d.rank; ++k)
-        v += __bfloat162float(d.BL[(size_t)j * d.rank + k]) * d.xa[(size_t)(r0 + r) * d.rank + k];
+  float inv = 1.f;
+  if (g) {
+    float ss = 0.f;
+    for (int i = threadIdx.x * 4; i < in_dim; i += kLdThreads * 4) {
+      const float4 a = __ldg(reinterpret_cast<const float4*>(xr + i));
+      ss += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
     }
-    if (d.resid) v += d.resid[(size_t)(r0 + r) * d.out_dim + j];
-    d.y[(size_t)(r0 + r) * d.out_dim + j] = v;
+    ss = warp_sum(ss);
+    if (lane == 0) red[warp] = ss;
+    __syncthreads();
+    ss = 0.f;
+#pragma unroll
+    for (int w = 0; w < kLdThreads / 32; ++w) ss += red[w];
+    inv = rsqrtf(ss / in_dim + eps);
+    __syncthreads();
   }
-}
-
-// xa[r, k] = scale * <A[k, :], x[r, :]>, one warp per (r, k).
-__global__ void lora_down_rows_kernel(const __nv_bfloat16* __restrict__ A, int rank, int in_dim,
-                                      const float* __restrict__ x, int rows, float scale,
-                                      float* __restrict__ xa) {
-  const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (w >= rows * rank) return;
-  const int r = w / rank, k = w % rank;
+  if (b >= n_dot) {  // normalised row for the GEMV that follows
+    for (int i = threadIdx.x; i < in_dim; i += kLdThreads)
+      xn[(size_t)r * in_dim + i] = xr[i] * inv * __bfloat162float(g[i]);
+    return;
+  }
+  const int mi = b / (rows * rank), k = b % rank;
+  const __nv_bfloat16* A = m.A[mi] + (size_t)k * in_dim;
   float s = 0.f;
-  for (int i = lane; i < in_dim; i += 32)
-    s += __bfloat162float(A[(size_t)k * in_dim + i]) * x[(size_t)r * in_dim + i];
+  for (int i = threadIdx.x * 8; i < in_dim; i += kLdThreads * 8) {
+    const uint4 u = __ldg(reinterpret_cast<const uint4*>(A + i));
+    const float4* xp = reinterpret_cast<const float4*>(xr + i);
+    float4 a = __ldg(xp), c = __ldg(xp + 1);
+    if (g) {
+      const uint4 gv = __ldg(reinterpret_cast<const uint4*>(g + i));
+      a.x *= inv * bf16_lo(gv.x); a.y *= inv * bf16_hi(gv.x); a.z *= inv * bf16_lo(gv.y);
+      a.w *= inv * bf16_hi(gv.y); c.x *= inv * bf16_lo(gv.z); c.y *= inv * bf16_hi(gv.z);
+      c.z *= inv * bf16_lo(gv.w); c.w *= inv * bf16_hi(gv.w);
+    }
+    s += bf16_lo(u.x) * a.x + bf16_hi(u.x) * a.y + bf16_lo(u.y) * a.z + bf16_hi(u.y) * a.w +
+         bf16_lo(u.z) * c.x + bf16_hi(u.z) * c.y + bf16_lo(u.w) * c.z + bf16_hi(u.w) * c.w;
+  }
   s = warp_sum(s);
-  if (lane == 0) xa[(size_t)r * rank + k] = s * scale;
+  if (lane == 0) red[warp] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kLdThreads / 32; ++w) t += red[w];
+    m.xa[mi][(size_t)r * rank + k] = t * scale;
+  }
 }
 
 // Rotate-half RoPE on fp32 rows x [rows, heads, d] at positions pos[r], angle in fp64.
@@ -491,19 +538,60 @@ cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv
   return cudaGetLastError();
 }
 
-cudaError_t launch_gemv(const GemvDesc& d, cudaStream_t stream) {
-  if (d.rows == 0 || d.out_dim == 0) return cudaSuccess;
-  if (d.in_dim % 8 != 0) return cudaErrorInvalidValue;
-  dim3 grid(cdiv(d.out_dim, kGemvWarps), cdiv(d.rows, kGemvMaxRows));
-  gemv_kernel<<<grid, kGemvWarps * 32, 0, stream>>>(d);
+template <int OPW>
+cudaError_t gemv_dispatch(const GemvLaunch& L, int blocks, cudaStream_t stream) {
+  if (L.d.rows == 1)
+    gemv_kernel<OPW, 1><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
+  else if (L.d.rows == 2)
+    gemv_kernel<OPW, 2><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
+  else if (L.d.rows <= 4)
+    gemv_kernel<OPW, 4><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
+  else
+    gemv_kernel<OPW, 8><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
   return cudaGetLastError();
 }
 
-cudaError_t launch_lora_down_rows(const __nv_bfloat16* A, int rank, int in_dim, const float* x,
-                                  int rows, float scale, float* xa, cudaStream_t stream) {
-  const int warps = rows * rank;
-  if (warps == 0) return cudaSuccess;
-  lora_down_rows_kernel<<<cdiv(warps, 8), 256, 0, stream>>>(A, rank, in_dim, x, rows, scale, xa);
+cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream) {
+  if (d.rows < 1 || d.rows > kGemvMaxRows || d.nseg < 1 || d.nseg > 3 || d.in_dim % 8 != 0)
+    return cudaErrorInvalidValue;
+  GemvLaunch L;
+  L.d = d;
+  int total_out = 0;
+  for (int s = 0; s < d.nseg; ++s) total_out += d.seg[s].out_dim;
+  if (total_out == 0) return cudaSuccess;
+  // outputs per warp: reuse x across weight rows when there are many outputs
+  L.opw = total_out >= 65536 ? 4 : total_out >= 16384 ? 2 : 1;
+  // split the input dimension until the warps cover the GPU (pieces of >= 256 inputs)
+  const int want_warps = 32 * num_sms;
+  L.ks = 1;
+  while (L.ks < kGemvWarps && (total_out / L.opw) * L.ks < want_warps &&
+         d.in_dim / (2 * L.ks) >= 256)
+    L.ks *= 2;
+  const int groups_per_block = kGemvWarps / L.ks;
+  int blocks = 0;
+  for (int s = 0; s < 3; ++s) {
+    L.block0[s] = blocks;
+    if (s < d.nseg) {
+      const int groups = (d.seg[s].out_dim + L.opw - 1) / L.opw;
+      blocks += (groups + groups_per_block - 1) / groups_per_block;
+    }
+  }
+  L.block0[3] = blocks;
+  switch (L.opw) {
+    case 4: return gemv_dispatch<4>(L, blocks, stream);
+    case 2: return gemv_dispatch<2>(L, blocks, stream);
+    default: return gemv_dispatch<1>(L, blocks, stream);
+  }
+}
+
+cudaError_t launch_lora_down_rows(const LoraDownRows& m, int rank, int in_dim, const float* x,
+                                  int rows, float scale, const __nv_bfloat16* norm_gain, float eps,
+                                  float* xn, cudaStream_t stream) {
+  const int blocks = m.n * rows * rank + (norm_gain ? rows : 0);
+  if (blocks == 0) return cudaSuccess;
+  if (in_dim % 8 != 0) return cudaErrorInvalidValue;
+  lora_down_rows_kernel<<<blocks, kLdThreads, 0, stream>>>(m, rank, in_dim, x, rows, scale,
+                                                           norm_gain, eps, xn);
   return cudaGetLastError();
 }
 
@@ -548,15 +636,20 @@ cudaError_t launch_gather_rows_f32(const __nv_bfloat16* src, const int64_t* row_
 }
 
 cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,
-                           float* logits, cudaStream_t stream) {
-  GemvDesc d{};
-  d.W = W;
-  d.out_dim = vocab;
-  d.in_dim = hidden;
-  d.x = h;
-  d.rows = rows;
-  d.y = logits;
-  return launch_gemv(d, stream);
+                           float* logits, int num_sms, cudaStream_t stream) {
+  for (int r0 = 0; r0 < rows; r0 += kGemvMaxRows) {
+    GemvDesc d{};
+    d.seg[0].W = W;
+    d.seg[0].out_dim = vocab;
+    d.seg[0].y = logits + (size_t)r0 * vocab;
+    d.nseg = 1;
+    d.in_dim = hidden;
+    d.x = h + (size_t)r0 * hidden;
+    d.rows = rows - r0 < kGemvMaxRows ? rows - r0 : kGemvMaxRows;
+    cudaError_t e = launch_gemv(d, num_sms, stream);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab, float* out,
