@@ -38,6 +38,10 @@ if ROOT not in sys.path:
 METRIC = "recomputed layer*tokens/s"
 UNIT = "layer*tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu --set full
+# capture of the kernel as it now stands, at the full launch size of the 7B-shape 16K workload
+# (profiles/gemm_gateup_swiglu_7b16k.md). An entry is removed whenever its kernel changes.
+NCU_TRAFFIC_BYTES = {"gemm_gateup_swiglu": 2.531287e9 + 0.611022e9}
 
 
 def load_peaks():
@@ -106,6 +110,23 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": float(rows[0][2]) if rows[0][2].replace(".", "").isdigit() else None,
                 "samples": len(rows), "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------- ranks
+def max_over_ranks(x: float, device="cpu") -> float:
+    """The largest value of x over all ranks (x itself without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: float, steps: int, world: int, max_ms: float) -> float:
+    """Whole-job rate: every rank's units over the slowest rank's time."""
+    return world * units_per_rank * steps / (max_ms / 1000.0)
 
 
 # ----------------------------------------------------------------------------- workload
@@ -400,12 +421,9 @@ def main():
     ctx.profile_enable(False)
     clk = clocks.stop()
     ctx.check()
-    if world > 1:
-        tt = torch.tensor([elapsed_ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(tt.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, device)
     ms_step = elapsed_ms / args.steps
-    value = world * units * args.steps / (elapsed_ms / 1000.0)
+    value = job_throughput(units, args.steps, world, elapsed_ms)
 
     # ---------------- end to end: restart state from pinned host memory, KL back to host
     h_host = st["ckpt"][s - 1].to("cpu").pin_memory() if s > 0 else None
@@ -429,13 +447,9 @@ def main():
         e2e_step()
     b.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = a.elapsed_time(b)
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e_ms = max_over_ranks(a.elapsed_time(b), device)
     h2d = (st["ckpt"][s - 1].numel() * 2 if s > 0 else 0)
-    e2e = {"value": world * units * args.steps / (e2e_ms / 1000.0), "unit": UNIT,
+    e2e = {"value": job_throughput(units, args.steps, world, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4,
            "ms_per_step": e2e_ms / args.steps, "kl_first_step": float(kl_host.item())}
 
@@ -465,7 +479,8 @@ def main():
     launches_dom = kernels[dom]["launches"]
     roofline = {"kernel": dom, "bound": "tensor", "achieved": kernels[dom]["tflops"],
                 "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                "frac": kernels[dom]["frac"], "traffic": None,
+                "frac": kernels[dom]["frac"],
+                "traffic": NCU_TRAFFIC_BYTES.get(dom) if wl.model.hidden == 3584 and n == 16384 else None,
                 "peak_source": f"bf16_tflops ({peak_src}, burst)",
                 "frac_of_sustained": round(kernels[dom]["tflops"] / peaks.get("bf16_tflops_sustained", 1700.0), 4),
                 "algorithmic_flops_per_launch": flops_layer[dom],

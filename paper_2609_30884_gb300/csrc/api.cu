@@ -202,7 +202,7 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_q = take(M * D.qd * 2);
   p.off_o = take(M * D.qd * 2);
   p.off_mlp = take(M * D.f * 2);
-  p.off_xa = take(M * 64 * 2);
+  p.off_xa = take(M * kXaCols * 2);
   p.off_rope = take(static_cast<size_t>(p.max_n) * (D.d / 2) * sizeof(float2));
   p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
   p.splits = dec_splits(p.max_n);
@@ -277,7 +277,7 @@ cudaError_t lora_down(const LayerCtx& c, int l, const void* X, int M, int K, con
   g.epi = kEpiScaleBf16;
   g.scale = c.scale;
   g.out = XA;
-  g.ldo = 64;
+  g.ldo = kXaCols;
   g.status = c.ctx->status_dev;
   return launch_gemm(g, nm * kRankPad, c.ctx->num_sms, c.st);
 }
@@ -333,7 +333,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
       g.bias[m] = D.bias ? w.bias[m] : nullptr;
     }
     g.XA = XA;
-    g.ldxa = 64;
+    g.ldxa = kXaCols;
     g.rank = rank;
     g.epi = kEpiQkv;
     g.rope = rope;
@@ -392,7 +392,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.group_cols[0] = D.h;
     if (lo) {
       g.XA = XA;
-      g.ldxa = 64;
+      g.ldxa = kXaCols;
       g.BL[0] = c.ad->B[l * 7 + m];
       g.rank = rank;
       g.lora_on[0][0] = 1;
@@ -444,7 +444,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     }
     g.group_cols[0] = D.f;
     g.XA = XA;
-    g.ldxa = 64;
+    g.ldxa = kXaCols;
     g.rank = rank;
     g.epi = kEpiSwiGLU;
     g.out = MLP;

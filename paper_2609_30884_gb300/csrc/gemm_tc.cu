@@ -164,8 +164,13 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
       if (!row_ok || col >= ncols) continue;
       const int n = min(16, ncols - col);
       if (a.epi == kEpiScaleBf16) {
+        // hi = bf16(v), lo = bf16(v - hi): the pair carries the product to ~16 mantissa bits
 #pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r0[j]) * a.scale;
+        for (int j = 0; j < 16; ++j) {
+          v[j] = __uint_as_float(r0[j]) * a.scale;
+          w[j] = v[j] - __bfloat162float(__float2bfloat16_rn(v[j]));
+        }
+        store_bf16_n(a.out + (size_t)row * a.ldo + kXaLoCol + col, w, n);
       } else {
         if (n >= 16) {
           load16_bf16(a.resid + (size_t)row * a.ld_resid + col, w);
@@ -340,14 +345,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           } else {
             // Extension block: per adapted segment s, the XA slice [128 x 16] of that
             // module (A slot + s * 4 KB) and the B-factor rows of the tile (B slot).
+            // A slot: [hi | lo] slices of 4 KB per adapted segment (at most 2 segments here)
             uint32_t bytes = 0;
             for (int s = 0; s < a.nseg; ++s)
-              if (a.lora_on[tl.g][s]) bytes += BM * kRankPad * 2 + seg_rows * kRankPad * 2;
+              if (a.lora_on[tl.g][s]) bytes += 2 * BM * kRankPad * 2 + seg_rows * kRankPad * 2;
             mbar_arrive_expect_tx(&full_bar[stage], bytes);
             for (int s = 0; s < a.nseg; ++s) {
               if (!a.lora_on[tl.g][s]) continue;
-              tma_load_2d(sa + s * BM * kRankPad * 2, &a.tmXA, &full_bar[stage],
+              tma_load_2d(sa + (2 * s) * BM * kRankPad * 2, &a.tmXA, &full_bar[stage],
                           a.xa_col[tl.g][s], m0);
+              tma_load_2d(sa + (2 * s + 1) * BM * kRankPad * 2, &a.tmXA, &full_bar[stage],
+                          a.xa_col[tl.g][s] + kXaLoCol, m0);
               tma_load_2d(sb + s * seg_rows * kRankPad * 2, &a.tmBL[tl.g + s], &full_bar[stage], 0,
                           tl.n_loc * seg_rows);
             }
@@ -409,9 +417,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint32_t idesc_seg = idesc_bf16_f32(BM, seg_rows);
             for (int s = 0; s < a.nseg; ++s) {
               if (!a.lora_on[tl.g][s]) continue;
-              const uint64_t ad = smem_desc(sa + s * BM * kRankPad * 2, 16, 256, kSwizzle32B);
               const uint64_t bd = smem_desc(sb + s * seg_rows * kRankPad * 2, 16, 256, kSwizzle32B);
-              mma_bf16_ss(d_tmem + s * seg_rows, ad, bd, idesc_seg, 1u);
+#pragma unroll
+              for (int h = 0; h < 2; ++h) {
+                const uint64_t ad =
+                    smem_desc(sa + (2 * s + h) * BM * kRankPad * 2, 16, 256, kSwizzle32B);
+                mma_bf16_ss(d_tmem + s * seg_rows, ad, bd, idesc_seg, 1u);
+              }
             }
           }
           issued = true;
@@ -526,6 +538,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
   bool any_lora = false;
   for (int g = 0; g < 3; ++g)
     for (int s = 0; s < 3; ++s) any_lora |= d.lora_on[g][s] != 0;
+  if (any_lora && d.nseg > 2) return cudaErrorInvalidValue;  // A slot holds 2 hi/lo pairs
   if (any_lora) {
     if (!make_map(&a.tmXA, d.XA, d.M, d.ldxa, d.ldxa, BM, kRankPad, CU_TENSOR_MAP_SWIZZLE_32B))
       return cudaErrorInvalidValue;

@@ -12,6 +12,10 @@ namespace crf {
 constexpr int kMaxReq = 32;   // equals CRF_MAX_REQUESTS
 constexpr int kPage = 16;
 constexpr int kRankPad = 16;  // LoRA rank padded to one K=16 MMA step
+// The scaled LoRA down product is kept as a bf16 pair hi + lo (lo = bf16(v - hi)); the lo
+// half of module slot j sits kXaLoCol columns after its hi half in the [rows, kXaCols] buffer.
+constexpr int kXaLoCol = 64;
+constexpr int kXaCols = 128;
 
 // Rows of a batched activation matrix that belong to each request.
 struct ReqTable {
@@ -22,7 +26,7 @@ struct ReqTable {
 };
 
 enum EpiKind : int {
-  kEpiScaleBf16 = 0,  // out = bf16(acc * scale)                        (LoRA down product)
+  kEpiScaleBf16 = 0,  // out = hi/lo bf16 pair of acc * scale            (LoRA down product)
   kEpiQkv = 1,        // +bias, RoPE(q,k); q -> qbuf, k/v -> KV pages    (Eq. S3)
   kEpiResid = 2,      // out = bf16(resid + acc)                         (o / down projection)
   kEpiSwiGLU = 3      // out = bf16(silu(gate) * up), tile = [gate | up]  (MLP)
@@ -40,7 +44,7 @@ struct GemmDesc {
   int B_rows[3];          // rows of each B matrix
   int ldb[3];
   int group_cols[3];      // valid output columns per group (plain) / per segment (stacked)
-  // LoRA extension: D += XA[:, xa_col] * BL^T (K = 16); XA already scaled by alpha/r
+  // LoRA extension: D += (XA_hi + XA_lo)[:, xa_col] * BL^T (two K = 16 steps); XA scaled by alpha/r
   const void* XA;
   int ldxa;
   const void* BL[3];

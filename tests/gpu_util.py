@@ -5,7 +5,7 @@ import numpy as np
 import torch
 
 import synth
-from oracle import build as obuild, cache as C
+from oracle import build as obuild, cache as C, decoder as Dec
 from oracle.decoder import LayerAdapter
 
 # Tolerances stated for the recomputation path (bf16 compute, fp32 accumulate):
@@ -76,3 +76,53 @@ def free_slots(t: torch.Tensor, free: np.ndarray) -> torch.Tensor:
     """Entries of a pool layer [P, Hkv, 16, d] at the (page, slot) pairs where ``free`` is True."""
     m = torch.from_numpy(free).to(t.device)
     return t.permute(0, 2, 1, 3)[m]
+
+
+def bf16_round(a) -> np.ndarray:
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).bfloat16().float().numpy()
+
+
+def bf16_execution_recover(om, oa, pool, req, s, e, restart):
+    """The window recovery executed the way a bf16 tensor pipeline runs it.
+
+    The paper computes in bfloat16 throughout (Section 5.1): every op's output tensor is bf16
+    while arithmetic inside an op accumulates in fp32. This runs the oracle's steps that way
+    (projections, LoRA factors, RoPE outputs, attention output, residual sums, norms, the MLP
+    activation and the cache K/V all rounded to bf16 as they are produced); the last row then
+    continues through the tail in fp32, as the decode path does. Its distance from the plain fp32
+    oracle measures how strongly the problem at hand amplifies bf16 rounding (large when deep-layer
+    adapters dominate and attention is near one-hot). Returns (per-layer K, V, H dicts, final row).
+    """
+    R = bf16_round
+    dims = om.dims
+    n = req.n
+
+    def proj(xin, P, A, m, bias):
+        y = xin @ P.W[m].T
+        if bias and m in P.bias:
+            y = y + P.bias[m]
+        y = R(y)
+        if m in A.AB:
+            Am, Bm = A.AB[m]
+            y = R(y + R(A.scale * R(R(xin @ Am.T) @ Bm.T)))
+        return y
+
+    cos, sin = Dec.rope_angles(np.arange(n), dims.head_dim, dims.rope_theta)
+    x = R(restart)
+    ks, vs, hs = {}, {}, {}
+    for l in range(s, e):
+        P, A = om.layers[l], oa.layers[l]
+        xn = R(Dec.rmsnorm(x, P.ln1, dims.rms_eps))
+        q = proj(xn, P, A, "q", True).reshape(n, dims.n_q_heads, dims.head_dim)
+        k = proj(xn, P, A, "k", True).reshape(n, dims.n_kv_heads, dims.head_dim)
+        v = proj(xn, P, A, "v", True).reshape(n, dims.n_kv_heads, dims.head_dim)
+        q, k = R(Dec.apply_rope(q, cos, sin)), R(Dec.apply_rope(k, cos, sin))
+        o = R(Dec.causal_gqa_attention(q, k, v))
+        x1 = R(x + proj(o.reshape(n, -1), P, A, "o", False))
+        xn2 = R(Dec.rmsnorm(x1, P.ln2, dims.rms_eps))
+        mlp = R(R(Dec.silu(proj(xn2, P, A, "gate", False))) * proj(xn2, P, A, "up", False))
+        x = R(x1 + proj(mlp, P, A, "down", False))
+        pool.write(l, req.page_table, k, v)
+        ks[l], vs[l], hs[l] = k, v, x
+    final = C.tail_decode(om, oa, pool, req, e, x[-1])
+    return ks, vs, hs, final

@@ -1,0 +1,64 @@
+"""Host logic of bench.py: max-over-ranks timing and whole-job throughput on two gloo ranks (CPU)."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import bench
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        ms = 10.0 + 5.0 * rank                # the slower rank sets the job time
+        got = bench.max_over_ranks(ms)
+        out[rank] = got
+        out[world + rank] = bench.job_throughput(100.0, 4, world, got)
+    finally:
+        dist.destroy_process_group()
+
+
+def test_max_over_ranks_and_throughput_gloo():
+    world = 2
+    out = mp.get_context("spawn").Manager().list([0.0] * (2 * world))
+    mp.start_processes(_rank_main, args=(world, _free_port(), out), nprocs=world, join=True,
+                       start_method="spawn")
+    assert list(out[:world]) == [15.0, 15.0]
+    # 2 ranks x 100 units x 4 steps in 15 ms
+    assert out[world] == pytest.approx(2 * 100 * 4 / 0.015)
+    assert out[world] == out[world + 1]
+
+
+def test_single_process_defaults():
+    assert bench.max_over_ranks(3.5) == 3.5
+    assert bench.job_throughput(65536, 20, 1, 1000.0) == pytest.approx(65536 * 20)
+
+
+def test_reference_arm_nonzero_rank_does_no_work(monkeypatch):
+    monkeypatch.setenv("RANK", "1")
+    args = type("A", (), {"workload": "7b-16k-w4", "ref_rows": 8, "steps": 1, "warmup": 0,
+                          "gpus": 2})()
+    assert bench.run_reference(args) == 0
+
+
+def test_algorithmic_work_7b_matches_hand_count():
+    import synth
+    wl = synth.workload("7b-16k-w4")
+    flops, byts = bench.algorithmic_work(wl.model, wl.lora, 16384)
+    # base GEMMs: 2 * n * sum(in * out) over the seven projections
+    h, f, qd, kvd = 3584, 18944, 3584, 512
+    base = 2 * 16384 * (h * (qd + 2 * kvd) + qd * h + 2 * h * f + f * h)
+    gemm = sum(v for k, v in flops.items() if k.startswith("gemm_") and k != "gemm_lora_down")
+    lora_up = 2 * 16384 * 16 * (qd + 2 * kvd + h + 2 * f + h)
+    assert gemm == base + lora_up
+    assert flops["attn_prefill_paged"] == 4 * 28 * 128 * 16384 * 16385 // 2
