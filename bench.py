@@ -149,64 +149,120 @@ def algorithmic_work(cfg, lc, n):
     return flops, byts
 
 
-def build_state(wl, device, ctx):
+def shard_requests(loads, world):
+    """Split independent requests over ranks (longest first onto the least-loaded rank).
+
+    Returns one list of request indices per rank; with a single request every rank gets it
+    (independent replicas).
+    """
+    if len(loads) == 1:
+        return [[0] for _ in range(world)]
+    order = sorted(range(len(loads)), key=lambda i: -loads[i])
+    bins = [[] for _ in range(world)]
+    tot = [0.0] * world
+    for i in order:
+        r = min(range(world), key=lambda k: (tot[k], k))
+        bins[r].append(i)
+        tot[r] += loads[i]
+    return [sorted(b) for b in bins]
+
+
+def build_state(wl, device, ctx, rank=0, world=1):
+    """Model, adapters, stale cache, checkpoints and the step's requests for this rank's share.
+
+    Every request's cache and checkpoints are built by a stale prefill under its own older
+    adapter version (current - gap); its fresh reference final row by a prefill under the
+    current version. Only the checkpoints the window reads or rewrites are kept.
+    """
     import torch
     import synth
     import paper_2609_30884_gb300 as crf
-    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed
+    from harness import DeviceAdapter, DeviceModel, make_pool, split_page_tables
 
     cfg, lc = wl.model, wl.lora
-    n = wl.n_tokens[0]
-    s, e = wl.windows[0]
     N = cfg.n_layers
-    st = {"cfg": cfg, "lc": lc, "n": n, "s": s, "e": e}
+    loads = [(e - s) * n for n, (s, e) in zip(wl.n_tokens, wl.windows)]
+    mine = shard_requests(loads, world)[rank]
+    ns = [wl.n_tokens[i] for i in mine]
+    wins = [wl.windows[i] for i in mine]
+    cur_v = wl.cur_version
+    stale_v = [cur_v - wl.stale_gap[i] for i in mine]
     dm = DeviceModel(cfg, device)
-    v_old = DeviceAdapter(cfg, lc, 0, device)
-    v_cur = DeviceAdapter(cfg, lc, 1, device)
-    P = pages_needed(n)
+    versions = {v: DeviceAdapter(cfg, lc, v, device) for v in sorted(set(stale_v) | {cur_v})}
+    v_cur = versions[cur_v]
+    P = sum((n + 15) // 16 for n in ns)
     pool = make_pool(cfg, P, device)
-    pt = synth.page_permutation(P, 1, device)
-    tokens = synth.token_ids(cfg, n, device=device)
-    ckpt = [torch.empty(n, cfg.hidden, dtype=torch.bfloat16, device=device) for _ in range(N)]
-    fresh_fin = torch.empty(cfg.hidden, dtype=torch.bfloat16, device=device)
-    full_req = crf.Request(pt, 0, N, tokens=tokens, hidden_out=ckpt, final_hidden_out=fresh_fin)
-    ws = ctx.workspace(dm.crf, v_cur.crf, [full_req])
-    # fresh reference (current adapter) on a scratch pool, then the stale cache (old adapter)
-    fresh_pool = make_pool(cfg, P, device)
-    ctx.recompute_window(dm.crf, v_cur.crf, fresh_pool,
-                         [crf.Request(pt, 0, N, tokens=tokens, final_hidden_out=fresh_fin)], ws)
-    torch.cuda.synchronize()
-    del fresh_pool
-    ctx.recompute_window(dm.crf, v_old.crf, pool, [crf.Request(pt, 0, N, tokens=tokens, hidden_out=ckpt)], ws)
+    pts = split_page_tables(ns, P, seed=1, device=device)
+    R = len(mine)
+    fin = torch.empty(R, cfg.hidden, dtype=torch.bfloat16, device=device)
+    fresh = torch.empty(R, cfg.hidden, dtype=torch.bfloat16, device=device)
+    # size the workspace for the largest of the set-up prefills and the batched step
+    prefills = [crf.Request(pts[k], 0, N, n_tokens=ns[k], final_hidden_out=fresh[k]) for k in range(R)]
+    step_reqs0 = [crf.Request(pts[k], wins[k][0], wins[k][1], n_tokens=ns[k], final_hidden_out=fin[k])
+                  for k in range(R)]
+    ws_bytes = max(ctx.workspace_size(dm.crf, v_cur.crf, [r]) for r in prefills)
+    ws_bytes = max(ws_bytes, ctx.workspace_size(dm.crf, v_cur.crf, step_reqs0))
+    ws = torch.empty(ws_bytes + 256, dtype=torch.uint8, device=device)
+    tokens, h_in, h_out, reqs = [], [], [], []
+    for k in range(R):
+        n, (s, e) = ns[k], wins[k]
+        tok = synth.token_ids(cfg, n, request=mine[k], device=device)
+        ctx.recompute_window(dm.crf, v_cur.crf, pool,
+                             [crf.Request(pts[k], 0, N, tokens=tok, final_hidden_out=fresh[k])], ws)
+        ck = [torch.empty(n, cfg.hidden, dtype=torch.bfloat16, device=device) for _ in range(N)]
+        ctx.recompute_window(dm.crf, versions[stale_v[k]].crf, pool,
+                             [crf.Request(pts[k], 0, N, tokens=tok, hidden_out=ck)], ws)
+        torch.cuda.synchronize()
+        tokens.append(tok)
+        h_in.append(ck[s - 1] if s > 0 else None)
+        h_out.append(ck[s:e])
+        reqs.append(crf.Request(pts[k], s, e, n_tokens=n, tokens=tok, hidden_in=h_in[k],
+                                hidden_out=h_out[k], final_hidden_out=fin[k]))
+        del ck
     ctx.check()
-    fin = torch.empty(cfg.hidden, dtype=torch.bfloat16, device=device)
-    h_in = ckpt[s - 1] if s > 0 else None
-    req = crf.Request(pt, s, e, n_tokens=n, tokens=tokens, hidden_in=h_in, hidden_out=ckpt[s:e],
-                      final_hidden_out=fin)
-    out_sq = torch.empty(N, 7, 2, dtype=torch.float32, device=device)
-    dws = ctx.drift_workspace(dm.crf.dims_c, v_cur.crf.dims_c)
-    out_kl = torch.empty(1, dtype=torch.float32, device=device)
-    kws = ctx.kl_workspace(1, cfg.vocab, cfg.hidden)
-    st.update(dm=dm, v_old=v_old, v_cur=v_cur, pool=pool, pt=pt, tokens=tokens, ckpt=ckpt,
-              fresh_fin=fresh_fin, fin=fin, req=req, ws=ws, out_sq=out_sq, dws=dws, out_kl=out_kl,
-              kws=kws, anchors=[v_old.crf] * N)
+    # each layer's anchor: the stale version of the first request whose window covers it
+    anchor_v = []
+    for l in range(N):
+        cover = [k for k in range(R) if wins[k][0] <= l < wins[k][1]]
+        anchor_v.append(stale_v[cover[0] if cover else 0])
+    st = {"cfg": cfg, "lc": lc, "mine": mine, "ns": ns, "wins": wins, "dm": dm,
+          "versions": versions, "v_cur": v_cur, "pool": pool, "pts": pts, "tokens": tokens,
+          "h_in": h_in, "h_out": h_out, "reqs": reqs, "ws": ws, "fin": fin, "fresh": fresh,
+          "anchors": [versions[v].crf for v in anchor_v],
+          "out_sq": torch.empty(N, 7, 2, dtype=torch.float32, device=device),
+          "dws": ctx.drift_workspace(dm.crf.dims_c, v_cur.crf.dims_c),
+          "out_kl": torch.empty(R, dtype=torch.float32, device=device),
+          "kws": ctx.kl_workspace(R, cfg.vocab, cfg.hidden),
+          "units": sum((e - s) * n for n, (s, e) in zip(ns, wins))}
     return st
 
 
 def run_step(ctx, st):
     ctx.drift(st["dm"].crf.dims_c, st["v_cur"].crf, st["anchors"], st["out_sq"], st["dws"])
-    ctx.recompute_window(st["dm"].crf, st["v_cur"].crf, st["pool"], [st["req"]], st["ws"])
-    ctx.kl(st["dm"].crf, st["fresh_fin"][None], st["fin"][None], st["out_kl"], st["cfg"].vocab,
-           st["kws"])
+    ctx.recompute_window(st["dm"].crf, st["v_cur"].crf, st["pool"], st["reqs"], st["ws"])
+    ctx.kl(st["dm"].crf, st["fresh"], st["fin"], st["out_kl"], st["cfg"].vocab, st["kws"])
 
 
 def time_refresh(ctx, st, s, e, reps=3):
     """ms of crf_recompute_window alone for window [s, e) (no tail decode)."""
     import torch
     import paper_2609_30884_gb300 as crf
-    n = st["n"]
-    req = crf.Request(st["pt"], s, e, n_tokens=n, tokens=st["tokens"],
-                      hidden_in=st["ckpt"][s - 1] if s > 0 else None, hidden_out=st["ckpt"][s:e])
+    n = st["ns"][0]
+    w0 = st["wins"][0]
+    # the window's restart state is the layer s-1 checkpoint; rewrite into scratch outputs
+    import torch as _t
+    if s == 0:
+        hin = None
+    elif s == w0[0]:
+        hin = st["h_in"][0]
+    elif w0[0] <= s - 1 < w0[1]:
+        hin = st["h_out"][0][s - 1 - w0[0]]
+    else:
+        return None
+    outs = [_t.empty(n, st["cfg"].hidden, dtype=_t.bfloat16, device=st["fin"].device)
+            for _ in range(e - s)]
+    req = crf.Request(st["pts"][0], s, e, n_tokens=n, tokens=st["tokens"][0], hidden_in=hin,
+                      hidden_out=outs)
     ctx.recompute_window(st["dm"].crf, st["v_cur"].crf, st["pool"], [req], st["ws"])
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -277,11 +333,17 @@ def run_reference(args):
 
 
 def config_of(wl):
-    s, e = wl.windows[0]
-    return {"workload": f"{args_workload_name(wl)}: {wl.name}", "prefix_tokens": wl.n_tokens[0],
-            "window": [s, e], "layers_recomputed": e - s, "n_layers": wl.model.n_layers,
-            "lora_rank": wl.lora.rank, "lora_modules": list(wl.lora.modules),
-            "page_tokens": 16, "l2": "inputs larger than L2 (1.9 GB of window weights per step)"}
+    cfg = {"workload": f"{args_workload_name(wl)}: {wl.name}", "n_layers": wl.model.n_layers,
+           "lora_rank": wl.lora.rank, "lora_modules": list(wl.lora.modules), "page_tokens": 16,
+           "l2": "inputs larger than L2 (window weights of >= 466 MB per layer per step)"}
+    if len(wl.n_tokens) == 1:
+        s, e = wl.windows[0]
+        cfg.update(prefix_tokens=wl.n_tokens[0], window=[s, e], layers_recomputed=e - s)
+    else:
+        cfg.update(requests=len(wl.n_tokens), prefix_tokens=list(wl.n_tokens),
+                   windows=[list(w) for w in wl.windows], stale_gaps=list(wl.stale_gap),
+                   layer_tokens=sum((e - s) * n for n, (s, e) in zip(wl.n_tokens, wl.windows)))
+    return cfg
 
 
 def args_workload_name(wl):
@@ -393,9 +455,9 @@ def main():
     wl = synth.workload(args.workload)
     cfg, lc = wl.model, wl.lora
     ctx = crf.Context(local)
-    st = build_state(wl, device, ctx)
-    n, s, e = st["n"], st["s"], st["e"]
-    units = (e - s) * n
+    st = build_state(wl, device, ctx, rank, world)
+    n, (s, e) = st["ns"][0], st["wins"][0]
+    units = st["units"]
 
     for _ in range(args.warmup):
         run_step(ctx, st)
@@ -426,13 +488,14 @@ def main():
     value = job_throughput(units, args.steps, world, elapsed_ms)
 
     # ---------------- end to end: restart state from pinned host memory, KL back to host
-    h_host = st["ckpt"][s - 1].to("cpu").pin_memory() if s > 0 else None
-    kl_host = torch.empty(1, dtype=torch.float32).pin_memory()
+    h_host = [h.to("cpu").pin_memory() if h is not None else None for h in st["h_in"]]
+    kl_host = torch.empty(st["out_kl"].numel(), dtype=torch.float32).pin_memory()
     stream = torch.cuda.current_stream()
 
     def e2e_step():
-        if h_host is not None:
-            st["ckpt"][s - 1].copy_(h_host, non_blocking=True)
+        for h_dev, hh in zip(st["h_in"], h_host):
+            if hh is not None:
+                h_dev.copy_(hh, non_blocking=True)
         run_step(ctx, st)
         kl_host.copy_(st["out_kl"], non_blocking=True)
 
@@ -448,15 +511,23 @@ def main():
     b.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(a.elapsed_time(b), device)
-    h2d = (st["ckpt"][s - 1].numel() * 2 if s > 0 else 0)
+    h2d = sum(h.numel() * 2 for h in st["h_in"] if h is not None)
     e2e = {"value": job_throughput(units, args.steps, world, e2e_ms), "unit": UNIT,
-           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4,
-           "ms_per_step": e2e_ms / args.steps, "kl_first_step": float(kl_host.item())}
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4 * kl_host.numel(),
+           "ms_per_step": e2e_ms / args.steps,
+           "kl_first_step": [round(float(v), 6) for v in kl_host.tolist()]}
 
     # ---------------- per-kernel roofline from the live events
     peaks, peak_src = load_peaks()
-    flops_layer, bytes_layer = algorithmic_work(cfg, lc, n)
-    layers_per_step = e - s
+    # algorithmic work of one step: per request, (e - s) layers over its own prefix length
+    flops_step, bytes_step = {}, {}
+    for n_i, (s_i, e_i) in zip(st["ns"], st["wins"]):
+        fl, by = algorithmic_work(cfg, lc, n_i)
+        for k, v in fl.items():
+            flops_step[k] = flops_step.get(k, 0) + v * (e_i - s_i)
+        for k, v in by.items():
+            bytes_step[k] = bytes_step.get(k, 0) + v * (e_i - s_i)
+    flops_layer, _ = algorithmic_work(cfg, lc, n)
     kernels = {}
     gpu_launches = 0
     for name, (ms, cnt) in prof.items():
@@ -465,17 +536,17 @@ def main():
         gpu_launches += cnt
         entry = {"launches": cnt, "ms_total": round(ms, 4),
                  "ms_per_step": round(ms / args.steps, 4)}
-        if name in flops_layer:
-            fl = flops_layer[name] * layers_per_step * args.steps
+        if name in flops_step:
+            fl = flops_step[name] * args.steps
             tf = fl / (ms / 1000.0) / 1e12
             entry.update(bound="tensor", tflops=round(tf, 1),
                          frac=round(tf / peaks["bf16_tflops"], 4))
-        if name in bytes_layer:
-            by = bytes_layer[name] * layers_per_step * args.steps
+        if name in bytes_step:
+            by = bytes_step[name] * args.steps
             gbs = by / (ms / 1000.0) / 1e9
             entry.update(bound="hbm", gbs=round(gbs, 1), frac=round(gbs / peaks["hbm_gbs"], 4))
         kernels[name] = entry
-    dom = max((k for k in kernels if k in flops_layer), key=lambda k: kernels[k]["ms_total"])
+    dom = max((k for k in kernels if k in flops_step), key=lambda k: kernels[k]["ms_total"])
     launches_dom = kernels[dom]["launches"]
     roofline = {"kernel": dom, "bound": "tensor", "achieved": kernels[dom]["tflops"],
                 "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
@@ -483,16 +554,16 @@ def main():
                 "traffic": NCU_TRAFFIC_BYTES.get(dom) if wl.model.hidden == 3584 and n == 16384 else None,
                 "peak_source": f"bf16_tflops ({peak_src}, burst)",
                 "frac_of_sustained": round(kernels[dom]["tflops"] / peaks.get("bf16_tflops_sustained", 1700.0), 4),
-                "algorithmic_flops_per_launch": flops_layer[dom],
+                "algorithmic_flops_per_launch": flops_step[dom] / max(1, kernels[dom]["launches"] // args.steps),
                 "launches": launches_dom}
-    gemm_names = [k for k in kernels if k.startswith("gemm_") and k in flops_layer]
-    gemm_fl = sum(flops_layer[k] for k in gemm_names) * layers_per_step * args.steps
+    gemm_names = [k for k in kernels if k.startswith("gemm_") and k in flops_step]
+    gemm_fl = sum(flops_step[k] for k in gemm_names) * args.steps
     gemm_ms = sum(kernels[k]["ms_total"] for k in gemm_names)
     gemm_tf = gemm_fl / (gemm_ms / 1000.0) / 1e12 if gemm_ms else 0.0
 
     # ---------------- window sweep (ms per 16K-prefix refresh)
     sweep = {}
-    if not args.no_sweep:
+    if not args.no_sweep and len(st["ns"]) == 1:
         for ln in (1, 2, 4):
             sweep[f"window_{ln}"] = round(time_refresh(ctx, st, s, min(s + ln, cfg.n_layers)), 3)
         sweep["full_prefill_28"] = round(time_refresh(ctx, st, 0, cfg.n_layers, reps=2), 3)
@@ -507,13 +578,15 @@ def main():
             "gemm_tflops_all": round(gemm_tf, 1),
             "gemm_frac_all": round(gemm_tf / peaks["bf16_tflops"], 4),
             "ms_per_refresh": sweep, "kernels": kernels,
-            "step": "drift(28x7) + recompute_window[14,18) + tail decode 18..27 + KL(first step)"}
+            "step": ("drift(N x 7) + crf_recompute_window over every request's window (rows of "
+                     "requests active at a layer batched) + tail decode of each last row through "
+                     "layers e..N-1 + first-step KL per request")}
 
     # ---------------- CPU oracle baseline (rank 0, one GPU only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         w = {k: v.to("cpu") for k, v in st["dm"].layers[s].items()}
         ad = {m: (a.to("cpu"), b.to("cpu")) for m, (a, b) in st["v_cur"].layers[s].items()}
-        x = st["ckpt"][s - 1][:args.cpu_rows].float().cpu().numpy() if s > 0 else None
+        x = st["h_in"][0][:args.cpu_rows].float().cpu().numpy() if s > 0 else None
         secs = cpu_oracle_sample(wl, args.cpu_rows, s, x, w, ad)
         line["cpu_baseline"] = {
             "value": args.cpu_rows / secs, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",

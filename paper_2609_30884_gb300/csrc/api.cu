@@ -206,10 +206,10 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_rope = take(static_cast<size_t>(p.max_n) * (D.d / 2) * sizeof(float2));
   p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
   p.splits = dec_splits(p.max_n);
-  // decode scratch, fp32: x, xn, x1, q, k, v, o, xa, gu, m, part
-  const size_t dec = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 3 * kRankPad + 3 * D.f) * 4 +
-                     static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
-  p.dec_bytes = align256(dec);
+  // decode scratch per row, fp32: x, xn, x1, q, k, v, o, xa (3 slots), gu, m, attention partials
+  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 3 * kRankPad + 3 * D.f) * 4 +
+                         static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
+  p.dec_bytes = align256(dec_row * std::max(1, p.dec_rows));
   p.off_dec = take(p.dec_rows ? p.dec_bytes : 0);
   p.total = o;
   return p;
@@ -459,71 +459,94 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
   return CRF_OK;
 }
 
-// ---------------------------------------------------------------- decode row
-// Carry one row (fp32) through layers [l0, N) at position `pos`, reading each
-// layer's cached K/V at positions < pos from the pages.
-crf_status decode_row(const LayerCtx& c, int l0, const __nv_bfloat16* start_row, int pos,
-                      const int32_t* page_table, void* out_bf16) {
+// ---------------------------------------------------------------- decode rows
+// Carry the last prefix row of every listed request through layers [e_i, N) against each
+// layer's cached K/V at positions < n_i - 1 (fp32 rows). Rows are ordered by window end, so
+// the rows active at a layer are a prefix of the batch and each layer's weights are read once
+// for all of them (GEMV launches of up to 8 rows).
+struct DecodeRow {
+  int e;            // first layer to run
+  int pos;          // position of the row (= n - 1)
+  const int32_t* page_table;
+  const __nv_bfloat16* start;  // bf16 [h]
+  void* out;        // bf16 [h]
+};
+
+crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
   const Dims& D = *c.D;
-  const bool ad_qkv = adapted(c.ad, 0) || adapted(c.ad, 1) || adapted(c.ad, 2);
-  const bool ad_gu = adapted(c.ad, CRF_MOD_GATE) || adapted(c.ad, CRF_MOD_UP);
-  (void)ad_qkv;
-  (void)ad_gu;
-  const int lora_launches = adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN);
-  // per layer: 2 norm + LoRA-down launches, other LoRA downs, 4 GEMVs, 1 RoPE, 2 attention,
-  // 1 SwiGLU; + 2 converts
-  ProfScope ps(c.ctx, kPDecode, c.st, (D.N - l0) * (10 + lora_launches) + 2);
   const Plan& p = *c.plan;
-  float* base = reinterpret_cast<float*>(c.ws + p.off_dec);
-  float* x = base;
-  float* xn = x + D.h;
-  float* x1 = xn + D.h;
-  float* q = x1 + D.h;  // q | k | v contiguous
-  float* k = q + D.qd;
-  float* v = k + D.kvd;
-  float* o = v + D.kvd;
-  float* xa = o + D.qd;  // three rank-padded slots
-  float* gu = xa + 3 * kRankPad;
-  float* m = gu + 2 * D.f;
-  float* part = m + D.f;
+  const int R = static_cast<int>(rows.size());
+  if (R == 0) return CRF_OK;
+  std::stable_sort(rows.begin(), rows.end(), [](const DecodeRow& a, const DecodeRow& b) { return a.e < b.e; });
+  const int l0 = rows[0].e;
+  const size_t Rs = static_cast<size_t>(R);
+  float* x = reinterpret_cast<float*>(c.ws + p.off_dec);
+  float* xn = x + Rs * D.h;
+  float* x1 = xn + Rs * D.h;
+  float* q = x1 + Rs * D.h;
+  float* k = q + Rs * D.qd;
+  float* v = k + Rs * D.kvd;
+  float* o = v + Rs * D.kvd;
+  float* xa = o + Rs * D.qd;  // three slots of [R, rank]
+  float* gu = xa + 3 * Rs * kRankPad;
+  float* m = gu + Rs * 2 * D.f;
+  float* part = m + Rs * D.f;
   const int rank = c.ad->dims.rank;
-  CRF_CUDA(launch_bf16_to_f32(start_row, x, D.h, c.st));
-  // segments [mods] sharing input `in`: LoRA down products of the adapted ones, then one GEMV
-  // norm_gain: normalise `raw` into `in` inside the LoRA-down launch (replaces the RMSNorm)
-  auto proj = [&](int l, const int* mods, int nm, const float* raw, const void* norm_gain, float* in,
-                  int in_dim, float* const* ys, const int* outs, const float* resid) -> cudaError_t {
+  // kernels per layer with up to 8 rows: 2 norm + LoRA-down launches, the o/down LoRA downs,
+  // 4 GEMVs, 2 RoPE, 2 attention, 1 SwiGLU; plus a conversion in and out per row
+  int launches = 2 * R;
+  for (int l = l0; l < D.N; ++l) {
+    int nr = 0;
+    for (const auto& r : rows) nr += r.e <= l;
+    launches += 9 + adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN) + 4 * ((nr + 7) / 8);
+  }
+  ProfScope ps(c.ctx, kPDecode, c.st, launches);
+  for (int i = 0; i < R; ++i)
+    CRF_CUDA(launch_bf16_to_f32(rows[i].start, x + i * static_cast<size_t>(D.h), D.h, c.st));
+  // segments [mods] sharing the fp32 rows `raw` (optionally RMS-normalised into `in` inside the
+  // LoRA-down launch), one GEMV per group of up to 8 rows
+  auto proj = [&](int l, int nr, const int* mods, int nm, const float* raw, const void* norm_gain,
+                  float* in, int in_dim, float* const* ys, const int* outs, const float* resid,
+                  int resid_ld) -> cudaError_t {
     if (!norm_gain) in = const_cast<float*>(raw);
     LoraDownRows ld{};
-    GemvDesc g{};
-    g.nseg = nm;
-    g.in_dim = in_dim;
-    g.x = in;
-    g.rows = 1;
-    g.rank = rank;
-    for (int s = 0; s < nm; ++s) {
-      const int mod = mods[s];
-      GemvSeg& sg = g.seg[s];
-      sg.W = static_cast<const __nv_bfloat16*>(c.model->layers[l].W[mod]);
-      sg.out_dim = outs[s];
-      sg.bias = (mod < 3 && D.bias) ? static_cast<const __nv_bfloat16*>(c.model->layers[l].bias[mod])
-                                    : nullptr;
-      sg.y = ys[s];
-      sg.resid = resid;
-      if (adapted(c.ad, mod)) {
-        sg.BL = static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + mod]);
-        sg.xa = xa + s * kRankPad;
-        ld.A[ld.n] = static_cast<const __nv_bfloat16*>(c.ad->A[l * 7 + mod]);
-        ld.xa[ld.n] = xa + s * kRankPad;
+    for (int s = 0; s < nm; ++s)
+      if (adapted(c.ad, mods[s])) {
+        ld.A[ld.n] = static_cast<const __nv_bfloat16*>(c.ad->A[l * 7 + mods[s]]);
+        ld.xa[ld.n] = xa + s * Rs * kRankPad;
         ++ld.n;
       }
-    }
     if (ld.n || norm_gain) {
-      cudaError_t e = launch_lora_down_rows(ld, rank, in_dim, raw, 1, c.scale,
+      cudaError_t e = launch_lora_down_rows(ld, rank, in_dim, raw, nr, c.scale,
                                             static_cast<const __nv_bfloat16*>(norm_gain), D.eps,
                                             in, c.st);
       if (e != cudaSuccess) return e;
     }
-    return launch_gemv(g, c.ctx->num_sms, c.st);
+    for (int r0 = 0; r0 < nr; r0 += 8) {
+      GemvDesc g{};
+      g.nseg = nm;
+      g.in_dim = in_dim;
+      g.x = in + static_cast<size_t>(r0) * in_dim;
+      g.rows = std::min(8, nr - r0);
+      g.rank = rank;
+      for (int s = 0; s < nm; ++s) {
+        const int mod = mods[s];
+        GemvSeg& sg = g.seg[s];
+        sg.W = static_cast<const __nv_bfloat16*>(c.model->layers[l].W[mod]);
+        sg.out_dim = outs[s];
+        sg.bias = (mod < 3 && D.bias) ? static_cast<const __nv_bfloat16*>(c.model->layers[l].bias[mod])
+                                      : nullptr;
+        sg.y = ys[s] + static_cast<size_t>(r0) * outs[s];
+        sg.resid = resid ? resid + static_cast<size_t>(r0) * resid_ld : nullptr;
+        if (adapted(c.ad, mod)) {
+          sg.BL = static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + mod]);
+          sg.xa = xa + s * Rs * kRankPad + static_cast<size_t>(r0) * rank;
+        }
+      }
+      cudaError_t e = launch_gemv(g, c.ctx->num_sms, c.st);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
   };
   const int m_qkv[3] = {CRF_MOD_Q, CRF_MOD_K, CRF_MOD_V};
   const int o_qkv[3] = {D.qd, D.kvd, D.kvd};
@@ -531,14 +554,18 @@ crf_status decode_row(const LayerCtx& c, int l0, const __nv_bfloat16* start_row,
   const int m_o[1] = {CRF_MOD_O}, o_o[1] = {D.h};
   float* const y_o[1] = {x1};
   const int m_gu[2] = {CRF_MOD_GATE, CRF_MOD_UP}, o_gu[2] = {D.f, D.f};
-  float* const y_gu[2] = {gu, gu + D.f};
+  float* const y_gu[2] = {gu, gu + Rs * D.f};
   const int m_d[1] = {CRF_MOD_DOWN}, o_d[1] = {D.h};
   float* const y_d[1] = {x};
+  RowPositions rp{};
+  for (int i = 0; i < R; ++i) rp.pos[i] = rows[i].pos;
   for (int l = l0; l < D.N; ++l) {
+    int nr = 0;
+    while (nr < R && rows[nr].e <= l) ++nr;
     const crf_layer_weights& w = c.model->layers[l];
-    CRF_CUDA(proj(l, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr));
-    // q and k heads are contiguous: one rotation launch
-    CRF_CUDA(launch_rope_rows(q, 1, D.hq + D.hkv, D.d, pos, D.theta, c.st));
+    CRF_CUDA(proj(l, nr, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr, 0));
+    CRF_CUDA(launch_rope_rows(q, nr, D.hq, D.d, rp, D.theta, c.st));
+    CRF_CUDA(launch_rope_rows(k, nr, D.hkv, D.d, rp, D.theta, c.st));
     DecodeAttnDesc a;
     std::memset(&a, 0, sizeof(a));
     a.q = q;
@@ -546,23 +573,27 @@ crf_status decode_row(const LayerCtx& c, int l0, const __nv_bfloat16* start_row,
     a.v_self = v;
     a.kpages = static_cast<const __nv_bfloat16*>(c.pool->k_pages[l]);
     a.vpages = static_cast<const __nv_bfloat16*>(c.pool->v_pages[l]);
-    a.page_table[0] = page_table;
-    a.pos[0] = pos;
+    for (int i = 0; i < nr; ++i) {
+      a.page_table[i] = rows[i].page_table;
+      a.pos[i] = rows[i].pos;
+    }
     a.out = o;
     a.part = part;
-    a.rows = 1;
+    a.rows = nr;
     a.n_q_heads = D.hq;
     a.n_kv_heads = D.hkv;
     a.head_dim = D.d;
     a.splits = p.splits;
-    a.max_pos = pos;
     CRF_CUDA(launch_decode_attention(a, c.st));
-    CRF_CUDA(proj(l, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x));
-    CRF_CUDA(proj(l, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr));
-    CRF_CUDA(launch_swiglu_f32(gu, m, 1, D.f, c.st));
-    CRF_CUDA(proj(l, m_d, 1, m, nullptr, nullptr, D.f, y_d, o_d, x1));
+    CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
+    CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
+    // gate rows then up rows: SwiGLU over [nr, f] with the up half Rs * f further on
+    CRF_CUDA(launch_swiglu_split_f32(gu, gu + Rs * D.f, m, nr * D.f, c.st));
+    CRF_CUDA(proj(l, nr, m_d, 1, m, nullptr, nullptr, D.f, y_d, o_d, x1, D.h));
   }
-  CRF_CUDA(launch_f32_to_bf16(x, static_cast<__nv_bfloat16*>(out_bf16), D.h, c.st));
+  for (int i = 0; i < R; ++i)
+    CRF_CUDA(launch_f32_to_bf16(x + i * static_cast<size_t>(D.h),
+                                static_cast<__nv_bfloat16*>(rows[i].out), D.h, c.st));
   return CRF_OK;
 }
 
@@ -827,17 +858,18 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
   }
 
   // first-step state: the last prefix row through layers e..N-1 on the historical cache
+  std::vector<DecodeRow> dec;
   for (int i = 0; i < n_req; ++i) {
     const crf_request& r = reqs[i];
     if (!r.final_hidden_out) continue;
-    const __nv_bfloat16* start = dx0 + static_cast<size_t>(i) * D.h;
+    __nv_bfloat16* start = dx0 + static_cast<size_t>(i) * D.h;
     if (r.s == r.e) {
       ProfScope ps(ctx, r.s == 0 ? kPEmbed : kPCopy, st, r.s == 0 ? 1 : 0);
       if (r.s == 0) {
         CRF_CUDA(launch_embed(static_cast<const __nv_bfloat16*>(model->embed), r.tokens + (r.n_tokens - 1),
-                              dx0 + static_cast<size_t>(i) * D.h, 1, D.h, st));
+                              start, 1, D.h, st));
       } else {
-        CRF_CUDA(cudaMemcpyAsync(dx0 + static_cast<size_t>(i) * D.h,
+        CRF_CUDA(cudaMemcpyAsync(start,
                                  static_cast<const __nv_bfloat16*>(r.hidden_in) +
                                      static_cast<size_t>(r.n_tokens - 1) * D.h,
                                  row_bytes, cudaMemcpyDeviceToDevice, st));
@@ -847,10 +879,11 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
       ProfScope ps(ctx, kPCopy, st, 0);
       CRF_CUDA(cudaMemcpyAsync(r.final_hidden_out, start, row_bytes, cudaMemcpyDeviceToDevice, st));
     } else {
-      s = decode_row(c, r.e, start, r.n_tokens - 1, r.page_table, r.final_hidden_out);
-      if (s != CRF_OK) return s;
+      dec.push_back({r.e, r.n_tokens - 1, r.page_table, start, r.final_hidden_out});
     }
   }
+  s = decode_rows(c, dec);
+  if (s != CRF_OK) return s;
   CRF_CUDA(cudaGetLastError());
   return CRF_OK;
 }

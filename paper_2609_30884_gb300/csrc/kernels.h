@@ -145,9 +145,15 @@ struct DecodeAttnDesc {
   int rows, n_q_heads, n_kv_heads, head_dim, splits, max_pos;
 };
 cudaError_t launch_decode_attention(const DecodeAttnDesc& d, cudaStream_t stream);
-cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, int pos,
+struct RowPositions {
+  int pos[kMaxReq];
+};
+// Rotate-half RoPE on fp32 rows x [rows, heads, head_dim], row r at position pos.pos[r].
+cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, const RowPositions& pos,
                              double theta, cudaStream_t stream);
 cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream);
+cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
+                                    cudaStream_t stream);
 cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream);
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStream_t stream);
 cudaError_t launch_gather_rows_f32(const __nv_bfloat16* src, const int64_t* row_index, float* dst,

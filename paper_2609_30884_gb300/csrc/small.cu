@@ -246,15 +246,16 @@ __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
   }
 }
 
-// Rotate-half RoPE on fp32 rows x [rows, heads, d] at positions pos[r], angle in fp64.
-__global__ void rope_rows_kernel(float* x, int rows, int heads, int d, int pos, double theta) {
+// Rotate-half RoPE on fp32 rows x [rows, heads, d], row r at position pos[r]; angle in fp64.
+__global__ void rope_rows_kernel(float* x, int rows, int heads, int d, const RowPositions pos,
+                                 double theta) {
   const int half = d / 2;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= rows * heads * half) return;
   const int i = idx % half;
   const int h = (idx / half) % heads;
   const int r = idx / (half * heads);
-  double turns = static_cast<double>(pos) * pow(theta, -2.0 * i / d) * 0.15915494309189535;
+  double turns = static_cast<double>(pos.pos[r]) * pow(theta, -2.0 * i / d) * 0.15915494309189535;
   turns -= floor(turns);
   float s, c;
   sincospif(static_cast<float>(2.0 * turns), &s, &c);
@@ -271,6 +272,12 @@ __global__ void swiglu_f32_kernel(const float* gu, float* m, int rows, int ffn) 
   const int r = idx / ffn, j = idx % ffn;
   const float g = gu[(size_t)r * 2 * ffn + j], u = gu[(size_t)r * 2 * ffn + ffn + j];
   m[idx] = g / (1.f + __expf(-g)) * u;
+}
+
+// m[i] = silu(g[i]) * u[i] over n elements (gate and up in separate buffers)
+__global__ void swiglu_split_f32_kernel(const float* g, const float* u, float* m, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) m[i] = g[i] / (1.f + __expf(-g[i])) * u[i];
 }
 
 __global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int n) {
@@ -602,7 +609,7 @@ cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y,
   return cudaGetLastError();
 }
 
-cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, int pos,
+cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, const RowPositions& pos,
                              double theta, cudaStream_t stream) {
   const int n = rows * heads * head_dim / 2;
   if (n == 0) return cudaSuccess;
@@ -614,6 +621,13 @@ cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cuda
   const int n = rows * ffn;
   if (n == 0) return cudaSuccess;
   swiglu_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(gu, m, rows, ffn);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
+                                    cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  swiglu_split_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(g, u, m, n);
   return cudaGetLastError();
 }
 

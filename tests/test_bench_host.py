@@ -62,3 +62,16 @@ def test_algorithmic_work_7b_matches_hand_count():
     lora_up = 2 * 16384 * 16 * (qd + 2 * kvd + h + 2 * f + h)
     assert gemm == base + lora_up
     assert flops["attn_prefill_paged"] == 4 * 28 * 128 * 16384 * 16385 // 2
+
+
+def test_shard_requests_partitions_and_balances():
+    import synth
+    wl = synth.workload("7b-batch8")
+    loads = [(e - s) * n for n, (s, e) in zip(wl.n_tokens, wl.windows)]
+    for world in (1, 2, 4, 8):
+        parts = bench.shard_requests(loads, world)
+        flat = sorted(i for p in parts for i in p)
+        assert flat == list(range(len(loads)))          # every request exactly once
+        tot = [sum(loads[i] for i in p) for p in parts]
+        assert max(tot) - min(tot) <= max(loads)        # greedy LPT balance bound
+    assert bench.shard_requests([7], 3) == [[0], [0], [0]]   # one prefix: replicas
