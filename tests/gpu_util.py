@@ -82,6 +82,39 @@ def bf16_round(a) -> np.ndarray:
     return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).bfloat16().float().numpy()
 
 
+def _bf16_proj(xin, P, A, m, bias):
+    """One adapted projection as a bf16 tensor pipeline runs it (op outputs rounded to bf16)."""
+    R = bf16_round
+    y = xin @ P.W[m].T
+    if bias and m in P.bias:
+        y = y + P.bias[m]
+    y = R(y)
+    if m in A.AB:
+        Am, Bm = A.AB[m]
+        y = R(y + R(A.scale * R(R(xin @ Am.T) @ Bm.T)))
+    return y
+
+
+def bf16_layer_rows(x, P, A, dims, rows):
+    """Layer output at `rows` (attention over all positions <= row) run as a bf16 tensor pipeline."""
+    R = bf16_round
+    n = x.shape[0]
+    x = R(x)
+    xn = R(Dec.rmsnorm(x, P.ln1, dims.rms_eps))
+    cos, sin = Dec.rope_angles(np.arange(n), dims.head_dim, dims.rope_theta)
+    q = R(Dec.apply_rope(_bf16_proj(xn, P, A, "q", True).reshape(n, dims.n_q_heads, dims.head_dim), cos, sin))
+    k = R(Dec.apply_rope(_bf16_proj(xn, P, A, "k", True).reshape(n, dims.n_kv_heads, dims.head_dim), cos, sin))
+    v = _bf16_proj(xn, P, A, "v", True).reshape(n, dims.n_kv_heads, dims.head_dim)
+    out = []
+    for t in rows:
+        o = R(Dec.single_query_attention(q[t], k[:t + 1], v[:t + 1])).reshape(1, -1)
+        x1 = R(x[t:t + 1] + _bf16_proj(o, P, A, "o", False))
+        xn2 = R(Dec.rmsnorm(x1, P.ln2, dims.rms_eps))
+        m = R(R(Dec.silu(_bf16_proj(xn2, P, A, "gate", False))) * _bf16_proj(xn2, P, A, "up", False))
+        out.append(R(x1 + _bf16_proj(m, P, A, "down", False))[0])
+    return np.stack(out)
+
+
 def bf16_execution_recover(om, oa, pool, req, s, e, restart):
     """The window recovery executed the way a bf16 tensor pipeline runs it.
 
@@ -96,16 +129,7 @@ def bf16_execution_recover(om, oa, pool, req, s, e, restart):
     R = bf16_round
     dims = om.dims
     n = req.n
-
-    def proj(xin, P, A, m, bias):
-        y = xin @ P.W[m].T
-        if bias and m in P.bias:
-            y = y + P.bias[m]
-        y = R(y)
-        if m in A.AB:
-            Am, Bm = A.AB[m]
-            y = R(y + R(A.scale * R(R(xin @ Am.T) @ Bm.T)))
-        return y
+    proj = _bf16_proj
 
     cos, sin = Dec.rope_angles(np.arange(n), dims.head_dim, dims.rope_theta)
     x = R(restart)
