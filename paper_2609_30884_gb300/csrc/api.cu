@@ -167,11 +167,22 @@ struct Plan {
   int max_n = 0;
   int dec_rows = 0;   // requests asking for the first-step state
   int splits = 1;
-  size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_rope;
+  size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_bx, off_rope;
   size_t off_dx0, off_dec;  // decode: bf16 starting rows, fp32 scratch
   size_t dec_bytes;
   size_t total;
 };
+
+// output rows of module m (q, k, v, o, gate, up, down) and their sum
+int module_rows(const Dims& D, int m) {
+  const int r[7] = {D.qd, D.kvd, D.kvd, D.h, D.f, D.f, D.h};
+  return r[m];
+}
+int module_rows_total(const Dims& D) {
+  int t = 0;
+  for (int m = 0; m < 7; ++m) t += module_rows(D, m);
+  return t;
+}
 
 // decode attention partials: one per 256-position chunk of the longest prefix
 int dec_splits(int max_n) { return std::max(1, (max_n + 255) / 256); }
@@ -203,6 +214,7 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_o = take(M * D.qd * 2);
   p.off_mlp = take(M * D.f * 2);
   p.off_xa = take(M * kXaCols * 2);
+  p.off_bx = take(static_cast<size_t>(module_rows_total(D)) * kBxCols * 2);
   p.off_rope = take(static_cast<size_t>(p.max_n) * (D.d / 2) * sizeof(float2));
   p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
   p.splits = dec_splits(p.max_n);
@@ -297,6 +309,29 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
   auto* rope = reinterpret_cast<const float2*>(ws + p.off_rope);
   const int rank = c.ad->dims.rank;
 
+  // BX = [B | B] rows of every module of layer l under its XA slot (up follows gate when both
+  // are adapted, so one K block carries the stacked gate|up pair)
+  __nv_bfloat16* BX[7];
+  {
+    auto* bx = reinterpret_cast<__nv_bfloat16*>(ws + p.off_bx);
+    BextDesc bd{};
+    bool any = false;
+    for (int m = 0; m < 7; ++m) {
+      BX[m] = bx;
+      bd.B[m] = adapted(c.ad, m) ? static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + m]) : nullptr;
+      bd.out[m] = bx;
+      bd.rows[m] = module_rows(D, m);
+      bd.col_off[m] = (m == CRF_MOD_UP && adapted(c.ad, CRF_MOD_GATE)) ? 32 : 0;
+      bx += static_cast<size_t>(bd.rows[m]) * kBxCols;
+      any |= adapted(c.ad, m);
+    }
+    bd.n = 7;
+    if (any) {
+      ProfScope ps(c.ctx, kPLoraDown, c.st);
+      CRF_CUDA(launch_lora_bext(bd, rank, c.st));
+    }
+  }
+
   // 1. RMSNorm before attention
   {
     ProfScope ps(c.ctx, kPNorm, c.st);
@@ -318,23 +353,22 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.ngroups = 3;
     g.nseg = 1;
     const int rows[3] = {D.qd, D.kvd, D.kvd};
-    int xa = 0;
+    int slot = 0;
     for (int m = 0; m < 3; ++m) {
       g.B[m] = w.W[m];
       g.B_rows[m] = rows[m];
       g.ldb[m] = D.h;
       g.group_cols[m] = rows[m];
       if (adapted(c.ad, m)) {
-        g.BL[m] = c.ad->B[l * 7 + m];
-        g.lora_on[m][0] = 1;
-        g.xa_col[m][0] = xa;
-        xa += kRankPad;
+        g.BX[m] = BX[m];
+        g.ext_on[m] = 1;
+        g.ext_steps[m] = 2;
+        g.xa_base[m] = 32 * slot++;
       }
       g.bias[m] = D.bias ? w.bias[m] : nullptr;
     }
     g.XA = XA;
     g.ldxa = kXaCols;
-    g.rank = rank;
     g.epi = kEpiQkv;
     g.rope = rope;
     g.head_dim = D.d;
@@ -393,10 +427,10 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     if (lo) {
       g.XA = XA;
       g.ldxa = kXaCols;
-      g.BL[0] = c.ad->B[l * 7 + m];
-      g.rank = rank;
-      g.lora_on[0][0] = 1;
-      g.xa_col[0][0] = 0;
+      g.BX[0] = BX[m];
+      g.ext_on[0] = 1;
+      g.ext_steps[0] = 2;
+      g.xa_base[0] = 0;
     }
     g.epi = kEpiResid;
     g.out = out;
@@ -429,23 +463,21 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.lda = D.h;
     g.ngroups = 1;
     g.nseg = 2;
-    int xa = 0;
     for (int s = 0; s < 2; ++s) {
       const int m = CRF_MOD_GATE + s;
       g.B[s] = w.W[m];
       g.B_rows[s] = D.f;
       g.ldb[s] = D.h;
-      if (adapted(c.ad, m)) {
-        g.BL[s] = c.ad->B[l * 7 + m];
-        g.lora_on[0][s] = 1;
-        g.xa_col[0][s] = xa;
-        xa += kRankPad;
-      }
+      g.BX[s] = BX[m];  // all-zero rows for a module without adapter
+    }
+    if (nm) {
+      g.ext_on[0] = 1;
+      g.ext_steps[0] = 2 * nm;
+      g.xa_base[0] = 0;
     }
     g.group_cols[0] = D.f;
     g.XA = XA;
     g.ldxa = kXaCols;
-    g.rank = rank;
     g.epi = kEpiSwiGLU;
     g.out = MLP;
     g.ldo = D.f;

@@ -1,23 +1,34 @@
 // Persistent tcgen05 GEMM for sm_103a with fused LoRA-up and fused epilogues.
 //
-//   D[128 x BN] = A[128 x K] * B[BN x K]^T  (+ XA[128 x 16] * BL[BN x 16]^T)
+//   D[BM*PAIR x BN] = A[BM*PAIR x K] * B[BN x K]^T  (+ XA[. x 64] * BX[BN x 64]^T)
 //
-// One CTA per SM; warp 0 issues TMA loads into a STAGES-deep shared-memory
-// ring, warp 1 allocates TMEM and issues tcgen05.mma from one thread into one
-// of two TMEM accumulators (so the epilogue of tile i overlaps the main loop of
-// tile i+1), warps 2..5 drain the accumulator (one TMEM lane = one output row
-// per thread) through the fused epilogue. Operands are bf16, K-major, staged
-// with 128-byte swizzle; accumulation is fp32 in TMEM.
+// PAIR = 2 (the projection GEMMs): a cluster of two CTAs on one TPC works on a
+// 256 x 256 tile with cta_group::2 MMAs. Each CTA stages its own 128 rows of A
+// and its own half of the B rows, so the operand bytes each SM pulls through L2
+// per FLOP are two thirds of the single-CTA 128 x 256 tile's. The even CTA
+// issues the MMAs; both CTAs hold 128 accumulator lanes in their own TMEM and
+// drain them through the same epilogue. PAIR = 1: one CTA per tile (the narrow
+// LoRA-down products).
+//
+// Per CTA: warp 0 issues TMA loads into a STAGES-deep shared-memory ring, warp 1
+// owns TMEM (two accumulators, so the epilogue of tile i overlaps the main loop
+// of tile i+1) and, in the MMA-issuing CTA, issues tcgen05.mma from one thread;
+// warps 2..5 drain the accumulator (one TMEM lane = one output row per thread)
+// through the fused epilogue. Operands are bf16, K-major, staged with 128-byte
+// swizzle; accumulation is fp32 in TMEM.
 //
 // The unmerged adapter term (alpha/r) (x A^T) B^T of every adapted projection
-// (Eq. S3 with W = W0 + (alpha/r) B A) enters as one extra K = 16 block per
-// tile: the rank-padded down product XA (computed by this same kernel with a
-// narrow tile, epilogue kEpiScaleBf16) against the B factor rows of the tile.
+// (Eq. S3 with W = W0 + (alpha/r) B A) enters as one extra 64-wide K block per
+// tile: A side = the scaled down product of the tile's rows stored as a bf16
+// pair [hi | lo] per module (16 + 16 columns), B side = rows of BX = [B | B]
+// placed under that module's columns (zeros elsewhere), so one K block serves
+// up to two stacked modules and the two halves of a pair alike.
 #include "common.cuh"
 #include "kernels.h"
 
 #include <algorithm>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 
 namespace crf {
@@ -33,13 +44,14 @@ struct GemmArgs {
   CUtensorMap tmA;
   CUtensorMap tmB[3];
   CUtensorMap tmXA;
-  CUtensorMap tmBL[3];
+  CUtensorMap tmBX[3];
   int M, K, num_kb;
   int ngroups, nseg;
   int group_tiles[3];
   int group_cols[3];
-  int lora_on[3][3];
-  int xa_col[3][3];
+  int ext_on[3];      // per group: tile has the LoRA K block
+  int ext_steps[3];   // per group: K = 16 steps of that block that carry data
+  int xa_base[3];     // per group: first XA column of that block
   int row_tiles, total_n, total_tiles;
   int epi;
   float scale;
@@ -79,10 +91,6 @@ __device__ __forceinline__ Tile decode_tile(int t, const GemmArgs& a) {
   r.g = g;
   r.n_loc = n;
   return r;
-}
-
-__device__ __forceinline__ bool group_has_lora(const GemmArgs& a, int g) {
-  return a.lora_on[g][0] | a.lora_on[g][1] | a.lora_on[g][2];
 }
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
@@ -147,8 +155,7 @@ __device__ __forceinline__ bool row_lookup(const ReqTable& rt, int row, int& pos
 
 template <int BN>
 __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl, uint32_t tacc,
-                                              int row_in_tile) {
-  const int row = tl.m_blk * BM + row_in_tile;
+                                              int row) {
   const bool row_ok = row < a.M;
   uint32_t r0[16], r1[16];
   float v[16], w[16];
@@ -164,13 +171,16 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
       if (!row_ok || col >= ncols) continue;
       const int n = min(16, ncols - col);
       if (a.epi == kEpiScaleBf16) {
-        // hi = bf16(v), lo = bf16(v - hi): the pair carries the product to ~16 mantissa bits
+        // hi = bf16(v), lo = bf16(v - hi): the pair carries the product to ~16 mantissa bits.
+        // Module slot j = col / 16 keeps hi at columns 32j.. and lo at 32j + 16..
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
           v[j] = __uint_as_float(r0[j]) * a.scale;
           w[j] = v[j] - __bfloat162float(__float2bfloat16_rn(v[j]));
         }
-        store_bf16_n(a.out + (size_t)row * a.ldo + kXaLoCol + col, w, n);
+        store_bf16_n(a.out + (size_t)row * a.ldo + 2 * col + 16, w, n);
+        store_bf16_n(a.out + (size_t)row * a.ldo + 2 * col, v, n);
+        continue;
       } else {
         if (n >= 16) {
           load16_bf16(a.resid + (size_t)row * a.ld_resid + col, w);
@@ -269,10 +279,11 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
   }
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, int PAIR>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
+  constexpr int CTA_ROWS = BN / PAIR;  // B rows staged by this CTA
   constexpr int A_BYTES = BM * BK * 2;
-  constexpr int B_BYTES = BN * BK * 2;
+  constexpr int B_BYTES = CTA_ROWS * BK * 2;
   constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   constexpr uint32_t TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128
                                                     : (2 * BN <= 256) ? 256 : 512;
@@ -289,6 +300,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR == 2 ? cluster_ctarank() : 0u;
+  const bool leader = rank == 0;
+  const int unit = blockIdx.x / PAIR;
+  const int n_units = gridDim.x / PAIR;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -297,7 +312,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);
-      mbar_init(&tempty_bar[i], 4);
+      mbar_init(&tempty_bar[i], 4 * PAIR);
     }
     mbar_init(&drain_bar, 1);
     abort_flag = 0;
@@ -308,27 +323,41 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     for (int i = 0; i < 3; ++i) tma_prefetch_desc(&a.tmB[i]);
   }
   if (warp == 1) {
-    tmem_alloc(&tmem_base_sh, TMEM_COLS);
-    tmem_relinquish();
+    if constexpr (PAIR == 2) {
+      tmem_alloc_pair(&tmem_base_sh, TMEM_COLS);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(&tmem_base_sh, TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if constexpr (PAIR == 2) cluster_sync(); else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = tmem_base_sh;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+    // ------------------------------------------------------------ TMA producer (every CTA)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       int armed_parity[STAGES];
       for (int s = 0; s < STAGES; ++s) armed_parity[s] = -1;
       bool ok = true;
-      for (int t = blockIdx.x; t < a.total_tiles && ok; t += gridDim.x) {
+      for (int t = unit; t < a.total_tiles && ok; t += n_units) {
         const Tile tl = decode_tile(t, a);
-        const int m0 = tl.m_blk * BM;
-        const int seg_rows = BN / a.nseg;
-        const int nkb = a.num_kb + (group_has_lora(a, tl.g) ? 1 : 0);
+        const int m0 = tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM;
+        const bool ext_tile = a.ext_on[tl.g] != 0;
+        const int nkb = a.num_kb + (ext_tile ? 1 : 0);
+        const int nseg = a.nseg;
+        const int seg_rows = BN / nseg;
+        const int per = nseg / PAIR;
+        // B rows of this CTA: the tile's CTA share (one segment) or its stacked segments
+        const int g0 = nseg == 1 ? tl.g : tl.g + static_cast<int>(rank) * per;
+        const int nb = nseg == 1 ? 1 : per;
+        const int yb = nseg == 1 ? tl.n_loc * BN + static_cast<int>(rank) * CTA_ROWS : tl.n_loc * seg_rows;
+        const int b_step = nseg == 1 ? 0 : seg_rows * BK * 2;
+        const int xa_ext = a.xa_base[tl.g];
         for (int kb = 0; kb < nkb; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1, &abort_flag, a.status)) {
             ok = false;
@@ -336,31 +365,24 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           }
           uint8_t* sa = smem + stage * STAGE_BYTES;
           uint8_t* sb = sa + A_BYTES;
-          if (kb < a.num_kb) {
-            mbar_arrive_expect_tx(&full_bar[stage], STAGE_BYTES);
-            tma_load_2d(sa, &a.tmA, &full_bar[stage], kb * BK, m0);
-            for (int s = 0; s < a.nseg; ++s)
-              tma_load_2d(sb + s * seg_rows * BK * 2, &a.tmB[tl.g + s], &full_bar[stage], kb * BK,
-                          tl.n_loc * seg_rows);
-          } else {
-            // Extension block: per adapted segment s, the XA slice [128 x 16] of that
-            // module (A slot + s * 4 KB) and the B-factor rows of the tile (B slot).
-            // A slot: [hi | lo] slices of 4 KB per adapted segment (at most 2 segments here)
-            uint32_t bytes = 0;
-            for (int s = 0; s < a.nseg; ++s)
-              if (a.lora_on[tl.g][s]) bytes += 2 * BM * kRankPad * 2 + seg_rows * kRankPad * 2;
-            mbar_arrive_expect_tx(&full_bar[stage], bytes);
-            for (int s = 0; s < a.nseg; ++s) {
-              if (!a.lora_on[tl.g][s]) continue;
-              tma_load_2d(sa + (2 * s) * BM * kRankPad * 2, &a.tmXA, &full_bar[stage],
-                          a.xa_col[tl.g][s], m0);
-              tma_load_2d(sa + (2 * s + 1) * BM * kRankPad * 2, &a.tmXA, &full_bar[stage],
-                          a.xa_col[tl.g][s] + kXaLoCol, m0);
-              tma_load_2d(sb + s * seg_rows * kRankPad * 2, &a.tmBL[tl.g + s], &full_bar[stage], 0,
-                          tl.n_loc * seg_rows);
-            }
+          // the MMA-issuing CTA's full barrier counts the bytes of both CTAs
+          if (leader) {
+            mbar_arrive_expect_tx(&full_bar[stage], PAIR * STAGE_BYTES);
+            armed_parity[stage] = phase;
           }
-          armed_parity[stage] = phase;
+          const bool ext = kb == a.num_kb;
+          const CUtensorMap* mA = ext ? &a.tmXA : &a.tmA;
+          const CUtensorMap* mB = ext ? &a.tmBX[g0] : &a.tmB[g0];
+          const int xa = ext ? xa_ext : kb * BK;
+          const int xb = ext ? 0 : kb * BK;
+          if constexpr (PAIR == 2) {
+            const uint32_t bar = mapa_shared(&full_bar[stage], 0);
+            tma_load_2d_pair(sa, mA, bar, xa, m0);
+            for (int j = 0; j < nb; ++j) tma_load_2d_pair(sb + j * b_step, mB + j, bar, xb, yb);
+          } else {
+            tma_load_2d(sa, mA, &full_bar[stage], xa, m0);
+            for (int j = 0; j < nb; ++j) tma_load_2d(sb + j * b_step, mB + j, &full_bar[stage], xb, yb);
+          }
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
@@ -368,86 +390,99 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
       }
       if (!ok) {
-        // Let every copy already issued land before the CTA can exit.
-        for (int s = 0; s < STAGES; ++s)
-          if (armed_parity[s] >= 0) {
-            volatile int never = 0;
-            mbar_wait(&full_bar[s], static_cast<uint32_t>(armed_parity[s]), &never, nullptr);
+        if (leader) {
+          // Let every copy already issued land before the CTA can exit.
+          for (int s = 0; s < STAGES; ++s)
+            if (armed_parity[s] >= 0) {
+              volatile int never = 0;
+              mbar_wait(&full_bar[s], static_cast<uint32_t>(armed_parity[s]), &never, nullptr);
+            }
+        } else {
+          // The peer's copies complete on the other CTA's barriers: give them time to land.
+          const unsigned long long t0 = globaltimer_ns();
+          while (globaltimer_ns() - t0 < 200000ull) {
           }
+        }
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // ------------------------------------------------------------ MMA issuer (even CTA)
+    if (lane == 0 && leader) {
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
       bool ok = true;
       bool issued = false;
-      const uint32_t idesc_main = idesc_bf16_f32(BM, BN);
-      for (int t = blockIdx.x; t < a.total_tiles && ok; t += gridDim.x, ++it) {
+      const uint32_t idesc = idesc_bf16_f32(BM * PAIR, BN);
+      for (int t = unit; t < a.total_tiles && ok; t += n_units, ++it) {
         const Tile tl = decode_tile(t, a);
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
-        if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1, &abort_flag, a.status)) {
+        if (!mbar_wait<PAIR == 2>(&tempty_bar[acc], acc_phase ^ 1, &abort_flag, a.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        const bool lora = group_has_lora(a, tl.g);
-        const int seg_rows = BN / a.nseg;
-        const int nkb = a.num_kb + (lora ? 1 : 0);
-        for (int kb = 0; kb < nkb; ++kb) {
+        const int ext_steps = a.ext_on[tl.g] ? a.ext_steps[tl.g] : 0;
+        auto mma = [&](uint64_t ad, uint64_t bd, uint32_t accum) {
+          if constexpr (PAIR == 2)
+            mma_bf16_ss_pair(d_tmem, ad, bd, idesc, accum);
+          else
+            mma_bf16_ss(d_tmem, ad, bd, idesc, accum);
+        };
+        auto release = [&]() {
+          if constexpr (PAIR == 2) mma_commit_pair(&empty_bar[stage], 0x3); else mma_commit(&empty_bar[stage]);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        };
+        for (int kb = 0; kb < a.num_kb; ++kb) {
           if (!mbar_wait(&full_bar[stage], phase, &abort_flag, a.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
-          const uint32_t sb = sa + A_BYTES;
-          if (kb < a.num_kb) {
+          const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
+          const uint64_t bd = smem_desc(sa + A_BYTES, 16, 1024, kSwizzle128B);
+          // K = 16 steps advance 32 bytes = 2 units of the descriptor's start-address field
 #pragma unroll
-            for (int k = 0; k < BK / 16; ++k) {
-              const uint64_t ad = smem_desc(sa + k * 32, 16, 1024, kSwizzle128B);
-              const uint64_t bd = smem_desc(sb + k * 32, 16, 1024, kSwizzle128B);
-              mma_bf16_ss(d_tmem, ad, bd, idesc_main, (kb > 0 || k > 0) ? 1u : 0u);
-            }
-          } else {
-            const uint32_t idesc_seg = idesc_bf16_f32(BM, seg_rows);
-            for (int s = 0; s < a.nseg; ++s) {
-              if (!a.lora_on[tl.g][s]) continue;
-              const uint64_t bd = smem_desc(sb + s * seg_rows * kRankPad * 2, 16, 256, kSwizzle32B);
-#pragma unroll
-              for (int h = 0; h < 2; ++h) {
-                const uint64_t ad =
-                    smem_desc(sa + (2 * s + h) * BM * kRankPad * 2, 16, 256, kSwizzle32B);
-                mma_bf16_ss(d_tmem + s * seg_rows, ad, bd, idesc_seg, 1u);
-              }
-            }
-          }
+          for (int k = 0; k < BK / 16; ++k) mma(ad + 2 * k, bd + 2 * k, (kb > 0 || k > 0) ? 1u : 0u);
           issued = true;
-          mma_commit(&empty_bar[stage]);
-          if (++stage == STAGES) {
-            stage = 0;
-            phase ^= 1;
+          release();
+        }
+        if (ok && ext_steps > 0) {
+          if (!mbar_wait(&full_bar[stage], phase, &abort_flag, a.status)) {
+            ok = false;
+          } else {
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+            const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
+            const uint64_t bd = smem_desc(sa + A_BYTES, 16, 1024, kSwizzle128B);
+            for (int k = 0; k < ext_steps; ++k) mma(ad + 2 * k, bd + 2 * k, 1u);
+            release();
           }
         }
         if (!ok) break;
-        mma_commit(&tfull_bar[acc]);
+        if constexpr (PAIR == 2) mma_commit_pair(&tfull_bar[acc], 0x3); else mma_commit(&tfull_bar[acc]);
       }
       if (!ok && issued) {
-        mma_commit(&drain_bar);
+        if constexpr (PAIR == 2) mma_commit_pair(&drain_bar, 0x1); else mma_commit(&drain_bar);
         volatile int never = 0;
         mbar_wait(&drain_bar, 0, &never, nullptr);
       }
     }
   } else {
-    // ------------------------------------------------------------ epilogue (warps 2..5)
+    // ------------------------------------------------------------ epilogue (warps 2..5, every CTA)
     const int quarter = warp & 3;  // TMEM lane quarter this warp may access
-    const int row_in_tile = quarter * 32 + lane;
+    const int row_in_cta = quarter * 32 + lane;
+    uint32_t tempty_addr[2];
+    for (int i = 0; i < 2; ++i)
+      tempty_addr[i] = PAIR == 2 ? mapa_shared(&tempty_bar[i], 0) : smem_u32(&tempty_bar[i]);
     int it = 0;
-    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x, ++it) {
+    for (int t = unit; t < a.total_tiles; t += n_units, ++it) {
       const Tile tl = decode_tile(t, a);
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
@@ -456,18 +491,20 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<BN>(a, tl, tacc, row_in_tile);
+      epilogue_tile<BN>(a, tl, tacc, tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM + row_in_cta);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+      if (lane == 0) {
+        if constexpr (PAIR == 2) mbar_arrive_cluster(tempty_addr[acc]); else mbar_arrive(&tempty_bar[acc]);
+      }
     }
   }
 
   tc_fence_before();
-  __syncthreads();
+  if constexpr (PAIR == 2) cluster_sync(); else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    if constexpr (PAIR == 2) tmem_dealloc_pair(tmem_base, TMEM_COLS); else tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -505,57 +542,109 @@ bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int ld, int 
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, int PAIR>
 cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) {
-  constexpr int smem = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024;
-  auto kern = gemm_tc_kernel<BN, STAGES>;
-  static bool attr_set = false;
-  if (!attr_set) {
+  constexpr int smem = STAGES * (BM * BK * 2 + (BN / PAIR) * BK * 2) + 1024;
+  auto kern = gemm_tc_kernel<BN, STAGES, PAIR>;
+  static int max_units = 0;
+  if (max_units == 0) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    if (PAIR == 2) {
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 2;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(num_sms);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = smem;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int clusters = 0;
+      e = cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg);
+      if (e != cudaSuccess) return e;
+      max_units = std::max(1, std::min(clusters, num_sms / 2));
+    } else {
+      max_units = num_sms;
+    }
   }
-  const int grid = std::max(1, std::min(num_sms, args.total_tiles));
-  kern<<<grid, kThreads, smem, stream>>>(args);
-  return cudaGetLastError();
+  const int units = std::max(1, std::min(max_units, args.total_tiles));
+  if (PAIR == 1) {
+    kern<<<units, kThreads, smem, stream>>>(args);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(2 * units);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args);
 }
 
 }  // namespace
 
+bool pair_mode_enabled() {
+  static int on = -1;
+  if (on < 0) {
+    const char* v = std::getenv("CRF_GEMM_PAIR");
+    on = (v && v[0] == '0') ? 0 : 1;
+  }
+  return on == 1;
+}
+
 cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream) {
   GemmArgs a;
   std::memset(&a, 0, sizeof(a));
-  const int seg_rows = bn / d.nseg;
+  const int pair = (bn == 256 && pair_mode_enabled() && (d.nseg == 1 || d.nseg == 2)) ? 2 : 1;
+  // rows of one B load: the CTA's share of the tile (plain) or one stacked segment
+  const int b_box = d.nseg == 1 ? bn / pair : bn / d.nseg;
   if (!make_map(&a.tmA, d.A, d.M, d.K, d.lda, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
   const int nmaps = d.ngroups + d.nseg - 1;
   for (int i = 0; i < 3; ++i) {
     const int src = i < nmaps ? i : 0;  // unused slots alias a valid map
-    if (!make_map(&a.tmB[i], d.B[src], d.B_rows[src], d.K, d.ldb[src], seg_rows, BK,
+    if (!make_map(&a.tmB[i], d.B[src], d.B_rows[src], d.K, d.ldb[src], b_box, BK,
                   CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
   }
-  bool any_lora = false;
-  for (int g = 0; g < 3; ++g)
-    for (int s = 0; s < 3; ++s) any_lora |= d.lora_on[g][s] != 0;
-  if (any_lora && d.nseg > 2) return cudaErrorInvalidValue;  // A slot holds 2 hi/lo pairs
-  if (any_lora) {
-    if (!make_map(&a.tmXA, d.XA, d.M, d.ldxa, d.ldxa, BM, kRankPad, CU_TENSOR_MAP_SWIZZLE_32B))
+  bool any_ext = false;
+  for (int g = 0; g < d.ngroups; ++g) any_ext |= d.ext_on[g] != 0;
+  if (any_ext) {
+    if (!d.XA || d.ldxa < kXaCols) return cudaErrorInvalidValue;
+    if (!make_map(&a.tmXA, d.XA, d.M, d.ldxa, d.ldxa, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
     for (int i = 0; i < 3; ++i) {
-      int src = -1;
-      if (i < nmaps && d.BL[i]) src = i;
+      int src = (i < nmaps && d.BX[i]) ? i : -1;
       if (src < 0)
         for (int j = 0; j < nmaps; ++j)
-          if (d.BL[j]) src = j;
+          if (d.BX[j]) src = j;
       if (src < 0) return cudaErrorInvalidValue;
-      if (!make_map(&a.tmBL[i], d.BL[src], d.B_rows[src], d.rank, d.rank, seg_rows, kRankPad,
-                    CU_TENSOR_MAP_SWIZZLE_32B))
+      if (!make_map(&a.tmBX[i], d.BX[src], d.B_rows[src], BK, BK, b_box, BK,
+                    CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
+    }
+    for (int g = 0; g < d.ngroups; ++g) {
+      if (!d.ext_on[g]) continue;
+      // the 64-wide block must lie inside the XA row, 16-byte aligned (TMA x coordinate)
+      if (d.xa_base[g] < 0 || d.xa_base[g] % 8 != 0 || d.xa_base[g] + BK > kXaCols ||
+          d.ext_steps[g] < 1 || d.ext_steps[g] > BK / 16)
+        return cudaErrorInvalidValue;
+      for (int s = 0; s < (d.ngroups == 1 ? d.nseg : 1); ++s)
+        if (!d.BX[g + s]) return cudaErrorInvalidValue;
     }
   } else {
     a.tmXA = a.tmA;
-    for (int i = 0; i < 3; ++i) a.tmBL[i] = a.tmB[i];
+    for (int i = 0; i < 3; ++i) a.tmBX[i] = a.tmB[i];
   }
   a.M = d.M;
   a.K = d.K;
@@ -564,19 +653,17 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
   a.nseg = d.nseg;
   a.total_n = 0;
   for (int g = 0; g < d.ngroups; ++g) {
-    const int cols_per_tile = (d.nseg > 1 && d.epi == kEpiSwiGLU) ? seg_rows : bn;
+    const int cols_per_tile = (d.nseg > 1 && d.epi == kEpiSwiGLU) ? bn / d.nseg : bn;
     a.group_cols[g] = d.group_cols[g];
     a.group_tiles[g] = (d.nseg > 1 && d.epi != kEpiSwiGLU) ? 1
                                                             : (d.group_cols[g] + cols_per_tile - 1) /
                                                                   cols_per_tile;
     a.total_n += a.group_tiles[g];
+    a.ext_on[g] = d.ext_on[g];
+    a.ext_steps[g] = d.ext_steps[g];
+    a.xa_base[g] = d.xa_base[g];
   }
-  for (int g = 0; g < 3; ++g)
-    for (int s = 0; s < 3; ++s) {
-      a.lora_on[g][s] = d.lora_on[g][s];
-      a.xa_col[g][s] = d.xa_col[g][s];
-    }
-  a.row_tiles = (d.M + BM - 1) / BM;
+  a.row_tiles = (d.M + BM * pair - 1) / (BM * pair);
   a.total_tiles = a.row_tiles * a.total_n;
   a.epi = d.epi;
   a.scale = d.scale;
@@ -595,12 +682,12 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
   a.req = d.req;
   a.status = d.status;
   if (a.total_tiles == 0) return cudaSuccess;
+  if (pair == 2) return launch_impl<256, 6, 2>(a, num_sms, stream);
   switch (bn) {
-    case 256: return launch_impl<256, 4>(a, num_sms, stream);
-    case 128: return launch_impl<128, 6>(a, num_sms, stream);
-    case 48: return launch_impl<48, 8>(a, num_sms, stream);
-    case 32: return launch_impl<32, 8>(a, num_sms, stream);
-    case 16: return launch_impl<16, 8>(a, num_sms, stream);
+    case 256: return launch_impl<256, 4, 1>(a, num_sms, stream);
+    case 48: return launch_impl<48, 8, 1>(a, num_sms, stream);
+    case 32: return launch_impl<32, 8, 1>(a, num_sms, stream);
+    case 16: return launch_impl<16, 8, 1>(a, num_sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -12,10 +12,11 @@ namespace crf {
 constexpr int kMaxReq = 32;   // equals CRF_MAX_REQUESTS
 constexpr int kPage = 16;
 constexpr int kRankPad = 16;  // LoRA rank padded to one K=16 MMA step
-// The scaled LoRA down product is kept as a bf16 pair hi + lo (lo = bf16(v - hi)); the lo
-// half of module slot j sits kXaLoCol columns after its hi half in the [rows, kXaCols] buffer.
-constexpr int kXaLoCol = 64;
+// The scaled LoRA down product is kept as a bf16 pair hi + lo (lo = bf16(v - hi)): module
+// slot j holds hi at columns [32j, 32j + 16) and lo at [32j + 16, 32j + 32) of a [rows, kXaCols]
+// buffer. The GEMM reads it as one 64-wide K block against BX = [B | B] rows (kBxCols wide).
 constexpr int kXaCols = 128;
+constexpr int kBxCols = 64;
 
 // Rows of a batched activation matrix that belong to each request.
 struct ReqTable {
@@ -44,13 +45,14 @@ struct GemmDesc {
   int B_rows[3];          // rows of each B matrix
   int ldb[3];
   int group_cols[3];      // valid output columns per group (plain) / per segment (stacked)
-  // LoRA extension: D += (XA_hi + XA_lo)[:, xa_col] * BL^T (two K = 16 steps); XA scaled by alpha/r
+  // LoRA extension (one extra K block): D += XA[:, xa_base[g] .. + 64] * BX^T, where XA holds the
+  // (alpha/r)-scaled down products as hi/lo pairs and BX [B_rows, 64] the matching B rows
   const void* XA;
   int ldxa;
-  const void* BL[3];
-  int rank;
-  int lora_on[3][3];
-  int xa_col[3][3];
+  const void* BX[3];      // map index g + s, like B
+  int ext_on[3];          // per group
+  int ext_steps[3];       // K = 16 steps of the block that carry data (2 per module)
+  int xa_base[3];
   // epilogue
   int epi;
   float scale;
@@ -69,8 +71,21 @@ struct GemmDesc {
   int* status;
 };
 
-// Launch the tcgen05 GEMM. bn: 256 or 128 for projections; 16/32/48 for LoRA down.
+// Launch the tcgen05 GEMM. bn: 256 for projections (CTA pairs with 256-row tiles unless the
+// environment sets CRF_GEMM_PAIR=0); 16/32/48 for LoRA down (single CTAs).
 cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream);
+
+// BX rows of up to 7 modules in one launch: out[m][r, :] = 0 except columns
+// [col_off[m], col_off[m] + 32) = [B_m[r, 0:16] | B_m[r, 0:16]] (rank padded with zeros); a null
+// B_m gives all-zero rows.
+struct BextDesc {
+  const __nv_bfloat16* B[7];
+  __nv_bfloat16* out[7];
+  int rows[7];
+  int col_off[7];
+  int n;
+};
+cudaError_t launch_lora_bext(const BextDesc& d, int rank, cudaStream_t stream);
 
 // ------------------------------------------------------------------ other kernels
 cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double theta,

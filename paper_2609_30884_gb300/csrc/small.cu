@@ -265,6 +265,30 @@ __global__ void rope_rows_kernel(float* x, int rows, int heads, int d, const Row
   base[i + half] = x2 * c + x1 * s;
 }
 
+// BX rows: one thread per (row, 8-column chunk) of module blockIdx.y.
+__global__ void lora_bext_kernel(const BextDesc d, int rank) {
+  const int m = blockIdx.y;
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= d.rows[m] * (kBxCols / 8)) return;
+  const int r = idx / (kBxCols / 8);
+  const int c0 = (idx % (kBxCols / 8)) * 8;
+  const __nv_bfloat16* B = d.B[m];
+  const int off = d.col_off[m];
+  uint32_t w[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    float v[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = c0 + 2 * j + h - off;
+      const int k = c & 15;
+      v[h] = (B && c >= 0 && c < 32 && k < rank) ? __bfloat162float(B[(size_t)r * rank + k]) : 0.f;
+    }
+    w[j] = pack_bf16(v[0], v[1]);
+  }
+  *reinterpret_cast<uint4*>(d.out[m] + (size_t)r * kBxCols + c0) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // gu [rows, 2, ffn] (gate then up) -> m [rows, ffn]
 __global__ void swiglu_f32_kernel(const float* gu, float* m, int rows, int ffn) {
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
@@ -614,6 +638,15 @@ cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, const 
   const int n = rows * heads * head_dim / 2;
   if (n == 0) return cudaSuccess;
   rope_rows_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, rows, heads, head_dim, pos, theta);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lora_bext(const BextDesc& d, int rank, cudaStream_t stream) {
+  int rows = 0;
+  for (int m = 0; m < d.n; ++m) rows = rows > d.rows[m] ? rows : d.rows[m];
+  if (d.n == 0 || rows == 0) return cudaSuccess;
+  if (rank < 1 || rank > kRankPad) return cudaErrorInvalidValue;
+  lora_bext_kernel<<<dim3(cdiv(rows * (kBxCols / 8), 256), d.n), 256, 0, stream>>>(d, rank);
   return cudaGetLastError();
 }
 
