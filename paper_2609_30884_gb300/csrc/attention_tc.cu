@@ -2,15 +2,17 @@
 // paged cache of the layer being recomputed.
 //
 // softmax(q k^T / sqrt(d) + causal mask) v over the whole prefix for every
-// query head; query head h reads kv head h / (Hq / Hkv). One CTA takes 128
-// query rows of two query heads that share a kv head (GQA), so every K/V tile
-// is fetched once for both. Warp roles:
+// query head; query head h reads kv head h / (Hq / Hkv). One CTA takes two
+// consecutive 128-row query tiles of one head (rows q0 .. q0+255): both read
+// the same K/V tiles except the last, which only the second tile needs, so
+// each K/V tile is fetched once for 256 query rows whatever the group size.
+// Warp roles:
 //   warp 0      TMA producer: the two Q tiles, then K and V tiles (8 pages of
 //               16 tokens each) into a 2-deep shared-memory ring
 //   warp 1      allocates TMEM and issues tcgen05.mma from one thread:
 //               S_t = Q_t K^T into TMEM, then O_t += P_t V with P_t read
 //               from TMEM (A operand) and V an MN-major shared operand
-//   warps 2-5   softmax of head 0, warps 6-9 softmax of head 1: one thread
+//   warps 2-5   softmax of query tile 0, warps 6-9 of query tile 1: one thread
 //               per query row; S from TMEM, online max / sum in fp32, P back
 //               into TMEM as bf16 over the S columns; O rescaled in TMEM only
 //               when the running max grows by more than 2^8
@@ -38,29 +40,26 @@ struct AttnTcArgs {
   CUtensorMap tmV;
   __nv_bfloat16* out;
   int ldo;
-  int n_q_heads, n_kv_heads, group, pairs;
+  int n_q_heads, n_kv_heads, group;
   int total_items;
   ReqTable req;
   int* status;
 };
 
 struct AttnWork {
-  int req, qt, g, h0, h1;
+  int req, qp, head, g;
 };
 
+// Items: (request, 256-row query pair, head), longest (latest) query pairs first.
 __device__ __forceinline__ bool attn_work(const AttnTcArgs& a, int idx, AttnWork& w) {
-  const int per_qt = a.n_kv_heads * a.pairs;
   for (int i = 0; i < a.req.n; ++i) {
-    const int nqt = (a.req.len[i] + kM - 1) / kM;
-    const int items = nqt * per_qt;
+    const int nqp = (a.req.len[i] + 2 * kM - 1) / (2 * kM);
+    const int items = nqp * a.n_q_heads;
     if (idx < items) {
       w.req = i;
-      w.qt = nqt - 1 - idx / per_qt;  // longest (latest) query tiles first
-      const int rem = idx % per_qt;
-      w.g = rem / a.pairs;
-      const int pp = rem % a.pairs;
-      w.h0 = w.g * a.group + 2 * pp;
-      w.h1 = (2 * pp + 1 < a.group) ? w.h0 + 1 : -1;
+      w.qp = nqp - 1 - idx / a.n_q_heads;
+      w.head = idx % a.n_q_heads;
+      w.g = w.head / a.group;
       return true;
     }
     idx -= items;
@@ -162,11 +161,12 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
   const int n = a.req.len[w.req];
   const int row0 = a.req.row0[w.req];
   const int32_t* pt = a.req.page_table[w.req];
-  const int q0 = w.qt * kM;
-  const int kv_end = min(q0 + kM, n);
-  const int J = (kv_end + kN - 1) / kN;
+  const int q0 = w.qp * 2 * kM;
+  const int ntiles = q0 + kM < n ? 2 : 1;
+  const int kv_end = min(q0 + ntiles * kM, n);
+  const int J = (kv_end + kN - 1) / kN;    // kv tiles of the last query tile
+  const int J0 = ntiles == 2 ? J - 1 : J;  // kv tiles of query tile 0 (its diagonal is tile J0-1)
   const int n_pages = (n + kPage - 1) / kPage;
-  const int ntiles = w.h1 >= 0 ? 2 : 1;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -200,12 +200,10 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
       bool ok = true;
       int armed_k[2] = {-1, -1}, armed_v[2] = {-1, -1};
       mbar_arrive_expect_tx(&q_full, ntiles * Q_BYTES);
-      for (int t = 0; t < ntiles; ++t) {
-        const int head = t == 0 ? w.h0 : w.h1;
+      for (int t = 0; t < ntiles; ++t)
         for (int h = 0; h < HALVES; ++h)
-          tma_load_2d(sQ + t * Q_BYTES + h * (kM * 128), &a.tmQ, &q_full, head * D + 64 * h,
-                      row0 + q0);
-      }
+          tma_load_2d(sQ + t * Q_BYTES + h * (kM * 128), &a.tmQ, &q_full, w.head * D + 64 * h,
+                      row0 + q0 + t * kM);
       for (int j = 0; j < J && ok; ++j) {
         const int st = j & 1;
         const uint32_t ph = (j >> 1) & 1;
@@ -241,8 +239,9 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     // Order: S0(0) S1(0) | PV0(j) S0(j+1) PV1(j) S1(j+1) | ... so that the softmax of one
-    // head overlaps the products of the other. tcgen05.mma of one thread execute in issue
-    // order, so S_t(j+1) overwrites the S/P columns only after PV_t(j) has read P_t(j).
+    // query tile overlaps the products of the other; query tile 0 stops one kv tile early
+    // (its diagonal), after which tile 1 runs alone. tcgen05.mma of one thread execute in
+    // issue order, so S_t(j+1) overwrites the S/P columns only after PV_t(j) has read P_t(j).
     if (lane == 0) {
       bool ok = mbar_wait(&q_full, 0, &abort_flag, a.status);
       bool issued = false;
@@ -275,7 +274,8 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
           break;
         }
         const uint32_t vb = smem_u32(sV + st * KV_BYTES);
-        for (int t = 0; t < ntiles && ok; ++t) {
+        bool k_ready = false;
+        for (int t = (j < J0 ? 0 : 1); t < ntiles && ok; ++t) {
           if (!mbar_wait(&p_full[t], j & 1, &abort_flag, a.status)) {
             ok = false;
             break;
@@ -288,13 +288,14 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
                         smem_desc(vb + kk * 2048, HALF_ROWS_BYTES, 1024, kSwizzle128B), idesc_o,
                         (j > 0 || kk > 0) ? 1u : 0u);
           }
-          if (more) {
-            if (t == 0) {
+          if (j + 1 < (t == 0 ? J0 : J)) {
+            if (!k_ready) {
               if (!mbar_wait(&k_full[nst], ((j + 1) >> 1) & 1, &abort_flag, a.status)) {
                 ok = false;
                 break;
               }
               tc_fence_after();
+              k_ready = true;
             }
             issue_s(t, nst);
           }
@@ -316,37 +317,38 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
     const int t = (warp - 2) >> 2;
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;  // query row within the tile (= TMEM lane)
-    const int head = t == 0 ? w.h0 : w.h1;
-    if (head >= 0) {
+    if (t < ntiles) {
       const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
       const uint32_t tS = tmem + lane_off + t * 128;
       const uint32_t tO = tmem + lane_off + 256 + t * 128;
       const float sl2 = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
-      const int qrow = q0 + r;
+      const int qrow = q0 + t * kM + r;
+      const int Jt = t == 0 ? J0 : J;
       float m_run = -INFINITY, l_run = 0.f;  // running max in raw score units
       bool ok = true;
-      for (int j = 0; j < J && ok; ++j) {
+      for (int j = 0; j < Jt && ok; ++j) {
         // warp-uniform outcome: the TMEM accesses below are warp-collective
         ok = __all_sync(0xffffffffu, mbar_wait(&s_full[t], j & 1, &abort_flag, a.status));
         if (!ok) break;
         tc_fence_after();
         const int k0 = j * kN;
-        const bool last = j == J - 1;
+        const bool last = j == Jt - 1;
         if (last) {
           // keys above min(query row, prefix end - 1) are masked on the diagonal tile
           softmax_tile<D, true>(tS, tO, j == 0, min(qrow, kv_end - 1) - k0, sl2, m_run, l_run);
         } else {
           softmax_tile<D, false>(tS, tO, j == 0, 0, sl2, m_run, l_run);
         }
-        if (last && t == 0 && kv_end - k0 < kN) {
-          // zero V rows past the prefix so that 0 * stale data cannot produce NaN
+        if (last && t == ntiles - 1 && kv_end - k0 < kN) {
+          // zero V rows past the prefix so that 0 * stale data cannot produce NaN (only the
+          // last query tile reads the last kv tile)
           const int st = j & 1;
           ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (j >> 1) & 1, &abort_flag, a.status));
           if (ok) {
             uint8_t* vt = sV + st * KV_BYTES;
             const int zr0 = kv_end - k0;
             const int chunks = (kN - zr0) * HALVES * 8;
-            for (int i = threadIdx.x - 64; i < chunks; i += 128) {
+            for (int i = threadIdx.x - 64 - 128 * t; i < chunks; i += 128) {
               const int rr = zr0 + i / (HALVES * 8);
               const int h = (i / 8) % HALVES;
               const int ch = i % 8;
@@ -365,7 +367,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
         tc_fence_after();
         const float inv = l_run > 0.f ? 1.0f / l_run : 0.f;
         const bool store = qrow < n;
-        __nv_bfloat16* dst = a.out + (size_t)(row0 + qrow) * a.ldo + head * D;
+        __nv_bfloat16* dst = a.out + (size_t)(row0 + qrow) * a.ldo + w.head * D;
         for (int c = 0; c < D / 32; ++c) {
           uint32_t o[32];
           tmem_ld32(tO + c * 32, o);
@@ -452,12 +454,11 @@ cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows
   a.n_q_heads = d.n_q_heads;
   a.n_kv_heads = d.n_kv_heads;
   a.group = d.n_q_heads / d.n_kv_heads;
-  a.pairs = (a.group + 1) / 2;
   a.req = d.req;
   a.status = d.status;
   a.total_items = 0;
   for (int i = 0; i < d.req.n; ++i)
-    a.total_items += ((d.req.len[i] + kM - 1) / kM) * d.n_kv_heads * a.pairs;
+    a.total_items += ((d.req.len[i] + 2 * kM - 1) / (2 * kM)) * d.n_q_heads;
   if (a.total_items == 0) return cudaSuccess;
   if (D == 128) return launch_tc<128>(a, stream);
   if (D == 64) return launch_tc<64>(a, stream);
