@@ -6,13 +6,16 @@
 // consecutive 128-row query tiles of one head (rows q0 .. q0+255): both read
 // the same K/V tiles except the last, which only the second tile needs, so
 // each K/V tile is fetched once for 256 query rows whatever the group size.
-// Warp roles:
-//   warp 0      TMA producer: the two Q tiles, then K and V tiles (8 pages of
-//               16 tokens each) into a 2-deep shared-memory ring
+// Warp roles (three warpgroups; setmaxnreg moves registers from the first to
+// the two softmax warpgroups):
+//   warp 0      TMA producer: the two Q tiles, then K0, V0, K1, V1, ... (8
+//               pages of 16 tokens each per tile) through one ring of kSlots
+//               shared-memory slots, so page gathers run two kv tiles ahead
 //   warp 1      allocates TMEM and issues tcgen05.mma from one thread:
 //               S_t = Q_t K^T into TMEM, then O_t += P_t V with P_t read
 //               from TMEM (A operand) and V an MN-major shared operand
-//   warps 2-5   softmax of query tile 0, warps 6-9 of query tile 1: one thread
+//   warps 2-3   idle
+//   warps 4-7   softmax of query tile 0, warps 8-11 of query tile 1: one thread
 //               per query row; S from TMEM, online max / sum in fp32, P back
 //               into TMEM as bf16 over the S columns; O rescaled in TMEM only
 //               when the running max grows by more than 2^8
@@ -31,7 +34,13 @@ namespace {
 constexpr int kM = 128;          // query rows per tile
 constexpr int kN = 128;          // keys per kv tile
 constexpr int kPagesPerTile = kN / kPage;
-constexpr int kThreadsAttn = 320;
+constexpr int kSlots = 5;        // K/V ring: slot of sequence item i = i % kSlots (K(j): 2j, V(j): 2j+1)
+constexpr int kThreadsAttn = 384;
+// setmaxnreg split: warpgroup 0 (producer, MMA) keeps kRegsCtl registers per thread, the
+// two softmax warpgroups take kRegsSoftmax; the sum must fit what the CTA launched with.
+constexpr int kRegsCtl = 56;
+constexpr int kRegsSoftmax = 208;
+constexpr int kRegsNeeded = 128 * kRegsCtl + 256 * kRegsSoftmax;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 struct AttnTcArgs {
@@ -78,26 +87,23 @@ __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, bool firs
 #pragma unroll
   for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
   tmem_ld_wait();
-  float mx0 = -INFINITY, mx1 = -INFINITY;
+  // eight independent max chains (one thread owns the whole row)
+  float mx[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
 #pragma unroll
   for (int c = 0; c < 4; ++c)
 #pragma unroll
-    for (int i = 0; i < 32; i += 2) {
-      float x0 = __uint_as_float(sr[c][i]), x1 = __uint_as_float(sr[c][i + 1]);
-      if (MASK) {
-        if (c * 32 + i > lim) {
-          x0 = -INFINITY;
-          sr[c][i] = __float_as_uint(x0);
-        }
-        if (c * 32 + i + 1 > lim) {
-          x1 = -INFINITY;
-          sr[c][i + 1] = __float_as_uint(x1);
-        }
+    for (int i = 0; i < 32; ++i) {
+      float x = __uint_as_float(sr[c][i]);
+      if (MASK && c * 32 + i > lim) {
+        x = -INFINITY;
+        sr[c][i] = __float_as_uint(x);
       }
-      mx0 = fmaxf(mx0, x0);
-      mx1 = fmaxf(mx1, x1);
+      mx[i & 7] = fmaxf(mx[i & 7], x);
     }
-  const float mt = fmaxf(mx0, mx1);
+  const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                         fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
   // the running max is kept in raw score units; p = 2^(s * sl2 - m_run * sl2)
   const bool grow = (mt - m_run) * sl2 > kRescaleThreshold;
   const float alpha = grow ? ex2_approx((m_run - mt) * sl2) : 1.0f;
@@ -118,23 +124,32 @@ __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, bool firs
     m_run = mt;
   }
   const float neg_m = -m_run * sl2;
-  float rs0 = 0.f, rs1 = 0.f;
+  float rs[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
   for (int c = 0; c < 4; ++c) {
     // keys 32c .. 32c+31 -> packed bf16 P columns 16c .. 16c+15 (S already in registers)
     uint32_t pk[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c][2 * i]), sl2, neg_m));
-      const float p1 = ex2_approx(fmaf(__uint_as_float(sr[c][2 * i + 1]), sl2, neg_m));
-      rs0 += p0;
-      rs1 += p1;
+      const float x0 = fmaf(__uint_as_float(sr[c][2 * i]), sl2, neg_m);
+      const float x1 = fmaf(__uint_as_float(sr[c][2 * i + 1]), sl2, neg_m);
+      const float p0 = ex2_approx(x0);
+      const float p1 = ex2_approx(x1);
+      rs[(2 * i) & 3] += p0;
+      rs[(2 * i + 1) & 3] += p1;
       pk[i] = pack_bf16(p0, p1);
     }
     tmem_st16(tS + 16 * c, pk);
   }
   tmem_st_wait();
-  l_run += rs0 + rs1;
+  l_run += (rs[0] + rs[1]) + (rs[2] + rs[3]);
+}
+
+__device__ __forceinline__ void regs_dec_ctl() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsCtl));
+}
+__device__ __forceinline__ void regs_inc_softmax() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSoftmax));
 }
 
 template <int D>
@@ -148,10 +163,9 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sQ = smem;
-  uint8_t* sK = sQ + 2 * Q_BYTES;
-  uint8_t* sV = sK + 2 * KV_BYTES;
+  uint8_t* sKV = sQ + 2 * Q_BYTES;  // kSlots x KV_BYTES
   __shared__ __align__(8) uint64_t q_full, o_full, drain_bar;
-  __shared__ __align__(8) uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
+  __shared__ __align__(8) uint64_t kv_full[kSlots], kv_empty[kSlots];
   __shared__ __align__(8) uint64_t s_full[2], p_full[2];
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_flag;
@@ -175,12 +189,13 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
     mbar_init(&o_full, 1);
     mbar_init(&drain_bar, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&k_full[i], 1);
-      mbar_init(&k_empty[i], 1);
-      mbar_init(&v_full[i], 1);
-      mbar_init(&v_empty[i], 1);
+
       mbar_init(&s_full[i], 1);
       mbar_init(&p_full[i], 4);
+    }
+    for (int i = 0; i < kSlots; ++i) {
+      mbar_init(&kv_full[i], 1);
+      mbar_init(&kv_empty[i], 1);
     }
     abort_flag = 0;
     fence_barrier_init();
@@ -194,50 +209,52 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
   tc_fence_after();
   const uint32_t tmem = tmem_base_sh;
 
-  if (warp == 0) {
-    // ---------------------------------------------------------------- producer
-    if (lane == 0) {
+  if (warp < 4) {
+    // setmaxnreg inside each role's branch: the softmax code is never reachable from here
+    regs_dec_ctl();
+    if (warp == 0 && lane == 0) {
+      // ---------------------------------------------------------------- producer
       bool ok = true;
-      int armed_k[2] = {-1, -1}, armed_v[2] = {-1, -1};
+      int armed[kSlots];
+      for (int i = 0; i < kSlots; ++i) armed[i] = -1;
       mbar_arrive_expect_tx(&q_full, ntiles * Q_BYTES);
       for (int t = 0; t < ntiles; ++t)
         for (int h = 0; h < HALVES; ++h)
           tma_load_2d(sQ + t * Q_BYTES + h * (kM * 128), &a.tmQ, &q_full, w.head * D + 64 * h,
                       row0 + q0 + t * kM);
-      for (int j = 0; j < J && ok; ++j) {
-        const int st = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        for (int kv = 0; kv < 2 && ok; ++kv) {
-          uint64_t* full = kv == 0 ? &k_full[st] : &v_full[st];
-          uint64_t* empty = kv == 0 ? &k_empty[st] : &v_empty[st];
-          if (!mbar_wait(empty, ph ^ 1, &abort_flag, a.status)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(full, KV_BYTES);
-          uint8_t* dst = (kv == 0 ? sK : sV) + st * KV_BYTES;
-          const CUtensorMap* map = kv == 0 ? &a.tmK : &a.tmV;
-          for (int p = 0; p < kPagesPerTile; ++p) {
-            // pages past the prefix repeat the last page: finite data, masked below
-            const int page = pt[min(j * kPagesPerTile + p, n_pages - 1)];
-            const int row = (page * a.n_kv_heads + w.g) * kPage;
-            for (int h = 0; h < HALVES; ++h)
-              tma_load_2d(dst + h * HALF_ROWS_BYTES + p * kPage * 128, map, full, 64 * h, row);
-          }
-          (kv == 0 ? armed_k : armed_v)[st] = ph;
+      int slot = 0;
+      uint32_t ph = 0;
+      for (int i = 0; i < 2 * J && ok; ++i) {
+        const int j = i >> 1;
+        const int kv = i & 1;
+        if (!mbar_wait(&kv_empty[slot], ph ^ 1, &abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&kv_full[slot], KV_BYTES);
+        uint8_t* dst = sKV + slot * KV_BYTES;
+        const CUtensorMap* map = kv == 0 ? &a.tmK : &a.tmV;
+        for (int p = 0; p < kPagesPerTile; ++p) {
+          // pages past the prefix repeat the last page: finite data, masked below
+          const int page = pt[min(j * kPagesPerTile + p, n_pages - 1)];
+          const int row = (page * a.n_kv_heads + w.g) * kPage;
+          for (int h = 0; h < HALVES; ++h)
+            tma_load_2d(dst + h * HALF_ROWS_BYTES + p * kPage * 128, map, &kv_full[slot], 64 * h, row);
+        }
+        armed[slot] = ph;
+        if (++slot == kSlots) {
+          slot = 0;
+          ph ^= 1;
         }
       }
       if (!ok) {
         volatile int never = 0;
-        for (int s = 0; s < 2; ++s) {
-          if (armed_k[s] >= 0) mbar_wait(&k_full[s], armed_k[s], &never, nullptr);
-          if (armed_v[s] >= 0) mbar_wait(&v_full[s], armed_v[s], &never, nullptr);
-        }
+        for (int i = 0; i < kSlots; ++i)
+          if (armed[i] >= 0) mbar_wait(&kv_full[i], armed[i], &never, nullptr);
         mbar_wait(&q_full, 0, &never, nullptr);
       }
-    }
-  } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
+    } else if (warp == 1) {
+      // -------------------------------------------------------------- MMA issuer
     // Order: S0(0) S1(0) | PV0(j) S0(j+1) PV1(j) S1(j+1) | ... so that the softmax of one
     // query tile overlaps the products of the other; query tile 0 stops one kv tile early
     // (its diagonal), after which tile 1 runs alone. tcgen05.mma of one thread execute in
@@ -247,8 +264,11 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
       bool issued = false;
       const uint32_t idesc_s = idesc_bf16_f32(kM, kN);
       const uint32_t idesc_o = idesc_bf16_f32(kM, D, false, true);
-      auto issue_s = [&](int t, int st) {
-        const uint32_t kb = smem_u32(sK + st * KV_BYTES);
+      // ring position of sequence item i (K(j): i = 2j, V(j): i = 2j + 1)
+      auto slot_of = [](int i) { return i % kSlots; };
+      auto parity_of = [](int i) { return static_cast<uint32_t>((i / kSlots) & 1); };
+      auto issue_s = [&](int t, int ks) {
+        const uint32_t kb = smem_u32(sKV + ks * KV_BYTES);
         const uint32_t qb = smem_u32(sQ + t * Q_BYTES);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
@@ -258,22 +278,22 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
         }
         mma_commit(&s_full[t]);
       };
-      if (ok) ok = mbar_wait(&k_full[0], 0, &abort_flag, a.status);
+      if (ok) ok = mbar_wait(&kv_full[slot_of(0)], parity_of(0), &abort_flag, a.status);
       if (ok) {
         tc_fence_after();
-        for (int t = 0; t < ntiles; ++t) issue_s(t, 0);
-        mma_commit(&k_empty[0]);
+        for (int t = 0; t < ntiles; ++t) issue_s(t, slot_of(0));
+        mma_commit(&kv_empty[slot_of(0)]);
         issued = true;
       }
       for (int j = 0; j < J && ok; ++j) {
-        const int st = j & 1;
-        const int nst = (j + 1) & 1;
+        const int vs = slot_of(2 * j + 1);
+        const int ks = slot_of(2 * j + 2);
         const bool more = j + 1 < J;
-        if (!mbar_wait(&v_full[st], (j >> 1) & 1, &abort_flag, a.status)) {
+        if (!mbar_wait(&kv_full[vs], parity_of(2 * j + 1), &abort_flag, a.status)) {
           ok = false;
           break;
         }
-        const uint32_t vb = smem_u32(sV + st * KV_BYTES);
+        const uint32_t vb = smem_u32(sKV + vs * KV_BYTES);
         bool k_ready = false;
         for (int t = (j < J0 ? 0 : 1); t < ntiles && ok; ++t) {
           if (!mbar_wait(&p_full[t], j & 1, &abort_flag, a.status)) {
@@ -290,19 +310,19 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
           }
           if (j + 1 < (t == 0 ? J0 : J)) {
             if (!k_ready) {
-              if (!mbar_wait(&k_full[nst], ((j + 1) >> 1) & 1, &abort_flag, a.status)) {
+              if (!mbar_wait(&kv_full[ks], parity_of(2 * j + 2), &abort_flag, a.status)) {
                 ok = false;
                 break;
               }
               tc_fence_after();
               k_ready = true;
             }
-            issue_s(t, nst);
+            issue_s(t, ks);
           }
         }
         if (!ok) break;
-        mma_commit(&v_empty[st]);
-        if (more) mma_commit(&k_empty[nst]);
+        mma_commit(&kv_empty[vs]);
+        if (more) mma_commit(&kv_empty[ks]);
       }
       if (ok) {
         mma_commit(&o_full);
@@ -312,9 +332,11 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
         mbar_wait(&drain_bar, 0, &never, nullptr);
       }
     }
+    }
   } else {
+    regs_inc_softmax();
     // ---------------------------------------------------------------- softmax + epilogue
-    const int t = (warp - 2) >> 2;
+    const int t = (warp - 4) >> 2;
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;  // query row within the tile (= TMEM lane)
     if (t < ntiles) {
@@ -342,13 +364,13 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
         if (last && t == ntiles - 1 && kv_end - k0 < kN) {
           // zero V rows past the prefix so that 0 * stale data cannot produce NaN (only the
           // last query tile reads the last kv tile)
-          const int st = j & 1;
-          ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (j >> 1) & 1, &abort_flag, a.status));
+          const int vi = 2 * j + 1;
+          ok = __all_sync(0xffffffffu, mbar_wait(&kv_full[vi % kSlots], (vi / kSlots) & 1, &abort_flag, a.status));
           if (ok) {
-            uint8_t* vt = sV + st * KV_BYTES;
+            uint8_t* vt = sKV + (vi % kSlots) * KV_BYTES;
             const int zr0 = kv_end - k0;
             const int chunks = (kN - zr0) * HALVES * 8;
-            for (int i = threadIdx.x - 64 - 128 * t; i < chunks; i += 128) {
+            for (int i = threadIdx.x - 128 - 128 * t; i < chunks; i += 128) {
               const int rr = zr0 + i / (HALVES * 8);
               const int h = (i / 8) % HALVES;
               const int ch = i % 8;
@@ -428,11 +450,17 @@ bool map2d(CUtensorMap* m, const void* base, long rows, int cols, int box_rows) 
 
 template <int D>
 cudaError_t launch_tc(const AttnTcArgs& args, cudaStream_t stream) {
-  constexpr int smem = 2 * kM * D * 2 + 4 * kN * D * 2 + 1024;
+  constexpr int smem = 2 * kM * D * 2 + kSlots * kN * D * 2 + 1024;
   static bool set = false;
   if (!set) {
     cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
+    // setmaxnreg.inc waits until the CTA's register pool can serve it: refuse to launch a
+    // build whose per-thread launch count leaves the split short
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, attn_tc_kernel<D>);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs * kThreadsAttn < kRegsNeeded) return cudaErrorInvalidConfiguration;
     set = true;
   }
   attn_tc_kernel<D><<<args.total_items, kThreadsAttn, smem, stream>>>(args);
