@@ -184,8 +184,8 @@ int module_rows_total(const Dims& D) {
   return t;
 }
 
-// decode attention partials: one per 256-position chunk of the longest prefix
-int dec_splits(int max_n) { return std::max(1, (max_n + 255) / 256); }
+// decode attention partials: one per chunk of the longest prefix
+int dec_splits(int max_n) { return decode_attention_splits(max_n); }
 
 Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   Plan p;
@@ -616,7 +616,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
     a.n_kv_heads = D.hkv;
     a.head_dim = D.d;
     a.splits = p.splits;
-    CRF_CUDA(launch_decode_attention(a, c.st));
+    CRF_CUDA(launch_decode_attention(a, c.pool->num_pages, c.ctx->status_dev, c.st));
     CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
     CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
     // gate rows then up rows: SwiGLU over [nr, f] with the up half Rs * f further on

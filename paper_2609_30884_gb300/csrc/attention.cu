@@ -1,6 +1,5 @@
-// Causal grouped-query prefill attention over the paged KV cache, and the
-// single-row decode attention used to carry the last prefix row through the
-// layers after a recomputed window.
+// Causal grouped-query prefill attention over the paged KV cache on mma.sync
+// (the alternative to the tcgen05 kernel, selected with CRF_ATTENTION=mma).
 //
 // Prefill: softmax(q k^T / sqrt(d) + causal mask) v over the whole prefix, per
 // query head; query head h reads kv head h / (Hq / Hkv). q arrives already
@@ -31,27 +30,6 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                          uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7},"
-      " {%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 // Row `r`, 16-byte chunk `c` of a tile whose rows are D*2 bytes: XOR-swizzled chunk.
@@ -262,176 +240,6 @@ __global__ void __launch_bounds__(kWarps * 32, 1) attn_prefill_kernel(const Attn
   }
 }
 
-// ---------------------------------------------------------------- decode attention
-// One decode row per request: q [Hq*d] (fp32, rotated) attends to the request's
-// cached keys at positions < pos (from the pages) plus its own fresh k/v at pos.
-// A block takes one kv head and one chunk of 256 positions and serves every query
-// head of that kv group, so each K/V row is read once per chunk:
-//   1. thread t scores position chunk0 + t against all heads of the group,
-//   2. warp h turns head h's scores into exp(s - max) and their sum,
-//   3. warp w accumulates positions 32w..32w+31 into per-lane 4-dim slices of O,
-//      and the 8 warp partials are summed through shared memory.
-// The chunk partials (max, sum, O) are merged by decode_attn_combine.
-constexpr int kDecThreads = 256;
-constexpr int kDecChunk = 256;
-constexpr int kDecMaxGroup = 8;
-
-template <int D>
-__global__ void __launch_bounds__(kDecThreads) decode_attn_partial(const DecodeAttnDesc p) {
-  constexpr int DPL = D / 32;  // dims per lane in the PV accumulation
-  const int r = blockIdx.z;
-  const int g = blockIdx.y;
-  const int chunk = blockIdx.x;
-  const int pos = p.pos[r];
-  const int grp = p.n_q_heads / p.n_kv_heads;
-  const int32_t* pt = p.page_table[r];
-  const int total = pos + 1;
-  const int t0 = chunk * kDecChunk;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __shared__ float q_s[kDecMaxGroup][D];
-  __shared__ float sc[kDecMaxGroup][kDecChunk];
-  __shared__ float stat[kDecMaxGroup][2];
-  __shared__ float red[kDecThreads / 32][kDecMaxGroup][D];
-  __shared__ int page_s[kDecChunk / kPage];
-  if (t0 >= total) return;
-  const float scale = rsqrtf(static_cast<float>(D));
-  for (int i = threadIdx.x; i < grp * D; i += kDecThreads)
-    q_s[i / D][i % D] = p.q[(size_t)r * p.n_q_heads * D + (g * grp + i / D) * D + i % D] * scale;
-  if (threadIdx.x < kDecChunk / kPage) {
-    const int t = t0 + threadIdx.x * kPage;
-    page_s[threadIdx.x] = t < pos ? pt[t / kPage] : 0;
-  }
-  __syncthreads();
-  // 1. scores
-  {
-    const int t = t0 + threadIdx.x;
-    float dot[kDecMaxGroup];
-#pragma unroll
-    for (int h = 0; h < kDecMaxGroup; ++h) dot[h] = 0.f;
-    if (t < total) {
-      if (t < pos) {
-        const uint4* kr = reinterpret_cast<const uint4*>(
-            p.kpages + (((size_t)page_s[threadIdx.x / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D);
-#pragma unroll 4
-        for (int i = 0; i < D / 8; ++i) {
-          const uint4 u = kr[i];
-          const float k8[8] = {bf16_lo(u.x), bf16_hi(u.x), bf16_lo(u.y), bf16_hi(u.y),
-                               bf16_lo(u.z), bf16_hi(u.z), bf16_lo(u.w), bf16_hi(u.w)};
-#pragma unroll
-          for (int h = 0; h < kDecMaxGroup; ++h)
-            if (h < grp)
-#pragma unroll
-              for (int e = 0; e < 8; ++e) dot[h] += q_s[h][8 * i + e] * k8[e];
-        }
-      } else {
-        const float* kr = p.k_self + (size_t)r * p.n_kv_heads * D + g * D;
-        for (int i = 0; i < D; ++i) {
-          const float kv = kr[i];
-#pragma unroll
-          for (int h = 0; h < kDecMaxGroup; ++h)
-            if (h < grp) dot[h] += q_s[h][i] * kv;
-        }
-      }
-    }
-#pragma unroll
-    for (int h = 0; h < kDecMaxGroup; ++h)
-      if (h < grp) sc[h][threadIdx.x] = t < total ? dot[h] : -FLT_MAX;
-  }
-  __syncthreads();
-  // 2. per-head max, exponentials, sum (warp h)
-  if (warp < grp) {
-    float m = -FLT_MAX;
-    for (int i = lane; i < kDecChunk; i += 32) m = fmaxf(m, sc[warp][i]);
-    m = warp_max(m);
-    float l = 0.f;
-    for (int i = lane; i < kDecChunk; i += 32) {
-      const float e = sc[warp][i] == -FLT_MAX ? 0.f : __expf(sc[warp][i] - m);
-      sc[warp][i] = e;
-      l += e;
-    }
-    l = warp_sum(l);
-    if (lane == 0) {
-      stat[warp][0] = m;
-      stat[warp][1] = l;
-    }
-  }
-  __syncthreads();
-  // 3. O partial: warp w takes positions t0 + 32w .. t0 + 32w + 31
-  float acc[kDecMaxGroup][DPL];
-#pragma unroll
-  for (int h = 0; h < kDecMaxGroup; ++h)
-#pragma unroll
-    for (int e = 0; e < DPL; ++e) acc[h][e] = 0.f;
-  const int kb = warp * 32;
-  const int kend = max(0, min(32, total - t0 - kb));
-#pragma unroll 8
-  for (int k = 0; k < kend; ++k) {
-    const int t = t0 + kb + k;
-    float v[DPL];
-    if (t < pos) {
-      const __nv_bfloat16* vr = p.vpages +
-          (((size_t)page_s[(kb + k) / kPage] * p.n_kv_heads + g) * kPage + t % kPage) * D + lane * DPL;
-      if (DPL == 4) {
-        const uint2 u = __ldg(reinterpret_cast<const uint2*>(vr));
-        v[0] = bf16_lo(u.x);
-        v[1 % DPL] = bf16_hi(u.x);
-        v[2 % DPL] = bf16_lo(u.y);
-        v[3 % DPL] = bf16_hi(u.y);
-      } else {
-        const uint32_t u = __ldg(reinterpret_cast<const uint32_t*>(vr));
-        v[0] = bf16_lo(u);
-        v[1 % DPL] = bf16_hi(u);
-      }
-    } else {
-      const float* vr = p.v_self + (size_t)r * p.n_kv_heads * D + g * D + lane * DPL;
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) v[e] = vr[e];
-    }
-#pragma unroll
-    for (int h = 0; h < kDecMaxGroup; ++h)
-      if (h < grp) {
-        const float ph = sc[h][kb + k];
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) acc[h][e] += ph * v[e];
-      }
-  }
-#pragma unroll
-  for (int h = 0; h < kDecMaxGroup; ++h)
-    if (h < grp)
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) red[warp][h][lane * DPL + e] = acc[h][e];
-  __syncthreads();
-  for (int i = threadIdx.x; i < grp * D; i += kDecThreads) {
-    const int h = i / D, d = i % D;
-    float o = 0.f;
-#pragma unroll
-    for (int w = 0; w < kDecThreads / 32; ++w) o += red[w][h][d];
-    float* part = p.part + (((size_t)r * p.n_q_heads + g * grp + h) * p.splits + chunk) * (D + 2);
-    part[d] = o;
-    if (d == 0) {
-      part[D] = stat[h][0];
-      part[D + 1] = stat[h][1];
-    }
-  }
-}
-
-template <int D>
-__global__ void decode_attn_combine(const DecodeAttnDesc p) {
-  const int r = blockIdx.y, h = blockIdx.x;
-  const int dd = threadIdx.x;
-  const int n_chunks = (p.pos[r] + 1 + kDecChunk - 1) / kDecChunk;
-  const float* base = p.part + ((size_t)r * p.n_q_heads + h) * p.splits * (D + 2);
-  float m = -FLT_MAX;
-  for (int s = 0; s < n_chunks; ++s) m = fmaxf(m, base[s * (D + 2) + D]);
-  float l = 0.f, acc = 0.f;
-  for (int s = 0; s < n_chunks; ++s) {
-    const float f = __expf(base[s * (D + 2) + D] - m);
-    l += f * base[s * (D + 2) + D + 1];
-    if (dd < D) acc += f * base[s * (D + 2) + dd];
-  }
-  if (dd < D) p.out[(size_t)r * p.n_q_heads * D + h * D + dd] = acc / l;
-}
-
 }  // namespace
 
 cudaError_t launch_attention(const AttnDesc& d, int num_sms, cudaStream_t stream) {
@@ -465,23 +273,5 @@ cudaError_t launch_attention(const AttnDesc& d, int num_sms, cudaStream_t stream
   return cudaGetLastError();
 }
 
-cudaError_t launch_decode_attention(const DecodeAttnDesc& d, cudaStream_t stream) {
-  if (d.n_q_heads / d.n_kv_heads > kDecMaxGroup) return cudaErrorInvalidValue;
-  int max_pos = 0;
-  for (int r = 0; r < d.rows; ++r) max_pos = max(max_pos, d.pos[r]);
-  const int chunks = (max_pos + 1 + kDecChunk - 1) / kDecChunk;
-  if (chunks > d.splits) return cudaErrorInvalidValue;
-  dim3 g1(chunks, d.n_kv_heads, d.rows), g2(d.n_q_heads, d.rows);
-  if (d.head_dim == 128) {
-    decode_attn_partial<128><<<g1, kDecThreads, 0, stream>>>(d);
-    decode_attn_combine<128><<<g2, 128, 0, stream>>>(d);
-  } else if (d.head_dim == 64) {
-    decode_attn_partial<64><<<g1, kDecThreads, 0, stream>>>(d);
-    decode_attn_combine<64><<<g2, 64, 0, stream>>>(d);
-  } else {
-    return cudaErrorInvalidValue;
-  }
-  return cudaGetLastError();
-}
 
 }  // namespace crf

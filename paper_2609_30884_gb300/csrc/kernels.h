@@ -159,7 +159,11 @@ struct DecodeAttnDesc {
   float* part;             // scratch [rows, Hq, splits, d + 2]
   int rows, n_q_heads, n_kv_heads, head_dim, splits, max_pos;
 };
-cudaError_t launch_decode_attention(const DecodeAttnDesc& d, cudaStream_t stream);
+// Chunked decode attention (TMA-staged pages, 128 positions per block) + merge. `splits` in
+// the descriptor must be at least decode_attention_splits(max position + 1).
+cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int* status,
+                                    cudaStream_t stream);
+int decode_attention_splits(int max_positions);
 struct RowPositions {
   int pos[kMaxReq];
 };
