@@ -525,12 +525,12 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
   float* part = m + Rs * D.f;
   const int rank = c.ad->dims.rank;
   // kernels per layer with up to 8 rows: 2 norm + LoRA-down launches, the o/down LoRA downs,
-  // 4 GEMVs, 2 RoPE, 2 attention, 1 SwiGLU; plus a conversion in and out per row
+  // 4 GEMVs, 1 RoPE, 2 attention, 1 SwiGLU; plus a conversion in and out per row
   int launches = 2 * R;
   for (int l = l0; l < D.N; ++l) {
     int nr = 0;
     for (const auto& r : rows) nr += r.e <= l;
-    launches += 9 + adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN) + 4 * ((nr + 7) / 8);
+    launches += 6 + adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN) + 4 * ((nr + 7) / 8);
   }
   ProfScope ps(c.ctx, kPDecode, c.st, launches);
   for (int i = 0; i < R; ++i)
@@ -596,8 +596,8 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
     while (nr < R && rows[nr].e <= l) ++nr;
     const crf_layer_weights& w = c.model->layers[l];
     CRF_CUDA(proj(l, nr, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr, 0));
-    CRF_CUDA(launch_rope_rows(q, nr, D.hq, D.d, rp, D.theta, c.st));
-    CRF_CUDA(launch_rope_rows(k, nr, D.hkv, D.d, rp, D.theta, c.st));
+    CRF_CUDA(launch_rope_rows(q, D.hq, k, D.hkv, nr, D.d,
+                              reinterpret_cast<const float2*>(c.ws + p.off_rope), rp, c.st));
     DecodeAttnDesc a;
     std::memset(&a, 0, sizeof(a));
     a.q = q;

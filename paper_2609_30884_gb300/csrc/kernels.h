@@ -167,9 +167,10 @@ int decode_attention_splits(int max_positions);
 struct RowPositions {
   int pos[kMaxReq];
 };
-// Rotate-half RoPE on fp32 rows x [rows, heads, head_dim], row r at position pos.pos[r].
-cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, const RowPositions& pos,
-                             double theta, cudaStream_t stream);
+// Rotate-half RoPE on the fp32 q [rows, hq, head_dim] and k [rows, hkv, head_dim] of decode
+// rows, row r at position pos.pos[r]; (cos, sin) from `table` [positions][head_dim / 2].
+cudaError_t launch_rope_rows(float* q, int hq, float* k, int hkv, int rows, int head_dim,
+                             const float2* table, const RowPositions& pos, cudaStream_t stream);
 cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream);
 cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
                                     cudaStream_t stream);

@@ -246,23 +246,22 @@ __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
   }
 }
 
-// Rotate-half RoPE on fp32 rows x [rows, heads, d], row r at position pos[r]; angle in fp64.
-__global__ void rope_rows_kernel(float* x, int rows, int heads, int d, const RowPositions pos,
-                                 double theta) {
+// Rotate-half RoPE on the fp32 q [rows, hq, d] and k [rows, hkv, d] of decode rows, row r at
+// position pos[r], angles from the (cos, sin) table of the window pass.
+__global__ void rope_rows_kernel(float* q, int hq, float* k, int hkv, int rows, int d,
+                                 const float2* __restrict__ table, const RowPositions pos) {
   const int half = d / 2;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  const int heads = hq + hkv;
   if (idx >= rows * heads * half) return;
   const int i = idx % half;
   const int h = (idx / half) % heads;
   const int r = idx / (half * heads);
-  double turns = static_cast<double>(pos.pos[r]) * pow(theta, -2.0 * i / d) * 0.15915494309189535;
-  turns -= floor(turns);
-  float s, c;
-  sincospif(static_cast<float>(2.0 * turns), &s, &c);
-  float* base = x + ((size_t)r * heads + h) * d;
+  const float2 cs = table[(size_t)pos.pos[r] * half + i];
+  float* base = h < hq ? q + ((size_t)r * hq + h) * d : k + ((size_t)r * hkv + (h - hq)) * d;
   const float x1 = base[i], x2 = base[i + half];
-  base[i] = x1 * c - x2 * s;
-  base[i + half] = x2 * c + x1 * s;
+  base[i] = x1 * cs.x - x2 * cs.y;
+  base[i + half] = x2 * cs.x + x1 * cs.y;
 }
 
 // BX rows: one thread per (row, 8-column chunk) of module blockIdx.y.
@@ -633,11 +632,11 @@ cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y,
   return cudaGetLastError();
 }
 
-cudaError_t launch_rope_rows(float* x, int rows, int heads, int head_dim, const RowPositions& pos,
-                             double theta, cudaStream_t stream) {
-  const int n = rows * heads * head_dim / 2;
+cudaError_t launch_rope_rows(float* q, int hq, float* k, int hkv, int rows, int head_dim,
+                             const float2* table, const RowPositions& pos, cudaStream_t stream) {
+  const int n = rows * (hq + hkv) * head_dim / 2;
   if (n == 0) return cudaSuccess;
-  rope_rows_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, rows, heads, head_dim, pos, theta);
+  rope_rows_kernel<<<cdiv(n, 256), 256, 0, stream>>>(q, hq, k, hkv, rows, head_dim, table, pos);
   return cudaGetLastError();
 }
 
