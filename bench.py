@@ -41,7 +41,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu --set full
 # capture of the kernel as it now stands, at the full launch size of the 7B-shape 16K workload
 # (profiles/gemm_gateup_swiglu_7b16k.md). An entry is removed whenever its kernel changes.
-NCU_TRAFFIC_BYTES = {}
+NCU_TRAFFIC_BYTES = {"gemm_gateup_swiglu": 2.712589e9 + 0.614191e9}
 
 
 def load_peaks():
@@ -410,6 +410,46 @@ def run_window_only(args):
     return 0
 
 
+def run_decode_only(args):
+    """The last layer as the window and its last row through the tail: the small profiling case
+    of the decode-row kernels (layers N-2, N-1 of the workload's shape, one KV pool)."""
+    import torch
+    import synth
+    import paper_2609_30884_gb300 as crf
+    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+
+    wl = synth.workload(args.workload)
+    cfg, lc = wl.model, wl.lora
+    n = args.tokens or wl.n_tokens[0]
+    s, e = cfg.n_layers - 2, cfg.n_layers - 1
+    device = "cuda:0"
+    ctx = crf.Context(0)
+    dm = DeviceModel(cfg, device, layers=range(s, cfg.n_layers), with_head=False)
+    cur = DeviceAdapter(cfg, lc, 1, device, layers=range(s, cfg.n_layers))
+    P = pages_needed(n)
+    pool = make_pool(cfg, P, device, fill="random", seed=11)
+    pt = split_page_tables([n], P, seed=5, device=device)[0]
+    h_in = synth.hidden_state(cfg, n, "restart", s - 1, device=device)
+    fin = torch.empty(cfg.hidden, dtype=torch.bfloat16, device=device)
+    req = crf.Request(pt, s, e, hidden_in=h_in, final_hidden_out=fin)
+    ws = ctx.workspace(dm.crf, cur.crf, [req])
+    for _ in range(args.warmup):
+        ctx.recompute_window(dm.crf, cur.crf, pool, [req], ws)
+    ctx.check()
+    ctx.profile_enable(True, 4096)
+    for _ in range(args.steps):
+        ctx.recompute_window(dm.crf, cur.crf, pool, [req], ws)
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    ctx.check()
+    kern = {k: {"ms_per_call": round(kms / args.steps, 4), "launches": cnt // args.steps}
+            for k, (kms, cnt) in prof.items() if k != "_dropped" and cnt}
+    print(json.dumps({"case": "decode-only", "workload": args.workload, "tokens": n,
+                      "window": [s, e], "tail_layers": cfg.n_layers - e, "kernels": kern}))
+    ctx.close()
+    return 0
+
+
 # ----------------------------------------------------------------------------- main
 def main():
     ap = argparse.ArgumentParser()
@@ -422,12 +462,15 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=1024, help="tokens per reference-arm step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
-    ap.add_argument("--case", default="step", choices=["step", "window-only"],
-                    help="window-only: the small profiling case (window layers only)")
+    ap.add_argument("--case", default="step", choices=["step", "window-only", "decode-only"],
+                    help="window-only / decode-only: small profiling cases (window layers only / "
+                         "the last layer and its first-step row)")
     ap.add_argument("--tokens", type=int, default=0, help="prefix length for --case window-only")
     args = ap.parse_args()
     if args.case == "window-only":
         return run_window_only(args)
+    if args.case == "decode-only":
+        return run_decode_only(args)
     if args.warmup < 3 and args.impl == "crf":
         args.warmup = 3
     if args.impl == "reference":
