@@ -305,7 +305,7 @@ def run_reference(args):
     if rank != 0:
         return 0
     import synth
-    wl = synth.workload(args.workload)
+    wl = workload_of(args)
     n_rows = args.ref_rows
     s, _ = wl.windows[0]
     weights = synth.layer_weights(wl.model, s)
@@ -365,7 +365,7 @@ def run_window_only(args):
     import paper_2609_30884_gb300 as crf
     from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed
 
-    wl = synth.workload(args.workload)
+    wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
     n = args.tokens or wl.n_tokens[0]
     s, e = wl.windows[0]
@@ -418,7 +418,7 @@ def run_decode_only(args):
     import paper_2609_30884_gb300 as crf
     from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 
-    wl = synth.workload(args.workload)
+    wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
     n = args.tokens or wl.n_tokens[0]
     s, e = cfg.n_layers - 2, cfg.n_layers - 1
@@ -450,6 +450,19 @@ def run_decode_only(args):
     return 0
 
 
+def workload_of(args):
+    """The named workload, with the adapter's rank / modules replaced when the flags ask for it
+    (alpha / r stays 2, as in the specified configurations)."""
+    import synth
+    from dataclasses import replace
+    wl = synth.workload(args.workload)
+    if args.lora_rank or args.lora_modules:
+        rank = args.lora_rank or wl.lora.rank
+        mods = tuple(args.lora_modules.split(",")) if args.lora_modules else wl.lora.modules
+        wl = replace(wl, lora=replace(wl.lora, rank=rank, alpha=2.0 * rank, modules=mods))
+    return wl
+
+
 # ----------------------------------------------------------------------------- main
 def main():
     ap = argparse.ArgumentParser()
@@ -466,6 +479,9 @@ def main():
                     help="window-only / decode-only: small profiling cases (window layers only / "
                          "the last layer and its first-step row)")
     ap.add_argument("--tokens", type=int, default=0, help="prefix length for --case window-only")
+    ap.add_argument("--lora-rank", type=int, default=0, help="adapter rank override (4, 8 or 16)")
+    ap.add_argument("--lora-modules", default="",
+                    help="adapter modules override, comma separated (e.g. v or q,v)")
     args = ap.parse_args()
     if args.case == "window-only":
         return run_window_only(args)
@@ -495,7 +511,7 @@ def main():
     import synth
     import paper_2609_30884_gb300 as crf
 
-    wl = synth.workload(args.workload)
+    wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
     ctx = crf.Context(local)
     st = build_state(wl, device, ctx, rank, world)

@@ -81,7 +81,7 @@ typedef struct crf_model_dims {
 } crf_model_dims;
 
 /* LoRA adapter shape: every adapted module m (bit m of module_mask) uses
- * W_m + (alpha / rank) * B_m A_m, kept unmerged. rank must be 8 or 16. */
+ * W_m + (alpha / rank) * B_m A_m, kept unmerged. rank must be 4, 8 or 16. */
 typedef struct crf_lora_dims {
   int rank;
   float alpha;

@@ -153,7 +153,8 @@ crf_status check_dims(const crf_model_dims& m) {
 }
 
 crf_status check_lora(const crf_lora_dims& l) {
-  if (l.rank != 8 && l.rank != 16) return fail(CRF_EUNSUPPORTED, "LoRA rank %d unsupported (8 or 16)", l.rank);
+  if (l.rank != 4 && l.rank != 8 && l.rank != 16)
+    return fail(CRF_EUNSUPPORTED, "LoRA rank %d unsupported (4, 8 or 16)", l.rank);
   if (!std::isfinite(l.alpha)) return fail(CRF_EINVAL, "LoRA alpha must be finite");
   if (l.module_mask & ~0x7Fu) return fail(CRF_EINVAL, "module_mask has bits beyond the 7 modules");
   return CRF_OK;

@@ -719,6 +719,9 @@ cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, float* g
     } else if (rank == 8) {
       drift_partial_kernel<16><<<g1, 256, 0, stream>>>(b, blocks_per_side, grams);
       drift_final_kernel<16><<<b.n_items, 256, 0, stream>>>(b, blocks_per_side, grams, out_sq);
+    } else if (rank == 4) {
+      drift_partial_kernel<8><<<g1, 256, 0, stream>>>(b, blocks_per_side, grams);
+      drift_final_kernel<8><<<b.n_items, 256, 0, stream>>>(b, blocks_per_side, grams, out_sq);
     } else {
       return cudaErrorInvalidValue;
     }
