@@ -450,6 +450,37 @@ def run_decode_only(args):
     return 0
 
 
+def run_trajectory_case(args):
+    """The recovery policy over a synthetic 32-version adapter trajectory (RQ4-style)."""
+    import torch
+    import paper_2609_30884_gb300 as crf
+    import trajectory
+    from harness import DeviceModel
+
+    wl = workload_of(args)
+    cfg, lc = wl.model, wl.lora
+    n = args.tokens or wl.n_tokens[0]
+    ctx = crf.Context(0)
+    dm = DeviceModel(cfg, "cuda:0")
+    layer = args.update_layer if args.update_layer >= 0 else cfg.n_layers // 2
+    t0 = time.time()
+    res = trajectory.run(ctx, dm, cfg, lc, n, versions=args.versions, calib_versions=args.calib_versions,
+                         layer=layer, module=args.update_module, std=args.update_std, base_version=0)
+    line = {"case": "trajectory", "workload": f"{args.workload}: {wl.name}", "tokens": n,
+            "versions": args.versions,
+            "update": {"layer": layer, "module": args.update_module, "std_per_entry": args.update_std,
+                       "version_0": "the workload adapter before any perturbation (A ~ N(0, 0.02^2), "
+                                    "B ~ N(0, 0.01^2))",
+                       "factors": "A and B, every entry, one seeded N(0, std^2) step per version"},
+            "maintenance": "crf_drift queries + crf_recompute_window of the chosen window (+ host decision), "
+                           "CUDA events, summed over the versions",
+            "data": "synthetic (seeded random-init decoder, uniform token ids)",
+            "wall_s": round(time.time() - t0, 1), **res}
+    print(json.dumps(line))
+    ctx.close()
+    return 0
+
+
 def workload_of(args):
     """The named workload, with the adapter's rank / modules replaced when the flags ask for it
     (alpha / r stays 2, as in the specified configurations)."""
@@ -475,9 +506,15 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=1024, help="tokens per reference-arm step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
-    ap.add_argument("--case", default="step", choices=["step", "window-only", "decode-only"],
+    ap.add_argument("--case", default="step", choices=["step", "window-only", "decode-only", "trajectory"],
                     help="window-only / decode-only: small profiling cases (window layers only / "
-                         "the last layer and its first-step row)")
+                         "the last layer and its first-step row); trajectory: the recovery policy "
+                         "over a synthetic continual-adapter trajectory")
+    ap.add_argument("--versions", type=int, default=32, help="trajectory: adapter updates replayed")
+    ap.add_argument("--calib-versions", type=int, default=8, help="trajectory: calibration updates")
+    ap.add_argument("--update-layer", type=int, default=-1, help="trajectory: updated layer (-1: N // 2)")
+    ap.add_argument("--update-module", default="v", help="trajectory: updated module")
+    ap.add_argument("--update-std", type=float, default=0.1, help="trajectory: step std per entry")
     ap.add_argument("--tokens", type=int, default=0, help="prefix length for --case window-only")
     ap.add_argument("--lora-rank", type=int, default=0, help="adapter rank override (4, 8 or 16)")
     ap.add_argument("--lora-modules", default="",
@@ -487,6 +524,8 @@ def main():
         return run_window_only(args)
     if args.case == "decode-only":
         return run_decode_only(args)
+    if args.case == "trajectory":
+        return run_trajectory_case(args)
     if args.warmup < 3 and args.impl == "crf":
         args.warmup = 3
     if args.impl == "reference":

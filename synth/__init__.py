@@ -268,6 +268,21 @@ def adapter_version(cfg: ModelCfg, lcfg: LoraCfg, version: int, layer: int, seed
     return out
 
 
+def trajectory_factors(cfg: ModelCfg, lcfg: LoraCfg, base_version: int, layer: int, module: str,
+                       t: int, std: float, seed: int = 0, device="cpu",
+                       base_seed: int = 0) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(A, B) of ``module`` at ``layer`` after t updates of a continual trajectory: the factors of
+    adapter version ``base_version`` (drawn with ``base_seed``), plus t independent fp32 steps
+    ~ N(0, std^2) on every entry of A and of B (drawn with ``seed``, in order 1..t), rounded to
+    bf16 once."""
+    a, b = adapter_version(cfg, lcfg, base_version, layer, base_seed, device)[module]
+    a, b = a.float(), b.float()
+    for k in range(1, t + 1):
+        a = a + normal(tuple(a.shape), f"traj_dA_{module}_{k}", layer, std, seed, device)
+        b = b + normal(tuple(b.shape), f"traj_dB_{module}_{k}", layer, std, seed, device)
+    return a.to(torch.bfloat16), b.to(torch.bfloat16)
+
+
 def embedding(cfg: ModelCfg, seed: int = 0, device="cpu") -> torch.Tensor:
     return bf16_normal((cfg.vocab, cfg.hidden), "embed", 0, W_STD, seed, device)
 

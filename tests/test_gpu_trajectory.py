@@ -1,0 +1,119 @@
+"""The recovery policy over a short continual-adapter trajectory: GPU run against an oracle replay.
+
+The GPU side is the benchmark's driver (package policy + crf_drift + crf_recompute_window + crf_kl
+on device caches). The oracle side replays the same seeded trajectory with the oracle's decoder on
+its own fp32 caches, the oracle's policy functions (Eq. 6-9, anchors of Section 4.2) and the
+oracle's drift and KL. Sensitivities and the drift-only threshold are fixed from oracle-computed
+version distances (calibration itself is covered by the CPU policy tests). Every method must take
+the same window at every version, and the first-step KL must agree within 1e-3.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from harness import DeviceModel, pages_needed, split_page_tables
+from oracle import cache as C, drift as odrift, fidelity, policy as OP
+from oracle.decoder import LayerAdapter
+from tests.gpu_util import KL_ABS, oracle_model
+
+pytestmark = pytest.mark.gpu
+
+CFG, LC = synth.TINY, synth.LORA_TINY
+N_TOK, LAYER, MODULE, STD, VERSIONS, SEED, BASE = 300, 2, "v", 1e-2, 6, 202, 0
+
+
+def _oracle_adapter(t):
+    layers = []
+    for l in range(CFG.n_layers):
+        d = synth.adapter_version(CFG, LC, BASE, l)
+        if l == LAYER and t > 0:
+            d[MODULE] = synth.trajectory_factors(CFG, LC, BASE, LAYER, MODULE, t, STD, SEED)
+        layers.append(LayerAdapter({m: (a.float().numpy(), b.float().numpy()) for m, (a, b) in d.items()},
+                                   LC.scale))
+    return C.Adapter(layers), layers
+
+
+def _state_sq(la, lb):
+    return sum(odrift.param_sq(*la[l].AB[m], *lb[l].AB[m])
+               for l in range(CFG.n_layers) for m in la[l].AB)
+
+
+def _oracle_windows_and_kl(om, ads, tokens, pt, sens, thr):
+    N = CFG.n_layers
+    r = OP.restart_layer(MODULE, LAYER, N)
+    num_pages = pages_needed(N_TOK)
+    base_pool = C.PagedPool(N, num_pages, CFG.n_kv_heads, CFG.head_dim)
+    base_req = C.RequestCache(tokens, pt)
+    C.prefill(om, ads[0][0], base_pool, base_req)
+    dist2 = lambda a, b: _state_sq(ads[a][1], ads[b][1])
+    out = {}
+    for method in ("fresh_full", "exact_suffix", "stale_reuse", "cachereforge", "drift_only", "fixed_window_2"):
+        pool = base_pool.copy()
+        req = C.RequestCache(tokens, pt, dict(base_req.hidden))
+        anchors = [0] * N
+        wins, kls, qs = [], [], []
+        for t in range(1, VERSIONS + 1):
+            oa = ads[t][0]
+            fp = C.PagedPool(N, num_pages, CFG.n_kv_heads, CFG.head_dim)
+            freq = C.RequestCache(tokens, pt)
+            z_fresh = C.logits(om, C.prefill(om, oa, fp, freq)[-1])
+            if method == "fresh_full":
+                w = (0, N)
+            elif method == "exact_suffix":
+                w = (r, N)
+            elif method == "stale_reuse":
+                w = (r, r)
+            elif method == "fixed_window_2":
+                w = (r, min(N, r + 2))
+            else:
+                d = OP.displacement(anchors, t, lambda a: [[dist2(a, t)]])
+                q = OP.risk(sens, d) if method == "cachereforge" else [x / thr for x in d]
+                qs.extend(q)
+                w = OP.plan(r, q)
+            if w[1] > w[0]:
+                C.run_window(om, oa, pool, req, w[0], w[1])
+            anchors = OP.update_anchors(anchors, w, t)
+            b = w[1] if w[1] > w[0] else w[0]
+            h = C.tail_decode(om, oa, pool, req, b, req.hidden[b - 1][-1])
+            kls.append(fidelity.kl(z_fresh, C.logits(om, h))[0])
+            wins.append(list(w))
+        out[method] = (wins, kls, qs)
+    return out
+
+
+def test_trajectory_matches_oracle_replay():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_30884_gb300 as crf
+    import trajectory as T
+
+    ads = [_oracle_adapter(t) for t in range(VERSIONS + 1)]
+    d01 = math.sqrt(_state_sq(ads[0][1], ads[1][1]))
+    sens = [0.0] * CFG.n_layers
+    sens[LAYER] = 1.0 / (1.5 * d01)
+    sens[LAYER + 1] = 1.0 / (2.5 * d01)
+    thr = 2.0 * d01
+
+    dm = DeviceModel(CFG)
+    om = oracle_model(dm)
+    tokens = synth.token_ids(CFG, N_TOK).numpy().astype(np.int64)
+    pt = split_page_tables([N_TOK], pages_needed(N_TOK), seed=1, device="cpu")[0].numpy()
+    want = _oracle_windows_and_kl(om, ads, tokens, pt, sens, thr)
+    # the fixed inputs must keep every risk clear of the trigger (else rounding could decide)
+    for m, (_, _, qs) in want.items():
+        assert all(abs(q - 1.0) > 1e-3 for q in qs), m
+    assert any(w[1] > w[0] for w in want["cachereforge"][0]) and any(w[1] == w[0] for w in want["cachereforge"][0])
+
+    ctx = crf.Context(0)
+    got = T.run(ctx, dm, CFG, LC, N_TOK, versions=VERSIONS, layer=LAYER, module=MODULE, std=STD,
+                eval_seed=SEED, sensitivity=sens, threshold=thr, base_version=BASE)
+    for m, (wins, kls, _) in want.items():
+        g = got["methods"][m]
+        assert g["windows"] == wins, (m, g["windows"], wins)
+        np.testing.assert_allclose(g["kl"], kls, atol=KL_ABS, rtol=0, err_msg=m)
+    assert got["methods"]["fresh_full"]["recompute_pct"] == 100.0
+    assert got["methods"]["stale_reuse"]["recompute_pct"] == 0.0
+    assert max(got["methods"]["fresh_full"]["kl"]) <= 1e-4  # full recompute reproduces fresh
