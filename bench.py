@@ -481,6 +481,63 @@ def run_trajectory_case(args):
     return 0
 
 
+def run_tail_case(args):
+    """Offline tail-influence sweep: N + 1 hybrid first-step passes over a stale cache."""
+    import torch
+    import numpy as np
+    import paper_2609_30884_gb300 as crf
+    from paper_2609_30884_gb300 import tail
+    import trajectory
+    from harness import DeviceModel, make_pool, pages_needed, split_page_tables
+
+    wl = workload_of(args)
+    cfg, lc = wl.model, wl.lora
+    n = args.tokens or wl.n_tokens[0]
+    N = cfg.n_layers
+    layer = args.update_layer if args.update_layer >= 0 else N // 2
+    ctx = crf.Context(0)
+    dm = DeviceModel(cfg, "cuda:0")
+    vers = trajectory.Versions(cfg, lc, layer, args.update_module, args.update_std, 202, "cuda:0", 0)
+    old, cur = vers.adapter(0), vers.adapter(args.versions)
+    P = pages_needed(n)
+    pt = split_page_tables([n], P, seed=1, device="cuda:0")[0]
+    tokens = synth_tokens(cfg, n)
+    stale, fresh = make_pool(cfg, P, "cuda:0"), make_pool(cfg, P, "cuda:0")
+    H = [torch.empty(n, cfg.hidden, dtype=torch.bfloat16, device="cuda:0") for _ in range(N)]
+    for ad, pool, hid in ((old, stale, None), (cur, fresh, H)):
+        req = crf.Request(pt, 0, N, n_tokens=n, tokens=tokens, hidden_out=hid)
+        ctx.recompute_window(dm.crf, ad, pool, [req], ctx.workspace(dm.crf, ad, [req]))
+    tail.sweep(ctx, dm.crf, cur, stale, pt, n, tokens, H, cfg.vocab)   # warm-up
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record()
+    rows = torch.empty(N + 1, cfg.hidden, dtype=torch.bfloat16, device="cuda:0")
+    tail.hybrid_rows(ctx, dm.crf, cur, stale, pt, n, tokens, H, rows)
+    b.record()
+    torch.cuda.synchronize()
+    ms_rows = a.elapsed_time(b)
+    res = tail.sweep(ctx, dm.crf, cur, stale, pt, n, tokens, H, cfg.vocab)
+    r = layer
+    print(json.dumps({
+        "case": "tail-influence", "workload": f"{args.workload}: {wl.name}", "tokens": n,
+        "update": {"layer": layer, "module": args.update_module, "std_per_entry": args.update_std,
+                   "versions": args.versions},
+        "ms_hybrid_rows": round(ms_rows, 3), "hybrid_passes": N + 1,
+        "kl": [round(float(x), 6) for x in res.kl], "tail_T": [round(float(x), 4) for x in res.tail],
+        "margin": round(res.margin, 4), "top1": [bool(x) for x in res.top1],
+        "kl_certificate_holds": int(res.kl_certificate_holds.sum()),
+        "top1_certificate_holds": int(res.top1_certificate_holds.sum()),
+        "horizon_eps_0.05": res.horizon(r, 0.05),
+        "data": "synthetic (seeded random-init decoder, uniform token ids)"}))
+    ctx.close()
+    return 0
+
+
+def synth_tokens(cfg, n):
+    import synth
+    return synth.token_ids(cfg, n, device="cuda:0")
+
+
 def workload_of(args):
     """The named workload, with the adapter's rank / modules replaced when the flags ask for it
     (alpha / r stays 2, as in the specified configurations)."""
@@ -506,10 +563,12 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=1024, help="tokens per reference-arm step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
-    ap.add_argument("--case", default="step", choices=["step", "window-only", "decode-only", "trajectory"],
+    ap.add_argument("--case", default="step",
+                    choices=["step", "window-only", "decode-only", "trajectory", "tail-influence"],
                     help="window-only / decode-only: small profiling cases (window layers only / "
                          "the last layer and its first-step row); trajectory: the recovery policy "
-                         "over a synthetic continual-adapter trajectory")
+                         "over a synthetic continual-adapter trajectory; tail-influence: the offline "
+                         "N + 1 hybrid-pass sweep (the update and --versions as for trajectory)")
     ap.add_argument("--versions", type=int, default=32, help="trajectory: adapter updates replayed")
     ap.add_argument("--calib-versions", type=int, default=8, help="trajectory: calibration updates")
     ap.add_argument("--update-layer", type=int, default=-1, help="trajectory: updated layer (-1: N // 2)")
@@ -526,6 +585,8 @@ def main():
         return run_decode_only(args)
     if args.case == "trajectory":
         return run_trajectory_case(args)
+    if args.case == "tail-influence":
+        return run_tail_case(args)
     if args.warmup < 3 and args.impl == "crf":
         args.warmup = 3
     if args.impl == "reference":
