@@ -533,6 +533,65 @@ def run_tail_case(args):
     return 0
 
 
+def run_decode_case(args):
+    """Greedy generation on the paged cache: R requests of the workload's prefix length, T steps."""
+    import torch
+    import paper_2609_30884_gb300 as crf
+    import synth
+    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+
+    wl = workload_of(args)
+    cfg, lc = wl.model, wl.lora
+    n = args.tokens or wl.n_tokens[0]
+    R, T = args.decode_rows, args.decode_steps
+    N = cfg.n_layers
+    ctx = crf.Context(0)
+    dm = DeviceModel(cfg, "cuda:0")
+    ad = DeviceAdapter(cfg, lc, wl.cur_version, "cuda:0")
+    P = R * pages_needed(n + T + args.warmup)
+    pts = split_page_tables([n + T + args.warmup] * R, P, seed=1, device="cuda:0")
+    pool = make_pool(cfg, P, "cuda:0")
+    for i in range(R):
+        tok = synth.token_ids(cfg, n, request=i, device="cuda:0")
+        req = crf.Request(pts[i], 0, N, n_tokens=n, tokens=tok)
+        ctx.recompute_window(dm.crf, ad.crf, pool, [req], ctx.workspace(dm.crf, ad.crf, [req]))
+    cur = synth.token_ids(cfg, R, request=99, device="cuda:0")
+    nxt = torch.empty(R, dtype=torch.int32, device="cuda:0")
+    pos = [n] * R
+    ws = ctx.decode_workspace(dm.crf, ad.crf, [n + T + args.warmup] * R, pts, cur)
+    for _ in range(args.warmup):
+        ctx.decode_step(dm.crf, ad.crf, pool, pos, pts, cur, nxt, ws)
+        cur, nxt = nxt, cur
+        pos = [p_ + 1 for p_ in pos]
+    ctx.check()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record()
+    for _ in range(T):
+        ctx.decode_step(dm.crf, ad.crf, pool, pos, pts, cur, nxt, ws)
+        cur, nxt = nxt, cur
+        pos = [p_ + 1 for p_ in pos]
+    b.record()
+    torch.cuda.synchronize()
+    ctx.check()
+    ms = a.elapsed_time(b)
+    h, f, qd, kvd, V = cfg.hidden, cfg.ffn, cfg.n_q_heads * cfg.head_dim, cfg.n_kv_heads * cfg.head_dim, cfg.vocab
+    w_bytes = 2 * N * (h * (qd + 2 * kvd) + qd * h + 2 * h * f + f * h) + 2 * V * h
+    kv_bytes = sum(2 * N * 2 * kvd * (p_ - T // 2) for p_ in pos)   # mean cached length over the run
+    step_ms = ms / T
+    peaks, src = load_peaks()
+    gbs = (w_bytes + kv_bytes) / (step_ms / 1000.0) / 1e9
+    print(json.dumps({"case": "decode", "workload": f"{args.workload}: {wl.name}", "prefix_tokens": n,
+                      "rows": R, "steps": T, "ms_per_step": round(step_ms, 3),
+                      "tokens_per_s": round(R * T / (ms / 1000.0), 1),
+                      "hbm": {"bytes_per_step": w_bytes + kv_bytes, "achieved_gbs": round(gbs, 1),
+                              "peak_gbs": peaks["hbm_gbs"], "frac": round(gbs / peaks["hbm_gbs"], 4),
+                              "peak_source": src},
+                      "data": "synthetic (seeded random-init decoder, uniform token ids)"}))
+    ctx.close()
+    return 0
+
+
 def synth_tokens(cfg, n):
     import synth
     return synth.token_ids(cfg, n, device="cuda:0")
@@ -564,12 +623,14 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--case", default="step",
-                    choices=["step", "window-only", "decode-only", "trajectory", "tail-influence"],
+                    choices=["step", "window-only", "decode-only", "trajectory", "tail-influence", "decode"],
                     help="window-only / decode-only: small profiling cases (window layers only / "
                          "the last layer and its first-step row); trajectory: the recovery policy "
                          "over a synthetic continual-adapter trajectory; tail-influence: the offline "
                          "N + 1 hybrid-pass sweep (the update and --versions as for trajectory)")
     ap.add_argument("--versions", type=int, default=32, help="trajectory: adapter updates replayed")
+    ap.add_argument("--decode-rows", type=int, default=8, help="decode: requests generating together")
+    ap.add_argument("--decode-steps", type=int, default=32, help="decode: timed generation steps")
     ap.add_argument("--calib-versions", type=int, default=8, help="trajectory: calibration updates")
     ap.add_argument("--update-layer", type=int, default=-1, help="trajectory: updated layer (-1: N // 2)")
     ap.add_argument("--update-module", default="v", help="trajectory: updated module")
@@ -587,6 +648,8 @@ def main():
         return run_trajectory_case(args)
     if args.case == "tail-influence":
         return run_tail_case(args)
+    if args.case == "decode":
+        return run_decode_case(args)
     if args.warmup < 3 and args.impl == "crf":
         args.warmup = 3
     if args.impl == "reference":

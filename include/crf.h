@@ -19,6 +19,10 @@
  *                         the current adapter from each layer's anchor.
  *   crf_kl                Section S2.1: forward KL(p* || p) at the first
  *                         generated-token step, fresh logits as reference.
+ *   crf_decode_step       one generated token per request on the recovered
+ *                         (mixed-version) paged cache: the step that consumes
+ *                         the refreshed cache (Section 3.1, first generated
+ *                         tokens); greedy next token and optional logits.
  *
  * Conventions (every entry point):
  *   - Device pointers are CUDA device memory on the context's device; host
@@ -171,6 +175,31 @@ CRF_API crf_status crf_workspace_size(crf_ctx* ctx, const crf_model* model, cons
 CRF_API crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_adapter* cur,
                                 const crf_kv_pool* pool, const crf_request* reqs, int n_req,
                                 void* workspace, size_t ws_bytes, void* stream);
+
+/* One generation step for each row: the token at position `pos` (the number
+ * of positions already cached for that request) is embedded and carried through
+ * layers 0..N-1 under `cur`; at every layer it attends to the cached keys and
+ * values at positions 0..pos-1 of its page table plus its own, and its post-RoPE
+ * K and V are written into slot pos % 16 of page page_table[pos / 16] of that
+ * layer (so the next step sees them). The final row goes through the final norm
+ * and the LM head; next_tokens[i] = argmax of row i's logits (lowest index
+ * among equal maxima).
+ *   page_table: device int32 [pos / 16 + 1]; pages must be distinct across rows.
+ *   token:      device int32, one entry: the input token id of the row.
+ * next_tokens: device int32 [n_rows]. logits: NULL or device fp32 [n_rows][vocab].
+ * The model needs embed, final_norm and lm_head; 1 <= n_rows <= CRF_MAX_REQUESTS.
+ * `workspace` >= crf_decode_workspace_size bytes, 256-byte aligned. */
+typedef struct {
+  int pos;
+  const int32_t* page_table;
+  const int32_t* token;
+} crf_decode_row;
+CRF_API crf_status crf_decode_workspace_size(crf_ctx* ctx, const crf_model* model, const crf_lora_dims* lora,
+                                     const crf_decode_row* rows, int n_rows, size_t* bytes);
+CRF_API crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const crf_adapter* cur,
+                           const crf_kv_pool* pool, const crf_decode_row* rows, int n_rows,
+                           int32_t* next_tokens, float* logits, void* workspace, size_t ws_bytes,
+                           void* stream);
 
 /* Eq. 8 drift. anchors: host array [n_layers] of adapters (anchors[l] is the
  * version that produced layer l's cache; all of the same lora dims as cur).

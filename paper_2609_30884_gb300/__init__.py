@@ -168,6 +168,34 @@ class Context:
                                                 workspace.data_ptr(), workspace.numel(),
                                                 _stream(stream)))
 
+    # -------------------------------------------------------------- generation
+    @staticmethod
+    def _decode_rows(positions: Sequence[int], page_tables: Sequence[torch.Tensor],
+                     tokens: torch.Tensor):
+        n = len(positions)
+        arr = (abi.DecodeRow * n)()
+        for i in range(n):
+            arr[i] = abi.DecodeRow(int(positions[i]), page_tables[i].data_ptr(), tokens[i:i + 1].data_ptr())
+        return arr
+
+    def decode_workspace(self, model: Model, adapter: Adapter, positions: Sequence[int],
+                         page_tables: Sequence[torch.Tensor], tokens: torch.Tensor) -> torch.Tensor:
+        n = c_size_t()
+        arr = self._decode_rows(positions, page_tables, tokens)
+        abi.check(self.lib.crf_decode_workspace_size(self.h, byref(model.c), byref(adapter.dims_c), arr,
+                                                     len(positions), byref(n)))
+        return torch.empty(max(256, n.value), dtype=torch.uint8, device=f"cuda:{self.device}")
+
+    def decode_step(self, model: Model, adapter: Adapter, pool: KVPool, positions: Sequence[int],
+                    page_tables: Sequence[torch.Tensor], tokens: torch.Tensor, next_tokens: torch.Tensor,
+                    workspace: torch.Tensor, logits: Optional[torch.Tensor] = None, stream=None) -> None:
+        """One generated token per row: tokens[i] (device int32) sits at positions[i]; its K/V are
+        written into the row's pages and next_tokens[i] receives the greedy next token."""
+        arr = self._decode_rows(positions, page_tables, tokens)
+        abi.check(self.lib.crf_decode_step(self.h, byref(model.c), byref(adapter.c), byref(pool.c), arr,
+                                           len(positions), next_tokens.data_ptr(), _ptr(logits),
+                                           workspace.data_ptr(), workspace.numel(), _stream(stream)))
+
     # -------------------------------------------------------------- drift
     def drift_workspace(self, dims_c, lora_dims_c) -> torch.Tensor:
         n = c_size_t()

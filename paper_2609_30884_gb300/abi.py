@@ -23,7 +23,7 @@ MAX_REQUESTS = 32
 EXPORTS = ("crf_create", "crf_destroy", "crf_last_error", "crf_check", "crf_workspace_size",
            "crf_recompute_window", "crf_drift_workspace_size", "crf_drift",
            "crf_kl_workspace_size", "crf_kl", "crf_kl_logits_noalloc", "crf_profile_enable",
-           "crf_profile_read")
+           "crf_profile_read", "crf_decode_workspace_size", "crf_decode_step")
 
 
 class ModelDims(ctypes.Structure):
@@ -61,6 +61,10 @@ class Request(ctypes.Structure):
                 ("hidden_out", POINTER(c_void_p)), ("final_hidden_out", c_void_p)]
 
 
+class DecodeRow(ctypes.Structure):
+    _fields_ = [("pos", c_int), ("page_table", c_void_p), ("token", c_void_p)]
+
+
 _lib = None
 
 
@@ -87,6 +91,10 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "crf_drift": ([P, POINTER(ModelDims), POINTER(Adapter), POINTER(POINTER(Adapter)), P, P,
                        c_size_t, P], c_int),
         "crf_kl_workspace_size": ([P, c_int, c_int, c_int, POINTER(c_size_t)], c_int),
+        "crf_decode_workspace_size": ([P, POINTER(Model), POINTER(LoraDims), POINTER(DecodeRow), c_int,
+                                       POINTER(c_size_t)], c_int),
+        "crf_decode_step": ([P, POINTER(Model), POINTER(Adapter), POINTER(KVPool), POINTER(DecodeRow),
+                             c_int, P, P, P, c_size_t, P], c_int),
         "crf_kl": ([P, POINTER(Model), P, P, c_int, c_int, P, P, P, c_size_t, P], c_int),
         "crf_kl_logits_noalloc": ([c_int, P, P, c_int, c_int, P, P], c_int),
         "crf_profile_enable": ([P, c_int, c_int], c_int),

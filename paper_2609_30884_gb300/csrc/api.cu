@@ -501,11 +501,20 @@ struct DecodeRow {
   int e;            // first layer to run
   int pos;          // position of the row (= n - 1)
   const int32_t* page_table;
-  const __nv_bfloat16* start;  // bf16 [h]
-  void* out;        // bf16 [h]
+  const __nv_bfloat16* start;  // bf16 [h], or null when the row starts from `token`'s embedding
+  void* out;        // bf16 [h], or null (the final fp32 rows stay in the decode scratch)
+  const int32_t* token = nullptr;  // device, the row's input token (generation steps)
 };
 
-crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
+// Generation steps (crf_decode_step) write each layer's k, v of the row into its page slot and
+// take RoPE angles from a table of the rows' own positions; the first-step rows of a window do
+// neither (their positions are in the window's full table, and the historical cache stays).
+struct DecodeOpts {
+  bool write_kv = false;
+  const float2* rope_by_row = nullptr;
+};
+
+crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const DecodeOpts& opt = DecodeOpts()) {
   const Dims& D = *c.D;
   const Plan& p = *c.plan;
   const int R = static_cast<int>(rows.size());
@@ -527,15 +536,32 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
   const int rank = c.ad->dims.rank;
   // kernels per layer with up to 8 rows: 2 norm + LoRA-down launches, the o/down LoRA downs,
   // 4 GEMVs, 1 RoPE, 2 attention, 1 SwiGLU; plus a conversion in and out per row
-  int launches = 2 * R;
+  int launches = 0;
+  for (const auto& r : rows) launches += (r.start ? 1 : 0) + (r.out ? 1 : 0);
+  bool any_token = false;
+  for (const auto& r : rows) any_token |= r.token != nullptr;
+  launches += any_token ? 1 : 0;
   for (int l = l0; l < D.N; ++l) {
     int nr = 0;
     for (const auto& r : rows) nr += r.e <= l;
-    launches += 6 + adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN) + 4 * ((nr + 7) / 8);
+    launches += 6 + (opt.write_kv ? 1 : 0) + adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN) +
+                4 * ((nr + 7) / 8);
   }
   ProfScope ps(c.ctx, kPDecode, c.st, launches);
-  for (int i = 0; i < R; ++i)
-    CRF_CUDA(launch_bf16_to_f32(rows[i].start, x + i * static_cast<size_t>(D.h), D.h, c.st));
+  TokenRows tr{};
+  for (int i = 0; i < R; ++i) {
+    if (rows[i].token) {
+      tr.token[i] = rows[i].token;
+    } else {
+      CRF_CUDA(launch_bf16_to_f32(rows[i].start, x + i * static_cast<size_t>(D.h), D.h, c.st));
+    }
+  }
+  if (any_token) {
+    // token rows are the whole batch (a generation step), so one launch covers them
+    for (int i = 0; i < R; ++i)
+      if (!rows[i].token) return fail(CRF_EINVAL, "decode rows mix token and hidden starts");
+    CRF_CUDA(launch_embed_rows_f32(static_cast<const __nv_bfloat16*>(c.model->embed), tr, R, x, D.h, c.st));
+  }
   // segments [mods] sharing the fp32 rows `raw` (optionally RMS-normalised into `in` inside the
   // LoRA-down launch), one GEMV per group of up to 8 rows
   auto proj = [&](int l, int nr, const int* mods, int nm, const float* raw, const void* norm_gain,
@@ -598,7 +624,9 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
     const crf_layer_weights& w = c.model->layers[l];
     CRF_CUDA(proj(l, nr, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr, 0));
     CRF_CUDA(launch_rope_rows(q, D.hq, k, D.hkv, nr, D.d,
-                              reinterpret_cast<const float2*>(c.ws + p.off_rope), rp, c.st));
+                              opt.rope_by_row ? opt.rope_by_row
+                                              : reinterpret_cast<const float2*>(c.ws + p.off_rope),
+                              rp, opt.rope_by_row != nullptr, c.st));
     DecodeAttnDesc a;
     std::memset(&a, 0, sizeof(a));
     a.q = q;
@@ -618,6 +646,14 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
     a.head_dim = D.d;
     a.splits = p.splits;
     CRF_CUDA(launch_decode_attention(a, c.pool->num_pages, c.ctx->status_dev, c.st));
+    if (opt.write_kv) {
+      RowPages pg{};
+      for (int i = 0; i < nr; ++i) {
+        pg.page_table[i] = rows[i].page_table;
+        pg.pos[i] = rows[i].pos;
+      }
+      CRF_CUDA(launch_kv_write_rows(k, v, c.pool->k_pages[l], c.pool->v_pages[l], pg, nr, D.hkv, D.d, c.st));
+    }
     CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
     CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
     // gate rows then up rows: SwiGLU over [nr, f] with the up half Rs * f further on
@@ -625,8 +661,9 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows) {
     CRF_CUDA(proj(l, nr, m_d, 1, m, nullptr, nullptr, D.f, y_d, o_d, x1, D.h));
   }
   for (int i = 0; i < R; ++i)
-    CRF_CUDA(launch_f32_to_bf16(x + i * static_cast<size_t>(D.h),
-                                static_cast<__nv_bfloat16*>(rows[i].out), D.h, c.st));
+    if (rows[i].out)
+      CRF_CUDA(launch_f32_to_bf16(x + i * static_cast<size_t>(D.h),
+                                  static_cast<__nv_bfloat16*>(rows[i].out), D.h, c.st));
   return CRF_OK;
 }
 
@@ -676,6 +713,61 @@ crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const c
     }
   }
   (void)ctx;
+  return CRF_OK;
+}
+
+// Workspace of one generation step: the decode-row scratch, the rows' RoPE angles, the final
+// normalised rows and (when the caller passes no buffer) the logits.
+struct StepPlan {
+  Plan p;
+  size_t off_angles, off_norm, off_logits, total;
+};
+
+StepPlan make_step_plan(const Dims& D, const crf_decode_row* rows, int n) {
+  StepPlan sp;
+  Plan& p = sp.p;
+  p.dec_rows = n;
+  p.max_n = 1;
+  for (int i = 0; i < n; ++i) p.max_n = std::max(p.max_n, rows[i].pos + 1);
+  p.splits = dec_splits(p.max_n);
+  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 3 * kRankPad + 3 * D.f) * 4 +
+                         static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
+  p.dec_bytes = align256(dec_row * std::max(1, n));
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = align256(o + bytes);
+    return at;
+  };
+  p.off_dec = take(p.dec_bytes);
+  p.off_rope = 0;
+  sp.off_angles = take(static_cast<size_t>(n) * (D.d / 2) * sizeof(float2));
+  sp.off_norm = take(static_cast<size_t>(n) * D.h * 4);
+  sp.off_logits = take(static_cast<size_t>(n) * D.V * 4);
+  sp.total = p.total = o;
+  return sp;
+}
+
+crf_status validate_decode_rows(const crf_kv_pool* pool, const crf_decode_row* rows, int n,
+                                cudaStream_t st) {
+  if (n < 1 || n > CRF_MAX_REQUESTS) return fail(CRF_EINVAL, "n_rows %d outside [1, %d]", n, CRF_MAX_REQUESTS);
+  if (!pool || !pool->k_pages || !pool->v_pages || pool->num_pages < 1) return fail(CRF_EINVAL, "kv pool missing");
+  std::vector<char> seen(static_cast<size_t>(pool->num_pages), 0);
+  for (int i = 0; i < n; ++i) {
+    const crf_decode_row& r = rows[i];
+    if (r.pos < 0) return fail(CRF_EINVAL, "row %d: negative position", i);
+    if (!r.page_table || !r.token) return fail(CRF_EINVAL, "row %d: page_table or token is null", i);
+    const int np = r.pos / kPage + 1;
+    std::vector<int32_t> pt(np);
+    CRF_CUDA(cudaMemcpyAsync(pt.data(), r.page_table, np * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+    CRF_CUDA(cudaStreamSynchronize(st));
+    for (int j = 0; j < np; ++j) {
+      if (pt[j] < 0 || pt[j] >= pool->num_pages)
+        return fail(CRF_EINVAL, "row %d: page id %d out of range [0,%d)", i, pt[j], pool->num_pages);
+      if (seen[pt[j]]) return fail(CRF_EINVAL, "row %d: page %d used twice", i, pt[j]);
+      seen[pt[j]] = 1;
+    }
+  }
   return CRF_OK;
 }
 
@@ -925,6 +1017,97 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
 static int drift_blocks_per_side(const crf_ctx* ctx, int n_items) {
   const int want = (4 * ctx->num_sms + 2 * n_items - 1) / std::max(1, 2 * n_items);
   return std::max(1, std::min(16, want));
+}
+
+crf_status crf_decode_workspace_size(crf_ctx* ctx, const crf_model* model, const crf_lora_dims* lora,
+                                     const crf_decode_row* rows, int n_rows, size_t* bytes) {
+  if (!ctx || !model || !lora || !rows || !bytes) return fail(CRF_EINVAL, "null argument");
+  crf_status s = check_dims(model->dims);
+  if (s != CRF_OK) return s;
+  s = check_lora(*lora);
+  if (s != CRF_OK) return s;
+  if (n_rows < 1 || n_rows > CRF_MAX_REQUESTS) return fail(CRF_EINVAL, "n_rows out of range");
+  for (int i = 0; i < n_rows; ++i)
+    if (rows[i].pos < 0) return fail(CRF_EINVAL, "row %d: negative position", i);
+  *bytes = make_step_plan(dims_of(model->dims), rows, n_rows).total;
+  return CRF_OK;
+}
+
+crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const crf_adapter* cur,
+                           const crf_kv_pool* pool, const crf_decode_row* rows, int n_rows,
+                           int32_t* next_tokens, float* logits, void* workspace, size_t ws_bytes,
+                           void* stream) {
+  if (!ctx || !model || !cur || !pool || !rows || !next_tokens) return fail(CRF_EINVAL, "null argument");
+  if (!model->layers) return fail(CRF_EINVAL, "model layers missing");
+  if (!model->embed || !model->final_norm || !model->lm_head)
+    return fail(CRF_EINVAL, "model embedding, final norm or LM head is null");
+  if (!cur->A || !cur->B) return fail(CRF_EINVAL, "adapter tables missing");
+  crf_status s = check_dims(model->dims);
+  if (s != CRF_OK) return s;
+  s = check_lora(cur->dims);
+  if (s != CRF_OK) return s;
+  CRF_CUDA(cudaSetDevice(ctx->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const Dims D = dims_of(model->dims);
+  s = check_model_layers(model, 0, D.N, D);
+  if (s != CRF_OK) return s;
+  s = check_adapter_layers(cur, 0, D.N);
+  if (s != CRF_OK) return s;
+  for (int l = 0; l < D.N; ++l)
+    if (!pool || !pool->k_pages || !pool->v_pages || !pool->k_pages[l] || !pool->v_pages[l] ||
+        !aligned16(pool->k_pages[l]) || !aligned16(pool->v_pages[l]))
+      return fail(CRF_EINVAL, "kv pool layer %d null or misaligned", l);
+  s = validate_decode_rows(pool, rows, n_rows, st);
+  if (s != CRF_OK) return s;
+  const StepPlan sp = make_step_plan(D, rows, n_rows);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return fail(CRF_EINVAL, "workspace null or not 256-byte aligned");
+  if (ws_bytes < sp.total) return fail(CRF_ENOMEM, "workspace %zu bytes, %zu needed", ws_bytes, sp.total);
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  LayerCtx c;
+  c.D = &D;
+  c.ctx = ctx;
+  c.model = model;
+  c.ad = cur;
+  c.pool = pool;
+  c.st = st;
+  c.ws = ws;
+  c.plan = &sp.p;
+  c.scale = cur->dims.alpha / cur->dims.rank;
+  RowPositions rp{};
+  std::vector<DecodeRow> dec;
+  for (int i = 0; i < n_rows; ++i) {
+    rp.pos[i] = rows[i].pos;
+    DecodeRow d{};
+    d.e = 0;
+    d.pos = rows[i].pos;
+    d.page_table = rows[i].page_table;
+    d.token = rows[i].token;
+    dec.push_back(d);
+  }
+  auto* angles = reinterpret_cast<float2*>(ws + sp.off_angles);
+  {
+    ProfScope ps(ctx, kPRope, st);
+    CRF_CUDA(launch_rope_table_rows(angles, rp, n_rows, D.d, D.theta, st));
+  }
+  DecodeOpts opt;
+  opt.write_kv = true;
+  opt.rope_by_row = angles;
+  s = decode_rows(c, dec, opt);
+  if (s != CRF_OK) return s;
+  // final norm, LM head, greedy token: the fp32 rows are the head of the decode scratch
+  float* x = reinterpret_cast<float*>(ws + sp.p.off_dec);
+  float* hn = reinterpret_cast<float*>(ws + sp.off_norm);
+  float* z = logits ? logits : reinterpret_cast<float*>(ws + sp.off_logits);
+  {
+    ProfScope ps(ctx, kPLmHead, st, 3);
+    CRF_CUDA(launch_rmsnorm_f32(x, static_cast<const __nv_bfloat16*>(model->final_norm), hn, n_rows, D.h, D.eps, st));
+    CRF_CUDA(launch_lm_head(static_cast<const __nv_bfloat16*>(model->lm_head), hn, n_rows, D.V, D.h, z,
+                            ctx->num_sms, st));
+    CRF_CUDA(launch_argmax_rows(z, n_rows, D.V, next_tokens, st));
+  }
+  return CRF_OK;
 }
 
 crf_status crf_drift_workspace_size(crf_ctx* ctx, const crf_model_dims* dims,

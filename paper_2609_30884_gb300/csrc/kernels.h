@@ -168,9 +168,31 @@ struct RowPositions {
   int pos[kMaxReq];
 };
 // Rotate-half RoPE on the fp32 q [rows, hq, head_dim] and k [rows, hkv, head_dim] of decode
-// rows, row r at position pos.pos[r]; (cos, sin) from `table` [positions][head_dim / 2].
+// rows, row r at position pos.pos[r]; (cos, sin) from `table` [positions][head_dim / 2], or with
+// table_by_row from row r of a [rows][head_dim / 2] table of the rows' own positions.
 cudaError_t launch_rope_rows(float* q, int hq, float* k, int hkv, int rows, int head_dim,
-                             const float2* table, const RowPositions& pos, cudaStream_t stream);
+                             const float2* table, const RowPositions& pos, bool table_by_row,
+                             cudaStream_t stream);
+// (cos, sin) of the rows' positions: table [rows][head_dim / 2].
+cudaError_t launch_rope_table_rows(float2* table, const RowPositions& pos, int rows, int head_dim,
+                                   double theta, cudaStream_t stream);
+struct TokenRows {
+  const int32_t* token[kMaxReq];  // device pointer to each row's input token id
+};
+// x [rows, hidden] fp32 = embed[token_r].
+cudaError_t launch_embed_rows_f32(const __nv_bfloat16* embed, const TokenRows& t, int rows, float* x,
+                                  int hidden, cudaStream_t stream);
+struct RowPages {
+  const int32_t* page_table[kMaxReq];
+  int pos[kMaxReq];
+};
+// Rows' fp32 k, v [rows, hkv * head_dim] into their page slot (page_table[pos / 16], pos % 16).
+cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, void* vpages,
+                                 const RowPages& rp, int rows, int hkv, int head_dim,
+                                 cudaStream_t stream);
+// out[r] = argmax of logits row r (lowest index among equal maxima).
+cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
+                               cudaStream_t stream);
 cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream);
 cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
                                     cudaStream_t stream);

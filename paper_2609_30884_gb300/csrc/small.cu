@@ -249,7 +249,7 @@ __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
 // Rotate-half RoPE on the fp32 q [rows, hq, d] and k [rows, hkv, d] of decode rows, row r at
 // position pos[r], angles from the (cos, sin) table of the window pass.
 __global__ void rope_rows_kernel(float* q, int hq, float* k, int hkv, int rows, int d,
-                                 const float2* __restrict__ table, const RowPositions pos) {
+                                 const float2* __restrict__ table, const RowPositions pos, int by_row) {
   const int half = d / 2;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   const int heads = hq + hkv;
@@ -257,7 +257,7 @@ __global__ void rope_rows_kernel(float* q, int hq, float* k, int hkv, int rows, 
   const int i = idx % half;
   const int h = (idx / half) % heads;
   const int r = idx / (half * heads);
-  const float2 cs = table[(size_t)pos.pos[r] * half + i];
+  const float2 cs = table[(size_t)(by_row ? r : pos.pos[r]) * half + i];
   float* base = h < hq ? q + ((size_t)r * hq + h) * d : k + ((size_t)r * hkv + (h - hq)) * d;
   const float x1 = base[i], x2 = base[i + half];
   base[i] = x1 * cs.x - x2 * cs.y;
@@ -633,10 +633,123 @@ cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y,
 }
 
 cudaError_t launch_rope_rows(float* q, int hq, float* k, int hkv, int rows, int head_dim,
-                             const float2* table, const RowPositions& pos, cudaStream_t stream) {
+                             const float2* table, const RowPositions& pos, bool table_by_row,
+                             cudaStream_t stream) {
   const int n = rows * (hq + hkv) * head_dim / 2;
   if (n == 0) return cudaSuccess;
-  rope_rows_kernel<<<cdiv(n, 256), 256, 0, stream>>>(q, hq, k, hkv, rows, head_dim, table, pos);
+  rope_rows_kernel<<<cdiv(n, 256), 256, 0, stream>>>(q, hq, k, hkv, rows, head_dim, table, pos,
+                                                     table_by_row ? 1 : 0);
+  return cudaGetLastError();
+}
+
+// (cos, sin) of the rows' own positions only: table[r][i] for position pos[r].
+__global__ void rope_table_rows_kernel(float2* table, int rows, int half, const RowPositions pos,
+                                       const __grid_constant__ RopeFreqs f) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * half) return;
+  const int r = idx / half, i = idx % half;
+  double turns = static_cast<double>(pos.pos[r]) * f.turns_per_pos[i];
+  turns -= floor(turns);
+  float s, c;
+  sincospif(static_cast<float>(2.0 * turns), &s, &c);
+  table[idx] = make_float2(c, s);
+}
+
+// x[r] = embed[token_r] as fp32, the token read from device memory.
+__global__ void embed_rows_f32_kernel(const __nv_bfloat16* __restrict__ embed, const TokenRows t,
+                                      float* __restrict__ x, int hidden) {
+  const int r = blockIdx.y;
+  const int32_t tok = *t.token[r];
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < hidden; i += gridDim.x * blockDim.x)
+    x[(size_t)r * hidden + i] = __bfloat162float(embed[(size_t)tok * hidden + i]);
+}
+
+// The rows' fp32 k, v [rows, Hkv * d] into slot pos % 16 of page page_table[pos / 16], bf16.
+__global__ void kv_write_rows_kernel(const float* __restrict__ k, const float* __restrict__ v,
+                                     __nv_bfloat16* kpages, __nv_bfloat16* vpages, const RowPages rp,
+                                     int hkv, int d) {
+  const int r = blockIdx.y;
+  const int pos = rp.pos[r];
+  const int page = rp.page_table[r][pos / kPage];
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < hkv * d; i += gridDim.x * blockDim.x) {
+    const int h = i / d, j = i % d;
+    const size_t dst = (((size_t)page * hkv + h) * kPage + pos % kPage) * d + j;
+    kpages[dst] = __float2bfloat16_rn(k[(size_t)r * hkv * d + i]);
+    vpages[dst] = __float2bfloat16_rn(v[(size_t)r * hkv * d + i]);
+  }
+}
+
+// out[r] = argmax_i logits[r, i], the lowest index among equal maxima.
+__global__ void argmax_rows_kernel(const float* __restrict__ logits, int vocab, int32_t* out) {
+  const int r = blockIdx.x;
+  const float* z = logits + (size_t)r * vocab;
+  float best = -INFINITY;
+  int arg = 0x7fffffff;
+  for (int i = threadIdx.x; i < vocab; i += blockDim.x) {
+    const float v = z[i];
+    if (v > best || (v == best && i < arg)) {
+      best = v;
+      arg = i;
+    }
+  }
+  __shared__ float sb[32];
+  __shared__ int sa[32];
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oa = __shfl_xor_sync(0xffffffffu, arg, o);
+    if (ob > best || (ob == best && oa < arg)) {
+      best = ob;
+      arg = oa;
+    }
+  }
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    sb[w] = best;
+    sa[w] = arg;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < static_cast<int>(blockDim.x >> 5); ++i)
+      if (sb[i] > best || (sb[i] == best && sa[i] < arg)) {
+        best = sb[i];
+        arg = sa[i];
+      }
+    out[r] = arg;
+  }
+}
+
+cudaError_t launch_rope_table_rows(float2* table, const RowPositions& pos, int rows, int head_dim,
+                                   double theta, cudaStream_t stream) {
+  const int half = head_dim / 2;
+  if (rows == 0) return cudaSuccess;
+  if (half > 64) return cudaErrorInvalidValue;
+  RopeFreqs f{};
+  for (int i = 0; i < half; ++i)
+    f.turns_per_pos[i] = std::pow(theta, -2.0 * i / head_dim) / (2.0 * 3.14159265358979323846);
+  rope_table_rows_kernel<<<cdiv(rows * half, 256), 256, 0, stream>>>(table, rows, half, pos, f);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_embed_rows_f32(const __nv_bfloat16* embed, const TokenRows& t, int rows, float* x,
+                                  int hidden, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  embed_rows_f32_kernel<<<dim3(cdiv(hidden, 256), rows), 256, 0, stream>>>(embed, t, x, hidden);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, void* vpages,
+                                 const RowPages& rp, int rows, int hkv, int head_dim,
+                                 cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  kv_write_rows_kernel<<<dim3(cdiv(hkv * head_dim, 256), rows), 256, 0, stream>>>(
+      k, v, static_cast<__nv_bfloat16*>(kpages), static_cast<__nv_bfloat16*>(vpages), rp, hkv, head_dim);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
+                               cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  argmax_rows_kernel<<<rows, 1024, 0, stream>>>(logits, vocab, out);
   return cudaGetLastError();
 }
 
