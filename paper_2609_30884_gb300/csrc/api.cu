@@ -602,7 +602,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
           sg.xa = xa + s * Rs * kRankPad + static_cast<size_t>(r0) * rank;
         }
       }
-      cudaError_t e = launch_gemv(g, c.ctx->num_sms, c.st);
+      cudaError_t e = launch_gemv(g, c.ctx->num_sms, c.st, nr);
       if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

@@ -132,7 +132,12 @@ struct GemvDesc {
   int rows;        // 1..8
   int rank;
 };
-cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream);
+// Tensor-core GEMV (mma.sync, rows as a bf16 hi/lo pair); launch_gemv uses it when the call's
+// rows (total_rows, the rows of all chunks one caller splits into launches of <= 8; 0 = d.rows)
+// number three or more, unless the environment sets CRF_GEMV=scalar (then always the CUDA-core
+// kernel). One kernel per call keeps equal rows equal across chunks.
+cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int total_rows = 0);
+cudaError_t launch_gemv_tc(const GemvDesc& d, int num_sms, cudaStream_t stream);
 // xa_m[r, k] = scale * sum_i A_m[k, i] x[r, i] for up to three modules m sharing x
 struct LoraDownRows {
   const __nv_bfloat16* A[3];

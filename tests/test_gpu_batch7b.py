@@ -1,9 +1,10 @@
 """GPU parity of the batched 7B-shape workload: 8 cached prefixes of 2K-16K tokens, each with
 its own window, one shared pool with a randomly permuted page table.
 
-* Batching is invisible: the batched call gives bit-identical pages, refreshed checkpoints and
-  first-step rows to running every request alone (each row is computed the same way whatever
-  else shares its tile or launch).
+* Batching is invisible in the window: the batched call gives bit-identical pages and refreshed
+  checkpoints to running every request alone (each row is computed the same way whatever else
+  shares its tile or launch); the first-step rows agree to bf16 rounding (their GEMV kernel
+  depends on how many rows share a weight pass).
 * Against the oracle, per request, on what it computes one by one at this size: K and V of every
   position of the request's first window layer, and that layer's output at sampled rows, held to
   1e-2 plus twice the largest distance that rounding-sized changes move the same rows (a bf16
@@ -78,7 +79,9 @@ def test_batch7b_equals_single_and_oracle(ctx):
             assert torch.equal(request_kv_t(pool.k_pages[l], pts[i], n), request_kv_t(got_k[l], pts[i], n)), (i, l)
             assert torch.equal(request_kv_t(pool.v_pages[l], pts[i], n), request_kv_t(got_v[l], pts[i], n)), (i, l)
             assert torch.equal(keep1[i][2][l - s], keep[i][2][l - s]), (i, l)
-        assert torch.equal(keep1[i][3], keep[i][3]), i
+        # the first-step row takes the tensor-core GEMV when >= 3 rows share a weight pass and the
+        # CUDA-core one alone: both fp32-accurate, so only bf16 rounding of the output may differ
+        assert rel_frob(to_np(keep1[i][3]), to_np(keep[i][3])) <= 5e-3, i
 
     # untouched slots and layers, bit-exact
     free = untouched_mask(P, list(zip(pts, wl.n_tokens)))
