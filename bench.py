@@ -592,6 +592,48 @@ def run_decode_case(args):
     return 0
 
 
+def run_drift_case(args):
+    """crf_drift alone (every layer and module of the workload's adapter against a per-layer anchor):
+    the small profiling case of the drift kernels (adapters only on the device)."""
+    import torch
+    import paper_2609_30884_gb300 as crf
+    from harness import DeviceAdapter, DeviceModel
+
+    wl = workload_of(args)
+    cfg, lc = wl.model, wl.lora
+    ctx = crf.Context(0)
+    dm = DeviceModel(cfg, "cuda:0", layers=[], with_head=False)
+    cur = DeviceAdapter(cfg, lc, 3, "cuda:0")
+    anchors = [DeviceAdapter(cfg, lc, v, "cuda:0") for v in (0, 1, 2)]
+    which = [anchors[l % 3].crf for l in range(cfg.n_layers)]
+    out = torch.empty(cfg.n_layers, 7, 2, dtype=torch.float32, device="cuda:0")
+    ws = ctx.drift_workspace(dm.crf.dims_c, cur.crf.dims_c)
+    for _ in range(args.warmup):
+        ctx.drift(dm.crf.dims_c, cur.crf, which, out, ws)
+    ctx.check()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record()
+    for _ in range(args.steps):
+        ctx.drift(dm.crf.dims_c, cur.crf, which, out, ws)
+    b.record()
+    torch.cuda.synchronize()
+    ctx.check()
+    ms = a.elapsed_time(b) / args.steps
+    factor_bytes = 0
+    for l in range(cfg.n_layers):
+        for m, (A, B) in cur.layers[l].items():
+            factor_bytes += 2 * (A.numel() + B.numel()) * 2   # both versions, bf16
+    peaks, src = load_peaks()
+    gbs = factor_bytes / (ms / 1000.0) / 1e9
+    print(json.dumps({"case": "drift", "workload": f"{args.workload}: {wl.name}", "rank": lc.rank,
+                      "modules": list(lc.modules), "ms_per_call": round(ms, 4),
+                      "hbm": {"bytes": factor_bytes, "achieved_gbs": round(gbs, 1),
+                              "frac": round(gbs / peaks["hbm_gbs"], 4), "peak_source": src}}))
+    ctx.close()
+    return 0
+
+
 def synth_tokens(cfg, n):
     import synth
     return synth.token_ids(cfg, n, device="cuda:0")
@@ -623,7 +665,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--case", default="step",
-                    choices=["step", "window-only", "decode-only", "trajectory", "tail-influence", "decode"],
+                    choices=["step", "window-only", "decode-only", "trajectory", "tail-influence", "decode",
+                             "drift"],
                     help="window-only / decode-only: small profiling cases (window layers only / "
                          "the last layer and its first-step row); trajectory: the recovery policy "
                          "over a synthetic continual-adapter trajectory; tail-influence: the offline "
@@ -650,6 +693,8 @@ def main():
         return run_tail_case(args)
     if args.case == "decode":
         return run_decode_case(args)
+    if args.case == "drift":
+        return run_drift_case(args)
     if args.warmup < 3 and args.impl == "crf":
         args.warmup = 3
     if args.impl == "reference":

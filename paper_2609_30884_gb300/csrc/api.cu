@@ -1014,9 +1014,11 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
 }
 
 // ---------------------------------------------------------------- drift
-static int drift_blocks_per_side(const crf_ctx* ctx, int n_items) {
-  const int want = (4 * ctx->num_sms + 2 * n_items - 1) / std::max(1, 2 * n_items);
-  return std::max(1, std::min(16, want));
+// Blocks per Gram side: enough that the longest side (the ffn or the hidden rows) is cut into
+// pieces of <= 768 rows, so no block runs far longer than the rest.
+static int drift_blocks_per_side(const crf_model_dims& d) {
+  const int longest = std::max(std::max(d.hidden, d.ffn), d.n_q_heads * d.head_dim);
+  return std::max(1, std::min(32, (longest + 767) / 768));
 }
 
 crf_status crf_decode_workspace_size(crf_ctx* ctx, const crf_model* model, const crf_lora_dims* lora,
@@ -1118,7 +1120,7 @@ crf_status crf_drift_workspace_size(crf_ctx* ctx, const crf_model_dims* dims,
   int nm = 0;
   for (int m = 0; m < 7; ++m) nm += (lora->module_mask >> m) & 1;
   const int items = dims->n_layers * nm;
-  const int bps = drift_blocks_per_side(ctx, std::max(1, items));
+  const int bps = drift_blocks_per_side(*dims);
   const size_t r2 = 2 * lora->rank;
   *bytes = align256(static_cast<size_t>(items) * 2 * bps * r2 * r2 * sizeof(float));
   return CRF_OK;
@@ -1161,7 +1163,7 @@ crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   CRF_CUDA(cudaMemsetAsync(out_sq, 0, static_cast<size_t>(D.N) * 7 * 2 * sizeof(float), st));
   if (items.empty()) return CRF_OK;
-  const int bps = drift_blocks_per_side(ctx, static_cast<int>(items.size()));
+  const int bps = drift_blocks_per_side(*dims);
   ProfScope ps(ctx, kPDrift, st, 2 * ((static_cast<int>(items.size()) + 223) / 224));
   CRF_CUDA(launch_drift(items.data(), static_cast<int>(items.size()), cur->dims.rank,
                         static_cast<float*>(workspace), bps, out_sq, st));

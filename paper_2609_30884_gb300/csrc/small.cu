@@ -435,7 +435,8 @@ __global__ void __launch_bounds__(256) drift_partial_kernel(const __grid_constan
   const int item = blockIdx.z, side = blockIdx.y, blk = blockIdx.x;
   const DriftItem& it = batch.items[item];
   const int L = side == 0 ? it.out_dim : it.in_dim;
-  const int per = (L + blocks_per_side - 1) / blocks_per_side;
+  // pieces of whole 128-row chunks, so every chunk starts 16-byte aligned (L % 8 == 0)
+  const int per = (((L + blocks_per_side - 1) / blocks_per_side + kDriftRows - 1) / kDriftRows) * kDriftRows;
   const int l0 = blk * per, l1 = min(L, l0 + per);
   __shared__ float vec[kDriftRows][R2 + 1];
   constexpr int T = R2 / 4;  // 4x4 tiles per dimension
@@ -453,19 +454,33 @@ __global__ void __launch_bounds__(256) drift_partial_kernel(const __grid_constan
   for (int c0 = l0; c0 < l1; c0 += kDriftRows) {
     const int cn = min(kDriftRows, l1 - c0);
     __syncthreads();
-    for (int i = tid; i < cn * R; i += 256) {
+    // 4 consecutive bf16 per thread (8-byte loads): B rows are contiguous in k, A rows in the
+    // input dimension; cn and R are multiples of 4
+    for (int i = tid; i < cn * R / 4; i += 256) {
       if (side == 0) {
-        const int rr = i / R, k = i % R;
+        const int rr = i / (R / 4), k = (i % (R / 4)) * 4;
         const size_t off = (size_t)(c0 + rr) * R + k;
-        const float b0 = __bfloat162float(it.B0[off]), b1 = __bfloat162float(it.B1[off]);
-        vec[rr][k] = b1 - b0;
-        vec[rr][R + k] = b0;
+        const uint2 u0 = *reinterpret_cast<const uint2*>(it.B0 + off);
+        const uint2 u1 = *reinterpret_cast<const uint2*>(it.B1 + off);
+        const float b0[4] = {bf16_lo(u0.x), bf16_hi(u0.x), bf16_lo(u0.y), bf16_hi(u0.y)};
+        const float b1[4] = {bf16_lo(u1.x), bf16_hi(u1.x), bf16_lo(u1.y), bf16_hi(u1.y)};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          vec[rr][k + e] = b1[e] - b0[e];
+          vec[rr][R + k + e] = b0[e];
+        }
       } else {
-        const int k = i / cn, rr = i % cn;  // coalesced along the input dimension
+        const int k = i / (cn / 4), rr = (i % (cn / 4)) * 4;  // coalesced along the input dimension
         const size_t off = (size_t)k * it.in_dim + c0 + rr;
-        const float a0 = __bfloat162float(it.A0[off]), a1 = __bfloat162float(it.A1[off]);
-        vec[rr][k] = a1;
-        vec[rr][R + k] = a1 - a0;
+        const uint2 u0 = *reinterpret_cast<const uint2*>(it.A0 + off);
+        const uint2 u1 = *reinterpret_cast<const uint2*>(it.A1 + off);
+        const float a0[4] = {bf16_lo(u0.x), bf16_hi(u0.x), bf16_lo(u0.y), bf16_hi(u0.y)};
+        const float a1[4] = {bf16_lo(u1.x), bf16_hi(u1.x), bf16_lo(u1.y), bf16_hi(u1.y)};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          vec[rr + e][k] = a1[e];
+          vec[rr + e][R + k] = a1[e] - a0[e];
+        }
       }
     }
     __syncthreads();
@@ -482,23 +497,20 @@ __global__ void __launch_bounds__(256) drift_partial_kernel(const __grid_constan
         for (int b = 0; b < 4; ++b) acc[a][b] += x[a] * y[b];
     }
   }
-  // reduce the groups through shared memory (reuse vec as [GROUPS][R2*R2] is too big; do it in steps)
-  __shared__ float red[R2 * R2];
-  for (int gg = 0; gg < GROUPS; ++gg) {
-    __syncthreads();
-    if (grp == gg) {
+  // every thread's 4x4 tile into [GROUPS][R2 * R2] (256 x 16 floats whatever R2 is), then each
+  // output summed over the row groups in a fixed order
+  __shared__ float part[GROUPS * R2 * R2];
 #pragma unroll
-      for (int a = 0; a < 4; ++a)
+  for (int a = 0; a < 4; ++a)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          float& dst = red[(ti * 4 + a) * R2 + tj * 4 + b];
-          dst = (gg == 0 ? 0.f : dst) + acc[a][b];
-        }
-    }
-  }
+    for (int b = 0; b < 4; ++b) part[grp * R2 * R2 + (ti * 4 + a) * R2 + tj * 4 + b] = acc[a][b];
   __syncthreads();
   float* out = grams + (((size_t)item * 2 + side) * blocks_per_side + blk) * R2 * R2;
-  for (int i = tid; i < R2 * R2; i += 256) out[i] = red[i];
+  for (int i = tid; i < R2 * R2; i += 256) {
+    float v = 0.f;
+    for (int gg = 0; gg < GROUPS; ++gg) v += part[gg * R2 * R2 + i];
+    out[i] = v;
+  }
 }
 
 template <int R2>
