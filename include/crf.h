@@ -95,6 +95,7 @@ typedef struct crf_lora_dims {
 /* Base weights of one layer (device pointers, bf16):
  *   W[m]    [out_m, in_m]   q:[Hq*d,h] k,v:[Hkv*d,h] o:[h,Hq*d] gate,up:[f,h] down:[h,f]
  *   bias[j] [out_j] for q,k,v (j = 0..2), used iff dims.qkv_bias
+ * Every W[m] and bias[j] starts on a 16-byte boundary (CRF_EINVAL otherwise).
  *   ln1/ln2 [h] RMSNorm gains before attention / before the MLP. */
 typedef struct crf_layer_weights {
   const void* W[CRF_NUM_MODULES];

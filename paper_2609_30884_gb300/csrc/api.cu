@@ -237,7 +237,8 @@ crf_status check_model_layers(const crf_model* model, int l0, int l1, const Dims
     if (!w.ln1 || !w.ln2) return fail(CRF_EINVAL, "layer %d norm gain is null", l);
     if (D.bias)
       for (int j = 0; j < 3; ++j)
-        if (!w.bias[j]) return fail(CRF_EINVAL, "layer %d qkv bias %d is null", l, j);
+        if (!w.bias[j] || !aligned16(w.bias[j]))
+          return fail(CRF_EINVAL, "layer %d qkv bias %d null or misaligned", l, j);
   }
   return CRF_OK;
 }

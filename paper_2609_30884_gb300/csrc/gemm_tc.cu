@@ -163,9 +163,25 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
   if (a.epi == kEpiScaleBf16 || a.epi == kEpiResid) {
     const int col0 = tl.n_loc * BN;
     const int ncols = a.group_cols[tl.g];
+    const bool resid = a.epi == kEpiResid;
+    // residual chunk c + 16 is requested while chunk c is drained: its load latency overlaps
+    auto load_resid = [&](int col, float (&dst)[16]) {
+      const int n = min(16, ncols - col);
+      if (n >= 16) {
+        load16_bf16(a.resid + (size_t)row * a.ld_resid + col, dst);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          dst[j] = j < n ? __bfloat162float(a.resid[(size_t)row * a.ld_resid + col + j]) : 0.f;
+      }
+    };
+    float wn[16];
+    if (resid && row_ok && col0 < ncols) load_resid(col0, w);
 #pragma unroll 1
     for (int c = 0; c < BN; c += 16) {
       tmem_ld16(tacc + c, r0);
+      const bool more = resid && row_ok && c + 16 < BN && col0 + c + 16 < ncols;
+      if (more) load_resid(col0 + c + 16, wn);
       tmem_ld_wait();
       const int col = col0 + c;
       if (!row_ok || col >= ncols) continue;
@@ -182,17 +198,14 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
         store_bf16_n(a.out + (size_t)row * a.ldo + 2 * col, v, n);
         continue;
       } else {
-        if (n >= 16) {
-          load16_bf16(a.resid + (size_t)row * a.ld_resid + col, w);
-        } else {
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            w[j] = j < n ? __bfloat162float(a.resid[(size_t)row * a.ld_resid + col + j]) : 0.f;
-        }
 #pragma unroll
         for (int j = 0; j < 16; ++j) v[j] = w[j] + __uint_as_float(r0[j]);
       }
       store_bf16_n(a.out + (size_t)row * a.ldo + col, v, n);
+      if (more) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) w[j] = wn[j];
+      }
     }
     return;
   }
@@ -240,13 +253,27 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
       head_stride = (size_t)kPage * d;
     }
   }
-  const float2* rope_row = a.rope + (size_t)pos * half;
+  // Chunks of 16 rotation pairs outermost: a chunk's cos/sin (one row of the angle table,
+  // shared by every head of the tile) is loaded once, and the next chunk's is requested
+  // while this one is applied, so the table's load latency overlaps the TMEM drain.
+  const bool rot = have && g < 2;
+  const float4* rope4 = reinterpret_cast<const float4*>(a.rope + (size_t)pos * half);
+  float4 cs[8], csn[8];
+  if (rot) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) cs[k] = rope4[k];
+  }
 #pragma unroll 1
-  for (int hh = 0; hh < BN / d; ++hh) {
-    const int head = (tl.n_loc * BN) / d + hh;
-    const int gcol = head * d;
+  for (int i0 = 0; i0 < half; i0 += 16) {
+    const bool more = rot && i0 + 16 < half;
+    if (more) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) csn[k] = rope4[(i0 + 16) / 2 + k];
+    }
 #pragma unroll 1
-    for (int i0 = 0; i0 < half; i0 += 16) {
+    for (int hh = 0; hh < BN / d; ++hh) {
+      const int head = (tl.n_loc * BN) / d + hh;
+      const int gcol = head * d;
       tmem_ld16(tacc + hh * d + i0, r0);
       tmem_ld16(tacc + hh * d + half + i0, r1);
       tmem_ld_wait();
@@ -257,24 +284,32 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
         w[j] = __uint_as_float(r1[j]);
       }
       if (bias) {
+        float b0[16], b1[16];
+        load16_bf16(bias + gcol + i0, b0);
+        load16_bf16(bias + gcol + half + i0, b1);
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
-          v[j] += __bfloat162float(bias[gcol + i0 + j]);
-          w[j] += __bfloat162float(bias[gcol + half + i0 + j]);
+          v[j] += b0[j];
+          w[j] += b1[j];
         }
       }
       if (g < 2) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
-          const float2 cs = rope_row[i0 + j];
+          const float c = (j & 1) ? cs[j >> 1].z : cs[j >> 1].x;
+          const float sn = (j & 1) ? cs[j >> 1].w : cs[j >> 1].y;
           const float x1 = v[j], x2 = w[j];
-          v[j] = x1 * cs.x - x2 * cs.y;
-          w[j] = x2 * cs.x + x1 * cs.y;
+          v[j] = x1 * c - x2 * sn;
+          w[j] = x2 * c + x1 * sn;
         }
       }
       __nv_bfloat16* dst = dst_row + head * head_stride;
       store16_bf16(dst + i0, v);
       store16_bf16(dst + half + i0, w);
+    }
+    if (more) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) cs[k] = csn[k];
     }
   }
 }
@@ -492,10 +527,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       tc_fence_after();
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
       epilogue_tile<BN>(a, tl, tacc, tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM + row_in_cta);
+      // the accumulator is free once this warp's TMEM loads have completed (tcgen05.wait::ld in
+      // the epilogue); the tile's global stores need not be visible first, so the arrival on
+      // the MMA-issuing CTA's barrier is relaxed
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        if constexpr (PAIR == 2) mbar_arrive_cluster(tempty_addr[acc]); else mbar_arrive(&tempty_bar[acc]);
+        if constexpr (PAIR == 2) mbar_arrive_cluster_relaxed(tempty_addr[acc]); else mbar_arrive(&tempty_bar[acc]);
       }
     }
   }

@@ -167,3 +167,34 @@ def test_qwen7b_16k_window_layer_sampled(ctx):
             assert torch.equal(free_slots(pool.v_pages[l], free), free_slots(bv[l], free))
         else:
             assert torch.equal(pool.k_pages[l], bk[l])
+
+
+def test_misaligned_bias_rejected(ctx):
+    """The QKV epilogue reads biases as 16-byte vectors: a bias pointer off that boundary is
+    refused on the host (CRF_EINVAL) before anything is launched, and the pages stay untouched."""
+    import paper_2609_30884_gb300 as crf
+    cfg = replace(synth.QWEN15B, name="qwen2.5-1.5b-shape-2l", n_layers=2)
+    lc = synth.LORA_QWEN
+    dm = DeviceModel(cfg, with_head=False)
+    cur = DeviceAdapter(cfg, lc, 1)
+    n = 256
+    P = pages_needed(n)
+    pool = make_pool(cfg, P)
+    pt = split_page_tables([n], P, seed=3)[0]
+    h = synth.hidden_state(cfg, n, device="cuda")
+    layers = [dict(w) for w in dm.layers]
+    b = layers[1]["bias_k"]
+    padded = torch.empty(b.numel() + 1, dtype=b.dtype, device=b.device)
+    padded[1:].copy_(b)
+    layers[1]["bias_k"] = padded[1:]  # starts 2 bytes past a 16-byte boundary
+    bad = crf.Model(dm.crf.dims, layers)
+    req = crf.Request(pt, 1, 2, hidden_in=h)
+    ws = ctx.workspace(bad, cur.crf, [req])
+    bk = [k.clone() for k in pool.k_pages]
+    with pytest.raises(crf.CrfError) as ei:
+        ctx.recompute_window(bad, cur.crf, pool, [req], ws)
+    assert ei.value.status == crf.abi.EINVAL
+    torch.cuda.synchronize()
+    assert all(torch.equal(a, c) for a, c in zip(pool.k_pages, bk))
+    ctx.recompute_window(dm.crf, cur.crf, pool, [req], ws)  # the aligned model still runs
+    ctx.check()
