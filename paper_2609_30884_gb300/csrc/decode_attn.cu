@@ -13,8 +13,9 @@
 //                       P stays in registers as the A operand of P V, and the warps' partial
 //                       products are summed in shared memory in a fixed order. The chunk's
 //                       (max, sum, unnormalised o) are written in log2 units;
-//   decode_attn_merge   one block per (query head, row): rescales the chunk partials to
-//                       the common max and normalises.
+//   decode_attn_merge   one block per (query head, row, 32-column slice): rescales the chunk
+//                       partials to the common max and normalises, every chunk's loads
+//                       independent of the others.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -279,47 +280,37 @@ __global__ void __launch_bounds__(kThreadsChunk) decode_attn_chunk(const __grid_
   }
 }
 
-// One block per (query head, row): warp w takes chunks w, w + 8, ...; lane covers D / 32 dims.
+// One block per (query head, row, 32-column slice of o): warp w takes chunks w, w + 4, ...
+// (each chunk's loads independent of the others), lane = one output column; the warps'
+// sums meet in a fixed order.
 template <int D>
-__global__ void __launch_bounds__(256) decode_attn_merge(const DecodeAttnDesc p) {
-  constexpr int DPL = D / 32;
+__global__ void __launch_bounds__(128) decode_attn_merge(const DecodeAttnDesc p) {
   const int h = blockIdx.x, r = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int col = blockIdx.z * 32 + lane;
   const int n_chunks = p.pos[r] / kChunk + 1;
   const float* base = p.part + ((size_t)r * p.n_q_heads + h) * p.splits * (D + 2);
-  __shared__ float red[8];
-  __shared__ float red_o[8][D];
-  __shared__ float red_l[8];
+  __shared__ float red_m[4], red_l[4], red_o[4][32];
   float m = -INFINITY;
-  for (int s = tid; s < n_chunks; s += 256) m = fmaxf(m, base[(size_t)s * (D + 2) + D]);
+  for (int s = tid; s < n_chunks; s += 128) m = fmaxf(m, base[(size_t)s * (D + 2) + D]);
   m = warp_max(m);
-  if (lane == 0) red[warp] = m;
+  if (lane == 0) red_m[warp] = m;
   __syncthreads();
-  m = red[0];
-#pragma unroll
-  for (int i = 1; i < 8; ++i) m = fmaxf(m, red[i]);
-  float acc[DPL], l = 0.f;
-#pragma unroll
-  for (int e = 0; e < DPL; ++e) acc[e] = 0.f;
-#pragma unroll 4
-  for (int s = warp; s < n_chunks; s += 8) {
+  m = fmaxf(fmaxf(red_m[0], red_m[1]), fmaxf(red_m[2], red_m[3]));
+  float acc = 0.f, l = 0.f;
+#pragma unroll 8
+  for (int s = warp; s < n_chunks; s += 4) {
     const float* ps = base + (size_t)s * (D + 2);
     const float f = ex2_approx(ps[D] - m);
     l += f * ps[D + 1];
-#pragma unroll
-    for (int e = 0; e < DPL; ++e) acc[e] += f * ps[lane * DPL + e];
+    acc += f * ps[col];
   }
-#pragma unroll
-  for (int e = 0; e < DPL; ++e) red_o[warp][lane * DPL + e] = acc[e];
+  red_o[warp][lane] = acc;
   if (lane == 0) red_l[warp] = l;
   __syncthreads();
-  if (tid < D) {
-    float o = 0.f, L = 0.f;
-#pragma unroll
-    for (int w = 0; w < 8; ++w) {
-      o += red_o[w][tid];
-      L += red_l[w];
-    }
-    p.out[(size_t)r * p.n_q_heads * D + h * D + tid] = o / L;
+  if (warp == 0) {
+    const float o = (red_o[0][lane] + red_o[1][lane]) + (red_o[2][lane] + red_o[3][lane]);
+    const float L = (red_l[0] + red_l[1]) + (red_l[2] + red_l[3]);
+    p.out[(size_t)r * p.n_q_heads * D + h * D + col] = o / L;
   }
 }
 
@@ -364,7 +355,7 @@ cudaError_t launch_dec(const DecodeArgs& args, int chunks, cudaStream_t stream) 
   }
   const DecodeAttnDesc& d = args.d;
   decode_attn_chunk<D><<<dim3(chunks, d.n_kv_heads, d.rows), kThreadsChunk, smem, stream>>>(args);
-  decode_attn_merge<D><<<dim3(d.n_q_heads, d.rows), 256, 0, stream>>>(d);
+  decode_attn_merge<D><<<dim3(d.n_q_heads, d.rows, D / 32), 128, 0, stream>>>(d);
   return cudaGetLastError();
 }
 
