@@ -140,12 +140,16 @@ def algorithmic_work(cfg, lc, n):
         "gemm_o_resid": 2 * n * qd * h + up("o", h),
         "gemm_gateup_swiglu": 2 * n * h * 2 * f + up("gate", f) + up("up", f),
         "gemm_down_resid": 2 * n * f * h + up("down", h),
-        # down product x A^T of every adapted module: 2 n r in_m
-        "gemm_lora_down": 2 * n * r * (h * sum(ad(m) for m in ("q", "k", "v", "gate", "up"))
-                                       + qd * ad("o") + f * ad("down")),
         "attn_prefill_paged": 4 * cfg.n_q_heads * cfg.head_dim * n * (n + 1) // 2,
     }
-    byts = {"rmsnorm": 2 * (2 * n * h * 2)}   # two norms, read + write bf16
+    byts = {"rmsnorm": 2 * (2 * n * h * 2),   # two norms, read + write bf16
+            # down products x A^T (2 n r in_m FLOP, HBM-bound): each distinct input read once
+            # (the q/k/v and the gate/up modules share theirs), a bf16 hi/lo pair of r columns
+            # written per adapted module
+            "gemm_lora_down": 2 * n * (h * any(ad(m) for m in ("q", "k", "v"))
+                                       + h * any(ad(m) for m in ("gate", "up"))
+                                       + qd * ad("o") + f * ad("down"))
+                              + n * 2 * r * 2 * sum(ad(m) for m in ("q", "k", "v", "o", "gate", "up", "down"))}
     return flops, byts
 
 
