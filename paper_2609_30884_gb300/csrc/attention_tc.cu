@@ -31,8 +31,9 @@
 // K/V slot layout: the 128 keys of a tile in 16 groups of 8 keys, group c at
 // c * HALVES * 1024 bytes, and within a group one 1 KB 128B-swizzled atom per
 // 64-column half of the head dimension. A page (two groups, both halves) is
-// then one contiguous 4 KB box of a 4-D view of the pool, so a kv tile costs
-// 8 copies instead of 16 per half; both MMAs see a uniform 8-row stride.
+// then one contiguous 4 KB box of a 4-D view of the pool: a K or V tile is 8
+// copies (one per page, 16 with one copy per page and half); both MMAs see a
+// uniform 8-row stride.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -279,65 +280,65 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
       }
     } else if (warp == 1) {
       // -------------------------------------------------------------- MMA issuer
-    // Order: S0(0) S1(0) | PV0(j) S0(j+1) PV1(j) S1(j+1) | ... so that the softmax of one
-    // query tile overlaps the products of the other; query tile 0 stops one kv tile early
-    // (its diagonal), after which tile 1 runs alone. tcgen05.mma of one thread execute in
-    // issue order, so S_t(j+1) overwrites the S/P columns only after PV_t(j) has read P_t(j).
-    if (lane == 0) {
-      bool ok = mbar_wait(&q_full, 0, &abort_flag, a.status);
-      bool issued = false;
-      const uint32_t idesc_s = idesc_bf16_f32(kM, kN);
-      const uint32_t idesc_o = idesc_bf16_f32(kM, D, false, true);
-      // ring position of sequence item i (K(j): i = 2j, V(j): i = 2j + 1)
-      auto slot_of = [](int i) { return i % kSlots; };
-      auto parity_of = [](int i) { return static_cast<uint32_t>((i / kSlots) & 1); };
-      auto issue_s = [&](int t, int ks) {
-        const uint32_t kb = smem_u32(sKV + ks * KV_BYTES);
-        const uint32_t qb = smem_u32(sQ + t * Q_BYTES);
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t in_row = (kk & 3) * 32;
-          mma_bf16_ss(tmem + t * 128,
-                      smem_desc(qb + (kk >> 2) * HALF_ROWS_BYTES + in_row, 16, 1024, kSwizzle128B),
-                      smem_desc(kb + (kk >> 2) * 1024 + in_row, 16, GROUP_BYTES, kSwizzle128B),
-                      idesc_s, kk > 0 ? 1u : 0u);
-        }
-        mma_commit(&s_full[t]);
-      };
-      if (ok) ok = mbar_wait(&kv_full[slot_of(0)], parity_of(0), &abort_flag, a.status);
-      if (ok) {
-        tc_fence_after();
-        for (int t = 0; t < ntiles; ++t) issue_s(t, slot_of(0));
-        issued = true;
-      }
-      for (int j = 0; j < J && ok; ++j) {
-        const uint32_t vb = smem_u32(sKV + slot_of(2 * j + 1) * KV_BYTES);
-        const int ks = slot_of(2 * j + 2);
-        for (int t = (j < J0 ? 0 : 1); t < ntiles; ++t) {
-          // phase j of p_full[t]: P_t(j) is in TMEM, and V(j) and K(j + 1) have landed
-          if (!mbar_wait(&p_full[t], j & 1, &abort_flag, a.status)) {
-            ok = false;
-            break;
+      // Order: S0(0) S1(0) | PV0(j) S0(j+1) PV1(j) S1(j+1) | ... so that the softmax of one
+      // query tile overlaps the products of the other; query tile 0 stops one kv tile early
+      // (its diagonal), after which tile 1 runs alone. tcgen05.mma of one thread execute in
+      // issue order, so S_t(j+1) overwrites the S/P columns only after PV_t(j) has read P_t(j).
+      if (lane == 0) {
+        bool ok = mbar_wait(&q_full, 0, &abort_flag, a.status);
+        bool issued = false;
+        const uint32_t idesc_s = idesc_bf16_f32(kM, kN);
+        const uint32_t idesc_o = idesc_bf16_f32(kM, D, false, true);
+        // ring position of sequence item i (K(j): i = 2j, V(j): i = 2j + 1)
+        auto slot_of = [](int i) { return i % kSlots; };
+        auto parity_of = [](int i) { return static_cast<uint32_t>((i / kSlots) & 1); };
+        auto issue_s = [&](int t, int ks) {
+          const uint32_t kb = smem_u32(sKV + ks * KV_BYTES);
+          const uint32_t qb = smem_u32(sQ + t * Q_BYTES);
+  #pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t in_row = (kk & 3) * 32;
+            mma_bf16_ss(tmem + t * 128,
+                        smem_desc(qb + (kk >> 2) * HALF_ROWS_BYTES + in_row, 16, 1024, kSwizzle128B),
+                        smem_desc(kb + (kk >> 2) * 1024 + in_row, 16, GROUP_BYTES, kSwizzle128B),
+                        idesc_s, kk > 0 ? 1u : 0u);
           }
+          mma_commit(&s_full[t]);
+        };
+        if (ok) ok = mbar_wait(&kv_full[slot_of(0)], parity_of(0), &abort_flag, a.status);
+        if (ok) {
           tc_fence_after();
-#pragma unroll
-          for (int kk = 0; kk < kN / 16; ++kk) {
-            // P: 16 keys = 8 packed bf16x2 columns; V: 16 key rows = two 8-key groups
-            mma_bf16_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
-                        smem_desc(vb + kk * 2 * GROUP_BYTES, 1024, GROUP_BYTES, kSwizzle128B), idesc_o,
-                        (j > 0 || kk > 0) ? 1u : 0u);
+          for (int t = 0; t < ntiles; ++t) issue_s(t, slot_of(0));
+          issued = true;
+        }
+        for (int j = 0; j < J && ok; ++j) {
+          const uint32_t vb = smem_u32(sKV + slot_of(2 * j + 1) * KV_BYTES);
+          const int ks = slot_of(2 * j + 2);
+          for (int t = (j < J0 ? 0 : 1); t < ntiles; ++t) {
+            // phase j of p_full[t]: P_t(j) is in TMEM, and V(j) and K(j + 1) have landed
+            if (!mbar_wait(&p_full[t], j & 1, &abort_flag, a.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+  #pragma unroll
+            for (int kk = 0; kk < kN / 16; ++kk) {
+              // P: 16 keys = 8 packed bf16x2 columns; V: 16 key rows = two 8-key groups
+              mma_bf16_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
+                          smem_desc(vb + kk * 2 * GROUP_BYTES, 1024, GROUP_BYTES, kSwizzle128B), idesc_o,
+                          (j > 0 || kk > 0) ? 1u : 0u);
+            }
+            if (j + 1 < (t == 0 ? J0 : J)) issue_s(t, ks);
           }
-          if (j + 1 < (t == 0 ? J0 : J)) issue_s(t, ks);
+        }
+        if (ok) {
+          mma_commit(&o_full);
+        } else if (issued) {
+          mma_commit(&drain_bar);
+          volatile int never = 0;
+          mbar_wait(&drain_bar, 0, &never, nullptr);
         }
       }
-      if (ok) {
-        mma_commit(&o_full);
-      } else if (issued) {
-        mma_commit(&drain_bar);
-        volatile int never = 0;
-        mbar_wait(&drain_bar, 0, &never, nullptr);
-      }
-    }
     }
   } else {
     regs_inc_softmax();
