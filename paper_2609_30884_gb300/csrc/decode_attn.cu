@@ -27,9 +27,27 @@ namespace crf {
 
 namespace {
 
-constexpr int kChunk = 128;                     // positions per block
-constexpr int kThreadsChunk = 128;
+constexpr int kChunk = 128;                     // positions per chunk
+constexpr int kThreadsStream = 160;             // four compute warps + one copy warp
 constexpr int kMaxGroup = 8;
+
+__device__ __forceinline__ void named_bar_sync_dec(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+// Named barrier that also ANDs a flag over its threads: the compute warps take every later
+// barrier together even when one of them gave up on a timed-out wait.
+__device__ __forceinline__ bool named_bar_and_dec(int id, int nthreads, bool flag) {
+  uint32_t out;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.and.pred po, %2, %3, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(out)
+      : "r"(flag ? 1u : 0u), "r"(id), "r"(nthreads)
+      : "memory");
+  return out != 0;
+}
 
 struct DecodeArgs {
   CUtensorMap tmK;  // K pool of the layer viewed as [pages*Hkv*16, d], box {64, 16}
@@ -39,59 +57,98 @@ struct DecodeArgs {
 };
 
 template <int D>
-__global__ void __launch_bounds__(kThreadsChunk) decode_attn_chunk(const __grid_constant__ DecodeArgs a) {
+__global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __grid_constant__ DecodeArgs a) {
   constexpr int HALVES = D / 64;
   constexpr int HALF = kChunk * 128;     // bytes of one 64-column half of a K (or V) tile
   constexpr int TILE = HALVES * HALF;
   constexpr int QHALF = 16 * 128;        // one 64-column half of the 16-row Q tile
   const DecodeAttnDesc& p = a.d;
-  const int r = blockIdx.z, g = blockIdx.y, chunk = blockIdx.x;
+  // block -> (row, kv head, its chunks c_beg .. c_end - 1, partial slot)
+  int r = -1, g = 0, slot = 0, c_beg = 0, c_end = 0;
+  {
+    int b = blockIdx.x;
+    for (int i = 0; i < p.rows; ++i) {
+      const int chunks = p.pos[i] / kChunk + 1;
+      const int bpp = (chunks + p.chunks_per_block - 1) / p.chunks_per_block;
+      if (b < bpp * p.n_kv_heads) {
+        r = i;
+        g = b / bpp;
+        slot = b % bpp;
+        c_beg = slot * p.chunks_per_block;
+        c_end = min(chunks, c_beg + p.chunks_per_block);
+        break;
+      }
+      b -= bpp * p.n_kv_heads;
+    }
+  }
+  if (r < 0) return;
   const int pos = p.pos[r];
-  const int t0 = chunk * kChunk;
-  if (t0 > pos) return;
   const int grp = p.n_q_heads / p.n_kv_heads;
-  const int n_cached = min(kChunk, pos - t0);               // cached keys of this chunk
-  const bool has_self = pos < t0 + kChunk;                  // the row's own key falls here
-  const int n_valid = n_cached + (has_self ? 1 : 0);
-  const int pages = (n_cached + kPage - 1) / kPage;
+  const bool self_here = c_end - 1 == pos / kChunk;  // the chunk holding the row's own position
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sK = smem;
-  uint8_t* sV = smem + TILE;
-  uint8_t* sQ = smem + 2 * TILE;                            // hi: [HALVES][16 rows][128 B], swizzled
+  uint8_t* sKV = smem;                                      // [2 stages][K tile | V tile]
+  uint8_t* sQ = smem + 4 * TILE;                            // hi: [HALVES][16 rows][128 B], swizzled
   uint8_t* sQl = sQ + HALVES * QHALF;                       // lo, same layout
-  __shared__ __align__(16) float o_red[16][D];
-  __shared__ float red_m[kThreadsChunk / 32][16], red_l[kThreadsChunk / 32][16];
-  __shared__ float s_self[16], p_self[16];  // the row's own key: fp32 score, then weight
-  __shared__ __align__(8) uint64_t full;
+  __shared__ float red_m[4][16], red_l[4][16];
+  __shared__ float s_self[16];  // the row's own key, scored in fp32
+  __shared__ __align__(8) uint64_t full[2], empty[2];
   __shared__ volatile int abort_flag;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
-    mbar_init(&full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 4);
+    }
     abort_flag = 0;
     fence_barrier_init();
   }
   __syncthreads();
-  if (tid == 0 && pages > 0) {
-    const int32_t* pt = p.page_table[r];
-    mbar_arrive_expect_tx(&full, 2 * pages * HALVES * kPage * 128);
-    for (int i = 0; i < pages; ++i) {
-      const int row = (pt[t0 / kPage + i] * p.n_kv_heads + g) * kPage;
-      for (int h = 0; h < HALVES; ++h) {
-        const int off = h * HALF + i * (kPage * 128);
-        tma_load_2d(sK + off, &a.tmK, &full, 64 * h, row);
-        tma_load_2d(sV + off, &a.tmV, &full, 64 * h, row);
+
+  if (warp == 4) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      const int32_t* pt = p.page_table[r];
+      int armed[2] = {-1, -1};
+      for (int c = c_beg; c < c_end; ++c) {
+        const int i = c - c_beg, st = i & 1;
+        if (i >= 2 && !mbar_wait(&empty[st], ((i >> 1) - 1) & 1, &abort_flag, a.status)) break;
+        const int t0 = c * kChunk;
+        const int pages = (min(kChunk, pos - t0) + kPage - 1) / kPage;
+        uint8_t* sK = sKV + st * 2 * TILE;
+        uint8_t* sV = sK + TILE;
+        if (pages == 0) {
+          mbar_arrive(&full[st]);  // only the row's own key here: nothing to copy
+        } else {
+          mbar_arrive_expect_tx(&full[st], 2 * pages * HALVES * kPage * 128);
+          for (int pg = 0; pg < pages; ++pg) {
+            const int row = (pt[t0 / kPage + pg] * p.n_kv_heads + g) * kPage;
+            for (int h = 0; h < HALVES; ++h) {
+              const int off = h * HALF + pg * (kPage * 128);
+              tma_load_2d(sK + off, &a.tmK, &full[st], 64 * h, row);
+              tma_load_2d(sV + off, &a.tmV, &full[st], 64 * h, row);
+            }
+          }
+          armed[st] = (i >> 1) & 1;
+        }
       }
+      // copies still in flight land before the block's shared memory is released
+      volatile int never = 0;
+      for (int st = 0; st < 2; ++st)
+        if (armed[st] >= 0) mbar_wait(&full[st], armed[st], &never, nullptr);
     }
+    return;
   }
+
+  // -------------------------------------------------------------------- compute warps 0..3
   // q of the group's heads (rows >= grp zero) as bf16 hi + lo, pre-scaled so scores are in
   // log2 units
   const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
   const float* qrow0 = p.q + (size_t)r * p.n_q_heads * D + (size_t)(g * grp) * D;
-  for (int i = tid; i < 16 * (D / 2); i += kThreadsChunk) {
+  for (int i = tid; i < 16 * (D / 2); i += 128) {
     const int row = i / (D / 2), d = 2 * (i % (D / 2));
     float v0 = 0.f, v1 = 0.f;
     if (row < grp) {
@@ -105,175 +162,213 @@ __global__ void __launch_bounds__(kThreadsChunk) decode_attn_chunk(const __grid_
     *reinterpret_cast<uint32_t*>(sQ + off) = pack_bf16(h0, h1);
     *reinterpret_cast<uint32_t*>(sQl + off) = pack_bf16(v0 - h0, v1 - h1);
   }
-  // the row's own key, scored in fp32 (warp w takes heads w, w + 4)
-  if (has_self) {
+  if (self_here) {
+    // the row's own key, scored in fp32 (warp w takes heads w, w + 4)
     const float* ks = p.k_self + (size_t)r * p.n_kv_heads * D + g * D;
-    for (int h = warp; h < grp; h += kThreadsChunk / 32) {
+    for (int h = warp; h < grp; h += 4) {
       float dot = 0.f;
       for (int d = lane; d < D; d += 32) dot += qrow0[(size_t)h * D + d] * ks[d];
       dot = warp_sum(dot);
       if (lane == 0) s_self[h] = dot * qscale;
     }
   }
-  bool ok = true;
-  if (pages > 0) ok = mbar_wait(&full, 0, &abort_flag, a.status);
-  if (!__syncthreads_and(ok)) return;
-  // V rows from the row's own slot on are zeroed: its value is added in fp32 at the end, and
-  // 0 * stale data must not produce NaN in P V (masked scores need no cleaning)
-  if (has_self) {
-    for (int i = tid; i < (kChunk - n_cached) * HALVES * 8; i += kThreadsChunk) {
-      const int t2 = n_cached + i / (HALVES * 8);
-      const int hf = (i / 8) % HALVES, c = i % 8;
-      *reinterpret_cast<uint4*>(sV + hf * HALF + t2 * 128 + (c << 4)) = make_uint4(0, 0, 0, 0);
-    }
-  }
-  __syncthreads();
+  named_bar_sync_dec(1, 128);
 
-  // 1. S = Q K^T for this warp's 32 keys: 4 n-tiles of 8 keys
-  const uint32_t q_base = smem_u32(sQ), ql_base = smem_u32(sQl), k_base = smem_u32(sK),
-                 v_base = smem_u32(sV);
+  const uint32_t q_base = smem_u32(sQ), ql_base = smem_u32(sQl);
   const int mi = lane >> 3, li = lane & 7;  // ldmatrix: matrix index, row within it
-  float S[4][4];
-#pragma unroll
-  for (int nt = 0; nt < 4; ++nt)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) S[nt][e] = 0.f;
-#pragma unroll
-  for (int ks = 0; ks < D / 16; ++ks) {
-    const int hf = ks / 4;
-    uint32_t af[4], al[4];
-    {
-      const int row = (mi & 1) * 8 + li, c = 2 * (ks % 4) + (mi >> 1);
-      const uint32_t off = hf * QHALF + row * 128 + ((c ^ (row & 7)) << 4);
-      ldsm_x4(q_base + off, af[0], af[1], af[2], af[3]);
-      ldsm_x4(ql_base + off, al[0], al[1], al[2], al[3]);
-    }
-#pragma unroll
-    for (int np = 0; np < 2; ++np) {
-      const int key = warp * 32 + (2 * np + (mi >> 1)) * 8 + li, c = 2 * (ks % 4) + (mi & 1);
-      uint32_t b0, b1, b2, b3;
-      ldsm_x4(k_base + hf * HALF + key * 128 + ((c ^ (key & 7)) << 4), b0, b1, b2, b3);
-      mma16816(S[2 * np], af, b0, b1);
-      mma16816(S[2 * np + 1], af, b2, b3);
-      mma16816(S[2 * np], al, b0, b1);
-      mma16816(S[2 * np + 1], al, b2, b3);
-    }
-  }
-  // 2. mask, block row max, P = 2^(S - max), row sums
   const int r0 = lane >> 2, cq = 2 * (lane & 3);
-  float m0 = -INFINITY, m1 = -INFINITY;
+  // this warp's running state over its 32-key slice of every chunk: max and partial sum of
+  // rows r0 and r0 + 8 (log2 units), and its share of the unnormalised o
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  float O[D / 8][4];
 #pragma unroll
-  for (int nt = 0; nt < 4; ++nt)
+  for (int dn = 0; dn < D / 8; ++dn)
 #pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      const int key = warp * 32 + nt * 8 + cq + e;
-      const bool valid = key < n_valid;
-      S[nt][e] = valid ? S[nt][e] : -INFINITY;
-      S[nt][2 + e] = valid ? S[nt][2 + e] : -INFINITY;
-      if (has_self && key == n_cached) {
-        S[nt][e] = r0 < grp ? s_self[r0] : 0.f;
-        S[nt][2 + e] = r0 + 8 < grp ? s_self[r0 + 8] : 0.f;
+    for (int e = 0; e < 4; ++e) O[dn][e] = 0.f;
+  bool ok = true;
+  for (int c = c_beg; c < c_end; ++c) {
+    const int i = c - c_beg, st = i & 1;
+    const int t0 = c * kChunk;
+    const int n_cached = min(kChunk, pos - t0);  // cached keys of this chunk
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&full[st], (i >> 1) & 1, &abort_flag, a.status));
+    const uint32_t k_base = smem_u32(sKV + st * 2 * TILE), v_base = k_base + TILE;
+    if (n_cached < kChunk) {
+      // the last chunk: V rows from the row's own slot on are zeroed (its value is added in
+      // fp32 at the end, and 0 * stale data must not produce NaN in P V); all four warps read
+      // every row of V, so they meet before the products
+      if (ok) {
+        for (int q = tid; q < (kChunk - n_cached) * HALVES * 8; q += 128) {
+          const int t2 = n_cached + q / (HALVES * 8);
+          const int hf = (q / 8) % HALVES, cc = q % 8;
+          *reinterpret_cast<uint4*>(sKV + st * 2 * TILE + TILE + hf * HALF + t2 * 128 + (cc << 4)) =
+              make_uint4(0, 0, 0, 0);
+        }
       }
-      m0 = fmaxf(m0, S[nt][e]);
-      m1 = fmaxf(m1, S[nt][2 + e]);
+      ok = named_bar_and_dec(1, 128, ok);
     }
+    if (ok) {
+      // 1. S = Q K^T for this warp's 32 keys: 4 n-tiles of 8 keys
+      float S[4][4];
 #pragma unroll
-  for (int o = 1; o <= 2; o <<= 1) {
-    m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, o));
-    m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, o));
-  }
-  if ((lane & 3) == 0) {
-    red_m[warp][r0] = m0;
-    red_m[warp][r0 + 8] = m1;
-  }
-  __syncthreads();
-  float M0 = red_m[0][r0], M1 = red_m[0][r0 + 8];
+      for (int nt = 0; nt < 4; ++nt)
 #pragma unroll
-  for (int w = 1; w < kThreadsChunk / 32; ++w) {
-    M0 = fmaxf(M0, red_m[w][r0]);
-    M1 = fmaxf(M1, red_m[w][r0 + 8]);
-  }
-  float l0 = 0.f, l1 = 0.f;
+        for (int e = 0; e < 4; ++e) S[nt][e] = 0.f;
 #pragma unroll
-  for (int nt = 0; nt < 4; ++nt)
+      for (int ks = 0; ks < D / 16; ++ks) {
+        const int hf = ks / 4;
+        uint32_t af[4], al[4];
+        {
+          const int row = (mi & 1) * 8 + li, cc = 2 * (ks % 4) + (mi >> 1);
+          const uint32_t off = hf * QHALF + row * 128 + ((cc ^ (row & 7)) << 4);
+          ldsm_x4(q_base + off, af[0], af[1], af[2], af[3]);
+          ldsm_x4(ql_base + off, al[0], al[1], al[2], al[3]);
+        }
 #pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      S[nt][e] = ex2_approx(S[nt][e] - M0);
-      S[nt][2 + e] = ex2_approx(S[nt][2 + e] - M1);
-      l0 += S[nt][e];
-      l1 += S[nt][2 + e];
-      if (has_self && warp * 32 + nt * 8 + cq + e == n_cached) {
-        p_self[r0] = S[nt][e];
-        p_self[r0 + 8] = S[nt][2 + e];
+        for (int np = 0; np < 2; ++np) {
+          const int key = warp * 32 + (2 * np + (mi >> 1)) * 8 + li, cc = 2 * (ks % 4) + (mi & 1);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(k_base + hf * HALF + key * 128 + ((cc ^ (key & 7)) << 4), b0, b1, b2, b3);
+          mma16816(S[2 * np], af, b0, b1);
+          mma16816(S[2 * np + 1], af, b2, b3);
+          mma16816(S[2 * np], al, b0, b1);
+          mma16816(S[2 * np + 1], al, b2, b3);
+        }
+      }
+      // 2. mask the keys past this chunk's cached ones, online max / sum update of the slice
+      float c0 = -INFINITY, c1 = -INFINITY;
+#pragma unroll
+      for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const bool valid = warp * 32 + nt * 8 + cq + e < n_cached;
+          S[nt][e] = valid ? S[nt][e] : -INFINITY;
+          S[nt][2 + e] = valid ? S[nt][2 + e] : -INFINITY;
+          c0 = fmaxf(c0, S[nt][e]);
+          c1 = fmaxf(c1, S[nt][2 + e]);
+        }
+#pragma unroll
+      for (int o = 1; o <= 2; o <<= 1) {
+        c0 = fmaxf(c0, __shfl_xor_sync(0xffffffffu, c0, o));
+        c1 = fmaxf(c1, __shfl_xor_sync(0xffffffffu, c1, o));
+      }
+      const float n0 = fmaxf(m0, c0), n1 = fmaxf(m1, c1);
+      // a slice with nothing valid so far keeps max -inf: no rescale, P = 0
+      const float a0 = n0 == -INFINITY ? 1.f : ex2_approx(m0 - n0);
+      const float a1 = n1 == -INFINITY ? 1.f : ex2_approx(m1 - n1);
+      const float z0 = n0 == -INFINITY ? 0.f : n0, z1 = n1 == -INFINITY ? 0.f : n1;
+      m0 = n0;
+      m1 = n1;
+      l0 *= a0;
+      l1 *= a1;
+#pragma unroll
+      for (int dn = 0; dn < D / 8; ++dn) {
+        O[dn][0] *= a0;
+        O[dn][1] *= a0;
+        O[dn][2] *= a1;
+        O[dn][3] *= a1;
+      }
+#pragma unroll
+      for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          S[nt][e] = ex2_approx(S[nt][e] - z0);
+          S[nt][2 + e] = ex2_approx(S[nt][2 + e] - z1);
+          l0 += S[nt][e];
+          l1 += S[nt][2 + e];
+        }
+      // 3. O += P V over this warp's keys: P from the S fragments, V by transposing loads
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        uint32_t pa[4];
+        pa[0] = pack_bf16(S[2 * j][0], S[2 * j][1]);
+        pa[1] = pack_bf16(S[2 * j][2], S[2 * j][3]);
+        pa[2] = pack_bf16(S[2 * j + 1][0], S[2 * j + 1][1]);
+        pa[3] = pack_bf16(S[2 * j + 1][2], S[2 * j + 1][3]);
+        const int key = warp * 32 + 16 * j + (mi & 1) * 8 + li;
+#pragma unroll
+        for (int dp = 0; dp < D / 16; ++dp) {
+          const int gc = 2 * dp + (mi >> 1);  // 16-byte chunk of the row (8 dims)
+          const int hf = gc / 8, cc = gc % 8;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(v_base + hf * HALF + key * 128 + ((cc ^ (key & 7)) << 4), b0, b1, b2, b3);
+          mma16816(O[2 * dp], pa, b0, b1);
+          mma16816(O[2 * dp + 1], pa, b2, b3);
+        }
       }
     }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[st]);  // this warp is done with the stage
+  }
+
+  // 4. the warps' states (and the row's own key) meet at the common max, in a fixed order
 #pragma unroll
   for (int o = 1; o <= 2; o <<= 1) {
     l0 += __shfl_xor_sync(0xffffffffu, l0, o);
     l1 += __shfl_xor_sync(0xffffffffu, l1, o);
   }
   if ((lane & 3) == 0) {
-    red_l[warp][r0] = l0;
-    red_l[warp][r0 + 8] = l1;
+    red_m[warp][r0] = m0;
+    red_m[warp][r0 + 8] = m1;
   }
-  // 3. O += P V over this warp's keys: P from the S fragments, V by transposing loads
-  float O[D / 8][4];
+  ok = named_bar_and_dec(1, 128, ok);
+  float M0 = red_m[0][r0], M1 = red_m[0][r0 + 8];
 #pragma unroll
-  for (int dn = 0; dn < D / 8; ++dn)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) O[dn][e] = 0.f;
-#pragma unroll
-  for (int j = 0; j < 2; ++j) {
-    uint32_t pa[4];
-    pa[0] = pack_bf16(S[2 * j][0], S[2 * j][1]);
-    pa[1] = pack_bf16(S[2 * j][2], S[2 * j][3]);
-    pa[2] = pack_bf16(S[2 * j + 1][0], S[2 * j + 1][1]);
-    pa[3] = pack_bf16(S[2 * j + 1][2], S[2 * j + 1][3]);
-    const int key = warp * 32 + 16 * j + (mi & 1) * 8 + li;
-#pragma unroll
-    for (int dp = 0; dp < D / 16; ++dp) {
-      const int gc = 2 * dp + (mi >> 1);  // 16-byte chunk of the row (8 dims)
-      const int hf = gc / 8, c = gc % 8;
-      uint32_t b0, b1, b2, b3;
-      ldsm_x4_t(v_base + hf * HALF + key * 128 + ((c ^ (key & 7)) << 4), b0, b1, b2, b3);
-      mma16816(O[2 * dp], pa, b0, b1);
-      mma16816(O[2 * dp + 1], pa, b2, b3);
-    }
+  for (int w = 1; w < 4; ++w) {
+    M0 = fmaxf(M0, red_m[w][r0]);
+    M1 = fmaxf(M1, red_m[w][r0 + 8]);
   }
-  // 4. sum the warps' partial products in warp order (a fixed order keeps every row's result
-  // independent of what else is in the launch); write the chunk partial for the group's heads
-  for (int w = 0; w < kThreadsChunk / 32; ++w) {
-    if (warp == w) {
+  if (self_here) {
+    M0 = fmaxf(M0, r0 < grp ? s_self[r0] : -INFINITY);
+    M1 = fmaxf(M1, r0 + 8 < grp ? s_self[r0 + 8] : -INFINITY);
+  }
+  const float f0 = m0 == -INFINITY ? 0.f : ex2_approx(m0 - M0);
+  const float f1 = m1 == -INFINITY ? 0.f : ex2_approx(m1 - M1);
+  if ((lane & 3) == 0) {
+    red_l[warp][r0] = l0 * f0;
+    red_l[warp][r0 + 8] = l1 * f1;
+  }
+  // partial o of every warp summed over the stage-0 K tile (every copy has landed and been read)
+  float (*o_red)[D] = reinterpret_cast<float (*)[D]>(sKV);
+  static_assert(16 * D * 4 <= TILE, "partial products fit in a K tile");
+  for (int w = 0; w < 4; ++w) {
+    if (warp == w && ok) {
 #pragma unroll
       for (int dn = 0; dn < D / 8; ++dn) {
-        float* a0 = &o_red[r0][dn * 8 + cq];
-        float* a1 = &o_red[r0 + 8][dn * 8 + cq];
+        float* p0 = &o_red[r0][dn * 8 + cq];
+        float* p1 = &o_red[r0 + 8][dn * 8 + cq];
         if (w == 0) {
-          a0[0] = O[dn][0];
-          a0[1] = O[dn][1];
-          a1[0] = O[dn][2];
-          a1[1] = O[dn][3];
+          p0[0] = O[dn][0] * f0;
+          p0[1] = O[dn][1] * f0;
+          p1[0] = O[dn][2] * f1;
+          p1[1] = O[dn][3] * f1;
         } else {
-          a0[0] += O[dn][0];
-          a0[1] += O[dn][1];
-          a1[0] += O[dn][2];
-          a1[1] += O[dn][3];
+          p0[0] += O[dn][0] * f0;
+          p0[1] += O[dn][1] * f0;
+          p1[0] += O[dn][2] * f1;
+          p1[1] += O[dn][3] * f1;
         }
       }
     }
-    __syncthreads();
+    named_bar_sync_dec(1, 128);
   }
+  if (!ok) return;
   const float* vs = p.v_self + (size_t)r * p.n_kv_heads * D + g * D;
-  for (int i = tid; i < grp * D; i += kThreadsChunk) {
-    const int h = i / D, d = i % D;
-    float* out = p.part + (((size_t)r * p.n_q_heads + g * grp + h) * p.splits + chunk) * (D + 2);
-    out[d] = has_self ? o_red[h][d] + p_self[h] * vs[d] : o_red[h][d];
+  for (int q = tid; q < grp * D; q += 128) {
+    const int h = q / D, d = q % D;
+    float M = red_m[0][h];
+#pragma unroll
+    for (int w = 1; w < 4; ++w) M = fmaxf(M, red_m[w][h]);
+    float ps = 0.f;
+    if (self_here) {
+      M = fmaxf(M, s_self[h]);
+      ps = ex2_approx(s_self[h] - M);
+    }
+    float* out = p.part + (((size_t)r * p.n_q_heads + g * grp + h) * p.splits + slot) * (D + 2);
+    out[d] = o_red[h][d] + ps * vs[d];
     if (d == 0) {
-      float M = red_m[0][h], L = 0.f;
+      float L = ps;
 #pragma unroll
-      for (int w = 1; w < kThreadsChunk / 32; ++w) M = fmaxf(M, red_m[w][h]);
-#pragma unroll
-      for (int w = 0; w < kThreadsChunk / 32; ++w) L += red_l[w][h];
+      for (int w = 0; w < 4; ++w) L += red_l[w][h];
       out[D] = M;
       out[D + 1] = L;
     }
@@ -287,7 +382,7 @@ template <int D>
 __global__ void __launch_bounds__(128) decode_attn_merge(const DecodeAttnDesc p) {
   const int h = blockIdx.x, r = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int col = blockIdx.z * 32 + lane;
-  const int n_chunks = p.pos[r] / kChunk + 1;
+  const int n_chunks = (p.pos[r] / kChunk + p.chunks_per_block) / p.chunks_per_block;  // partials
   const float* base = p.part + ((size_t)r * p.n_q_heads + h) * p.splits * (D + 2);
   __shared__ float red_m[4], red_l[4], red_o[4][32];
   float m = -INFINITY;
@@ -345,17 +440,17 @@ bool pool_map(CUtensorMap* m, const void* base, long rows, int cols) {
 }
 
 template <int D>
-cudaError_t launch_dec(const DecodeArgs& args, int chunks, cudaStream_t stream) {
-  constexpr int smem = 2 * kChunk * D * 2 + 2 * 16 * D * 2 + 1024;
+cudaError_t launch_dec(const DecodeArgs& args, int blocks, cudaStream_t stream) {
+  constexpr int smem = 4 * kChunk * D * 2 + 2 * 16 * D * 2 + 1024;  // two K/V stages, q hi/lo
   static bool set = false;
   if (!set) {
-    cudaError_t e = cudaFuncSetAttribute(decode_attn_chunk<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(decode_attn_stream<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     set = true;
   }
   const DecodeAttnDesc& d = args.d;
-  decode_attn_chunk<D><<<dim3(chunks, d.n_kv_heads, d.rows), kThreadsChunk, smem, stream>>>(args);
-  decode_attn_merge<D><<<dim3(d.n_q_heads, d.rows, D / 32), 128, 0, stream>>>(d);
+  decode_attn_stream<D><<<blocks, kThreadsStream, smem, stream>>>(args);
+  decode_attn_merge<D><<<dim3(d.n_q_heads, d.rows, D / 32), 128, 0, stream>>>(d);  // d carries chunks_per_block
   return cudaGetLastError();
 }
 
@@ -370,17 +465,36 @@ cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int*
     return cudaErrorInvalidValue;
   int max_pos = 0;
   for (int r = 0; r < d.rows; ++r) max_pos = std::max(max_pos, d.pos[r]);
-  const int chunks = max_pos / kChunk + 1;
-  if (chunks > d.splits) return cudaErrorInvalidValue;
+  if (max_pos / kChunk + 1 > d.splits) return cudaErrorInvalidValue;
+  // one block per SM (two 64 KB K/V stages each), each streaming a run of consecutive chunks
+  // of one (row, kv head): the fewest chunks per block that keeps every block in one wave
+  static int num_sms = 0;
+  if (num_sms == 0) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess || num_sms < 1) return e != cudaSuccess ? e : cudaErrorInvalidValue;
+  }
+  long items = 0;
+  for (int r = 0; r < d.rows; ++r) items += static_cast<long>(d.n_kv_heads) * (d.pos[r] / kChunk + 1);
+  int cpb = static_cast<int>(std::max(1L, (items + num_sms - 1) / num_sms));
+  auto blocks_for = [&](int c) {
+    long b = 0;
+    for (int r = 0; r < d.rows; ++r) b += static_cast<long>(d.n_kv_heads) * ((d.pos[r] / kChunk + c) / c);
+    return b;
+  };
+  while (blocks_for(cpb) > num_sms) ++cpb;
+  const int blocks = static_cast<int>(blocks_for(cpb));
   DecodeArgs a;
   std::memset(&a, 0, sizeof(a));
   const long pool_rows = static_cast<long>(num_pages) * d.n_kv_heads * kPage;
   if (!pool_map(&a.tmK, d.kpages, pool_rows, d.head_dim)) return cudaErrorInvalidValue;
   if (!pool_map(&a.tmV, d.vpages, pool_rows, d.head_dim)) return cudaErrorInvalidValue;
   a.d = d;
+  a.d.chunks_per_block = cpb;
   a.status = status;
-  if (d.head_dim == 128) return launch_dec<128>(a, chunks, stream);
-  if (d.head_dim == 64) return launch_dec<64>(a, chunks, stream);
+  if (d.head_dim == 128) return launch_dec<128>(a, blocks, stream);
+  if (d.head_dim == 64) return launch_dec<64>(a, blocks, stream);
   return cudaErrorInvalidValue;
 }
 

@@ -163,9 +163,11 @@ struct DecodeAttnDesc {
   float* out;              // [rows, Hq*d]
   float* part;             // scratch [rows, Hq, splits, d + 2]
   int rows, n_q_heads, n_kv_heads, head_dim, splits, max_pos;
+  int chunks_per_block;    // set by launch_decode_attention
 };
-// Chunked decode attention (TMA-staged pages, 128 positions per block) + merge. `splits` in
-// the descriptor must be at least decode_attention_splits(max position + 1).
+// Decode attention streamed in 128-position chunks (TMA-staged pages, one block per SM walking
+// a run of chunks of one row and kv head) + merge of the blocks' partials. `splits` in the
+// descriptor must be at least decode_attention_splits(max position + 1).
 cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int* status,
                                     cudaStream_t stream);
 int decode_attention_splits(int max_positions);
