@@ -2,19 +2,22 @@
 // through layers e..N-1): for each decode row at position pos and query head h,
 //   o = softmax(q k^T / sqrt(d)) v over the cached keys 0..pos-1 of that layer plus the
 //   row's own fresh (k, v) at position pos.
-// The work is memory-bound (K and V of every cached position are read once), so the
-// positions are split into chunks of 128 that run as independent blocks:
-//   decode_attn_chunk   one block per (chunk, kv head, row): TMA gathers the chunk's K and
-//                       V pages (128-byte swizzle). The group's query heads (padded to 16
-//                       rows) are scored against the chunk with mma.sync m16n8k16 (each warp
-//                       takes 32 keys), q entering as a bf16 pair hi + lo so the scores keep
-//                       fp32 accuracy (K is exact in bf16); the row's own key is scored and
-//                       its value added in fp32. Softmax runs on the accumulator fragments,
-//                       P stays in registers as the A operand of P V, and the warps' partial
-//                       products are summed in shared memory in a fixed order. The chunk's
-//                       (max, sum, unnormalised o) are written in log2 units;
-//   decode_attn_merge   one block per (query head, row, 32-column slice): rescales the chunk
-//                       partials to the common max and normalises, every chunk's loads
+// The work is memory-bound (K and V of every cached position are read once): the positions
+// are cut into chunks of 128 and streamed.
+//   decode_attn_stream  one block per SM, walking a run of consecutive chunks of one (row,
+//                       kv head) through a two-stage ring: a copy warp gathers each chunk's
+//                       K and V pages with TMA (128-byte swizzle) while four compute warps
+//                       score the previous one. The group's query heads (padded to 16 rows)
+//                       meet the chunk on mma.sync m16n8k16 (each warp takes a 32-key slice),
+//                       q entering as a bf16 pair hi + lo so the scores keep fp32 accuracy (K
+//                       is exact in bf16). Every warp keeps an online-softmax state (running
+//                       max, sum and unnormalised o in registers, P as the A operand of P V)
+//                       over its slices; at the end the warps and the row's own key and value
+//                       (scored and added in fp32) meet at the common max in a fixed order and
+//                       the block writes one (max, sum, unnormalised o) partial in log2 units.
+//                       The chunks per block are the fewest that keep all blocks in one wave;
+//   decode_attn_merge   one block per (query head, row, 32-column slice): rescales the blocks'
+//                       partials to the common max and normalises, every partial's loads
 //                       independent of the others.
 #include "common.cuh"
 #include "kernels.h"
