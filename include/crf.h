@@ -177,7 +177,9 @@ CRF_API crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, co
                                 const crf_kv_pool* pool, const crf_request* reqs, int n_req,
                                 void* workspace, size_t ws_bytes, void* stream);
 
-/* One generation step for each row: the token at position `pos` (the number
+/* One generation step for each row (the decoding that consumes the recovered
+ * cache, Section 2.1; the first generated token is where Section S2.1 measures
+ * KL and top-1): the token at position `pos` (the number
  * of positions already cached for that request) is embedded and carried through
  * layers 0..N-1 under `cur`; at every layer it attends to the cached keys and
  * values at positions 0..pos-1 of its page table plus its own, and its post-RoPE
