@@ -164,6 +164,13 @@ CRF_API const char* crf_last_error(void);
  * last check (CRF_ETIMEOUT) or a pending CUDA error (CRF_ECUDA). */
 CRF_API crf_status crf_check(crf_ctx* ctx, void* stream);
 
+/* Failure-path self-test (no counterpart in the paper): launches one block on
+ * `stream` whose wait on a barrier that nothing completes runs out after the
+ * library's bounded-wait limit (2 s), exactly as a stalled kernel of the hot
+ * path would; the next crf_check then returns CRF_ETIMEOUT and clears the
+ * report, and the context stays usable. No fault is raised on the GPU. */
+CRF_API crf_status crf_selftest_timeout(crf_ctx* ctx, void* stream);
+
 /* Workspace bytes crf_recompute_window needs for these requests. */
 CRF_API crf_status crf_workspace_size(crf_ctx* ctx, const crf_model* model, const crf_lora_dims* lora,
                               const crf_request* reqs, int n_req, size_t* bytes);

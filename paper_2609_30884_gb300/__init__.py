@@ -226,6 +226,11 @@ class Context:
     def check(self, stream=None) -> None:
         abi.check(self.lib.crf_check(self.h, _stream(stream)))
 
+    def selftest_timeout(self, stream=None) -> None:
+        """Launch the bounded-wait self-test (its wait runs out after 2 s); the next check()
+        raises CRF_ETIMEOUT."""
+        abi.check(self.lib.crf_selftest_timeout(self.h, _stream(stream)))
+
     # -------------------------------------------------------------- profiling
     def profile_enable(self, on: bool = True, max_launches: int = 8192) -> None:
         abi.check(self.lib.crf_profile_enable(self.h, int(on), max_launches))

@@ -23,7 +23,8 @@ MAX_REQUESTS = 32
 EXPORTS = ("crf_create", "crf_destroy", "crf_last_error", "crf_check", "crf_workspace_size",
            "crf_recompute_window", "crf_drift_workspace_size", "crf_drift",
            "crf_kl_workspace_size", "crf_kl", "crf_kl_logits_noalloc", "crf_profile_enable",
-           "crf_profile_read", "crf_decode_workspace_size", "crf_decode_step")
+           "crf_profile_read", "crf_decode_workspace_size", "crf_decode_step",
+           "crf_selftest_timeout")
 
 
 class ModelDims(ctypes.Structure):
@@ -82,6 +83,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "crf_destroy": ([P], c_int),
         "crf_last_error": ([], c_char_p),
         "crf_check": ([P, P], c_int),
+        "crf_selftest_timeout": ([P, P], c_int),
         "crf_workspace_size": ([P, POINTER(Model), POINTER(LoraDims), POINTER(Request), c_int,
                                 POINTER(c_size_t)], c_int),
         "crf_recompute_window": ([P, POINTER(Model), POINTER(Adapter), POINTER(KVPool),

@@ -834,6 +834,13 @@ crf_status crf_check(crf_ctx* ctx, void* stream) {
   return CRF_OK;
 }
 
+crf_status crf_selftest_timeout(crf_ctx* ctx, void* stream) {
+  if (!ctx) return fail(CRF_EINVAL, "ctx is null");
+  CRF_CUDA(cudaSetDevice(ctx->device));
+  CRF_CUDA(launch_wait_selftest(ctx->status_dev, static_cast<cudaStream_t>(stream)));
+  return CRF_OK;
+}
+
 crf_status crf_workspace_size(crf_ctx* ctx, const crf_model* model, const crf_lora_dims* lora,
                               const crf_request* reqs, int n_req, size_t* bytes) {
   if (!ctx || !model || !lora || !reqs || !bytes) return fail(CRF_EINVAL, "null argument");

@@ -198,6 +198,9 @@ cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, v
                                  const RowPages& rp, int rows, int hkv, int head_dim,
                                  cudaStream_t stream);
 // out[r] = argmax of logits row r (lowest index among equal maxima).
+// One block whose wait on an mbarrier nothing arrives on runs out after the bounded-wait limit
+// and raises kStatusTimeout in *status (the failure path, exercised without a fault).
+cudaError_t launch_wait_selftest(int* status, cudaStream_t stream);
 cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
                                cudaStream_t stream);
 cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream);

@@ -655,6 +655,26 @@ cudaError_t launch_lora_down_rows(const LoraDownRows& m, int rank, int in_dim, c
   return cudaGetLastError();
 }
 
+// Bounded-wait self-test: thread 0 waits on an mbarrier that nothing arrives on. The wait
+// gives up after the library's limit, raises the status bit and the kernel returns, so the
+// context stays usable (the same path every kernel's waits take).
+__global__ void wait_selftest_kernel(int* status) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ volatile int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) (void)mbar_wait(&bar, 0, &abort_flag, status);
+}
+
+cudaError_t launch_wait_selftest(int* status, cudaStream_t stream) {
+  wait_selftest_kernel<<<1, 32, 0, stream>>>(status);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y, int rows,
                                int hidden, float eps, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
