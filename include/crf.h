@@ -38,6 +38,12 @@
  *   - A kernel that gives up on a bounded internal wait records it in the
  *     context; crf_check() reports it as CRF_ETIMEOUT. An asynchronous CUDA
  *     error is reported as CRF_ECUDA by the next call.
+ *   - Ids read from device memory are checked where they are used. A token id
+ *     outside [0, vocab) is read as token 0 and recorded; crf_check() then
+ *     returns CRF_EINVAL. Page ids are checked on the host before launch; a
+ *     library built with CRF_DEBUG defined (libcrf_debug.so) checks them again
+ *     at every device-side use, reads or writes page 0 in place of a bad id
+ *     and records it the same way.
  *   - Tensors are row-major, bf16 unless stated. Weights are [out, in].
  */
 #ifndef CRF_H
@@ -132,7 +138,7 @@ typedef struct crf_kv_pool {
 
 /* One cached prefix to refresh over the window [s, e) (0 <= s <= e <= N).
  *   page_table        device int32 [ceil(n_tokens/16)], distinct ids < num_pages
- *   tokens            device int32 [n_tokens]; required iff s == 0
+ *   tokens            device int32 [n_tokens]; required iff s == 0; ids in [0, vocab)
  *   hidden_in         device [n_tokens, h] = H_{s-1}; required iff s > 0
  *   hidden_out        NULL, or host array [e-s] of device [n_tokens, h]
  *                     buffers receiving H_s..H_{e-1} (refreshed checkpoints)
@@ -160,8 +166,10 @@ CRF_API crf_status crf_destroy(crf_ctx* ctx);
 /* Message for the last non-OK status returned on this thread. */
 CRF_API const char* crf_last_error(void);
 
-/* Synchronise `stream`, then report a device-side abandoned wait since the
- * last check (CRF_ETIMEOUT) or a pending CUDA error (CRF_ECUDA). */
+/* Synchronise `stream`, then report what the kernels recorded since the last
+ * check: a failed device-side bounds check (CRF_EINVAL, which takes
+ * precedence) or an abandoned bounded wait (CRF_ETIMEOUT); else a pending
+ * CUDA error (CRF_ECUDA). The record is cleared. */
 CRF_API crf_status crf_check(crf_ctx* ctx, void* stream);
 
 /* Failure-path self-test (no counterpart in the paper): launches one block on
@@ -195,7 +203,7 @@ CRF_API crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, co
  * and the LM head; next_tokens[i] = argmax of row i's logits (lowest index
  * among equal maxima).
  *   page_table: device int32 [pos / 16 + 1]; pages must be distinct across rows.
- *   token:      device int32, one entry: the input token id of the row.
+ *   token:      device int32, one entry: the input token id of the row, in [0, vocab).
  * next_tokens: device int32 [n_rows]. logits: NULL or device fp32 [n_rows][vocab].
  * The model needs embed, final_norm and lm_head; 1 <= n_rows <= CRF_MAX_REQUESTS.
  * `workspace` >= crf_decode_workspace_size bytes, 256-byte aligned. */

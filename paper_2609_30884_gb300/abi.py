@@ -10,7 +10,11 @@ import ctypes
 import os
 from ctypes import POINTER, c_char_p, c_float, c_int, c_size_t, c_uint32, c_void_p
 
-LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libcrf.so")
+LIB_DIR = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib")
+# CRF_LIB_VARIANT=debug selects the build with device-side page-id checks
+# (``build.build(debug=True)``); anything else, or unset, the release build.
+LIB_PATH = os.path.join(LIB_DIR, "libcrf_debug.so" if os.environ.get("CRF_LIB_VARIANT") == "debug"
+                        else "libcrf.so")
 
 OK, EINVAL, ESHAPE, EUNSUPPORTED, ENOMEM, ECUDA, ETIMEOUT = range(7)
 STATUS_NAMES = ["CRF_OK", "CRF_EINVAL", "CRF_ESHAPE", "CRF_EUNSUPPORTED", "CRF_ENOMEM",
@@ -75,7 +79,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     if _lib is not None:
         return _lib
     if not os.path.exists(path):
-        raise RuntimeError(f"libcrf.so not built at {path}; run paper_2609_30884_gb300.build.build()")
+        raise RuntimeError(f"{os.path.basename(path)} not built at {path}; run "
+                           "paper_2609_30884_gb300.build.build()"
+                           + ("" if path.endswith("libcrf.so") else " with debug=True"))
     lib = ctypes.CDLL(path)
     P = c_void_p
     sig = {

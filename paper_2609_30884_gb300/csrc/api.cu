@@ -561,7 +561,8 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
     // token rows are the whole batch (a generation step), so one launch covers them
     for (int i = 0; i < R; ++i)
       if (!rows[i].token) return fail(CRF_EINVAL, "decode rows mix token and hidden starts");
-    CRF_CUDA(launch_embed_rows_f32(static_cast<const __nv_bfloat16*>(c.model->embed), tr, R, x, D.h, c.st));
+    CRF_CUDA(launch_embed_rows_f32(static_cast<const __nv_bfloat16*>(c.model->embed), tr, R, x, D.h, D.V,
+                                   c.ctx->status_dev, c.st));
   }
   // segments [mods] sharing the fp32 rows `raw` (optionally RMS-normalised into `in` inside the
   // LoRA-down launch), one GEMV per group of up to 8 rows
@@ -653,7 +654,9 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
         pg.page_table[i] = rows[i].page_table;
         pg.pos[i] = rows[i].pos;
       }
-      CRF_CUDA(launch_kv_write_rows(k, v, c.pool->k_pages[l], c.pool->v_pages[l], pg, nr, D.hkv, D.d, c.st));
+      pg.num_pages = c.pool->num_pages;
+      CRF_CUDA(launch_kv_write_rows(k, v, c.pool->k_pages[l], c.pool->v_pages[l], pg, nr, D.hkv, D.d,
+                                    c.ctx->status_dev, c.st));
     }
     CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
     CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
@@ -666,6 +669,15 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
       CRF_CUDA(launch_f32_to_bf16(x + i * static_cast<size_t>(D.h),
                                   static_cast<__nv_bfloat16*>(rows[i].out), D.h, c.st));
   return CRF_OK;
+}
+
+// Page ids are read back and checked on the host before every launch. Only a CRF_DEBUG build run
+// with CRF_DEBUG_DEVICE_CHECKS_ONLY=1 skips that read, so that its device-side checks alone
+// stand between a bad id and the pool (the way its tests exercise them).
+bool host_page_check() {
+  if (!kDebugBuild) return true;
+  const char* e = std::getenv("CRF_DEBUG_DEVICE_CHECKS_ONLY");
+  return !(e && e[0] == '1');
 }
 
 crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const crf_adapter* cur,
@@ -702,6 +714,7 @@ crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const c
           !aligned16(pool->v_pages[l]))
         return fail(CRF_EINVAL, "kv pool layer %d null or misaligned", l);
     // page ids: in range and not shared between requests
+    if (!host_page_check()) continue;
     const int np = (r.n_tokens + kPage - 1) / kPage;
     std::vector<int32_t> pt(np);
     CRF_CUDA(cudaMemcpyAsync(pt.data(), r.page_table, np * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
@@ -758,6 +771,7 @@ crf_status validate_decode_rows(const crf_kv_pool* pool, const crf_decode_row* r
     const crf_decode_row& r = rows[i];
     if (r.pos < 0) return fail(CRF_EINVAL, "row %d: negative position", i);
     if (!r.page_table || !r.token) return fail(CRF_EINVAL, "row %d: page_table or token is null", i);
+    if (!host_page_check()) continue;
     const int np = r.pos / kPage + 1;
     std::vector<int32_t> pt(np);
     CRF_CUDA(cudaMemcpyAsync(pt.data(), r.page_table, np * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
@@ -829,6 +843,9 @@ crf_status crf_check(crf_ctx* ctx, void* stream) {
   CRF_CUDA(cudaMemcpy(&status, ctx->status_dev, sizeof(int), cudaMemcpyDeviceToHost));
   if (status) {
     CRF_CUDA(cudaMemset(ctx->status_dev, 0, sizeof(int)));
+    if (status & kStatusBounds)
+      return fail(CRF_EINVAL, "a device-side bounds check failed: a token id outside the vocabulary%s "
+                  "(status 0x%x)", kDebugBuild ? " or a page id outside the pool" : "", status);
     return fail(CRF_ETIMEOUT, "a kernel abandoned a bounded wait (status 0x%x)", status);
   }
   return CRF_OK;
@@ -916,6 +933,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
     if (act.empty()) continue;
     ReqTable rt;
     std::memset(&rt, 0, sizeof(rt));
+    rt.num_pages = pool->num_pages;
     int M = 0;
     for (int i : act) {
       rt.row0[rt.n] = M;
@@ -955,7 +973,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
           if (reqs[i].s == l && l == 0) {
             ProfScope ps(ctx, kPEmbed, st);
             CRF_CUDA(launch_embed(static_cast<const __nv_bfloat16*>(model->embed), reqs[i].tokens, dst,
-                                  reqs[i].n_tokens, D.h, st));
+                                  reqs[i].n_tokens, D.h, D.V, ctx->status_dev, st));
           } else {
             ProfScope ps(ctx, kPCopy, st, 0);
             CRF_CUDA(cudaMemcpyAsync(dst, curp[i], reqs[i].n_tokens * row_bytes,
@@ -1000,7 +1018,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
       ProfScope ps(ctx, r.s == 0 ? kPEmbed : kPCopy, st, r.s == 0 ? 1 : 0);
       if (r.s == 0) {
         CRF_CUDA(launch_embed(static_cast<const __nv_bfloat16*>(model->embed), r.tokens + (r.n_tokens - 1),
-                              start, 1, D.h, st));
+                              start, 1, D.h, D.V, ctx->status_dev, st));
       } else {
         CRF_CUDA(cudaMemcpyAsync(start,
                                  static_cast<const __nv_bfloat16*>(r.hidden_in) +

@@ -94,7 +94,7 @@ __global__ void __launch_bounds__(kWarps * 32, 1) attn_prefill_kernel(const Attn
       const int r = i / CH, c = i % CH;
       const int t = k0 + r;
       const bool ok = t < kv_end;
-      const int page = ok ? pt[t / kPage] : 0;
+      const int page = ok ? checked_page(pt[t / kPage], p.req.num_pages, p.status) : 0;
       const size_t off = (((size_t)page * p.n_kv_heads + g) * kPage + (t % kPage)) * D + c * 8;
       cp_async16(sK + buf * kBN * D * 2 + swz<D>(r, c), p.kpages + (ok ? off : 0), ok);
       cp_async16(sV + buf * kBN * D * 2 + swz<D>(r, c), p.vpages + (ok ? off : 0), ok);

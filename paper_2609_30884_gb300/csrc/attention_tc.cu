@@ -262,7 +262,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
         const CUtensorMap* map = kv == 0 ? &a.tmK : &a.tmV;
         for (int p = 0; p < kPagesPerTile; ++p) {
           // pages past the prefix repeat the last page: finite data, masked below
-          const int page = pt[min(j * kPagesPerTile + p, n_pages - 1)];
+          const int page = checked_page(pt[min(j * kPagesPerTile + p, n_pages - 1)], a.req.num_pages, a.status);
           const int group = (page * a.n_kv_heads + w.g) * (kPage / 8);
           tma_load_4d(dst + p * (kPage / 8) * GROUP_BYTES, map, &kv_full[slot], 0, 0, 0, group);
         }

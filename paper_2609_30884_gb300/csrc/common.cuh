@@ -11,7 +11,43 @@
 namespace crf {
 
 // Status bits a kernel may set in the context's device status word.
-enum : int { kStatusTimeout = 1 };
+enum : int { kStatusTimeout = 1, kStatusBounds = 2 };
+
+#ifdef CRF_DEBUG
+constexpr bool kDebugBuild = true;
+#else
+constexpr bool kDebugBuild = false;
+#endif
+
+// A token id read from device memory: one outside [0, vocab) sets kStatusBounds
+// and reads row 0 of the embedding instead. The host never sees the ids, so
+// this check stays on in every build.
+__device__ __forceinline__ int checked_token(int tok, int vocab, int* status) {
+  if (tok < 0 || tok >= vocab) {
+    if (status) atomicOr(status, kStatusBounds);
+    return 0;
+  }
+  return tok;
+}
+
+// Device-side bounds check on a page id read from a page table. In a build
+// with CRF_DEBUG defined, an id outside [0, num_pages) sets kStatusBounds and
+// comes back as page 0, so the copy that uses it stays inside the pool and
+// every barrier still completes; the host reports the bit. The host already
+// validates every page table before launch, so in the release build the
+// check compiles away and the id is returned unchanged.
+__device__ __forceinline__ int checked_page(int page, int num_pages, int* status) {
+#ifdef CRF_DEBUG
+  if (page < 0 || page >= num_pages) {
+    if (status) atomicOr(status, kStatusBounds);
+    return 0;
+  }
+#else
+  (void)num_pages;
+  (void)status;
+#endif
+  return page;
+}
 
 // Bounded waits give up after this many nanoseconds (a correct kernel never
 // waits more than microseconds on one barrier).

@@ -56,6 +56,7 @@ struct DecodeArgs {
   CUtensorMap tmK;  // K pool of the layer viewed as [pages*Hkv*16, d], box {64, 16}
   CUtensorMap tmV;
   DecodeAttnDesc d;
+  int num_pages;
   int* status;
 };
 
@@ -128,7 +129,8 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
         } else {
           mbar_arrive_expect_tx(&full[st], 2 * pages * HALVES * kPage * 128);
           for (int pg = 0; pg < pages; ++pg) {
-            const int row = (pt[t0 / kPage + pg] * p.n_kv_heads + g) * kPage;
+            const int page = checked_page(pt[t0 / kPage + pg], a.num_pages, a.status);
+            const int row = (page * p.n_kv_heads + g) * kPage;
             for (int h = 0; h < HALVES; ++h) {
               const int off = h * HALF + pg * (kPage * 128);
               tma_load_2d(sK + off, &a.tmK, &full[st], 64 * h, row);
@@ -495,6 +497,7 @@ cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int*
   if (!pool_map(&a.tmV, d.vpages, pool_rows, d.head_dim)) return cudaErrorInvalidValue;
   a.d = d;
   a.d.chunks_per_block = cpb;
+  a.num_pages = num_pages;
   a.status = status;
   if (d.head_dim == 128) return launch_dec<128>(a, blocks, stream);
   if (d.head_dim == 64) return launch_dec<64>(a, blocks, stream);

@@ -247,7 +247,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
       dst_row = a.qbuf + (size_t)row * a.ldq;
       head_stride = d;
     } else {
-      const int page = pt[pos / kPage];
+      const int page = checked_page(pt[pos / kPage], a.req.num_pages, a.status);
       __nv_bfloat16* base = (g == 1) ? a.kpages : a.vpages;
       dst_row = base + ((size_t)page * a.n_kv_heads * kPage + (pos % kPage)) * d;
       head_stride = (size_t)kPage * d;

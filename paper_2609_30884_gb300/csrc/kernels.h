@@ -21,6 +21,7 @@ constexpr int kBxCols = 64;
 // Rows of a batched activation matrix that belong to each request.
 struct ReqTable {
   int n;
+  int num_pages;  // pool size; page ids are checked against it in a CRF_DEBUG build
   int row0[kMaxReq];
   int len[kMaxReq];
   const int32_t* page_table[kMaxReq];
@@ -92,8 +93,9 @@ cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double the
                               cudaStream_t stream);
 cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bfloat16* y,
                            int rows, int hidden, float eps, cudaStream_t stream);
+// Token ids outside [0, vocab) read row 0 and set kStatusBounds in *status.
 cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv_bfloat16* out,
-                         int n, int hidden, cudaStream_t stream);
+                         int n, int hidden, int vocab, int* status, cudaStream_t stream);
 
 // Causal GQA prefill attention over the paged cache of the current layer.
 struct AttnDesc {
@@ -188,14 +190,15 @@ struct TokenRows {
 };
 // x [rows, hidden] fp32 = embed[token_r].
 cudaError_t launch_embed_rows_f32(const __nv_bfloat16* embed, const TokenRows& t, int rows, float* x,
-                                  int hidden, cudaStream_t stream);
+                                  int hidden, int vocab, int* status, cudaStream_t stream);
 struct RowPages {
   const int32_t* page_table[kMaxReq];
   int pos[kMaxReq];
+  int num_pages;
 };
 // Rows' fp32 k, v [rows, hkv * head_dim] into their page slot (page_table[pos / 16], pos % 16).
 cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, void* vpages,
-                                 const RowPages& rp, int rows, int hkv, int head_dim,
+                                 const RowPages& rp, int rows, int hkv, int head_dim, int* status,
                                  cudaStream_t stream);
 // out[r] = argmax of logits row r (lowest index among equal maxima).
 // One block whose wait on an mbarrier nothing arrives on runs out after the bounded-wait limit

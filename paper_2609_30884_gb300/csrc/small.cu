@@ -95,13 +95,16 @@ __global__ void rmsnorm_f32_kernel(const float* __restrict__ x, const __nv_bfloa
 
 // ------------------------------------------------------------------ embedding
 __global__ void embed_kernel(const __nv_bfloat16* __restrict__ e, const int32_t* __restrict__ tok,
-                             __nv_bfloat16* __restrict__ out, int n, int hidden) {
+                             __nv_bfloat16* __restrict__ out, int n, int hidden, int vocab,
+                             int* status) {
   const int nv = hidden / 8;
   const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (size_t)n * nv) return;
   const int t = static_cast<int>(idx / nv), c = static_cast<int>(idx % nv);
+  // Only the row's first chunk reports a bad id, so the status word sees one atomic per row.
+  const int id = checked_token(tok[t], vocab, c == 0 ? status : nullptr);
   reinterpret_cast<uint4*>(out + (size_t)t * hidden)[c] =
-      reinterpret_cast<const uint4*>(e + (size_t)tok[t] * hidden)[c];
+      reinterpret_cast<const uint4*>(e + (size_t)id * hidden)[c];
 }
 
 // ------------------------------------------------------------------ decode-path GEMV
@@ -575,10 +578,10 @@ cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_
 }
 
 cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv_bfloat16* out,
-                         int n, int hidden, cudaStream_t stream) {
+                         int n, int hidden, int vocab, int* status, cudaStream_t stream) {
   const long total = (long)n * (hidden / 8);
   if (total == 0) return cudaSuccess;
-  embed_kernel<<<cdiv(total, 256), 256, 0, stream>>>(embed, tokens, out, n, hidden);
+  embed_kernel<<<cdiv(total, 256), 256, 0, stream>>>(embed, tokens, out, n, hidden, vocab, status);
   return cudaGetLastError();
 }
 
@@ -707,9 +710,10 @@ __global__ void rope_table_rows_kernel(float2* table, int rows, int half, const 
 
 // x[r] = embed[token_r] as fp32, the token read from device memory.
 __global__ void embed_rows_f32_kernel(const __nv_bfloat16* __restrict__ embed, const TokenRows t,
-                                      float* __restrict__ x, int hidden) {
+                                      float* __restrict__ x, int hidden, int vocab, int* status) {
   const int r = blockIdx.y;
-  const int32_t tok = *t.token[r];
+  const int tok = checked_token(*t.token[r], vocab,
+                                blockIdx.x == 0 && threadIdx.x == 0 ? status : nullptr);
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < hidden; i += gridDim.x * blockDim.x)
     x[(size_t)r * hidden + i] = __bfloat162float(embed[(size_t)tok * hidden + i]);
 }
@@ -717,10 +721,11 @@ __global__ void embed_rows_f32_kernel(const __nv_bfloat16* __restrict__ embed, c
 // The rows' fp32 k, v [rows, Hkv * d] into slot pos % 16 of page page_table[pos / 16], bf16.
 __global__ void kv_write_rows_kernel(const float* __restrict__ k, const float* __restrict__ v,
                                      __nv_bfloat16* kpages, __nv_bfloat16* vpages, const RowPages rp,
-                                     int hkv, int d) {
+                                     int hkv, int d, int* status) {
   const int r = blockIdx.y;
   const int pos = rp.pos[r];
-  const int page = rp.page_table[r][pos / kPage];
+  const int page = checked_page(rp.page_table[r][pos / kPage], rp.num_pages,
+                                blockIdx.x == 0 && threadIdx.x == 0 ? status : nullptr);
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < hkv * d; i += gridDim.x * blockDim.x) {
     const int h = i / d, j = i % d;
     const size_t dst = (((size_t)page * hkv + h) * kPage + pos % kPage) * d + j;
@@ -781,18 +786,20 @@ cudaError_t launch_rope_table_rows(float2* table, const RowPositions& pos, int r
 }
 
 cudaError_t launch_embed_rows_f32(const __nv_bfloat16* embed, const TokenRows& t, int rows, float* x,
-                                  int hidden, cudaStream_t stream) {
+                                  int hidden, int vocab, int* status, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
-  embed_rows_f32_kernel<<<dim3(cdiv(hidden, 256), rows), 256, 0, stream>>>(embed, t, x, hidden);
+  embed_rows_f32_kernel<<<dim3(cdiv(hidden, 256), rows), 256, 0, stream>>>(embed, t, x, hidden, vocab,
+                                                                            status);
   return cudaGetLastError();
 }
 
 cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, void* vpages,
-                                 const RowPages& rp, int rows, int hkv, int head_dim,
+                                 const RowPages& rp, int rows, int hkv, int head_dim, int* status,
                                  cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
   kv_write_rows_kernel<<<dim3(cdiv(hkv * head_dim, 256), rows), 256, 0, stream>>>(
-      k, v, static_cast<__nv_bfloat16*>(kpages), static_cast<__nv_bfloat16*>(vpages), rp, hkv, head_dim);
+      k, v, static_cast<__nv_bfloat16*>(kpages), static_cast<__nv_bfloat16*>(vpages), rp, hkv, head_dim,
+      status);
   return cudaGetLastError();
 }
 

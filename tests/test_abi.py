@@ -80,3 +80,14 @@ def test_struct_layouts_match_c(tmp_path):
             assert int(got[f"{sname}.{f}"]) == getattr(cls, f).offset, f"{sname}.{f}"
     assert got["enum 6 16"] == str(abi.MAX_REQUESTS)
     assert abi.PAGE_SIZE == 16 and abi.NUM_MODULES == 7
+
+
+def test_debug_build_exports_every_declared_symbol():
+    """The CRF_DEBUG variant (device-side page-id checks) builds from the same sources."""
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("no nvcc")
+    path = build.build(debug=True)
+    assert os.path.basename(path) == "libcrf_debug.so"
+    dbg = ctypes.CDLL(path)
+    for name in declared_functions():
+        assert hasattr(dbg, name), name
