@@ -620,49 +620,54 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
   float* const y_d[1] = {x};
   RowPositions rp{};
   for (int i = 0; i < R; ++i) rp.pos[i] = rows[i].pos;
-  for (int l = l0; l < D.N; ++l) {
-    int nr = 0;
-    while (nr < R && rows[nr].e <= l) ++nr;
-    const crf_layer_weights& w = c.model->layers[l];
-    CRF_CUDA(proj(l, nr, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr, 0));
-    CRF_CUDA(launch_rope_rows(q, D.hq, k, D.hkv, nr, D.d,
-                              opt.rope_by_row ? opt.rope_by_row
-                                              : reinterpret_cast<const float2*>(c.ws + p.off_rope),
-                              rp, opt.rope_by_row != nullptr, c.st));
-    DecodeAttnDesc a;
-    std::memset(&a, 0, sizeof(a));
-    a.q = q;
-    a.k_self = k;
-    a.v_self = v;
-    a.kpages = static_cast<const __nv_bfloat16*>(c.pool->k_pages[l]);
-    a.vpages = static_cast<const __nv_bfloat16*>(c.pool->v_pages[l]);
-    for (int i = 0; i < nr; ++i) {
-      a.page_table[i] = rows[i].page_table;
-      a.pos[i] = rows[i].pos;
-    }
-    a.out = o;
-    a.part = part;
-    a.rows = nr;
-    a.n_q_heads = D.hq;
-    a.n_kv_heads = D.hkv;
-    a.head_dim = D.d;
-    a.splits = p.splits;
-    CRF_CUDA(launch_decode_attention(a, c.pool->num_pages, c.ctx->status_dev, c.st));
-    if (opt.write_kv) {
-      RowPages pg{};
+  {
+    // the layer loop is a chain of short kernels only: each may become resident and prefetch its
+    // weights while the one before it finishes
+    PdlScope pdl;
+    for (int l = l0; l < D.N; ++l) {
+      int nr = 0;
+      while (nr < R && rows[nr].e <= l) ++nr;
+      const crf_layer_weights& w = c.model->layers[l];
+      CRF_CUDA(proj(l, nr, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr, 0));
+      CRF_CUDA(launch_rope_rows(q, D.hq, k, D.hkv, nr, D.d,
+                                opt.rope_by_row ? opt.rope_by_row
+                                                : reinterpret_cast<const float2*>(c.ws + p.off_rope),
+                                rp, opt.rope_by_row != nullptr, c.st));
+      DecodeAttnDesc a;
+      std::memset(&a, 0, sizeof(a));
+      a.q = q;
+      a.k_self = k;
+      a.v_self = v;
+      a.kpages = static_cast<const __nv_bfloat16*>(c.pool->k_pages[l]);
+      a.vpages = static_cast<const __nv_bfloat16*>(c.pool->v_pages[l]);
       for (int i = 0; i < nr; ++i) {
-        pg.page_table[i] = rows[i].page_table;
-        pg.pos[i] = rows[i].pos;
+        a.page_table[i] = rows[i].page_table;
+        a.pos[i] = rows[i].pos;
       }
-      pg.num_pages = c.pool->num_pages;
-      CRF_CUDA(launch_kv_write_rows(k, v, c.pool->k_pages[l], c.pool->v_pages[l], pg, nr, D.hkv, D.d,
-                                    c.ctx->status_dev, c.st));
+      a.out = o;
+      a.part = part;
+      a.rows = nr;
+      a.n_q_heads = D.hq;
+      a.n_kv_heads = D.hkv;
+      a.head_dim = D.d;
+      a.splits = p.splits;
+      CRF_CUDA(launch_decode_attention(a, c.pool->num_pages, c.ctx->status_dev, c.st));
+      if (opt.write_kv) {
+        RowPages pg{};
+        for (int i = 0; i < nr; ++i) {
+          pg.page_table[i] = rows[i].page_table;
+          pg.pos[i] = rows[i].pos;
+        }
+        pg.num_pages = c.pool->num_pages;
+        CRF_CUDA(launch_kv_write_rows(k, v, c.pool->k_pages[l], c.pool->v_pages[l], pg, nr, D.hkv, D.d,
+                                      c.ctx->status_dev, c.st));
+      }
+      CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
+      CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
+      // gate rows then up rows: SwiGLU over [nr, f] with the up half Rs * f further on
+      CRF_CUDA(launch_swiglu_split_f32(gu, gu + Rs * D.f, m, nr * D.f, c.st));
+      CRF_CUDA(proj(l, nr, m_d, 1, m, nullptr, nullptr, D.f, y_d, o_d, x1, D.h));
     }
-    CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
-    CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
-    // gate rows then up rows: SwiGLU over [nr, f] with the up half Rs * f further on
-    CRF_CUDA(launch_swiglu_split_f32(gu, gu + Rs * D.f, m, nr * D.f, c.st));
-    CRF_CUDA(proj(l, nr, m_d, 1, m, nullptr, nullptr, D.f, y_d, o_d, x1, D.h));
   }
   for (int i = 0; i < R; ++i)
     if (rows[i].out)

@@ -133,6 +133,31 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// ---------------------------------------------------------------- dependent launch
+// A kernel launched with the programmatic-stream-serialization attribute may become resident
+// while the kernel before it in the stream is still running. griddep_wait() returns once that
+// kernel has completed and its writes are visible (at once for a kernel launched without the
+// attribute), so a kernel touches nothing that an earlier kernel of the stream may write before
+// it: only weights, which no kernel writes. griddep_launch_dependents() then lets the next kernel
+// of the stream start its own prologue; issuing it after the wait keeps at most one kernel ahead.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_begin() {
+  griddep_wait();
+  griddep_launch_dependents();
+}
+
+// Ask L2 for bytes [p, p + n), n < 4 GB (128-byte lines; the block's threads share the lines in turn).
+static __device__ __noinline__ void prefetch_l2_range(const void* p, size_t n) {
+  const char* c = static_cast<const char*>(p);
+  const uint32_t lines = static_cast<uint32_t>((n + 127) / 128);
+#pragma unroll 1
+  for (uint32_t i = threadIdx.x; i < lines; i += blockDim.x)
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(c + static_cast<size_t>(i) * 128));
+}
+
 // ---------------------------------------------------------------- clusters
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;

@@ -67,6 +67,7 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
   constexpr int TILE = HALVES * HALF;
   constexpr int QHALF = 16 * 128;        // one 64-column half of the 16-row Q tile
   const DecodeAttnDesc& p = a.d;
+  griddep_begin();  // q, k, v of the rows come from the kernel before
   // block -> (row, kv head, its chunks c_beg .. c_end - 1, partial slot)
   int r = -1, g = 0, slot = 0, c_beg = 0, c_end = 0;
   {
@@ -385,6 +386,7 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
 // sums meet in a fixed order.
 template <int D>
 __global__ void __launch_bounds__(128) decode_attn_merge(const DecodeAttnDesc p) {
+  griddep_begin();  // the partials come from decode_attn_stream
   const int h = blockIdx.x, r = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int col = blockIdx.z * 32 + lane;
   const int n_chunks = (p.pos[r] / kChunk + p.chunks_per_block) / p.chunks_per_block;  // partials
@@ -454,9 +456,10 @@ cudaError_t launch_dec(const DecodeArgs& args, int blocks, cudaStream_t stream) 
     set = true;
   }
   const DecodeAttnDesc& d = args.d;
-  decode_attn_stream<D><<<blocks, kThreadsStream, smem, stream>>>(args);
-  decode_attn_merge<D><<<dim3(d.n_q_heads, d.rows, D / 32), 128, 0, stream>>>(d);  // d carries chunks_per_block
-  return cudaGetLastError();
+  cudaError_t e = launch_kernel(decode_attn_stream<D>, dim3(blocks), dim3(kThreadsStream), smem, stream, args);
+  if (e != cudaSuccess) return e;
+  // d carries chunks_per_block
+  return launch_kernel(decode_attn_merge<D>, dim3(d.n_q_heads, d.rows, D / 32), dim3(128), 0, stream, d);
 }
 
 }  // namespace

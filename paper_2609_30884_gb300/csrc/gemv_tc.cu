@@ -46,7 +46,13 @@ __global__ void __launch_bounds__(kWarps * 32) gemv_tc_kernel(const __grid_const
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tl = warp / ks, kp = warp % ks;
   const int tiles_per_block = kWarps / ks;
-  const int j0 = ((static_cast<int>(blockIdx.x) - L.block0[s]) * tiles_per_block + tl) * 16;
+  const int tb = (static_cast<int>(blockIdx.x) - L.block0[s]) * tiles_per_block;
+  if (d.prefetch) {  // the block's weight rows are contiguous
+    const int jb0 = tb * 16, jb1 = min(sg.out_dim, jb0 + tiles_per_block * 16);
+    if (jb0 < jb1) prefetch_l2_range(sg.W + (size_t)jb0 * d.in_dim, (size_t)(jb1 - jb0) * d.in_dim * 2);
+  }
+  griddep_begin();  // x, xa and the residual come from the kernels before
+  const int j0 = (tb + tl) * 16;
   const int g = lane >> 2, c = lane & 3;
   const int K = d.in_dim;
   // K range of this warp in 32-column blocks (a 16-column tail goes to the last warp)
@@ -129,6 +135,7 @@ cudaError_t launch_gemv_tc(const GemvDesc& d, int num_sms, cudaStream_t stream) 
     return cudaErrorInvalidValue;
   GemvTcLaunch L;
   L.d = d;
+  L.d.prefetch = pdl_active() ? 1 : 0;
   int tiles = 0;
   for (int s = 0; s < d.nseg; ++s) tiles += (d.seg[s].out_dim + 15) / 16;
   if (tiles == 0) return cudaSuccess;
@@ -143,8 +150,7 @@ cudaError_t launch_gemv_tc(const GemvDesc& d, int num_sms, cudaStream_t stream) 
     if (s < d.nseg) blocks += ((d.seg[s].out_dim + 15) / 16 + tiles_per_block - 1) / tiles_per_block;
   }
   L.block0[3] = blocks;
-  gemv_tc_kernel<<<blocks, kWarps * 32, 0, stream>>>(L);
-  return cudaGetLastError();
+  return launch_kernel(gemv_tc_kernel, dim3(blocks), dim3(kWarps * 32), 0, stream, L);
 }
 
 }  // namespace crf

@@ -18,6 +18,41 @@ constexpr int kRankPad = 16;  // LoRA rank padded to one K=16 MMA step
 constexpr int kXaCols = 128;
 constexpr int kBxCols = 64;
 
+// Programmatic dependent launch for chains of short kernels. While a PdlScope is alive on the
+// calling thread, the launchers below that go through launch_kernel() give their kernels the
+// programmatic-stream-serialization attribute: such a kernel becomes resident while its
+// predecessor in the stream still runs, prefetches its weights and then waits for it
+// (griddep_wait). Every kernel launched this way calls griddep_wait before it touches memory
+// that an earlier kernel may write. The decode-row layer loop opens a scope; CRF_PDL=0 in the
+// environment turns the attribute off.
+class PdlScope {
+ public:
+  PdlScope();
+  ~PdlScope();
+  PdlScope(const PdlScope&) = delete;
+  PdlScope& operator=(const PdlScope&) = delete;
+
+ private:
+  bool prev_;
+};
+bool pdl_active();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                          cudaStream_t stream, Args&&... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_active() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // Rows of a batched activation matrix that belong to each request.
 struct ReqTable {
   int n;
@@ -133,6 +168,7 @@ struct GemvDesc {
   const float* x;  // [rows, in_dim] fp32
   int rows;        // 1..8
   int rank;
+  int prefetch;    // set by the launcher: prefetch the block's weight rows into L2 before the wait
 };
 // Tensor-core GEMV (mma.sync, rows as a bf16 hi/lo pair); launch_gemv uses it when the call's
 // rows (total_rows, the rows of all chunks one caller splits into launches of <= 8; 0 = d.rows)
@@ -145,6 +181,7 @@ struct LoraDownRows {
   const __nv_bfloat16* A[3];
   float* xa[3];
   int n;
+  int prefetch;  // set by the launcher: prefetch the block's A row into L2 before the wait
 };
 // With norm_gain != null, x is normalised first (rmsnorm(x) * norm_gain, eps) and the
 // normalised rows are also written to xn (so the launch replaces the separate RMSNorm).

@@ -133,7 +133,13 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const __grid_cons
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gl = warp / ks, kp = warp % ks;
   const int groups_per_block = kGemvWarps / ks;
-  const int g = (static_cast<int>(blockIdx.x) - L.block0[s]) * groups_per_block + gl;
+  const int gb = (static_cast<int>(blockIdx.x) - L.block0[s]) * groups_per_block;
+  if (d.prefetch) {  // the block's weight rows are contiguous
+    const int jb0 = gb * OPW, jb1 = min(sg.out_dim, jb0 + groups_per_block * OPW);
+    if (jb0 < jb1) prefetch_l2_range(sg.W + (size_t)jb0 * d.in_dim, (size_t)(jb1 - jb0) * d.in_dim * 2);
+  }
+  griddep_begin();  // x, xa and the residual come from the kernels before
+  const int g = gb + gl;
   const int j0 = g * OPW;
   const int n8 = d.in_dim / 8;
   const int per = (n8 + ks - 1) / ks;
@@ -195,12 +201,15 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const __grid_cons
 constexpr int kLdThreads = 256;
 
 __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
-    const LoraDownRows m, int rank, int in_dim, const float* __restrict__ x, int rows, float scale,
-    const __nv_bfloat16* __restrict__ g, float eps, float* __restrict__ xn) {
+    const __grid_constant__ LoraDownRows m, int rank, int in_dim, const float* __restrict__ x, int rows,
+    float scale, const __nv_bfloat16* __restrict__ g, float eps, float* __restrict__ xn) {
   __shared__ float red[kLdThreads / 32];
   const int b = blockIdx.x;
   const int n_dot = m.n * rows * rank;
   const int r = b < n_dot ? (b / rank) % rows : b - n_dot;
+  const int mi = b / (rows * rank), k = b % rank;
+  if (m.prefetch) prefetch_l2_range(b < n_dot ? m.A[mi] + (size_t)k * in_dim : g, g || b < n_dot ? in_dim * 2 : 0);
+  griddep_begin();  // x comes from the kernel before
   const float* xr = x + (size_t)r * in_dim;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float inv = 1.f;
@@ -224,7 +233,6 @@ __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
       xn[(size_t)r * in_dim + i] = xr[i] * inv * __bfloat162float(g[i]);
     return;
   }
-  const int mi = b / (rows * rank), k = b % rank;
   const __nv_bfloat16* A = m.A[mi] + (size_t)k * in_dim;
   float s = 0.f;
   for (int i = threadIdx.x * 8; i < in_dim; i += kLdThreads * 8) {
@@ -255,6 +263,7 @@ __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
 // position pos[r], angles from the (cos, sin) table of the window pass.
 __global__ void rope_rows_kernel(float* q, int hq, float* k, int hkv, int rows, int d,
                                  const float2* __restrict__ table, const RowPositions pos, int by_row) {
+  griddep_begin();  // q, k come from the GEMV before
   const int half = d / 2;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   const int heads = hq + hkv;
@@ -304,6 +313,7 @@ __global__ void swiglu_f32_kernel(const float* gu, float* m, int rows, int ffn) 
 
 // m[i] = silu(g[i]) * u[i] over n elements (gate and up in separate buffers)
 __global__ void swiglu_split_f32_kernel(const float* g, const float* u, float* m, int n) {
+  griddep_begin();  // gate and up come from the GEMV before
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) m[i] = g[i] / (1.f + __expf(-g[i])) * u[i];
 }
@@ -587,16 +597,28 @@ cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv
 
 template <int OPW>
 cudaError_t gemv_dispatch(const GemvLaunch& L, int blocks, cudaStream_t stream) {
-  if (L.d.rows == 1)
-    gemv_kernel<OPW, 1><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
-  else if (L.d.rows == 2)
-    gemv_kernel<OPW, 2><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
-  else if (L.d.rows <= 4)
-    gemv_kernel<OPW, 4><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
-  else
-    gemv_kernel<OPW, 8><<<blocks, kGemvWarps * 32, 0, stream>>>(L);
-  return cudaGetLastError();
+  const dim3 grid(blocks), block(kGemvWarps * 32);
+  if (L.d.rows == 1) return launch_kernel(gemv_kernel<OPW, 1>, grid, block, 0, stream, L);
+  if (L.d.rows == 2) return launch_kernel(gemv_kernel<OPW, 2>, grid, block, 0, stream, L);
+  if (L.d.rows <= 4) return launch_kernel(gemv_kernel<OPW, 4>, grid, block, 0, stream, L);
+  return launch_kernel(gemv_kernel<OPW, 8>, grid, block, 0, stream, L);
 }
+
+namespace {
+thread_local bool t_pdl = false;
+bool pdl_env() {
+  static int v = -1;
+  if (v < 0) {
+    const char* e = std::getenv("CRF_PDL");
+    v = (e && std::strcmp(e, "0") == 0) ? 0 : 1;
+  }
+  return v == 1;
+}
+}  // namespace
+
+PdlScope::PdlScope() : prev_(t_pdl) { t_pdl = pdl_env(); }
+PdlScope::~PdlScope() { t_pdl = prev_; }
+bool pdl_active() { return t_pdl; }
 
 static bool gemv_scalar() {
   static int v = -1;
@@ -619,6 +641,7 @@ cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int
     return cudaErrorInvalidValue;
   GemvLaunch L;
   L.d = d;
+  L.d.prefetch = pdl_active() ? 1 : 0;
   int total_out = 0;
   for (int s = 0; s < d.nseg; ++s) total_out += d.seg[s].out_dim;
   if (total_out == 0) return cudaSuccess;
@@ -653,9 +676,10 @@ cudaError_t launch_lora_down_rows(const LoraDownRows& m, int rank, int in_dim, c
   const int blocks = m.n * rows * rank + (norm_gain ? rows : 0);
   if (blocks == 0) return cudaSuccess;
   if (in_dim % 8 != 0) return cudaErrorInvalidValue;
-  lora_down_rows_kernel<<<blocks, kLdThreads, 0, stream>>>(m, rank, in_dim, x, rows, scale,
-                                                           norm_gain, eps, xn);
-  return cudaGetLastError();
+  LoraDownRows mp = m;
+  mp.prefetch = pdl_active() ? 1 : 0;
+  return launch_kernel(lora_down_rows_kernel, dim3(blocks), dim3(kLdThreads), 0, stream, mp, rank, in_dim, x,
+                       rows, scale, norm_gain, eps, xn);
 }
 
 // Bounded-wait self-test: thread 0 waits on an mbarrier that nothing arrives on. The wait
@@ -690,9 +714,8 @@ cudaError_t launch_rope_rows(float* q, int hq, float* k, int hkv, int rows, int 
                              cudaStream_t stream) {
   const int n = rows * (hq + hkv) * head_dim / 2;
   if (n == 0) return cudaSuccess;
-  rope_rows_kernel<<<cdiv(n, 256), 256, 0, stream>>>(q, hq, k, hkv, rows, head_dim, table, pos,
-                                                     table_by_row ? 1 : 0);
-  return cudaGetLastError();
+  return launch_kernel(rope_rows_kernel, dim3(cdiv(n, 256)), dim3(256), 0, stream, q, hq, k, hkv, rows, head_dim,
+                       table, pos, table_by_row ? 1 : 0);
 }
 
 // (cos, sin) of the rows' own positions only: table[r][i] for position pos[r].
@@ -722,6 +745,7 @@ __global__ void embed_rows_f32_kernel(const __nv_bfloat16* __restrict__ embed, c
 __global__ void kv_write_rows_kernel(const float* __restrict__ k, const float* __restrict__ v,
                                      __nv_bfloat16* kpages, __nv_bfloat16* vpages, const RowPages rp,
                                      int hkv, int d, int* status) {
+  griddep_begin();  // k, v come from the kernels before
   const int r = blockIdx.y;
   const int pos = rp.pos[r];
   const int page = checked_page(rp.page_table[r][pos / kPage], rp.num_pages,
@@ -797,10 +821,9 @@ cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, v
                                  const RowPages& rp, int rows, int hkv, int head_dim, int* status,
                                  cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
-  kv_write_rows_kernel<<<dim3(cdiv(hkv * head_dim, 256), rows), 256, 0, stream>>>(
-      k, v, static_cast<__nv_bfloat16*>(kpages), static_cast<__nv_bfloat16*>(vpages), rp, hkv, head_dim,
-      status);
-  return cudaGetLastError();
+  return launch_kernel(kv_write_rows_kernel, dim3(cdiv(hkv * head_dim, 256), rows), dim3(256), 0, stream, k, v,
+                       static_cast<__nv_bfloat16*>(kpages), static_cast<__nv_bfloat16*>(vpages), rp, hkv,
+                       head_dim, status);
 }
 
 cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
@@ -829,8 +852,7 @@ cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cuda
 cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
                                     cudaStream_t stream) {
   if (n == 0) return cudaSuccess;
-  swiglu_split_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(g, u, m, n);
-  return cudaGetLastError();
+  return launch_kernel(swiglu_split_f32_kernel, dim3(cdiv(n, 256)), dim3(256), 0, stream, g, u, m, n);
 }
 
 cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream) {
