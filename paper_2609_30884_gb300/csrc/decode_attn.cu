@@ -5,9 +5,9 @@
 // The work is memory-bound (K and V of every cached position are read once): the positions
 // are cut into chunks of 128 and streamed.
 //   decode_attn_stream  one block per SM, walking a run of consecutive chunks of one (row,
-//                       kv head) through a two-stage ring: a copy warp gathers each chunk's
-//                       K and V pages with TMA (128-byte swizzle) while four compute warps
-//                       score the previous one. The group's query heads (padded to 16 rows)
+//                       kv head) through a two-stage ring: a copy warp gathers the next
+//                       chunk's K and V pages with TMA (128-byte swizzle) while four compute
+//                       warps score the current one. The group's query heads (padded to 16 rows)
 //                       meet the chunk on mma.sync m16n8k16 (each warp takes a 32-key slice),
 //                       q entering as a bf16 pair hi + lo so the scores keep fp32 accuracy (K
 //                       is exact in bf16). Every warp keeps an online-softmax state (running
@@ -31,6 +31,7 @@ namespace crf {
 namespace {
 
 constexpr int kChunk = 128;                     // positions per chunk
+constexpr int kStages = 2;                      // K/V ring depth (64 KB per stage at d = 128)
 constexpr int kThreadsStream = 160;             // four compute warps + one copy warp
 constexpr int kMaxGroup = 8;
 
@@ -94,17 +95,17 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sKV = smem;                                      // [2 stages][K tile | V tile]
-  uint8_t* sQ = smem + 4 * TILE;                            // hi: [HALVES][16 rows][128 B], swizzled
+  uint8_t* sKV = smem;                                      // [kStages][K tile | V tile]
+  uint8_t* sQ = smem + 2 * kStages * TILE;                  // hi: [HALVES][16 rows][128 B], swizzled
   uint8_t* sQl = sQ + HALVES * QHALF;                       // lo, same layout
   __shared__ float red_m[4][16], red_l[4][16];
   __shared__ float s_self[16];  // the row's own key, scored in fp32
-  __shared__ __align__(8) uint64_t full[2], empty[2];
+  __shared__ __align__(8) uint64_t full[kStages], empty[kStages];
   __shared__ volatile int abort_flag;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kStages; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 4);
     }
@@ -117,10 +118,11 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
     // ---------------------------------------------------------------- producer
     if (lane == 0) {
       const int32_t* pt = p.page_table[r];
-      int armed[2] = {-1, -1};
+      int armed[kStages];
+      for (int st = 0; st < kStages; ++st) armed[st] = -1;
       for (int c = c_beg; c < c_end; ++c) {
-        const int i = c - c_beg, st = i & 1;
-        if (i >= 2 && !mbar_wait(&empty[st], ((i >> 1) - 1) & 1, &abort_flag, a.status)) break;
+        const int i = c - c_beg, st = i % kStages;
+        if (i >= kStages && !mbar_wait(&empty[st], (i / kStages - 1) & 1, &abort_flag, a.status)) break;
         const int t0 = c * kChunk;
         const int pages = (min(kChunk, pos - t0) + kPage - 1) / kPage;
         uint8_t* sK = sKV + st * 2 * TILE;
@@ -138,12 +140,12 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
               tma_load_2d(sV + off, &a.tmV, &full[st], 64 * h, row);
             }
           }
-          armed[st] = (i >> 1) & 1;
+          armed[st] = (i / kStages) & 1;
         }
       }
       // copies still in flight land before the block's shared memory is released
       volatile int never = 0;
-      for (int st = 0; st < 2; ++st)
+      for (int st = 0; st < kStages; ++st)
         if (armed[st] >= 0) mbar_wait(&full[st], armed[st], &never, nullptr);
     }
     return;
@@ -193,10 +195,10 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
     for (int e = 0; e < 4; ++e) O[dn][e] = 0.f;
   bool ok = true;
   for (int c = c_beg; c < c_end; ++c) {
-    const int i = c - c_beg, st = i & 1;
+    const int i = c - c_beg, st = i % kStages;
     const int t0 = c * kChunk;
     const int n_cached = min(kChunk, pos - t0);  // cached keys of this chunk
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&full[st], (i >> 1) & 1, &abort_flag, a.status));
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&full[st], (i / kStages) & 1, &abort_flag, a.status));
     const uint32_t k_base = smem_u32(sKV + st * 2 * TILE), v_base = k_base + TILE;
     if (n_cached < kChunk) {
       // the last chunk: V rows from the row's own slot on are zeroed (its value is added in
@@ -448,7 +450,7 @@ bool pool_map(CUtensorMap* m, const void* base, long rows, int cols) {
 
 template <int D>
 cudaError_t launch_dec(const DecodeArgs& args, int blocks, cudaStream_t stream) {
-  constexpr int smem = 4 * kChunk * D * 2 + 2 * 16 * D * 2 + 1024;  // two K/V stages, q hi/lo
+  constexpr int smem = 2 * kStages * kChunk * D * 2 + 2 * 16 * D * 2 + 1024;  // K/V stages, q hi/lo
   static bool set = false;
   if (!set) {
     cudaError_t e = cudaFuncSetAttribute(decode_attn_stream<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);

@@ -215,6 +215,7 @@ __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
   float inv = 1.f;
   if (g) {
     float ss = 0.f;
+#pragma unroll 4
     for (int i = threadIdx.x * 4; i < in_dim; i += kLdThreads * 4) {
       const float4 a = __ldg(reinterpret_cast<const float4*>(xr + i));
       ss += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
@@ -235,6 +236,7 @@ __global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
   }
   const __nv_bfloat16* A = m.A[mi] + (size_t)k * in_dim;
   float s = 0.f;
+#pragma unroll 4
   for (int i = threadIdx.x * 8; i < in_dim; i += kLdThreads * 8) {
     const uint4 u = __ldg(reinterpret_cast<const uint4*>(A + i));
     const float4* xp = reinterpret_cast<const float4*>(xr + i);
@@ -759,18 +761,45 @@ __global__ void kv_write_rows_kernel(const float* __restrict__ k, const float* _
 }
 
 // out[r] = argmax_i logits[r, i], the lowest index among equal maxima.
+// One block per row; 16-byte loads, four in flight per thread before their compares.
 __global__ void argmax_rows_kernel(const float* __restrict__ logits, int vocab, int32_t* out) {
   const int r = blockIdx.x;
   const float* z = logits + (size_t)r * vocab;
   float best = -INFINITY;
   int arg = 0x7fffffff;
-  for (int i = threadIdx.x; i < vocab; i += blockDim.x) {
-    const float v = z[i];
+  auto take = [&](float v, int i) {
     if (v > best || (v == best && i < arg)) {
       best = v;
       arg = i;
     }
+  };
+  // elements before the row's first 16-byte boundary, then whole float4s, then the tail
+  const int mis = static_cast<int>(reinterpret_cast<uintptr_t>(z) & 15) / 4;
+  const int head = min(vocab, mis ? 4 - mis : 0);
+  for (int i = threadIdx.x; i < head; i += blockDim.x) take(z[i], i);
+  const int n4 = (vocab - head) / 4;
+  const float4* z4 = reinterpret_cast<const float4*>(z + head);
+  constexpr int kU = 4;
+  for (int i0 = threadIdx.x; i0 < n4; i0 += kU * blockDim.x) {
+    float4 v[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int i = i0 + u * blockDim.x;
+      v[u] = i < n4 ? __ldg(z4 + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n4) {
+        const int b = head + 4 * i;
+        take(v[u].x, b);
+        take(v[u].y, b + 1);
+        take(v[u].z, b + 2);
+        take(v[u].w, b + 3);
+      }
+    }
   }
+  for (int i = head + 4 * n4 + threadIdx.x; i < vocab; i += blockDim.x) take(z[i], i);
   __shared__ float sb[32];
   __shared__ int sa[32];
   for (int o = 16; o > 0; o >>= 1) {
