@@ -27,13 +27,18 @@ default, float64 in the pins); norms' mean-square, softmax normalisation, KL and
 drift accumulate in float64. Parameters arrive as the bf16 values the GPU gets,
 upcast, so input quantisation is not counted as error.
 
-Parity pins (tests/test_oracle_*.py): merged == unmerged LoRA; brute-force and
-library attention; library RMSNorm/SiLU; complex-number RoPE; window(0, N) ==
-prefill; identical adapters reproduce the stale cache; a one-layer window after
-a query/output/MLP update leaves that layer's K/V unchanged (Eq. S4); KL
+Parity pins (tests/test_oracle_*.py): merged == unmerged LoRA and the alpha / r
+scale; brute-force and library attention; library RMSNorm/SiLU; complex-number
+RoPE; a whole decoder layer against a composition of torch library ops with
+merged weights; the final norm + LM head and the embedding lookup against
+torch; window(0, N) == prefill; identical adapters reproduce the stale cache; a
+one-layer window after a query/output/MLP update leaves that layer's K/V
+unchanged (Eq. S4); tail decode over a fresh cache gives the fresh logits; KL
 identities and the Eq. 4 / Eq. 5 certificates; factored == dense drift; policy
-worked examples printed in the paper (tests/golden/). Absolute K/V/H values at
-the Qwen-shaped sizes have no printed worked example: beyond these structural
-pins they are "parity unpinned".
+worked examples printed in the paper (tests/golden/). Every function here has
+at least one such pin. The paper prints no worked example of K/V/H values for
+its models, so those values are pinned through the library composition at
+small sizes and through identities that hold at any size, not through stored
+numbers.
 """
 from . import decoder, cache, fidelity, drift, policy  # noqa: F401

@@ -14,7 +14,7 @@ import torch
 
 import synth
 from .cache import Adapter, Model
-from .decoder import Dims, LayerAdapter, LayerParams
+from .decoder import Dims, LayerAdapter, LayerParams, lora_scale
 
 
 def _np(t: torch.Tensor) -> np.ndarray:
@@ -37,7 +37,7 @@ def layer_params(cfg: synth.ModelCfg, layer: int, seed: int = 0,
 def layer_adapter(cfg: synth.ModelCfg, lcfg: synth.LoraCfg, version: int, layer: int,
                   seed: int = 0, tensors=None) -> LayerAdapter:
     ab = tensors if tensors is not None else synth.adapter_version(cfg, lcfg, version, layer, seed)
-    return LayerAdapter({m: (_np(a), _np(b)) for m, (a, b) in ab.items()}, lcfg.scale)
+    return LayerAdapter({m: (_np(a), _np(b)) for m, (a, b) in ab.items()}, lora_scale(lcfg.alpha, lcfg.rank))
 
 
 def model(cfg: synth.ModelCfg, seed: int = 0, layers: Optional[Iterable[int]] = None,

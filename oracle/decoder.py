@@ -136,9 +136,17 @@ class LayerParams:
 
 @dataclass
 class LayerAdapter:
-    """LoRA factors of one layer: m -> (A [r, in], B [out, r]); modules absent are unadapted."""
+    """LoRA factors of one layer: m -> (A [r, in], B [out, r]); modules absent are unadapted.
+
+    ``scale`` multiplies B A (``lora_scale``)."""
     AB: Dict[str, Tuple[np.ndarray, np.ndarray]]
     scale: float
+
+
+def lora_scale(alpha: float, rank: int) -> float:
+    """alpha / r: the factor of the low-rank update B A in the LoRA parameterisation the paper
+    adopts (Section 1, citing LoRA; the adapter of Section 5.1 is stated by rank and alpha)."""
+    return float(alpha) / float(rank)
 
 
 def _proj(x, P: LayerParams, ad: LayerAdapter, m: str, dt):

@@ -69,10 +69,6 @@ class LoraCfg:
     step_std: float = 0.005
 
     @property
-    def scale(self) -> float:
-        return self.alpha / self.rank
-
-    @property
     def mask(self) -> int:
         return sum(1 << MODULES.index(m) for m in self.modules)
 

@@ -36,7 +36,7 @@ def oracle_model(dm) -> C.Model:
 
 def oracle_adapter(da) -> C.Adapter:
     return C.Adapter([LayerAdapter({m: (to_np(a), to_np(b)) for m, (a, b) in d.items()},
-                                   da.lcfg.scale) if d is not None else None
+                                   Dec.lora_scale(da.lcfg.alpha, da.lcfg.rank)) if d is not None else None
                       for d in da.layers])
 
 

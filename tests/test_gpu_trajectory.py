@@ -16,7 +16,7 @@ import torch
 import synth
 from harness import DeviceModel, pages_needed, split_page_tables
 from oracle import cache as C, drift as odrift, fidelity, policy as OP
-from oracle.decoder import LayerAdapter
+from oracle.decoder import LayerAdapter, lora_scale
 from tests.gpu_util import KL_ABS, oracle_model
 
 pytestmark = pytest.mark.gpu
@@ -32,7 +32,7 @@ def _oracle_adapter(t):
         if l == LAYER and t > 0:
             d[MODULE] = synth.trajectory_factors(CFG, LC, BASE, LAYER, MODULE, t, STD, SEED)
         layers.append(LayerAdapter({m: (a.float().numpy(), b.float().numpy()) for m, (a, b) in d.items()},
-                                   LC.scale))
+                                   lora_scale(LC.alpha, LC.rank)))
     return C.Adapter(layers), layers
 
 

@@ -158,3 +158,30 @@ def test_recovery_with_restart_state_argument(tiny):
     x_a = C.run_window(model, v1, pool, req, 2, 4)
     x_b = C.run_window(model, v1, pool2, req2, 2, 4, restart=h1)
     np.testing.assert_array_equal(x_a, x_b)
+
+
+def test_logits_match_library_final_norm_and_head(tiny):
+    """z = W_lm (rmsnorm(h) * g_f): against torch's rms_norm and linear in float64."""
+    import torch
+    import torch.nn.functional as F
+    model, _, _ = tiny
+    rng = np.random.default_rng(11)
+    h = rng.standard_normal((3, CFG.hidden)) * 2.0
+    z = C.logits(model, h, np.float64)
+    t = lambda a: torch.tensor(np.asarray(a, np.float64))
+    want = F.linear(F.rms_norm(t(h), (CFG.hidden,), t(model.final_norm), CFG.rms_eps),
+                    t(model.lm_head)).numpy()
+    np.testing.assert_allclose(z, want, rtol=1e-12, atol=1e-12)
+    # a single row gives its row of the batch (up to the BLAS blocking of a 1-row product)
+    np.testing.assert_allclose(C.logits(model, h[1], np.float64)[0], z[1], rtol=1e-12, atol=1e-13)
+
+
+def test_embed_matches_library_lookup(tiny):
+    """H_{-1} = E[tokens]: against torch's embedding lookup, repeated ids included."""
+    import torch
+    import torch.nn.functional as F
+    model, _, _ = tiny
+    tokens = np.array([0, CFG.vocab - 1, 5, 5, 17])
+    got = C.embed(model, tokens, np.float64)
+    want = F.embedding(torch.tensor(tokens), torch.tensor(np.asarray(model.embed, np.float64))).numpy()
+    np.testing.assert_array_equal(got, want)

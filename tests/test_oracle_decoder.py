@@ -175,3 +175,14 @@ def test_float32_path_close_to_float64():
     h64, _, _ = D.decoder_layer(x, P, ad, dims, np.float64)
     h32, _, _ = D.decoder_layer(x, P, ad, dims, np.float32)
     assert np.linalg.norm(h32 - h64) / np.linalg.norm(h64) < 1e-5
+
+
+def test_lora_scale_is_alpha_over_rank():
+    """The adapter update enters as (alpha / r) B A: rank 8, alpha 16 -> 2; rank 16, alpha 32 -> 2."""
+    assert D.lora_scale(16.0, 8) == 2.0 and D.lora_scale(32.0, 16) == 2.0 and D.lora_scale(8.0, 4) == 2.0
+    # doubling the rank with the same factors padded by zeros halves the update at fixed alpha
+    W, A, B = _r(6, 5), _r(2, 5), _r(6, 2)
+    A2 = np.concatenate([A, np.zeros_like(A)]); B2 = np.concatenate([B, np.zeros_like(B)], 1)
+    d1 = D.merged_weight(W, A, B, D.lora_scale(4.0, 2)) - W
+    d2 = D.merged_weight(W, A2, B2, D.lora_scale(4.0, 4)) - W
+    np.testing.assert_allclose(d2, d1 / 2, rtol=1e-12, atol=1e-14)
