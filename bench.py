@@ -37,6 +37,9 @@ if ROOT not in sys.path:
 
 METRIC = "recomputed layer*tokens/s"
 UNIT = "layer*tokens/s"
+# refresh sweep of the single-prefix workloads: window lengths from the workload's window start,
+# and starts of complete affected suffixes (..N); full prefill is always timed. Default: 1, 2, 4.
+SWEEPS = {"1.5b-16k": ((1, 2, 4, 8), (14, 26))}
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu --set full
 # capture of the kernel as it now stands, at the full launch size of the 7B-shape 16K workload
@@ -277,7 +280,7 @@ def time_refresh(ctx, st, s, e, reps=3):
     elif w0[0] <= s - 1 < w0[1]:
         hin = st["h_out"][0][s - 1 - w0[0]]
     else:
-        return None
+        hin = st["h_in"][0]  # a stand-in restart state: the refresh's cost does not depend on its values
     outs = [_t.empty(n, st["cfg"].hidden, dtype=_t.bfloat16, device=st["fin"].device)
             for _ in range(e - s)]
     req = crf.Request(st["pts"][0], s, e, n_tokens=n, tokens=st["tokens"][0], hidden_in=hin,
@@ -884,8 +887,11 @@ def main():
     # ---------------- window sweep (ms per 16K-prefix refresh)
     sweep = {}
     if not args.no_sweep and len(st["ns"]) == 1:
-        for ln in (1, 2, 4):
+        lengths, suffix_starts = SWEEPS.get(args.workload, ((1, 2, 4), ()))
+        for ln in lengths:
             sweep[f"window_{ln}"] = round(time_refresh(ctx, st, s, min(s + ln, cfg.n_layers)), 3)
+        for s0 in suffix_starts:
+            sweep[f"suffix_{s0}_{cfg.n_layers}"] = round(time_refresh(ctx, st, s0, cfg.n_layers, reps=2), 3)
         sweep["full_prefill_28"] = round(time_refresh(ctx, st, 0, cfg.n_layers, reps=2), 3)
         sweep["layer_tokens_per_s_full"] = round(cfg.n_layers * n / (sweep["full_prefill_28"] / 1000.0))
 
