@@ -345,7 +345,7 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-            "data": "synthetic (seeded counter-based generator, random-init Qwen2.5-7B shape)",
+            "data": f"synthetic (seeded counter-based generator, random-init {wl.model.name})",
             "config": config_of(wl),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": sample},
@@ -898,7 +898,7 @@ def main():
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic (seeded counter-based generator, random-init Qwen2.5-7B shape)",
+            "data": f"synthetic (seeded counter-based generator, random-init {wl.model.name})",
             "config": config_of(wl), "gpu_launches": gpu_launches, "e2e": e2e,
             "roofline": roofline, "clocks": clk,
             "gemm_tflops_all": round(gemm_tf, 1),
