@@ -651,7 +651,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
       a.n_kv_heads = D.hkv;
       a.head_dim = D.d;
       a.splits = p.splits;
-      CRF_CUDA(launch_decode_attention(a, c.pool->num_pages, c.ctx->status_dev, c.st));
+      CRF_CUDA(launch_decode_attention(a, c.pool->num_pages, c.ctx->num_sms, c.ctx->status_dev, c.st));
       if (opt.write_kv) {
         RowPages pg{};
         for (int i = 0; i < nr; ++i) {

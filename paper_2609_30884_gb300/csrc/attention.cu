@@ -249,22 +249,24 @@ cudaError_t launch_attention(const AttnDesc& d, int num_sms, cudaStream_t stream
   if (items == 0) return cudaSuccess;
   if (d.head_dim == 128) {
     constexpr int smem = (kBM + 4 * kBN) * 128 * 2;
-    static bool set = false;
-    if (!set) {
+    static PerDevice once;
+    int dev = 0;
+    if (once.pending(&dev)) {
       cudaError_t e = cudaFuncSetAttribute(attn_prefill_kernel<128>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
       if (e != cudaSuccess) return e;
-      set = true;
+      once.done(dev);
     }
     attn_prefill_kernel<128><<<items, kWarps * 32, smem, stream>>>(d);
   } else if (d.head_dim == 64) {
     constexpr int smem = (kBM + 4 * kBN) * 64 * 2;
-    static bool set = false;
-    if (!set) {
+    static PerDevice once;
+    int dev = 0;
+    if (once.pending(&dev)) {
       cudaError_t e = cudaFuncSetAttribute(attn_prefill_kernel<64>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
       if (e != cudaSuccess) return e;
-      set = true;
+      once.done(dev);
     }
     attn_prefill_kernel<64><<<items, kWarps * 32, smem, stream>>>(d);
   } else {

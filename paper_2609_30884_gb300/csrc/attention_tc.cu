@@ -491,8 +491,9 @@ bool map2d(CUtensorMap* m, const void* base, long rows, int cols, int box_rows) 
 template <int D>
 cudaError_t launch_tc(const AttnTcArgs& args, cudaStream_t stream) {
   constexpr int smem = 2 * kM * D * 2 + kSlots * kN * D * 2 + 1024;
-  static bool set = false;
-  if (!set) {
+  static PerDevice once;
+  int dev = 0;
+  if (once.pending(&dev)) {
     cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     // setmaxnreg.inc waits until the CTA's register pool can serve it: refuse to launch a
@@ -501,7 +502,7 @@ cudaError_t launch_tc(const AttnTcArgs& args, cudaStream_t stream) {
     e = cudaFuncGetAttributes(&fa, attn_tc_kernel<D>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs * kThreadsAttn < kRegsNeeded) return cudaErrorInvalidConfiguration;
-    set = true;
+    once.done(dev);
   }
   attn_tc_kernel<D><<<args.total_items, kThreadsAttn, smem, stream>>>(args);
   return cudaGetLastError();

@@ -451,11 +451,12 @@ bool pool_map(CUtensorMap* m, const void* base, long rows, int cols) {
 template <int D>
 cudaError_t launch_dec(const DecodeArgs& args, int blocks, cudaStream_t stream) {
   constexpr int smem = 2 * kStages * kChunk * D * 2 + 2 * 16 * D * 2 + 1024;  // K/V stages, q hi/lo
-  static bool set = false;
-  if (!set) {
+  static PerDevice once;
+  int dev = 0;
+  if (once.pending(&dev)) {
     cudaError_t e = cudaFuncSetAttribute(decode_attn_stream<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    set = true;
+    once.done(dev);
   }
   const DecodeAttnDesc& d = args.d;
   cudaError_t e = launch_kernel(decode_attn_stream<D>, dim3(blocks), dim3(kThreadsStream), smem, stream, args);
@@ -468,7 +469,7 @@ cudaError_t launch_dec(const DecodeArgs& args, int blocks, cudaStream_t stream) 
 
 int decode_attention_splits(int max_positions) { return std::max(1, (max_positions + kChunk - 1) / kChunk); }
 
-cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int* status,
+cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int num_sms, int* status,
                                     cudaStream_t stream) {
   if (d.rows < 1) return cudaSuccess;
   if (d.n_q_heads % d.n_kv_heads != 0 || d.n_q_heads / d.n_kv_heads > kMaxGroup)
@@ -478,13 +479,7 @@ cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int*
   if (max_pos / kChunk + 1 > d.splits) return cudaErrorInvalidValue;
   // one block per SM (two 64 KB K/V stages each), each streaming a run of consecutive chunks
   // of one (row, kv head): the fewest chunks per block that keeps every block in one wave
-  static int num_sms = 0;
-  if (num_sms == 0) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess || num_sms < 1) return e != cudaSuccess ? e : cudaErrorInvalidValue;
-  }
+  if (num_sms < 1) return cudaErrorInvalidValue;
   long items = 0;
   for (int r = 0; r < d.rows; ++r) items += static_cast<long>(d.n_kv_heads) * (d.pos[r] / kChunk + 1);
   int cpb = static_cast<int>(std::max(1L, (items + num_sms - 1) / num_sms));

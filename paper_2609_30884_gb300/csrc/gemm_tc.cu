@@ -584,8 +584,13 @@ template <int BN, int STAGES, int PAIR>
 cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) {
   constexpr int smem = STAGES * (BM * BK * 2 + (BN / PAIR) * BK * 2) + 1024;
   auto kern = gemm_tc_kernel<BN, STAGES, PAIR>;
-  static int max_units = 0;
-  if (max_units == 0) {
+  // the attributes and the co-resident cluster count are per device
+  static PerDevice once;
+  static std::atomic<int> units_of[64];
+  int dev = 0, max_units = 0;
+  if (!once.pending(&dev)) {
+    max_units = units_of[dev].load(std::memory_order_relaxed);
+  } else {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     if (PAIR == 2) {
@@ -608,6 +613,8 @@ cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) 
     } else {
       max_units = num_sms;
     }
+    if (dev >= 0 && dev < 64) units_of[dev].store(max_units, std::memory_order_relaxed);
+    once.done(dev);
   }
   const int units = std::max(1, std::min(max_units, args.total_tiles));
   if (PAIR == 1) {
@@ -632,12 +639,11 @@ cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) 
 }  // namespace
 
 bool pair_mode_enabled() {
-  static int on = -1;
-  if (on < 0) {
+  static const bool on = [] {
     const char* v = std::getenv("CRF_GEMM_PAIR");
-    on = (v && v[0] == '0') ? 0 : 1;
-  }
-  return on == 1;
+    return !(v && v[0] == '0');
+  }();
+  return on;
 }
 
 cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream) {

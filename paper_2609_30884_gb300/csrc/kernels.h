@@ -7,7 +7,26 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace crf {
+
+// One-time set-up that CUDA keeps per device (kernel attributes): bit d of the mask records
+// device d. Host threads may race to do it; doing it twice is harmless.
+class PerDevice {
+ public:
+  // Sets *dev to the current device; true while its set-up is still to do.
+  bool pending(int* dev) const {
+    if (cudaGetDevice(dev) != cudaSuccess) *dev = -1;
+    return *dev < 0 || *dev >= 64 || !((mask_.load(std::memory_order_acquire) >> *dev) & 1u);
+  }
+  void done(int dev) {
+    if (dev >= 0 && dev < 64) mask_.fetch_or(1ull << dev, std::memory_order_acq_rel);
+  }
+
+ private:
+  std::atomic<uint64_t> mask_{0};
+};
 
 constexpr int kMaxReq = 32;   // equals CRF_MAX_REQUESTS
 constexpr int kPage = 16;
@@ -207,7 +226,7 @@ struct DecodeAttnDesc {
 // Decode attention streamed in 128-position chunks (TMA-staged pages, one block per SM walking
 // a run of chunks of one row and kv head) + merge of the blocks' partials. `splits` in the
 // descriptor must be at least decode_attention_splits(max position + 1).
-cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int* status,
+cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int num_sms, int* status,
                                     cudaStream_t stream);
 int decode_attention_splits(int max_positions);
 struct RowPositions {

@@ -609,12 +609,11 @@ cudaError_t gemv_dispatch(const GemvLaunch& L, int blocks, cudaStream_t stream) 
 namespace {
 thread_local bool t_pdl = false;
 bool pdl_env() {
-  static int v = -1;
-  if (v < 0) {
+  static const bool on = [] {
     const char* e = std::getenv("CRF_PDL");
-    v = (e && std::strcmp(e, "0") == 0) ? 0 : 1;
-  }
-  return v == 1;
+    return !(e && std::strcmp(e, "0") == 0);
+  }();
+  return on;
 }
 }  // namespace
 
@@ -623,12 +622,11 @@ PdlScope::~PdlScope() { t_pdl = prev_; }
 bool pdl_active() { return t_pdl; }
 
 static bool gemv_scalar() {
-  static int v = -1;
-  if (v < 0) {
+  static const bool on = [] {
     const char* e = std::getenv("CRF_GEMV");
-    v = (e && std::strcmp(e, "scalar") == 0) ? 1 : 0;
-  }
-  return v == 1;
+    return e && std::strcmp(e, "scalar") == 0;
+  }();
+  return on;
 }
 
 bool gemv_use_tensor(int total_rows, int in_dim) {
