@@ -34,7 +34,10 @@
  *     enqueued on it; results are valid once the stream has synchronised.
  *   - Every argument is validated on the host before anything is launched.
  *     A non-OK status means nothing was enqueued and nothing was written;
- *     crf_last_error() then returns a message (thread-local).
+ *     crf_last_error() then returns a message (thread-local). For the page
+ *     ids, crf_recompute_window and crf_decode_step read each page table back
+ *     to the host on `stream` and wait for it. That waits for the work already
+ *     on `stream`, and it keeps these two calls out of CUDA graph capture.
  *   - A kernel that gives up on a bounded internal wait records it in the
  *     context; crf_check() reports it as CRF_ETIMEOUT. An asynchronous CUDA
  *     error is reported as CRF_ECUDA by the next call.
