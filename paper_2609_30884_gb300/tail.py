@@ -76,9 +76,14 @@ def sweep(ctx: Context, model: Model, adapter: Adapter, stale: KVPool, page_tabl
     ws = ctx.kl_workspace(N + 1, vocab, hidden)
     ctx.kl(model, ref, rows, out_kl, vocab, ws, logits_out=logits)
     ctx.check()
-    z = logits[N + 1:].double().cpu().numpy()
-    z_star = z[N]
-    kl = out_kl.double().cpu().numpy()
+    return certificates(logits[N + 1:].double().cpu().numpy(), out_kl.double().cpu().numpy(), kl_slack)
+
+
+def certificates(z: np.ndarray, kl: np.ndarray, kl_slack: float = 1e-4) -> TailSweep:
+    """The host side of the sweep from the hybrid logits z [N + 1, V] (z[N] = z*) and their KLs."""
+    z = np.asarray(z, np.float64)
+    kl = np.asarray(kl, np.float64)
+    z_star = z[-1]
     v_norm = np.linalg.norm(z[:-1] - z[1:], axis=1)
     tail = np.concatenate([np.cumsum(v_norm[::-1])[::-1], [0.0]])
     top = np.sort(z_star)
