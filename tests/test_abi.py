@@ -54,6 +54,7 @@ STRUCTS = {
     "crf_kv_pool": (abi.KVPool, ["k_pages", "v_pages", "num_pages"]),
     "crf_request": (abi.Request, ["n_tokens", "s", "e", "page_table", "tokens", "hidden_in",
                                   "hidden_out", "final_hidden_out"]),
+    "crf_decode_row": (abi.DecodeRow, ["pos", "page_table", "token"]),
 }
 
 
