@@ -33,8 +33,14 @@
  *   - `stream` is a cudaStream_t (NULL = legacy default stream). Work is
  *     enqueued on it; results are valid once the stream has synchronised.
  *   - Every argument is validated on the host before anything is launched.
- *     A non-OK status means nothing was enqueued and nothing was written;
- *     crf_last_error() then returns a message (thread-local). For the page
+ *     A non-OK status from validation (CRF_EINVAL, CRF_ESHAPE,
+ *     CRF_EUNSUPPORTED, CRF_ENOMEM) means nothing was enqueued and nothing
+ *     was written. A CRF_ECUDA from a failed launch can leave the call's
+ *     earlier kernels enqueued; their outputs are then undefined.
+ *     crf_last_error() returns a message in either case (thread-local).
+ *   - A context is used by one host thread at a time: its device status word
+ *     and timing state are shared by its calls. Separate contexts may run
+ *     concurrently. For the page
  *     ids, crf_recompute_window and crf_decode_step read each page table back
  *     to the host on `stream` and wait for it. That waits for the work already
  *     on `stream`, and it keeps these two calls out of CUDA graph capture.
