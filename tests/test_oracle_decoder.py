@@ -100,6 +100,18 @@ def test_attention_matches_torch_sdpa_gqa():
     np.testing.assert_allclose(got, ref.transpose(0, 1).numpy(), rtol=1e-10, atol=1e-12)
 
 
+@pytest.mark.parametrize("hq,hkv,d,n,chunk", [(28, 4, 128, 300, 128), (12, 2, 128, 257, 64), (4, 2, 64, 129, 512)],
+                         ids=["7b-heads", "1.5b-heads", "tiny-heads"])
+def test_attention_matches_torch_sdpa_at_model_head_shapes(hq, hkv, d, n, chunk):
+    """The model families' head layouts (GQA 7:1 and 6:1 at d = 128, 2:1 at d = 64), lengths that
+    leave a ragged last query chunk, fp64 against the library routine."""
+    q, k, v = _r(n, hq, d), _r(n, hkv, d), _r(n, hkv, d)
+    got = D.causal_gqa_attention(q, k, v, chunk=chunk, dt=np.float64)
+    tq, tk, tv = (torch.tensor(t).transpose(0, 1)[None] for t in (q, k, v))
+    ref = F.scaled_dot_product_attention(tq, tk, tv, is_causal=True, enable_gqa=True)[0]
+    np.testing.assert_allclose(got, ref.transpose(0, 1).numpy(), rtol=1e-10, atol=1e-12)
+
+
 def test_single_query_attention_is_last_row_of_causal():
     q, k, v = _r(13, 4, 8), _r(13, 2, 8), _r(13, 2, 8)
     full = D.causal_gqa_attention(q, k, v, dt=np.float64)
