@@ -119,15 +119,17 @@ def test_single_query_attention_is_last_row_of_causal():
     np.testing.assert_allclose(row, full[-1], rtol=1e-12, atol=1e-13)
 
 
-def _tiny_layer(seed=0, bias=True):
+def _tiny_layer(seed=0, bias=True, dims=None, wstd=0.2):
     rng = np.random.default_rng(seed)
-    dims = D.Dims(hidden=32, n_q_heads=4, n_kv_heads=2, head_dim=8, ffn=48, rms_eps=1e-6,
-                  rope_theta=1e4)
-    shapes = {"q": (32, 32), "k": (16, 32), "v": (16, 32), "o": (32, 32), "gate": (48, 32),
-              "up": (48, 32), "down": (32, 48)}
-    W = {m: rng.standard_normal(s) * 0.2 for m, s in shapes.items()}
+    if dims is None:
+        dims = D.Dims(hidden=32, n_q_heads=4, n_kv_heads=2, head_dim=8, ffn=48, rms_eps=1e-6,
+                      rope_theta=1e4)
+    h, qd, kvd, f = dims.hidden, dims.n_q_heads * dims.head_dim, dims.n_kv_heads * dims.head_dim, dims.ffn
+    shapes = {"q": (qd, h), "k": (kvd, h), "v": (kvd, h), "o": (h, qd), "gate": (f, h),
+              "up": (f, h), "down": (h, f)}
+    W = {m: rng.standard_normal(s) * wstd for m, s in shapes.items()}
     b = {m: rng.standard_normal(shapes[m][0]) * 0.1 for m in ("q", "k", "v")} if bias else {}
-    P = D.LayerParams(W, b, 1 + 0.1 * rng.standard_normal(32), 1 + 0.1 * rng.standard_normal(32))
+    P = D.LayerParams(W, b, 1 + 0.1 * rng.standard_normal(h), 1 + 0.1 * rng.standard_normal(h))
     AB = {m: (rng.standard_normal((4, s[1])) * 0.1, rng.standard_normal((s[0], 4)) * 0.1)
           for m, s in shapes.items()}
     return dims, P, D.LayerAdapter(AB, 2.0)
@@ -170,6 +172,20 @@ def test_decoder_layer_matches_library_composition():
     np.testing.assert_allclose(h, rh, rtol=1e-10, atol=1e-11)
     np.testing.assert_allclose(k, rk, rtol=1e-10, atol=1e-11)
     np.testing.assert_allclose(v, rv, rtol=1e-10, atol=1e-11)
+
+
+def test_decoder_layer_matches_library_composition_at_head_dim_128():
+    """Head dim 128 with GQA 7:1 and theta 1e6 (the model families' RoPE frequencies), a ragged
+    last query chunk."""
+    dims = D.Dims(hidden=256, n_q_heads=7, n_kv_heads=1, head_dim=128, ffn=320, rms_eps=1e-6,
+                  rope_theta=1e6)
+    dims, P, ad = _tiny_layer(4, dims=dims, wstd=0.06)
+    x = _r(37, 256)
+    h, k, v = D.decoder_layer(x, P, ad, dims, np.float64, chunk=16)
+    rh, rk, rv = _torch_layer(x, dims, P, ad)
+    np.testing.assert_allclose(h, rh, rtol=1e-9, atol=1e-10)
+    np.testing.assert_allclose(k, rk, rtol=1e-9, atol=1e-10)
+    np.testing.assert_allclose(v, rv, rtol=1e-9, atol=1e-10)
 
 
 def test_decode_row_matches_prefill_last_row():
