@@ -15,7 +15,8 @@ Layout:
   prefill, executable window restart (Section 4.2) and the first-step
   next-token logits of a hybrid cache (Section 3.1, Section S1.2).
 * ``fidelity`` -- forward KL at the first generated-token step (Section S2.1),
-  top-1 agreement, tail influence and its certificates (Eq. 2, 4, 5, S7-S15).
+  top-1 agreement, tail influence and its certificates (Eq. 2, 4, 5; derived in
+  Section S1.2).
 * ``drift``    -- adapter displacement per layer and module (Eq. 8), dense and
   rank-factored.
 * ``policy``   -- host recovery policy: invalidation onset (Eq. S4), candidate

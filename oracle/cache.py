@@ -30,7 +30,8 @@ PAGE = 16
 
 
 class PagedPool:
-    """Per-layer K and V page pools, [num_pages, Hkv, 16, d] each."""
+    """Per-layer K and V page pools, [num_pages, Hkv, 16, d] each: the layerwise cache of Eq. 1,
+    stored in 16-token pages that requests address through page tables."""
 
     def __init__(self, n_layers: int, num_pages: int, n_kv_heads: int, head_dim: int,
                  dtype=np.float32):
@@ -40,20 +41,24 @@ class PagedPool:
 
     @staticmethod
     def slots(page_table: np.ndarray, n: int):
+        """(page, offset) of positions 0..n-1: page_table[t // 16], t % 16 (the Eq. 1 cache's layout)."""
         t = np.arange(n)
         return np.asarray(page_table)[t // PAGE], t % PAGE
 
     def write(self, layer: int, page_table: np.ndarray, k: np.ndarray, v: np.ndarray) -> None:
-        """Store k/v [n, Hkv, d] of positions 0..n-1 of one request at its slots of ``layer``."""
+        """Store k/v [n, Hkv, d] of positions 0..n-1 of one request at its slots of ``layer``: the
+        overwrite of a layer's K/V entries by recomputation (Section 4.2)."""
         pages, off = self.slots(page_table, k.shape[0])
         self.k[layer][pages, :, off, :] = k
         self.v[layer][pages, :, off, :] = v
 
     def read(self, layer: int, page_table: np.ndarray, n: int):
+        """K, V [n, Hkv, d] of positions 0..n-1 of one request at ``layer`` (Eq. 1 entries)."""
         pages, off = self.slots(page_table, n)
         return self.k[layer][pages, :, off, :], self.v[layer][pages, :, off, :]
 
     def copy(self) -> "PagedPool":
+        """An independent copy: a stale cache C^(t) kept while another is built (Eq. 1)."""
         out = PagedPool.__new__(PagedPool)
         out.k = [a.copy() for a in self.k]
         out.v = [a.copy() for a in self.v]
@@ -62,7 +67,8 @@ class PagedPool:
 
 @dataclass
 class Model:
-    """Base model: per-layer params, embedding, final norm and LM head (float arrays)."""
+    """Base model: per-layer params, embedding, final norm and LM head (float arrays); the frozen
+    base of Section 2.1."""
     dims: Dims
     layers: List[LayerParams]
     embed: np.ndarray
@@ -71,24 +77,27 @@ class Model:
 
     @property
     def n_layers(self) -> int:
+        """N, the layers 0..N-1 of Eq. 1."""
         return len(self.layers)
 
 
 @dataclass
 class Adapter:
-    """One adapter version theta_t: per-layer LoRA factors."""
+    """One adapter version theta_t: per-layer LoRA factors (Section 2.1, adapter evolution)."""
     layers: List[LayerAdapter]
 
 
 @dataclass
 class RequestCache:
-    """Per-request state: tokens, page table and retained hidden states H_l (l = -1..N-1)."""
+    """Per-request state: tokens, page table and retained hidden states H_l (l = -1..N-1), the
+    boundary states an executable restart reads (Section 4.2)."""
     tokens: np.ndarray
     page_table: np.ndarray
     hidden: Dict[int, np.ndarray] = field(default_factory=dict)
 
     @property
     def n(self) -> int:
+        """n, the prefix length x_{1:n} of Eq. 1."""
         return int(self.tokens.shape[0])
 
 
@@ -131,7 +140,8 @@ def tail_decode(model: Model, adapter: Adapter, pool: PagedPool, req: RequestCac
                 h_row: np.ndarray, dt=np.float32) -> np.ndarray:
     """Carry row n-1 through layers e..N-1 against the cached K/V of those layers.
 
-    Writes nothing: layers at and after the window end keep their historical cache.
+    Writes nothing: layers at and after the window end keep their historical cache. This is the
+    hybrid execution of Section 3.1 with boundary b = e, the first-step state of Section S2.1.
     """
     n = req.n
     x = np.asarray(h_row, dtype=dt).reshape(1, -1)
@@ -143,7 +153,9 @@ def tail_decode(model: Model, adapter: Adapter, pool: PagedPool, req: RequestCac
 
 
 def logits(model: Model, h_final: np.ndarray, dt=np.float32) -> np.ndarray:
-    """z = W_lm rmsnorm(h) * g_f for final hidden rows h [.., hidden]; returned in float64."""
+    """z = W_lm rmsnorm(h) * g_f for final hidden rows h [.., hidden]; returned in float64.
+
+    The first-step next-token logits z of Section 3.1 (z* for the fresh row)."""
     hn = rmsnorm(np.atleast_2d(h_final), model.final_norm, model.dims.rms_eps, dt)
     return (hn @ np.asarray(model.lm_head, dtype=dt).T).astype(np.float64)
 

@@ -27,6 +27,7 @@ MODULES = ("q", "k", "v", "o", "gate", "up", "down")
 
 @dataclass
 class Dims:
+    """Shape of the decoder block of the model family in Section 5.1 (Qwen2.5)."""
     hidden: int
     n_q_heads: int
     n_kv_heads: int
@@ -37,7 +38,9 @@ class Dims:
 
 
 def rmsnorm(x: np.ndarray, g: np.ndarray, eps: float, dt=np.float32) -> np.ndarray:
-    """Row-wise RMSNorm: x / sqrt(mean(x^2) + eps) * g, mean-square accumulated in fp64."""
+    """Row-wise RMSNorm: x / sqrt(mean(x^2) + eps) * g, mean-square accumulated in fp64.
+
+    The normalisation of the block input that Section S1.1 writes as the bar in H-bar (Eq. S3)."""
     x = np.asarray(x, dtype=dt)
     ms = np.mean(np.square(x.astype(np.float64)), axis=-1, keepdims=True)
     inv = (1.0 / np.sqrt(ms + eps)).astype(dt)
@@ -46,7 +49,10 @@ def rmsnorm(x: np.ndarray, g: np.ndarray, eps: float, dt=np.float32) -> np.ndarr
 
 def lora_linear(x: np.ndarray, W: np.ndarray, A: Optional[np.ndarray], B: Optional[np.ndarray],
                 scale: float, bias: Optional[np.ndarray] = None, dt=np.float32) -> np.ndarray:
-    """y = x W^T (+ b) + scale * (x A^T) B^T with W [out,in], A [r,in], B [out,r] (unmerged LoRA)."""
+    """y = x W^T (+ b) + scale * (x A^T) B^T with W [out,in], A [r,in], B [out,r] (unmerged LoRA).
+
+    A projection of Eq. S3 under the current adapter: frozen base weight plus the adapter's
+    low-rank update (Section 2.1, Section 5.1)."""
     x = np.asarray(x, dtype=dt)
     y = x @ np.asarray(W, dtype=dt).T
     if bias is not None:
@@ -58,7 +64,9 @@ def lora_linear(x: np.ndarray, W: np.ndarray, A: Optional[np.ndarray], B: Option
 
 
 def rope_angles(positions: np.ndarray, head_dim: int, theta: float) -> Tuple[np.ndarray, np.ndarray]:
-    """cos/sin of p * theta^(-2i/d) for i < d/2, computed in fp64. Shapes [n, d/2]."""
+    """cos/sin of p * theta^(-2i/d) for i < d/2, computed in fp64. Shapes [n, d/2].
+
+    The positional rotation that Eq. S3 suppresses, in the model family's rotate-half form."""
     i = np.arange(head_dim // 2, dtype=np.float64)
     inv_freq = theta ** (-2.0 * i / head_dim)
     ang = np.asarray(positions, dtype=np.float64)[:, None] * inv_freq[None, :]
@@ -66,7 +74,9 @@ def rope_angles(positions: np.ndarray, head_dim: int, theta: float) -> Tuple[np.
 
 
 def apply_rope(x: np.ndarray, cos: np.ndarray, sin: np.ndarray, dt=np.float32) -> np.ndarray:
-    """Rotate-half rotary embedding on x [n, H, d]: pairs (i, i + d/2) rotate by the angle of i."""
+    """Rotate-half rotary embedding on x [n, H, d]: pairs (i, i + d/2) rotate by the angle of i.
+
+    Applied to q and k before K is cached (the rotation Eq. S3 suppresses)."""
     x = np.asarray(x, dtype=dt)
     half = x.shape[-1] // 2
     c = cos.astype(dt)[:, None, :]
@@ -76,6 +86,7 @@ def apply_rope(x: np.ndarray, cos: np.ndarray, sin: np.ndarray, dt=np.float32) -
 
 
 def silu(x: np.ndarray) -> np.ndarray:
+    """x * sigmoid(x), the gate of the SwiGLU MLP of the model family's block (Section 5.1)."""
     with np.errstate(over="ignore"):
         return x / (1.0 + np.exp(-x))
 
@@ -91,7 +102,8 @@ def causal_gqa_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, chunk: int
     """softmax(q k^T / sqrt(d) + causal mask) v per query head, over the whole prefix.
 
     q [n, Hq, d], k/v [n, Hkv, d]; query head h reads kv head h // (Hq/Hkv). Query i sees keys
-    j <= i. Query rows are processed in chunks only to bound memory.
+    j <= i. Query rows are processed in chunks only to bound memory. The self-attention of the
+    block whose K, V form the cache of Eq. 1 (Eq. S3).
     """
     n, hq, d = q.shape
     hkv = k.shape[1]
@@ -113,7 +125,9 @@ def causal_gqa_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, chunk: int
 
 
 def single_query_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, dt=np.float32) -> np.ndarray:
-    """One query row q [Hq, d] over keys k/v [t, Hkv, d] (all visible)."""
+    """One query row q [Hq, d] over keys k/v [t, Hkv, d] (all visible).
+
+    The attention of a decoding row over a cache (Section 3.1: the first generated step)."""
     hq, d = q.shape
     grp = hq // k.shape[1]
     scale = dt(1.0 / np.sqrt(d))
@@ -127,7 +141,8 @@ def single_query_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, dt=np.fl
 
 @dataclass
 class LayerParams:
-    """Base weights of one layer (float arrays holding the bf16 values)."""
+    """Base weights of one layer (float arrays holding the bf16 values): the frozen base model
+    of Section 2.1."""
     W: Dict[str, np.ndarray]             # m -> [out, in]
     bias: Dict[str, np.ndarray]          # q/k/v -> [out] (empty when the model has none)
     ln1: np.ndarray
@@ -138,14 +153,16 @@ class LayerParams:
 class LayerAdapter:
     """LoRA factors of one layer: m -> (A [r, in], B [out, r]); modules absent are unadapted.
 
-    ``scale`` multiplies B A (``lora_scale``)."""
+    The layer's part theta_l of an adapter version (Section 2.1). ``scale`` multiplies B A
+    (``lora_scale``)."""
     AB: Dict[str, Tuple[np.ndarray, np.ndarray]]
     scale: float
 
 
 def lora_scale(alpha: float, rank: int) -> float:
     """alpha / r: the factor of the low-rank update B A in the LoRA parameterisation the paper
-    adopts (Section 1, citing LoRA; the adapter of Section 5.1 is stated by rank and alpha)."""
+    adopts (Section 1, citing LoRA). Section 5.1 gives the adapter's rank but not alpha, which the
+    workload fixes."""
     return float(alpha) / float(rank)
 
 
@@ -169,7 +186,7 @@ def qkv(x: np.ndarray, P: LayerParams, ad: LayerAdapter, dims: Dims, positions: 
 
 def post_attention(x: np.ndarray, o: np.ndarray, P: LayerParams, ad: LayerAdapter, dims: Dims,
                    dt=np.float32) -> np.ndarray:
-    """Output projection + residual, then the SwiGLU MLP + residual."""
+    """Output projection + residual, then the SwiGLU MLP + residual: the rest of F_l in Eq. S1."""
     n = x.shape[0]
     x1 = np.asarray(x, dt) + _proj(o.reshape(n, -1), P, ad, "o", dt)
     xn2 = rmsnorm(x1, P.ln2, dims.rms_eps, dt)
@@ -191,7 +208,8 @@ def decode_row(x_row: np.ndarray, pos: int, k_hist: np.ndarray, v_hist: np.ndarr
     """One row at position ``pos`` attending to cached k/v at positions < pos plus its own fresh k, v.
 
     k_hist/v_hist [pos, Hkv, d] are the cached (historical) post-rotation keys and values of this
-    layer. Returns (h_out [1, hidden], k_row, v_row).
+    layer. Returns (h_out [1, hidden], k_row, v_row). The row of a hybrid execution that reads
+    historical states at this layer (Section 3.1).
     """
     q, k, v = qkv(x_row.reshape(1, -1), P, ad, dims, np.array([pos]), dt)
     kk = np.concatenate([np.asarray(k_hist, dt), k], axis=0)
@@ -201,5 +219,6 @@ def decode_row(x_row: np.ndarray, pos: int, k_hist: np.ndarray, v_hist: np.ndarr
 
 
 def merged_weight(W: np.ndarray, A: np.ndarray, B: np.ndarray, scale: float) -> np.ndarray:
-    """W + scale * B A: the merged form of an adapted projection (used by the pins only)."""
+    """W + scale * B A: the merged form of an adapted projection (used by the pins only); the same
+    projection as ``lora_linear`` (Section 2.1)."""
     return np.asarray(W, np.float64) + scale * (np.asarray(B, np.float64) @ np.asarray(A, np.float64))

@@ -19,17 +19,23 @@ import numpy as np
 
 
 def param_sq(A0, B0, A1, B1) -> float:
+    """||A_1 - A_0||_F^2 + ||B_1 - B_0||_F^2: one module's share of ||theta_t - theta^anchor||_2^2
+    in Eq. 8 (the adapter compared as parameters)."""
     A0, B0, A1, B1 = (np.asarray(t, np.float64) for t in (A0, B0, A1, B1))
     return float(np.sum((A1 - A0) ** 2) + np.sum((B1 - B0) ** 2))
 
 
 def dense_sq(A0, B0, A1, B1) -> float:
+    """||B_1 A_1 - B_0 A_0||_F^2 formed explicitly: the weight-space reading of the Eq. 8
+    displacement (tiny shapes only)."""
     A0, B0, A1, B1 = (np.asarray(t, np.float64) for t in (A0, B0, A1, B1))
     d = B1 @ A1 - B0 @ A0
     return float(np.sum(d * d))
 
 
 def factored_sq(A0, B0, A1, B1) -> float:
+    """The same weight-space displacement as ``dense_sq`` (Eq. 8) through the rank-2r factors and
+    their 2r x 2r Grams."""
     A0, B0, A1, B1 = (np.asarray(t, np.float64) for t in (A0, B0, A1, B1))
     Bt = np.concatenate([B1 - B0, B0], axis=1)     # [out, 2r]
     At = np.concatenate([A1, A1 - A0], axis=0)     # [2r, in]
@@ -39,7 +45,8 @@ def factored_sq(A0, B0, A1, B1) -> float:
 
 
 def drift_table(anchor_layers, cur_layers, modules, dense: bool = False) -> np.ndarray:
-    """[N, 7, 2] table of (weight-space, parameter-space) squared drifts.
+    """[N, 7, 2] table of (weight-space, parameter-space) squared drifts (Eq. 8, per layer against
+    that layer's anchor, Section 4.2).
 
     ``anchor_layers[l]`` / ``cur_layers[l]`` map module -> (A, B). Modules without an adapter
     give zeros.

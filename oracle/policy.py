@@ -35,17 +35,19 @@ def r_kv(module: str, s: int, n_layers: int) -> int:
 
 
 def restart_layer(module: str, s: int, n_layers: int) -> Optional[int]:
-    """r(c): restart at s if any cache layer is affected, else None (nothing to recover)."""
+    """r(c): restart at s if any cache layer is affected, else None (nothing to recover): the
+    executable restart of Section 4.1 / Section 4.2 with the onset of Eq. S4."""
     return s if r_kv(module, s, n_layers) < n_layers else None
 
 
 def candidate_windows(r: int, n_layers: int, hs: Sequence[int] = CANDIDATE_H) -> List[int]:
-    """H_i: the distinct executable window lengths tried during calibration, ascending."""
+    """H_i: the distinct executable window lengths tried during calibration, ascending (the
+    candidate set of the offline calibration, Section 4.1)."""
     return sorted({min(h, n_layers - r) for h in hs} | {n_layers - r})
 
 
 def first_safe(cands: Sequence[int], safe: Callable[[int], bool]) -> Optional[int]:
-    """h*_i = min{h in H_i : S_i(h) = 1} (first hit, no monotonicity assumed)."""
+    """h*_i = min{h in H_i : S_i(h) = 1} (first hit, no monotonicity assumed; Section 4.1)."""
     for h in sorted(cands):
         if safe(h):
             return h

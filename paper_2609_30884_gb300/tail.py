@@ -1,4 +1,4 @@
-"""Offline tail-influence sweep on the device kernels (Section 3.2, Eq. 3-5).
+"""Offline tail-influence sweep on the device kernels (Sections 3.1-3.2, Eq. 2-5).
 
 For a stale cache and the current adapter, z^(b) are the first-step next-token logits when the
 cache is refreshed below layer b and historical from layer b on: the last prefix row restarts from
@@ -7,12 +7,12 @@ pages (b = 0 restarts from the embedding; z^(N) = z* is the fresh model). The sw
 hybrid rows as empty-window ``crf_recompute_window`` calls, then one ``crf_kl`` call over all of
 them with the fresh row as reference, and derives on the host:
 
-* v_l = z^(l) - z^(l+1) and the tail influence T_b = sum_{l >= b} ||v_l||_2 (Eq. 3),
+* v_l = z^(l) - z^(l+1) and the tail influence T_b = sum_{l >= b} ||v_l||_2 (Eq. 2),
 * the KL certificate KL(p* || p^(b)) <= T_b^2 / 4 (Eq. 4),
 * the top-1 certificate T_b < gamma*/2 => argmax z^(b) = argmax z* (Eq. 5), gamma* the fresh
   margin between the two largest logits,
 * the first boundary at or after the restart whose KL meets a tolerance (the recomputation
-  horizon of Eq. 2 counted from the restart).
+  horizon of Eq. 3 counted from the restart).
 """
 from __future__ import annotations
 

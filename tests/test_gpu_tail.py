@@ -1,4 +1,4 @@
-"""Offline tail-influence sweep on the device against the oracle (Section 3.2, Eq. 3-5).
+"""Offline tail-influence sweep on the device against the oracle (Sections 3.1-3.2, Eq. 2-5).
 
 A stale cache built under adapter version 0 and the current adapter version 3 (tiny decoder, every
 layer adapted): the device's N + 1 hybrid first-step distributions z^(b), their KL to the fresh

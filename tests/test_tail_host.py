@@ -1,5 +1,5 @@
 """Host side of the tail-influence sweep (paper_2609_30884_gb300.tail.certificates) against the
-oracle's restatement of Eq. 3-5, on synthetic hybrid logits (CPU)."""
+oracle's restatement of Eq. 2-5, on synthetic hybrid logits (CPU)."""
 import numpy as np
 
 from oracle import fidelity as Fi
