@@ -1,5 +1,6 @@
 // Causal grouped-query prefill attention over the paged KV cache on mma.sync
-// (the alternative to the tcgen05 kernel, selected with CRF_ATTENTION=mma).
+// (the alternative to the tcgen05 kernel, selected with CRF_ATTENTION=mma): the
+// self-attention of a recomputed layer (Section 4.2, Eq. 1, Eq. S3).
 //
 // Prefill: softmax(q k^T / sqrt(d) + causal mask) v over the whole prefix, per
 // query head; query head h reads kv head h / (Hq / Hkv). q arrives already

@@ -1,5 +1,7 @@
 // Causal grouped-query prefill attention on tcgen05, reading K/V from the
-// paged cache of the layer being recomputed.
+// paged cache of the layer being recomputed: the self-attention of every layer
+// that bounded recovery re-executes over the complete prefix (Section 4.2),
+// whose K/V are the cache entries of Eq. 1 (projections of Eq. S3).
 //
 // softmax(q k^T / sqrt(d) + causal mask) v over the whole prefix for every
 // query head; query head h reads kv head h / (Hq / Hkv). One CTA takes two

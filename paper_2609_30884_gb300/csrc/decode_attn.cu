@@ -1,5 +1,7 @@
 // Decode attention of single rows over the paged cache (the first-step rows carried
-// through layers e..N-1): for each decode row at position pos and query head h,
+// through layers e..N-1: the hybrid execution of Section 3.1 that reads historical states
+// from the window end on, and the generated tokens of Section S2.1): for each decode row at
+// position pos and query head h,
 //   o = softmax(q k^T / sqrt(d)) v over the cached keys 0..pos-1 of that layer plus the
 //   row's own fresh (k, v) at position pos.
 // The work is memory-bound (K and V of every cached position are read once): the positions

@@ -1,5 +1,6 @@
 // Multi-row GEMV on the tensor cores: y[r, j] = sum_i W[j, i] x[r, i] (+ bias, LoRA up, residual)
-// for up to 8 fp32 rows x (the first-step rows of a window and the rows of a generation step).
+// for up to 8 fp32 rows x (the first-step rows of a window and the rows of a generation step): the
+// adapted projections of Eq. S3 for single rows (Section 3.1 hybrid rows, Section S2.1 decoding).
 //
 // mma.sync m16n8k16 with W as the A operand (16 output rows per warp) and the rows as the B
 // operand (n = 8 row slots; slots past the row count are zero). x enters as a bf16 pair

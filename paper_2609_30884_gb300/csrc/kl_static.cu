@@ -1,5 +1,6 @@
-// crf_kl_logits_noalloc: the first-step KL from logits with its scratch in a
-// fixed device array instead of a caller-provided workspace.
+// crf_kl_logits_noalloc: the first-step KL from logits (forward KL, fresh
+// model as reference, Section S2.1) with its scratch in a fixed device array
+// instead of a caller-provided workspace.
 //
 // Some callers cannot allocate device memory at the point where they need the
 // fidelity number: a serving loop that runs under a fixed device-memory budget
