@@ -75,3 +75,26 @@ def test_shard_requests_partitions_and_balances():
         tot = [sum(loads[i] for i in p) for p in parts]
         assert max(tot) - min(tot) <= max(loads)        # greedy LPT balance bound
     assert bench.shard_requests([7], 3) == [[0], [0], [0]]   # one prefix: replicas
+
+
+def test_reference_arm_line_has_the_contract_keys(capsys, monkeypatch):
+    """The reference arm (the oracle on the host cores) prints one JSON line with the metric,
+    its own cpu_baseline and an e2e object that copies nothing between host and device."""
+    import json
+    monkeypatch.delenv("RANK", raising=False)
+    args = type("A", (), {"workload": "tiny", "ref_rows": 16, "steps": 1, "warmup": 0, "gpus": 1,
+                          "lora_rank": 0, "lora_modules": ""})()
+    assert bench.run_reference(args) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    for key in ("impl", "metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config",
+                "cpu_baseline", "e2e"):
+        assert key in line, key
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC and line["unit"] == bench.UNIT
+    assert line["higher_is_better"] is True and line["value"] > 0
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["cores"] >= 1 and cb["sample"]
+    e2e = line["e2e"]
+    assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
+    assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
+    assert "tiny" in line["config"]["workload"] and "tiny" in line["data"]
