@@ -98,3 +98,18 @@ def test_reference_arm_line_has_the_contract_keys(capsys, monkeypatch):
     assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
     assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
     assert "tiny" in line["config"]["workload"] and "tiny" in line["data"]
+
+
+def test_clock_summary_reports_median_and_active_reasons():
+    rows = ["0, 1950, 2070, 900.1, 0x4, Not Active, Not Active, Not Active, Active\n",
+            "0, 1980, 2070, 1200.5, 0x0, Not Active, Not Active, Not Active, Not Active\n",
+            "0, 1400, 2070, 1390.0, 0x4, Not Active, Not Active, Not Active, Active\n",
+            "garbage line\n"]
+    s = bench.ClockSampler.summarise(rows)
+    assert s["sm_mhz"] == 1950.0 and s["sm_max_mhz"] == 2070.0 and s["samples"] == 3
+    assert s["reasons"] == ["sw_power_cap"]
+    hot = bench.ClockSampler.summarise(["0, 1500, 2070, 1000, 0x40, Not Active, Active, Not Active, Not Active\n"])
+    assert hot["reasons"] == ["hw_thermal_slowdown"]
+    assert bench.ClockSampler.summarise([])["reasons"] == ["no samples"]
+    na = bench.ClockSampler.summarise(["0, [N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A]\n"])
+    assert na["sm_mhz"] is None and na["sm_max_mhz"] is None
