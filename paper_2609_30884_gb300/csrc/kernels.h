@@ -262,13 +262,10 @@ cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, v
 cudaError_t launch_wait_selftest(int* status, cudaStream_t stream);
 cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
                                cudaStream_t stream);
-cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream);
 cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
                                     cudaStream_t stream);
 cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream);
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStream_t stream);
-cudaError_t launch_gather_rows_f32(const __nv_bfloat16* src, const int64_t* row_index, float* dst,
-                                   int rows, int hidden, cudaStream_t stream);
 
 // LM head + KL: logits [2*rows, V] (ref rows first) from final-normed hidden rows.
 cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,

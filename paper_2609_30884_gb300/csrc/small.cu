@@ -304,15 +304,6 @@ __global__ void lora_bext_kernel(const BextDesc d, int rank) {
   *reinterpret_cast<uint4*>(d.out[m] + (size_t)r * kBxCols + c0) = make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-// gu [rows, 2, ffn] (gate then up) -> m [rows, ffn]
-__global__ void swiglu_f32_kernel(const float* gu, float* m, int rows, int ffn) {
-  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= rows * ffn) return;
-  const int r = idx / ffn, j = idx % ffn;
-  const float g = gu[(size_t)r * 2 * ffn + j], u = gu[(size_t)r * 2 * ffn + ffn + j];
-  m[idx] = g / (1.f + __expf(-g)) * u;
-}
-
 // m[i] = silu(g[i]) * u[i] over n elements (gate and up in separate buffers)
 __global__ void swiglu_split_f32_kernel(const float* g, const float* u, float* m, int n) {
   griddep_begin();  // gate and up come from the GEMV before
@@ -327,13 +318,6 @@ __global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int n) {
 __global__ void bf16_to_f32_kernel(const __nv_bfloat16* x, float* y, int n) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) y[i] = __bfloat162float(x[i]);
-}
-__global__ void gather_rows_f32_kernel(const __nv_bfloat16* src, const int64_t* row_index, float* dst,
-                                       int rows, int hidden) {
-  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= rows * hidden) return;
-  const int r = idx / hidden, c = idx % hidden;
-  dst[idx] = __bfloat162float(src[row_index[r] * hidden + c]);
 }
 
 // ------------------------------------------------------------------ KL
@@ -869,13 +853,6 @@ cudaError_t launch_lora_bext(const BextDesc& d, int rank, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_swiglu_f32(const float* gu, float* m, int rows, int ffn, cudaStream_t stream) {
-  const int n = rows * ffn;
-  if (n == 0) return cudaSuccess;
-  swiglu_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(gu, m, rows, ffn);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
                                     cudaStream_t stream) {
   if (n == 0) return cudaSuccess;
@@ -890,13 +867,6 @@ cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStre
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStream_t stream) {
   if (n == 0) return cudaSuccess;
   bf16_to_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, y, n);
-  return cudaGetLastError();
-}
-cudaError_t launch_gather_rows_f32(const __nv_bfloat16* src, const int64_t* row_index, float* dst,
-                                   int rows, int hidden, cudaStream_t stream) {
-  const int n = rows * hidden;
-  if (n == 0) return cudaSuccess;
-  gather_rows_f32_kernel<<<cdiv(n, 256), 256, 0, stream>>>(src, row_index, dst, rows, hidden);
   return cudaGetLastError();
 }
 
