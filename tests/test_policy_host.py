@@ -110,3 +110,26 @@ def test_trajectory_anchors_match_oracle():
         anchors = OP.update_anchors(anchors, w, t)
         assert pol.anchors == anchors
         assert pol.fraction(w) == OP.recompute_fraction(w, N)
+
+
+def test_layer_and_state_displacement_readings_of_eq8():
+    """The two readings of d_l (Eq. 8) from a [N][7][2] drift table: per layer, the root of the
+    layer's summed weight-space (or parameter-space) squares; over the whole adapter, the root of
+    every parameter-space square."""
+    import synth
+    from oracle import build as obuild, drift as odrift
+    HP = PP
+    cfg, lc = synth.TINY, synth.LORA_TINY
+    a0 = [obuild.layer_adapter(cfg, lc, 0, l).AB for l in range(cfg.n_layers)]
+    a2 = [obuild.layer_adapter(cfg, lc, 2, l).AB for l in range(cfg.n_layers)]
+    table = odrift.drift_table(a0, a2, synth.MODULES)
+    d_w = HP.layer_displacement(table)
+    d_p = HP.layer_displacement(table, weight_space=False)
+    for l in range(cfg.n_layers):
+        want_w = math.sqrt(sum(odrift.dense_sq(*a0[l][m], *a2[l][m]) for m in lc.modules))
+        want_p = math.sqrt(sum(odrift.param_sq(*a0[l][m], *a2[l][m]) for m in lc.modules))
+        assert d_w[l] == pytest.approx(want_w, rel=1e-10)
+        assert d_p[l] == pytest.approx(want_p, rel=1e-12)
+    assert HP.state_displacement(table) == pytest.approx(math.sqrt(sum(x * x for x in d_p)), rel=1e-12)
+    # identical versions: zero displacement everywhere
+    assert HP.layer_displacement(odrift.drift_table(a2, a2, synth.MODULES)) == [0.0] * cfg.n_layers
