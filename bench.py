@@ -191,7 +191,7 @@ def build_state(wl, device, ctx, rank=0, world=1):
     import torch
     import synth
     import paper_2609_30884_gb300 as crf
-    from harness import DeviceAdapter, DeviceModel, make_pool, split_page_tables
+    from tests.harness import DeviceAdapter, DeviceModel, make_pool, split_page_tables
 
     cfg, lc = wl.model, wl.lora
     N = cfg.n_layers
@@ -392,7 +392,7 @@ def run_window_only(args):
     import torch
     import synth
     import paper_2609_30884_gb300 as crf
-    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed
+    from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed
 
     wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
@@ -445,7 +445,7 @@ def run_decode_only(args):
     import torch
     import synth
     import paper_2609_30884_gb300 as crf
-    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+    from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 
     wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
@@ -483,8 +483,8 @@ def run_trajectory_case(args):
     """The recovery policy over a synthetic 32-version adapter trajectory (RQ4-style)."""
     import torch
     import paper_2609_30884_gb300 as crf
-    import trajectory
-    from harness import DeviceModel
+    from paper_2609_30884_gb300 import trajectory
+    from tests.harness import DeviceModel, Versions, pages_needed, split_page_tables
 
     wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
@@ -492,9 +492,13 @@ def run_trajectory_case(args):
     ctx = crf.Context(0)
     dm = DeviceModel(cfg, "cuda:0")
     layer = args.update_layer if args.update_layer >= 0 else cfg.n_layers // 2
+    pt = split_page_tables([n], pages_needed(n), seed=1, device="cuda:0")[0]
     t0 = time.time()
-    res = trajectory.run(ctx, dm, cfg, lc, n, versions=args.versions, calib_versions=args.calib_versions,
-                         layer=layer, module=args.update_module, std=args.update_std, base_version=0)
+    res = trajectory.run(ctx, dm.crf, synth_tokens(cfg, n), pt,
+                         lambda seed: Versions(cfg, lc, layer, args.update_module, args.update_std, seed,
+                                               "cuda:0", 0),
+                         versions=args.versions, calib_versions=args.calib_versions, layer=layer,
+                         module=args.update_module)
     line = {"case": "trajectory", "workload": f"{args.workload}: {wl.name}", "tokens": n,
             "versions": args.versions,
             "update": {"layer": layer, "module": args.update_module, "std_per_entry": args.update_std,
@@ -516,8 +520,7 @@ def run_tail_case(args):
     import numpy as np
     import paper_2609_30884_gb300 as crf
     from paper_2609_30884_gb300 import tail
-    import trajectory
-    from harness import DeviceModel, make_pool, pages_needed, split_page_tables
+    from tests.harness import DeviceModel, Versions, make_pool, pages_needed, split_page_tables
 
     wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
@@ -526,7 +529,7 @@ def run_tail_case(args):
     layer = args.update_layer if args.update_layer >= 0 else N // 2
     ctx = crf.Context(0)
     dm = DeviceModel(cfg, "cuda:0")
-    vers = trajectory.Versions(cfg, lc, layer, args.update_module, args.update_std, 202, "cuda:0", 0)
+    vers = Versions(cfg, lc, layer, args.update_module, args.update_std, 202, "cuda:0", 0)
     old, cur = vers.adapter(0), vers.adapter(args.versions)
     P = pages_needed(n)
     pt = split_page_tables([n], P, seed=1, device="cuda:0")[0]
@@ -567,7 +570,7 @@ def run_decode_case(args):
     import torch
     import paper_2609_30884_gb300 as crf
     import synth
-    from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+    from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 
     wl = workload_of(args)
     cfg, lc = wl.model, wl.lora
@@ -626,7 +629,7 @@ def run_drift_case(args):
     the small profiling case of the drift kernels (adapters only on the device)."""
     import torch
     import paper_2609_30884_gb300 as crf
-    from harness import DeviceAdapter, DeviceModel
+    from tests.harness import DeviceAdapter, DeviceModel
 
     wl = workload_of(args)
     cfg, lc = wl.model, wl.lora

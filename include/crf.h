@@ -255,16 +255,18 @@ CRF_API crf_status crf_kl(crf_ctx* ctx, const crf_model* model, const void* ref,
  * interface for callers that cannot allocate device memory when they need the
  * number, such as a serving loop under a fixed device-memory budget or a C
  * host without its own device allocator).
- * Same result as crf_kl with model == NULL, but its scratch is a fixed device
- * array inside the library (160 KiB, held by every GPU that loads it until
- * the process exits) instead of a caller workspace, so the call allocates
- * nothing. z_ref, z_cur: device fp32 [n_rows, vocab]; out_kl: device fp32
- * [n_rows]. n_rows must be 1..32 (CRF_EUNSUPPORTED beyond). `device` is made
- * current for the call and restored after. The first call on a device looks
- * up the array's device address once; make that first call before any stream
- * capture. All calls share the one array: calls whose kernels overlap on the
- * GPU (different streams, or different host threads) race and must be
- * serialised by the caller. */
+ * Same arithmetic as crf_kl with model == NULL (the same vocabulary splits,
+ * reduced in the same order), but its scratch is a fixed device array inside
+ * the library (160 KiB, held by every GPU that loads it until the process
+ * exits) instead of a caller workspace, so the call allocates nothing.
+ * z_ref, z_cur: device fp32 [n_rows, vocab]; out_kl: device fp32 [n_rows].
+ * n_rows must be 1..32 (CRF_EUNSUPPORTED beyond). `device` is made current for
+ * the call and restored after. The first call on a device (and the first after
+ * that device's context is recreated, e.g. after cudaDeviceReset) looks up the
+ * array's device address; make that first call before any stream capture.
+ * All calls share the one array: calls whose kernels overlap on the GPU
+ * (different streams, or different host threads) race and must be serialised
+ * by the caller. */
 CRF_API crf_status crf_kl_logits_noalloc(int device, const float* z_ref, const float* z_cur,
                                          int n_rows, int vocab, float* out_kl, void* stream);
 

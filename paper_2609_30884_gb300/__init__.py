@@ -257,8 +257,21 @@ def kl_logits_noalloc(device: int, z_ref: torch.Tensor, z_cur: torch.Tensor, out
     """crf_kl_logits_noalloc: KL(softmax(z_ref) || softmax(z_cur)) per row with no workspace.
 
     For callers that cannot allocate device memory at call time; the library's fixed device
-    scratch serves every call, so calls must not overlap on the GPU.
+    scratch serves every call, so calls must not overlap on the GPU. The tensors are checked
+    here (fp32, contiguous, same shape, on ``device``, out_kl long enough) because the library
+    receives only their addresses.
     """
+    if z_ref.dim() != 2 or tuple(z_cur.shape) != tuple(z_ref.shape):
+        raise ValueError("z_ref and z_cur must be 2-D [n_rows, vocab] of the same shape")
+    for name, t in (("z_ref", z_ref), ("z_cur", z_cur), ("out_kl", out_kl)):
+        if t.dtype != torch.float32 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous float32 tensor")
+        if t.device.type != "cuda" or t.device.index != device:
+            raise ValueError(f"{name} must be on cuda:{device}")
+    if out_kl.numel() < z_ref.shape[0]:
+        raise ValueError("out_kl holds fewer entries than z_ref has rows")
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
     lib = abi.load()
     abi.check(lib.crf_kl_logits_noalloc(device, z_ref.data_ptr(), z_cur.data_ptr(),
                                         int(z_ref.shape[0]), int(z_ref.shape[1]),

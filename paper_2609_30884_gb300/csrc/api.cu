@@ -29,8 +29,6 @@ struct crf_ctx {
   int device;
   int num_sms;
   int* status_dev;
-  // CRF_ATTENTION=mma selects the mma.sync prefill attention instead of tcgen05
-  bool attn_mma_sync = false;
   // per-launch timing (crf_profile_enable)
   bool prof_on = false;
   std::vector<cudaEvent_t> ev;
@@ -400,10 +398,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     a.req = rt;
     a.status = c.ctx->status_dev;
     ProfScope ps(c.ctx, kPAttn, c.st);
-    if (c.ctx->attn_mma_sync)
-      CRF_CUDA(launch_attention(a, c.ctx->num_sms, c.st));
-    else
-      CRF_CUDA(launch_attention_tc(a, c.pool->num_pages, M, c.st));
+    CRF_CUDA(launch_attention_tc(a, c.pool->num_pages, M, c.st));
   }
 
   // 5-6. output projection + residual: X1 = X_in + O W_o^T (+ LoRA)
@@ -818,8 +813,6 @@ crf_status crf_create(crf_ctx** out, int device) {
   crf_ctx* c = new crf_ctx;
   c->device = device;
   c->num_sms = prop.multiProcessorCount;
-  const char* attn = std::getenv("CRF_ATTENTION");
-  c->attn_mma_sync = attn && std::strcmp(attn, "mma") == 0;
   c->status_dev = nullptr;
   cudaError_t e = cudaMalloc(&c->status_dev, sizeof(int));
   if (e == cudaSuccess) e = cudaMemset(c->status_dev, 0, sizeof(int));
@@ -1044,14 +1037,6 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
   return CRF_OK;
 }
 
-// ---------------------------------------------------------------- drift
-// Blocks per Gram side: enough that the longest side (the ffn or the hidden rows) is cut into
-// pieces of <= 768 rows, so no block runs far longer than the rest.
-static int drift_blocks_per_side(const crf_model_dims& d) {
-  const int longest = std::max(std::max(d.hidden, d.ffn), d.n_q_heads * d.head_dim);
-  return std::max(1, std::min(32, (longest + 767) / 768));
-}
-
 crf_status crf_decode_workspace_size(crf_ctx* ctx, const crf_model* model, const crf_lora_dims* lora,
                                      const crf_decode_row* rows, int n_rows, size_t* bytes) {
   if (!ctx || !model || !lora || !rows || !bytes) return fail(CRF_EINVAL, "null argument");
@@ -1148,12 +1133,10 @@ crf_status crf_drift_workspace_size(crf_ctx* ctx, const crf_model_dims* dims,
   if (!ctx || !dims || !lora || !bytes) return fail(CRF_EINVAL, "null argument");
   crf_status s = check_lora(*lora);
   if (s != CRF_OK) return s;
+  if (dims->n_layers < 1) return fail(CRF_EINVAL, "n_layers must be positive");
   int nm = 0;
   for (int m = 0; m < 7; ++m) nm += (lora->module_mask >> m) & 1;
-  const int items = dims->n_layers * nm;
-  const int bps = drift_blocks_per_side(*dims);
-  const size_t r2 = 2 * lora->rank;
-  *bytes = align256(static_cast<size_t>(items) * 2 * bps * r2 * r2 * sizeof(float));
+  *bytes = align256(drift_workspace_bytes(ctx->num_sms, lora->rank, dims->n_layers * nm));
   return CRF_OK;
 }
 
@@ -1166,6 +1149,8 @@ crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter
   if (s != CRF_OK) return s;
   if (!cur->A || !cur->B) return fail(CRF_EINVAL, "adapter tables missing");
   const Dims D = dims_of(*dims);
+  if (D.h % 8 || D.f % 8 || D.qd % 8 || D.kvd % 8)
+    return fail(CRF_EUNSUPPORTED, "drift needs every projection's input width to be a multiple of 8");
   std::vector<DriftItem> items;
   for (int l = 0; l < D.N; ++l) {
     const crf_adapter* an = anchors[l];
@@ -1181,6 +1166,8 @@ crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter
       it.B1 = static_cast<const __nv_bfloat16*>(cur->B[l * 7 + m]);
       if (!it.A0 || !it.B0 || !it.A1 || !it.B1)
         return fail(CRF_EINVAL, "layer %d module %d factor is null", l, m);
+      if (!aligned16(it.A0) || !aligned16(it.B0) || !aligned16(it.A1) || !aligned16(it.B1))
+        return fail(CRF_EINVAL, "layer %d module %d factor misaligned (16 bytes)", l, m);
       module_shape(D, m, it.out_dim, it.in_dim);
       it.out_index = l * 7 + m;
       items.push_back(it);
@@ -1189,22 +1176,21 @@ crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter
   size_t need = 0;
   s = crf_drift_workspace_size(ctx, dims, &cur->dims, &need);
   if (s != CRF_OK) return s;
-  if (!workspace || ws_bytes < need) return fail(CRF_ENOMEM, "drift workspace %zu < %zu", ws_bytes, need);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255) || ws_bytes < need)
+    return fail(CRF_ENOMEM, "drift workspace null, misaligned or %zu < %zu bytes", ws_bytes, need);
   CRF_CUDA(cudaSetDevice(ctx->device));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   CRF_CUDA(cudaMemsetAsync(out_sq, 0, static_cast<size_t>(D.N) * 7 * 2 * sizeof(float), st));
   if (items.empty()) return CRF_OK;
-  const int bps = drift_blocks_per_side(*dims);
-  ProfScope ps(ctx, kPDrift, st, 2 * ((static_cast<int>(items.size()) + 223) / 224));
+  ProfScope ps(ctx, kPDrift, st, drift_launches(static_cast<int>(items.size())));
   CRF_CUDA(launch_drift(items.data(), static_cast<int>(items.size()), cur->dims.rank,
-                        static_cast<float*>(workspace), bps, out_sq, st));
+                        static_cast<float*>(workspace), ctx->num_sms, out_sq, st));
   return CRF_OK;
 }
 
 // ---------------------------------------------------------------- KL
 static int kl_splits(const crf_ctx* ctx, int n_rows, int vocab) {
-  const int want = (2 * ctx->num_sms + n_rows - 1) / std::max(1, n_rows);
-  return std::max(1, std::min(want, (vocab + 1023) / 1024));
+  return kl_split_count(ctx->num_sms, n_rows, vocab);
 }
 
 crf_status crf_kl_workspace_size(crf_ctx* ctx, int n_rows, int vocab, int hidden, size_t* bytes) {

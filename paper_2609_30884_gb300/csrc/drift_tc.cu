@@ -1,0 +1,416 @@
+// Adapter drift (Eq. 8) on the tensor cores.
+//
+// Per (layer, module) item, the weight-space change of the unscaled LoRA update factors as
+//   B1 A1 - B0 A0 = [B1 - B0 | B0] [A1 ; A1 - A0],
+// so ||B1 A1 - B0 A0||_F^2 = tr(GB GA) with the 2r x 2r Grams GB = Bt^T Bt over the output rows
+// and GA = At At^T over the input columns; every Gram entry already scales with the change, so
+// nothing cancels. The parameter-space change ||A1 - A0||^2 + ||B1 - B0||^2 is the trace of the
+// two difference blocks.
+//
+// Both Grams are contractions over a long dimension (the output rows of B, the input columns of
+// A: 512..18944 at the Qwen2.5 shapes) and run here as bf16 mma.sync products with fp32
+// accumulation. The difference of two bf16 factors is exact in fp32 but not in bf16, so each
+// difference enters as a bf16 pair hi + lo (hi = bf16(d), lo = bf16(d - hi)); every product of
+// two bf16 values is exact in fp32, so the Grams carry the fp32-accumulated value of the exact
+// differences. Per long-dimension row the feature vector is [hi(d) | lo(d) | base] with
+// d = B1 - B0, base = B0 for the B side and d = A1 - A0, base = A1 for the A side, padded to
+// RP = max(r, 8) features per part (zeros), and the kernel accumulates the block-upper triangle
+// of its Gram (16 x 16 blocks).
+//
+// Work split: the long dimension of every (item, side) segment is cut into 128-row steps; the
+// steps of all segments are laid end to end and a persistent grid of G CTAs takes equal
+// consecutive ranges of them (stream-K). A CTA stages each step's rows of both versions with
+// cp.async (three stages in flight, no registers held), builds the hi/lo/base fragments in
+// registers from ldmatrix loads (transposed for the B side, whose rows are [r] wide), and its 8
+// warps each accumulate one 16-row slice. When its range leaves a segment (or ends) the CTA sums
+// its warps in a fixed order and writes one partial Gram to slot (b + seg), unique because a
+// CTA's segments follow the previous CTA's. The final kernel sums each segment's slots in CTA
+// order and forms tr(GB GA) and the parameter distance in fp64. The result does not depend on
+// timing: same inputs, same bits.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace crf {
+
+namespace {
+
+constexpr int kDtThreads = 256;
+constexpr int kDtRows = 128;   // long-dimension rows per step: 8 warps x 16
+constexpr int kDtStages = 3;
+constexpr int kDtCtasPerSm = 3;
+constexpr int kDtMaxItems = 224;
+constexpr int kDtMaxSegs = 2 * kDtMaxItems;
+constexpr int kDtAStride = kDtRows * 2 + 16;  // bytes per A row in a stage (+16: no bank conflicts)
+
+struct DriftTcArgs {
+  DriftItem items[kDtMaxItems];
+  int seg_step0[kDtMaxSegs + 1];  // first step of segment s = 2 * item + side; [n_segs] = total
+  int n_items, n_segs, total_steps, grid, rank;
+};
+
+template <int RP>
+struct DtShape {
+  static constexpr int kBStride = RP == 16 ? 48 : 16;          // bytes per B row in a stage
+  static constexpr int kBVersion = kDtRows * kBStride;          // one version of the B side
+  static constexpr int kAVersion = RP * kDtAStride;             // one version of the A side
+  static constexpr int kStage = 2 * (kBVersion > kAVersion ? kBVersion : kAVersion);
+  static constexpr int kBlocks = RP == 16 ? 3 : 2;              // 16-feature blocks of [hi|lo|base]
+  static constexpr int kPairs = kBlocks * (kBlocks + 1) / 2;    // block-upper triangle
+  static constexpr int kSlotFloats = kPairs * 256;
+};
+
+__device__ __forceinline__ void cp_async(uint32_t dst, const void* src, int bytes, bool valid) {
+  // bytes is 8 or 16; an invalid source copies nothing and fills the destination with zeros
+  if (bytes == 16)
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
+                 : "memory");
+  else
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(valid ? 8 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
+}
+
+// (hi, lo) of the exact fp32 differences of two bf16 pairs, and the pairs themselves
+__device__ __forceinline__ void split_diff(uint32_t a, uint32_t b, uint32_t& hi, uint32_t& lo) {
+  const float d0 = bf16_lo(a) - bf16_lo(b), d1 = bf16_hi(a) - bf16_hi(b);
+  hi = pack_bf16(d0, d1);
+  lo = pack_bf16(d0 - bf16_lo(hi), d1 - bf16_hi(hi));
+}
+
+// Step x of the grid-wide sequence: its segment, side and first long-dimension row.
+struct StepRef {
+  const DriftItem* it;
+  int side, row0, len;
+};
+
+__device__ __forceinline__ int seg_of(const DriftTcArgs& a, int x, int seg) {
+  while (seg + 1 < a.n_segs && x >= a.seg_step0[seg + 1]) ++seg;
+  return seg;
+}
+
+__device__ __forceinline__ StepRef step_ref(const DriftTcArgs& a, int x, int seg) {
+  StepRef s;
+  s.it = &a.items[seg >> 1];
+  s.side = seg & 1;
+  s.row0 = (x - a.seg_step0[seg]) * kDtRows;
+  s.len = s.side == 0 ? s.it->out_dim : s.it->in_dim;
+  return s;
+}
+
+// Issue the copies of one step into a stage: version 1 (current) then version 0 (anchor).
+template <int RP>
+__device__ __forceinline__ void load_step(const StepRef& s, int rank, uint32_t stage) {
+  using S = DtShape<RP>;
+  const int tid = threadIdx.x;
+  if (s.side == 0) {
+    // B [out, r]: row o holds r contiguous bf16; chunks of 16 bytes (8 bytes when r = 4)
+    const int cbytes = rank >= 8 ? 16 : 8;
+    const int cpr = rank * 2 / cbytes;  // chunks per row
+    const int total = 2 * kDtRows * cpr;
+    for (int i = tid; i < total; i += kDtThreads) {
+      const int v = i / (kDtRows * cpr), rem = i - v * kDtRows * cpr;
+      const int row = rem / cpr, ch = rem - row * cpr;
+      const int o = s.row0 + row;
+      const bool ok = o < s.len;
+      const __nv_bfloat16* base = v == 0 ? s.it->B1 : s.it->B0;
+      const __nv_bfloat16* src = base + (ok ? static_cast<size_t>(o) * rank + ch * (cbytes / 2) : 0);
+      cp_async(stage + v * S::kBVersion + row * S::kBStride + ch * 16, src, cbytes, ok);
+    }
+  } else {
+    // A [r, in]: rows k < r, 128 columns from row0 in 16-byte chunks (in % 8 == 0)
+    const int total = 2 * rank * (kDtRows / 8);
+    for (int i = tid; i < total; i += kDtThreads) {
+      const int v = i / (rank * (kDtRows / 8)), rem = i - v * rank * (kDtRows / 8);
+      const int k = rem / (kDtRows / 8), ch = rem - k * (kDtRows / 8);
+      const int c = s.row0 + ch * 8;
+      const bool ok = c < s.len;
+      const __nv_bfloat16* base = v == 0 ? s.it->A1 : s.it->A0;
+      const __nv_bfloat16* src = base + (ok ? static_cast<size_t>(k) * s.len + c : 0);
+      cp_async(stage + v * S::kAVersion + k * kDtAStride + ch * 16, src, 16, ok);
+    }
+  }
+}
+
+// This warp's 16-row slice of a staged step into its Gram accumulators.
+template <int RP>
+__device__ __forceinline__ void mma_step(int side, uint32_t stage, float (&acc)[DtShape<RP>::kPairs][2][4]) {
+  using S = DtShape<RP>;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m = lane >> 3, i = lane & 7;
+  uint32_t f1[4], f0[4];  // fragments of version 1 and version 0: {m0, m1, m2, m3} (RP = 8: m0, m2)
+  if (side == 0) {
+    // X[o][f] rows: matrix m covers rows k0 + (m >> 1) * 8 .. and features (m & 1) * 8 ..
+    if constexpr (RP == 16) {
+      const uint32_t off = (warp * 16 + (m >> 1) * 8 + i) * S::kBStride + (m & 1) * 16;
+      ldsm_x4_t(stage + off, f1[0], f1[1], f1[2], f1[3]);
+      ldsm_x4_t(stage + S::kBVersion + off, f0[0], f0[1], f0[2], f0[3]);
+    } else {
+      const uint32_t off = (warp * 16 + (m & 1) * 8 + i) * S::kBStride;
+      ldsm_x2_t(stage + off, f1[0], f1[2]);
+      ldsm_x2_t(stage + S::kBVersion + off, f0[0], f0[2]);
+    }
+  } else {
+    // Xt[f][c] rows: matrix m covers features (m & 1) * 8 .. and columns k0 + (m >> 1) * 8 ..
+    if constexpr (RP == 16) {
+      const uint32_t off = ((m & 1) * 8 + i) * kDtAStride + (warp * 16 + (m >> 1) * 8) * 2;
+      ldsm_x4(stage + off, f1[0], f1[1], f1[2], f1[3]);
+      ldsm_x4(stage + S::kAVersion + off, f0[0], f0[1], f0[2], f0[3]);
+    } else {
+      const uint32_t off = i * kDtAStride + (warp * 16 + (m & 1) * 8) * 2;
+      ldsm_x2(stage + off, f1[0], f1[2]);
+      ldsm_x2(stage + S::kAVersion + off, f0[0], f0[2]);
+    }
+  }
+  // base: B0 on the B side, A1 on the A side
+  uint32_t blk[S::kBlocks][4];
+  if constexpr (RP == 16) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      split_diff(f1[r], f0[r], blk[0][r], blk[1][r]);
+      blk[2][r] = side == 0 ? f0[r] : f1[r];
+    }
+  } else {
+    // block 0 = [hi (8 features) | lo (8)], block 1 = [base (8) | zeros]
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int r = 2 * h;
+      split_diff(f1[r], f0[r], blk[0][r], blk[0][r + 1]);
+      blk[1][r] = side == 0 ? f0[r] : f1[r];
+      blk[1][r + 1] = 0u;
+    }
+  }
+  int p = 0;
+#pragma unroll
+  for (int I = 0; I < S::kBlocks; ++I)
+#pragma unroll
+    for (int J = I; J < S::kBlocks; ++J, ++p) {
+      mma16816(acc[p][0], blk[I], blk[J][0], blk[J][2]);
+      mma16816(acc[p][1], blk[I], blk[J][1], blk[J][3]);
+    }
+}
+
+template <int RP>
+__global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
+    drift_tc_kernel(const __grid_constant__ DriftTcArgs a, float* __restrict__ slots) {
+  using S = DtShape<RP>;
+  extern __shared__ __align__(128) uint8_t dt_smem[];
+  float* red = reinterpret_cast<float*>(dt_smem + kDtStages * S::kStage);  // [32][kPairs * 8]
+  const uint32_t stage0 = smem_u32(dt_smem);
+  const int b = blockIdx.x;
+  const int x0 = static_cast<int>((static_cast<long long>(b) * a.total_steps) / a.grid);
+  const int x1 = static_cast<int>((static_cast<long long>(b + 1) * a.total_steps) / a.grid);
+  if (x0 >= x1) return;
+  // zero the stages once: the copies of a rank-4 adapter leave part of each row untouched
+  for (int i = threadIdx.x; i < kDtStages * S::kStage / 16; i += kDtThreads)
+    reinterpret_cast<uint4*>(dt_smem)[i] = make_uint4(0u, 0u, 0u, 0u);
+  __syncthreads();
+
+  float acc[S::kPairs][2][4];
+#pragma unroll
+  for (int p = 0; p < S::kPairs; ++p)
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int v = 0; v < 4; ++v) acc[p][h][v] = 0.f;
+
+  int lseg = seg_of(a, x0, 0);  // segment of the next step to load
+  int lx = x0;
+  auto issue = [&]() {
+    if (lx < x1) {
+      lseg = seg_of(a, lx, lseg);
+      load_step<RP>(step_ref(a, lx, lseg), a.rank, stage0 + ((lx - x0) % kDtStages) * S::kStage);
+    }
+    cp_async_commit();  // empty groups keep the count uniform
+    ++lx;
+  };
+  issue();
+  issue();
+  int seg = seg_of(a, x0, 0);
+  for (int x = x0; x < x1; ++x) {
+    issue();
+    cp_async_wait<kDtStages - 1>();
+    __syncthreads();
+    seg = seg_of(a, x, seg);
+    mma_step<RP>(seg & 1, stage0 + ((x - x0) % kDtStages) * S::kStage, acc);
+    const bool flush = x + 1 == x1 || x + 1 >= a.seg_step0[seg + 1];
+    if (flush) {
+      // the warps' partial Grams summed in warp order, then written as one slot
+      const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+      for (int w = 0; w < kDtThreads / 32; ++w) {
+        if (warp == w) {
+#pragma unroll
+          for (int p = 0; p < S::kPairs; ++p)
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+              for (int v = 0; v < 4; ++v) {
+                float* r = red + lane * (S::kPairs * 8) + p * 8 + h * 4 + v;
+                *r = (w == 0 ? 0.f : *r) + acc[p][h][v];
+              }
+        }
+        __syncthreads();
+      }
+      float* out = slots + static_cast<size_t>(b + seg) * S::kSlotFloats;
+      for (int e = threadIdx.x; e < S::kSlotFloats; e += kDtThreads) {
+        const int p = e >> 8, rr = (e >> 4) & 15, cc = e & 15;
+        const int ln = (rr & 7) * 4 + ((cc & 7) >> 1);
+        const int v = (rr >> 3) * 2 + (cc & 1);
+        out[e] = red[ln * (S::kPairs * 8) + p * 8 + (cc >> 3) * 4 + v];
+      }
+#pragma unroll
+      for (int p = 0; p < S::kPairs; ++p)
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[p][h][v] = 0.f;
+    }
+    __syncthreads();  // the stage read here is refilled two steps on; `red` is reused at the next flush
+  }
+  cp_async_wait<0>();
+}
+
+// One block per item: the segment's slots summed in CTA order, then tr(GB GA) and the
+// parameter distance from the [hi | lo | base] Grams, in fp64.
+template <int RP>
+__global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_constant__ DriftTcArgs a,
+                                                             const float* __restrict__ slots,
+                                                             float* __restrict__ out_sq) {
+  using S = DtShape<RP>;
+  __shared__ float g[2][S::kSlotFloats];
+  __shared__ double red[2][8];
+  const int item = blockIdx.x;
+  for (int side = 0; side < 2; ++side) {
+    const int seg = 2 * item + side;
+    const long long s0 = a.seg_step0[seg], s1 = a.seg_step0[seg + 1] - 1;
+    const int b_lo = static_cast<int>(((s0 + 1) * a.grid - 1) / a.total_steps);
+    const int b_hi = static_cast<int>(((s1 + 1) * a.grid - 1) / a.total_steps);
+    for (int e = threadIdx.x; e < S::kSlotFloats; e += 256) {
+      float v = 0.f;
+      for (int bb = b_lo; bb <= b_hi; ++bb) v += slots[static_cast<size_t>(bb + seg) * S::kSlotFloats + e];
+      g[side][e] = v;
+    }
+  }
+  __syncthreads();
+  // entry (f1, f2) of a side's symmetric feature Gram from its block-upper triangle
+  auto G = [&](int side, int f1, int f2) -> double {
+    int I = f1 >> 4, J = f2 >> 4;
+    if (I > J) {
+      const int t = f1; f1 = f2; f2 = t;
+      I = f1 >> 4; J = f2 >> 4;
+    }
+    const int p = I * S::kBlocks - I * (I - 1) / 2 + (J - I);
+    return static_cast<double>(g[side][p * 256 + (f1 & 15) * 16 + (f2 & 15)]);
+  };
+  // <d_i, d_j>, <d_i, base_j>, <base_i, base_j> with d = hi + lo; features hi_i = i,
+  // lo_i = RP + i, base_i = 2 RP + i
+  auto dd = [&](int s, int i, int j) {
+    return G(s, i, j) + G(s, i, RP + j) + G(s, RP + i, j) + G(s, RP + i, RP + j);
+  };
+  auto db = [&](int s, int i, int j) { return G(s, i, 2 * RP + j) + G(s, RP + i, 2 * RP + j); };
+  auto bb = [&](int s, int i, int j) { return G(s, 2 * RP + i, 2 * RP + j); };
+  const int r = a.rank, r2 = 2 * a.rank;
+  double t = 0.0, par = 0.0;
+  for (int idx = threadIdx.x; idx < r2 * r2; idx += 256) {
+    const int p = idx / r2, q = idx - p * r2;
+    // GB over [B1 - B0 | B0]; GA over [A1 ; A1 - A0]: base first on the A side
+    double gb, ga;
+    if (p < r && q < r) gb = dd(0, p, q);
+    else if (p < r) gb = db(0, p, q - r);
+    else if (q < r) gb = db(0, q, p - r);
+    else gb = bb(0, p - r, q - r);
+    if (p < r && q < r) ga = bb(1, p, q);
+    else if (p < r) ga = db(1, q - r, p);
+    else if (q < r) ga = db(1, p - r, q);
+    else ga = dd(1, p - r, q - r);
+    t += gb * ga;  // both Grams are symmetric: tr(GB GA) = sum_pq GB[p][q] GA[p][q]
+    if (p == q && p < r) par += dd(0, p, p) + dd(1, p, p);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    t += __shfl_xor_sync(0xffffffffu, t, o);
+    par += __shfl_xor_sync(0xffffffffu, par, o);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    red[0][threadIdx.x >> 5] = t;
+    red[1][threadIdx.x >> 5] = par;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double tt = 0.0, pp = 0.0;
+    for (int w = 0; w < 8; ++w) {
+      tt += red[0][w];
+      pp += red[1][w];
+    }
+    out_sq[a.items[item].out_index * 2 + 0] = static_cast<float>(tt);
+    out_sq[a.items[item].out_index * 2 + 1] = static_cast<float>(pp);
+  }
+}
+
+template <int RP>
+cudaError_t launch_rp(const DriftTcArgs& a, float* slots, float* out_sq, cudaStream_t stream) {
+  using S = DtShape<RP>;
+  constexpr int smem = kDtStages * S::kStage + 32 * S::kPairs * 8 * 4;
+  static PerDevice once;
+  int dev = 0;
+  if (once.pending(&dev)) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(drift_tc_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    once.done(dev);
+  }
+  drift_tc_kernel<RP><<<a.grid, kDtThreads, smem, stream>>>(a, slots);
+  drift_tc_final_kernel<RP><<<a.n_items, 256, 0, stream>>>(a, slots, out_sq);
+  return cudaGetLastError();
+}
+
+int slot_floats(int rank) { return rank == 16 ? DtShape<16>::kSlotFloats : DtShape<8>::kSlotFloats; }
+
+}  // namespace
+
+size_t drift_workspace_bytes(int num_sms, int rank, int n_items) {
+  const int items = n_items < kDtMaxItems ? n_items : kDtMaxItems;
+  const size_t slots = static_cast<size_t>(kDtCtasPerSm) * num_sms + 2 * static_cast<size_t>(items);
+  return slots * slot_floats(rank) * sizeof(float);
+}
+
+int drift_launches(int n_items) { return 2 * ((n_items + kDtMaxItems - 1) / kDtMaxItems); }
+
+cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, float* slots, int num_sms,
+                         float* out_sq, cudaStream_t stream) {
+  if (rank != 4 && rank != 8 && rank != 16) return cudaErrorInvalidValue;
+  for (int base = 0; base < n_items; base += kDtMaxItems) {
+    DriftTcArgs a;
+    a.n_items = n_items - base < kDtMaxItems ? n_items - base : kDtMaxItems;
+    a.n_segs = 2 * a.n_items;
+    a.rank = rank;
+    int steps = 0;
+    for (int i = 0; i < a.n_items; ++i) {
+      a.items[i] = items[base + i];
+      for (int side = 0; side < 2; ++side) {
+        a.seg_step0[2 * i + side] = steps;
+        const int len = side == 0 ? a.items[i].out_dim : a.items[i].in_dim;
+        steps += (len + kDtRows - 1) / kDtRows;
+      }
+    }
+    a.seg_step0[a.n_segs] = steps;
+    a.total_steps = steps;
+    const int want = kDtCtasPerSm * num_sms;
+    a.grid = steps < want ? steps : want;
+    if (a.grid < 1) continue;
+    const cudaError_t e = rank == 16 ? launch_rp<16>(a, slots, out_sq, stream)
+                                     : launch_rp<8>(a, slots, out_sq, stream);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace crf

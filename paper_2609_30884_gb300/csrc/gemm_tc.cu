@@ -638,18 +638,12 @@ cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) 
 
 }  // namespace
 
-bool pair_mode_enabled() {
-  static const bool on = [] {
-    const char* v = std::getenv("CRF_GEMM_PAIR");
-    return !(v && v[0] == '0');
-  }();
-  return on;
-}
-
 cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream) {
   GemmArgs a;
   std::memset(&a, 0, sizeof(a));
-  const int pair = (bn == 256 && pair_mode_enabled() && (d.nseg == 1 || d.nseg == 2)) ? 2 : 1;
+  // the 256-wide projection tiles run on CTA pairs; the narrow LoRA-down tiles on single CTAs
+  if (bn == 256 && d.nseg != 1 && d.nseg != 2) return cudaErrorInvalidValue;
+  const int pair = bn == 256 ? 2 : 1;
   // rows of one B load: the CTA's share of the tile (plain) or one stacked segment
   const int b_box = d.nseg == 1 ? bn / pair : bn / d.nseg;
   if (!make_map(&a.tmA, d.A, d.M, d.K, d.lda, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B))
@@ -728,7 +722,6 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
   if (a.total_tiles == 0) return cudaSuccess;
   if (pair == 2) return launch_impl<256, 6, 2>(a, num_sms, stream);
   switch (bn) {
-    case 256: return launch_impl<256, 4, 1>(a, num_sms, stream);
     case 48: return launch_impl<48, 8, 1>(a, num_sms, stream);
     case 32: return launch_impl<32, 8, 1>(a, num_sms, stream);
     case 16: return launch_impl<16, 8, 1>(a, num_sms, stream);

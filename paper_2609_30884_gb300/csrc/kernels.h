@@ -42,8 +42,7 @@ constexpr int kBxCols = 64;
 // programmatic-stream-serialization attribute: such a kernel becomes resident while its
 // predecessor in the stream still runs, prefetches its weights and then waits for it
 // (griddep_wait). Every kernel launched this way calls griddep_wait before it touches memory
-// that an earlier kernel may write. The decode-row layer loop opens a scope; CRF_PDL=0 in the
-// environment turns the attribute off.
+// that an earlier kernel may write. The decode-row layer loop opens a scope.
 class PdlScope {
  public:
   PdlScope();
@@ -126,8 +125,8 @@ struct GemmDesc {
   int* status;
 };
 
-// Launch the tcgen05 GEMM. bn: 256 for projections (CTA pairs with 256-row tiles unless the
-// environment sets CRF_GEMM_PAIR=0); 16/32/48 for LoRA down (single CTAs).
+// Launch the tcgen05 GEMM. bn: 256 for projections (CTA pairs with 256-row tiles); 16/32/48 for
+// LoRA down (single CTAs).
 cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream);
 
 // BX rows of up to 7 modules in one launch: out[m][r, :] = 0 except columns
@@ -163,8 +162,7 @@ struct AttnDesc {
   ReqTable req;
   int* status;
 };
-cudaError_t launch_attention(const AttnDesc& d, int num_sms, cudaStream_t stream);
-// tcgen05 version: num_pages of the pool, total_rows of q (for the TMA maps).
+// tcgen05, S and O in TMEM: num_pages of the pool, total_rows of q (for the TMA maps).
 cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows,
                                 cudaStream_t stream);
 
@@ -191,8 +189,8 @@ struct GemvDesc {
 };
 // Tensor-core GEMV (mma.sync, rows as a bf16 hi/lo pair); launch_gemv uses it when the call's
 // rows (total_rows, the rows of all chunks one caller splits into launches of <= 8; 0 = d.rows)
-// number three or more, unless the environment sets CRF_GEMV=scalar (then always the CUDA-core
-// kernel). One kernel per call keeps equal rows equal across chunks.
+// number three or more (one or two rows run faster on the CUDA-core kernel). One kernel per call
+// keeps equal rows equal across chunks.
 cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int total_rows = 0);
 cudaError_t launch_gemv_tc(const GemvDesc& d, int num_sms, cudaStream_t stream);
 // xa_m[r, k] = scale * sum_i A_m[k, i] x[r, i] for up to three modules m sharing x
@@ -270,9 +268,20 @@ cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStre
 // LM head + KL: logits [2*rows, V] (ref rows first) from final-normed hidden rows.
 cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,
                            float* logits, int num_sms, cudaStream_t stream);
-// KL per row from fp32 logits; part: scratch [rows][splits][4].
+// KL per row from fp32 logits; part: scratch [rows][splits][5].
 cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab, float* out,
                       float* part, int splits, cudaStream_t stream);
+// Vocabulary splits per row of the KL reduction: about two blocks per SM over all rows, at least
+// 1024 logits per split, at most kKlMaxSplits. Every KL entry point uses this count, so they
+// reduce in the same order.
+constexpr int kKlMaxSplits = 256;
+inline int kl_split_count(int num_sms, int n_rows, int vocab) {
+  int want = (2 * num_sms + n_rows - 1) / (n_rows > 0 ? n_rows : 1);
+  const int by_vocab = (vocab + 1023) / 1024;
+  want = want < by_vocab ? want : by_vocab;
+  want = want < kKlMaxSplits ? want : kKlMaxSplits;
+  return want < 1 ? 1 : want;
+}
 
 // Drift: per (layer, module) squared norms; see crf_drift.
 struct DriftItem {
@@ -281,7 +290,12 @@ struct DriftItem {
   int in_dim, out_dim;
   int out_index;           // layer * 7 + module
 };
-cudaError_t launch_drift(const DriftItem* items_dev, int n_items, int rank, float* grams,
-                         int blocks_per_side, float* out_sq, cudaStream_t stream);
+// Tensor-core drift (mma.sync Grams over the long dimensions, fp64 combine); `slots` is device
+// scratch of drift_workspace_bytes(num_sms, rank, n_items) bytes. Launches drift_launches(n)
+// kernels.
+size_t drift_workspace_bytes(int num_sms, int rank, int n_items);
+int drift_launches(int n_items);
+cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, float* slots, int num_sms,
+                         float* out_sq, cudaStream_t stream);
 
 }  // namespace crf

@@ -22,30 +22,69 @@ void set_last_error(const char* msg);
 namespace {
 
 constexpr int kNoallocMaxRows = 32;
-constexpr int kNoallocMaxSplits = 256;
 constexpr int kPartFloats = 5;  // (max*, sum*, dot*, max, sum) per (row, split)
 constexpr int kMaxDevices = 64;
 
 // Per-(row, split) partials of one call: 32 x 256 x 5 floats = 160 KiB.
-static __device__ __align__(256) float g_kl_scratch[kNoallocMaxRows * kNoallocMaxSplits * kPartFloats];
+static __device__ __align__(256) float g_kl_scratch[kNoallocMaxRows * crf::kKlMaxSplits * kPartFloats];
+
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+
+// cuCtxGetCurrent from the driver, through the runtime's entry-point query (the library links
+// only the runtime). Null if the driver does not provide it.
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      return reinterpret_cast<CtxGetCurrentFn>(p);
+    return static_cast<CtxGetCurrentFn>(nullptr);
+  }();
+  return fn;
+}
 
 std::mutex g_setup_mu;
-float* g_scratch_addr[kMaxDevices] = {};
+struct Setup {
+  CUcontext ctx;
+  float* addr;
+};
+Setup g_setup[kMaxDevices] = {};
 
-// Device address of g_kl_scratch on `device` (which must be current). Looked
-// up once per device; the host-side name of the array is not a device address.
+// Device address of g_kl_scratch on `device`, which must be current. The host-side name of the
+// array is not a device address, so the address is looked up with cudaGetSymbolAddress: once
+// per device and context. A device reset followed by a new primary context gives a new context
+// handle, and the address is looked up again for it instead of reusing the old context's.
 crf_status scratch_on(int device, float** out) {
+  CtxGetCurrentFn get = ctx_get_current();
+  if (!get) {
+    crf::set_last_error("crf_kl_logits_noalloc: cuCtxGetCurrent is unavailable");
+    return CRF_ECUDA;
+  }
+  // the runtime binds the device's primary context on first use; make that happen first
+  if (cudaFree(nullptr) != cudaSuccess) {
+    crf::set_last_error("crf_kl_logits_noalloc: cannot initialise the device context");
+    return CRF_ECUDA;
+  }
+  CUcontext cur = nullptr;
+  if (get(&cur) != CUDA_SUCCESS || !cur) {
+    crf::set_last_error("crf_kl_logits_noalloc: no current CUDA context");
+    return CRF_ECUDA;
+  }
   std::lock_guard<std::mutex> lock(g_setup_mu);
-  if (!g_scratch_addr[device]) {
+  Setup& s = g_setup[device];
+  if (s.ctx != cur || !s.addr) {
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_kl_scratch);
     if (e != cudaSuccess || !p) {
       crf::set_last_error(cudaGetErrorString(e));
       return CRF_ECUDA;
     }
-    g_scratch_addr[device] = static_cast<float*>(p);
+    s.ctx = cur;
+    s.addr = static_cast<float*>(p);
   }
-  *out = g_scratch_addr[device];
+  *out = s.addr;
   return CRF_OK;
 }
 
@@ -81,10 +120,8 @@ extern "C" crf_status crf_kl_logits_noalloc(int device, const float* z_ref, cons
   if (st == CRF_OK) {
     int sms = 1;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
-    int splits = (2 * sms + n_rows - 1) / n_rows;
-    splits = splits < (vocab + 1023) / 1024 ? splits : (vocab + 1023) / 1024;
-    splits = splits < kNoallocMaxSplits ? splits : kNoallocMaxSplits;
-    splits = splits < 1 ? 1 : splits;
+    // the same split count as crf_kl, so both reduce in the same order; at most kKlMaxSplits
+    const int splits = crf::kl_split_count(sms, n_rows, vocab);
     // Every (row, split) partial is written before it is read: nothing needs clearing.
     const cudaError_t e = crf::launch_kl(z_ref, z_cur, n_rows, vocab, out_kl, part, splits,
                                          static_cast<cudaStream_t>(stream));

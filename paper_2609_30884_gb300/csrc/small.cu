@@ -1,7 +1,6 @@
 // Memory-bound kernels: RMSNorm, embedding gather, RoPE angle table, the
 // small-M decode path (GEMV with fused LoRA, RoPE on rows, SwiGLU), the LM
-// head, the first-step KL reduction (Section S2.1) and the rank-factored
-// adapter drift (Eq. 8).
+// head and the first-step KL reduction (Section S2.1).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -414,141 +413,6 @@ __global__ void kl_final_kernel(const float* part, int splits, float* out, int r
   if (lane == 0) out[row] = Dr / Sr + (Mc + logf(Sc)) - (Mr + logf(Sr));
 }
 
-// ------------------------------------------------------------------ drift
-// Partial 2r x 2r Grams over a chunk of the long dimension, for one side of one
-// (layer, module) item. Side 0 (B): vector per output row o is
-// (B1[o,:] - B0[o,:], B0[o,:]); side 1 (A): vector per input column c is
-// (A1[:,c], A1[:,c] - A0[:,c]).
-constexpr int kDriftRows = 128;
-constexpr int kMaxDriftItems = 224;
-
-struct DriftBatch {
-  DriftItem items[kMaxDriftItems];
-  int n_items;
-};
-
-template <int R2>
-__global__ void __launch_bounds__(256) drift_partial_kernel(const __grid_constant__ DriftBatch batch,
-                                                            int blocks_per_side, float* grams) {
-  constexpr int R = R2 / 2;
-  const int item = blockIdx.z, side = blockIdx.y, blk = blockIdx.x;
-  const DriftItem& it = batch.items[item];
-  const int L = side == 0 ? it.out_dim : it.in_dim;
-  // pieces of whole 128-row chunks, so every chunk starts 16-byte aligned (L % 8 == 0)
-  const int per = (((L + blocks_per_side - 1) / blocks_per_side + kDriftRows - 1) / kDriftRows) * kDriftRows;
-  const int l0 = blk * per, l1 = min(L, l0 + per);
-  __shared__ float vec[kDriftRows][R2 + 1];
-  constexpr int T = R2 / 4;  // 4x4 tiles per dimension
-  // thread layout: group = tid / (T*T) splits the rows of each chunk
-  constexpr int TILES = T * T;
-  constexpr int GROUPS = 256 / TILES;
-  const int tid = threadIdx.x;
-  const int grp = tid / TILES, tt = tid % TILES;
-  const int ti = tt / T, tj = tt % T;
-  float acc[4][4];
-#pragma unroll
-  for (int a = 0; a < 4; ++a)
-#pragma unroll
-    for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
-  for (int c0 = l0; c0 < l1; c0 += kDriftRows) {
-    const int cn = min(kDriftRows, l1 - c0);
-    __syncthreads();
-    // 4 consecutive bf16 per thread (8-byte loads): B rows are contiguous in k, A rows in the
-    // input dimension; cn and R are multiples of 4
-    for (int i = tid; i < cn * R / 4; i += 256) {
-      if (side == 0) {
-        const int rr = i / (R / 4), k = (i % (R / 4)) * 4;
-        const size_t off = (size_t)(c0 + rr) * R + k;
-        const uint2 u0 = *reinterpret_cast<const uint2*>(it.B0 + off);
-        const uint2 u1 = *reinterpret_cast<const uint2*>(it.B1 + off);
-        const float b0[4] = {bf16_lo(u0.x), bf16_hi(u0.x), bf16_lo(u0.y), bf16_hi(u0.y)};
-        const float b1[4] = {bf16_lo(u1.x), bf16_hi(u1.x), bf16_lo(u1.y), bf16_hi(u1.y)};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          vec[rr][k + e] = b1[e] - b0[e];
-          vec[rr][R + k + e] = b0[e];
-        }
-      } else {
-        const int k = i / (cn / 4), rr = (i % (cn / 4)) * 4;  // coalesced along the input dimension
-        const size_t off = (size_t)k * it.in_dim + c0 + rr;
-        const uint2 u0 = *reinterpret_cast<const uint2*>(it.A0 + off);
-        const uint2 u1 = *reinterpret_cast<const uint2*>(it.A1 + off);
-        const float a0[4] = {bf16_lo(u0.x), bf16_hi(u0.x), bf16_lo(u0.y), bf16_hi(u0.y)};
-        const float a1[4] = {bf16_lo(u1.x), bf16_hi(u1.x), bf16_lo(u1.y), bf16_hi(u1.y)};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          vec[rr + e][k] = a1[e];
-          vec[rr + e][R + k] = a1[e] - a0[e];
-        }
-      }
-    }
-    __syncthreads();
-    for (int rr = grp; rr < cn; rr += GROUPS) {
-      float x[4], y[4];
-#pragma unroll
-      for (int a = 0; a < 4; ++a) {
-        x[a] = vec[rr][ti * 4 + a];
-        y[a] = vec[rr][tj * 4 + a];
-      }
-#pragma unroll
-      for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) acc[a][b] += x[a] * y[b];
-    }
-  }
-  // every thread's 4x4 tile into [GROUPS][R2 * R2] (256 x 16 floats whatever R2 is), then each
-  // output summed over the row groups in a fixed order
-  __shared__ float part[GROUPS * R2 * R2];
-#pragma unroll
-  for (int a = 0; a < 4; ++a)
-#pragma unroll
-    for (int b = 0; b < 4; ++b) part[grp * R2 * R2 + (ti * 4 + a) * R2 + tj * 4 + b] = acc[a][b];
-  __syncthreads();
-  float* out = grams + (((size_t)item * 2 + side) * blocks_per_side + blk) * R2 * R2;
-  for (int i = tid; i < R2 * R2; i += 256) {
-    float v = 0.f;
-    for (int gg = 0; gg < GROUPS; ++gg) v += part[gg * R2 * R2 + i];
-    out[i] = v;
-  }
-}
-
-template <int R2>
-__global__ void __launch_bounds__(256) drift_final_kernel(const __grid_constant__ DriftBatch batch,
-                                                          int blocks_per_side, const float* grams,
-                                                          float* out_sq) {
-  constexpr int R = R2 / 2;
-  const int item = blockIdx.x;
-  __shared__ float gb[R2 * R2], ga[R2 * R2];
-  for (int i = threadIdx.x; i < R2 * R2; i += 256) {
-    float sb = 0.f, sa = 0.f;
-    for (int b = 0; b < blocks_per_side; ++b) {
-      sb += grams[(((size_t)item * 2 + 0) * blocks_per_side + b) * R2 * R2 + i];
-      sa += grams[(((size_t)item * 2 + 1) * blocks_per_side + b) * R2 * R2 + i];
-    }
-    gb[i] = sb;
-    ga[i] = sa;
-  }
-  __syncthreads();
-  // trace(Gb Ga) = sum_ij Gb[i,j] Ga[j,i]
-  float t = 0.f;
-  for (int i = threadIdx.x; i < R2 * R2; i += 256) {
-    const int a = i / R2, b = i % R2;
-    t += gb[i] * ga[b * R2 + a];
-  }
-  __shared__ float red[8];
-  t = warp_sum(t);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = t;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float tot = 0.f;
-    for (int w = 0; w < 8; ++w) tot += red[w];
-    float par = 0.f;
-    for (int k = 0; k < R; ++k) par += gb[k * R2 + k] + ga[(R + k) * R2 + R + k];
-    out_sq[batch.items[item].out_index * 2 + 0] = tot;
-    out_sq[batch.items[item].out_index * 2 + 1] = par;
-  }
-}
-
 inline int cdiv(long a, long b) { return static_cast<int>((a + b - 1) / b); }
 
 }  // namespace
@@ -592,31 +456,16 @@ cudaError_t gemv_dispatch(const GemvLaunch& L, int blocks, cudaStream_t stream) 
 
 namespace {
 thread_local bool t_pdl = false;
-bool pdl_env() {
-  static const bool on = [] {
-    const char* e = std::getenv("CRF_PDL");
-    return !(e && std::strcmp(e, "0") == 0);
-  }();
-  return on;
-}
 }  // namespace
 
-PdlScope::PdlScope() : prev_(t_pdl) { t_pdl = pdl_env(); }
+PdlScope::PdlScope() : prev_(t_pdl) { t_pdl = true; }
 PdlScope::~PdlScope() { t_pdl = prev_; }
 bool pdl_active() { return t_pdl; }
-
-static bool gemv_scalar() {
-  static const bool on = [] {
-    const char* e = std::getenv("CRF_GEMV");
-    return e && std::strcmp(e, "scalar") == 0;
-  }();
-  return on;
-}
 
 bool gemv_use_tensor(int total_rows, int in_dim) {
   // the MMA path pays for its 16-row tiles and x splitting from three rows on (measured: 1-2 rows
   // run faster on the CUDA-core kernel, 3 rows 20% and 8 rows 45% faster on the tensor cores)
-  return !gemv_scalar() && total_rows >= 3 && in_dim % 16 == 0;
+  return total_rows >= 3 && in_dim % 16 == 0;
 }
 
 cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int total_rows) {
@@ -893,31 +742,6 @@ cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab,
   kl_partial_kernel<<<dim3(splits, rows), kKlThreads, 0, stream>>>(zref, zcur, vocab, splits, part);
   kl_final_kernel<<<cdiv(rows, 8), 256, 0, stream>>>(part, splits, out, rows);
   return cudaGetLastError();
-}
-
-cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, float* grams,
-                         int blocks_per_side, float* out_sq, cudaStream_t stream) {
-  for (int base = 0; base < n_items; base += kMaxDriftItems) {
-    DriftBatch b;
-    b.n_items = n_items - base < kMaxDriftItems ? n_items - base : kMaxDriftItems;
-    for (int i = 0; i < b.n_items; ++i) b.items[i] = items[base + i];
-    dim3 g1(blocks_per_side, 2, b.n_items);
-    if (rank == 16) {
-      drift_partial_kernel<32><<<g1, 256, 0, stream>>>(b, blocks_per_side, grams);
-      drift_final_kernel<32><<<b.n_items, 256, 0, stream>>>(b, blocks_per_side, grams, out_sq);
-    } else if (rank == 8) {
-      drift_partial_kernel<16><<<g1, 256, 0, stream>>>(b, blocks_per_side, grams);
-      drift_final_kernel<16><<<b.n_items, 256, 0, stream>>>(b, blocks_per_side, grams, out_sq);
-    } else if (rank == 4) {
-      drift_partial_kernel<8><<<g1, 256, 0, stream>>>(b, blocks_per_side, grams);
-      drift_final_kernel<8><<<b.n_items, 256, 0, stream>>>(b, blocks_per_side, grams, out_sq);
-    } else {
-      return cudaErrorInvalidValue;
-    }
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  return cudaSuccess;
 }
 
 }  // namespace crf

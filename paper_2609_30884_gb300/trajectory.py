@@ -13,7 +13,8 @@ paper's acceptance rule for a candidate window (KL <= 0.05 and the top-1 token k
 Maintenance = what a serving system runs per update: the drift queries the policy needs
 (``crf_drift``), the window's ``crf_recompute_window`` (refreshing K/V pages and checkpoints), and
 the host decision. The fresh reference and the evaluation of each method's first-step state are
-measured outside it. Used by ``bench.py --case trajectory`` and the GPU tests.
+measured outside it. Used by ``bench.py --case trajectory`` and the GPU tests, which supply the
+synthetic adapter versions, token ids and page table.
 """
 from __future__ import annotations
 
@@ -22,46 +23,27 @@ from typing import Dict, List, Optional, Sequence, Tuple
 
 import torch
 
-import synth
 import paper_2609_30884_gb300 as crf
-from harness import DeviceAdapter, make_pool, pages_needed, split_page_tables
 from paper_2609_30884_gb300 import policy as P
 
 KL_SAFE = 0.05
 METHODS = ("fresh_full", "exact_suffix", "stale_reuse", "cachereforge", "drift_only", "fixed_window_2")
 
 
-class Versions:
-    """Adapter versions 0..T of one trajectory: version 0 is the workload adapter (its version
-    ``base_version``); versions differ only in (layer, module)."""
-
-    def __init__(self, cfg, lcfg, layer: int, module: str, std: float, seed: int, device,
-                 base_version: int = 1):
-        self.cfg, self.lcfg, self.layer, self.module, self.std, self.seed = cfg, lcfg, layer, module, std, seed
-        self.device, self.base_version = device, base_version
-        self.base = DeviceAdapter(cfg, lcfg, base_version, device)
-        self._layers: Dict[int, list] = {}
-        self._ad: Dict[int, crf.Adapter] = {}
-
-    def adapter(self, t: int) -> crf.Adapter:
-        if t not in self._ad:
-            layers = list(self.base.layers)
-            if t > 0:
-                d = dict(layers[self.layer])
-                d[self.module] = synth.trajectory_factors(self.cfg, self.lcfg, self.base_version, self.layer,
-                                                          self.module, t, self.std, self.seed, self.device)
-                layers[self.layer] = d
-            self._layers[t] = layers  # keeps the tensors alive for the pointers below
-            self._ad[t] = crf.Adapter(self.lcfg.rank, self.lcfg.alpha, self.lcfg.modules, layers)
-        return self._ad[t]
+def zero_pool(dims: dict, num_pages: int, device) -> crf.KVPool:
+    """Per-layer K and V page pools of zeros, bf16 [num_pages, Hkv, 16, d]."""
+    shape = (num_pages, dims["n_kv_heads"], 16, dims["head_dim"])
+    return crf.KVPool([torch.zeros(shape, dtype=torch.bfloat16, device=device) for _ in range(dims["n_layers"])],
+                      [torch.zeros(shape, dtype=torch.bfloat16, device=device) for _ in range(dims["n_layers"])])
 
 
 class CacheState:
     """One method's cache of the prefix: K/V pages of every layer and the checkpoints H_l."""
 
-    def __init__(self, cfg, n: int, num_pages: int, device):
-        self.pool = make_pool(cfg, num_pages, device)
-        self.H = [torch.empty(n, cfg.hidden, dtype=torch.bfloat16, device=device) for _ in range(cfg.n_layers)]
+    def __init__(self, dims: dict, n: int, num_pages: int, device):
+        self.pool = zero_pool(dims, num_pages, device)
+        self.H = [torch.empty(n, dims["hidden"], dtype=torch.bfloat16, device=device)
+                  for _ in range(dims["n_layers"])]
 
     def copy_from(self, other: "CacheState") -> None:
         for a, b in zip(self.pool.k_pages + self.pool.v_pages + self.H,
@@ -70,37 +52,41 @@ class CacheState:
 
 
 class Trajectory:
-    def __init__(self, ctx: crf.Context, dm, cfg, lcfg, n: int, layer: int, module: str, std: float,
-                 device="cuda:0", seed: int = 0):
-        self.ctx, self.dm, self.cfg, self.lcfg, self.n = ctx, dm, cfg, lcfg, n
-        self.layer, self.module, self.std, self.device, self.seed = layer, module, std, device, seed
-        self.N = cfg.n_layers
-        self.num_pages = pages_needed(n)
-        self.pt = split_page_tables([n], self.num_pages, seed=1, device=device)[0]
-        self.tokens = synth.token_ids(cfg, n, device=device)
+    """One prefix (``tokens`` on the pages of ``page_table``) whose adapter changes at (layer, module)."""
+
+    def __init__(self, ctx: crf.Context, model: crf.Model, tokens: torch.Tensor, page_table: torch.Tensor,
+                 layer: int, module: str, device="cuda:0"):
+        dims = model.dims
+        self.ctx, self.model, self.dims = ctx, model, dims
+        self.n = int(tokens.shape[0])
+        self.layer, self.module, self.device = layer, module, device
+        self.N = dims["n_layers"]
+        self.num_pages = (self.n + 15) // 16
+        self.pt = page_table
+        self.tokens = tokens
         self.restart = P.restart_of([(module, layer)], self.N)
-        self.fin = torch.empty(cfg.hidden, dtype=torch.bfloat16, device=device)
-        self.fresh_fin = torch.empty(cfg.hidden, dtype=torch.bfloat16, device=device)
+        self.fin = torch.empty(dims["hidden"], dtype=torch.bfloat16, device=device)
+        self.fresh_fin = torch.empty(dims["hidden"], dtype=torch.bfloat16, device=device)
         self.out_kl = torch.empty(1, dtype=torch.float32, device=device)
-        self.logits = torch.empty(2, cfg.vocab, dtype=torch.float32, device=device)
-        self.kl_ws = ctx.kl_workspace(1, cfg.vocab, cfg.hidden)
+        self.logits = torch.empty(2, dims["vocab"], dtype=torch.float32, device=device)
+        self.kl_ws = ctx.kl_workspace(1, dims["vocab"], dims["hidden"])
         self.drift_out = torch.empty(self.N, 7, 2, dtype=torch.float32, device=device)
         self._ws: Dict[Tuple[int, int, bool], torch.Tensor] = {}
-        self.fresh_pool = make_pool(cfg, self.num_pages, device)
+        self.fresh_pool = zero_pool(dims, self.num_pages, device)
 
     # ------------------------------------------------------------------ device calls
     def _workspace(self, ad, req, key):
         if key not in self._ws:
-            self._ws[key] = self.ctx.workspace(self.dm.crf, ad, [req])
+            self._ws[key] = self.ctx.workspace(self.model, ad, [req])
         return self._ws[key]
 
     def prefill(self, ad: crf.Adapter, state: CacheState) -> None:
         req = crf.Request(self.pt, 0, self.N, n_tokens=self.n, tokens=self.tokens, hidden_out=state.H)
-        self.ctx.recompute_window(self.dm.crf, ad, state.pool, [req], self._workspace(ad, req, (0, self.N, False)))
+        self.ctx.recompute_window(self.model, ad, state.pool, [req], self._workspace(ad, req, (0, self.N, False)))
 
     def fresh_reference(self, ad: crf.Adapter) -> None:
         req = crf.Request(self.pt, 0, self.N, n_tokens=self.n, tokens=self.tokens, final_hidden_out=self.fresh_fin)
-        self.ctx.recompute_window(self.dm.crf, ad, self.fresh_pool, [req],
+        self.ctx.recompute_window(self.model, ad, self.fresh_pool, [req],
                                   self._workspace(ad, req, (0, self.N, True)))
 
     def refresh(self, ad: crf.Adapter, state: CacheState, window: Tuple[int, int]) -> None:
@@ -109,7 +95,7 @@ class Trajectory:
             return
         req = crf.Request(self.pt, s, e, n_tokens=self.n, tokens=self.tokens if s == 0 else None,
                           hidden_in=state.H[s - 1] if s > 0 else None, hidden_out=state.H[s:e])
-        self.ctx.recompute_window(self.dm.crf, ad, state.pool, [req], self._workspace(ad, req, (s, e, False)))
+        self.ctx.recompute_window(self.model, ad, state.pool, [req], self._workspace(ad, req, (s, e, False)))
 
     def first_step(self, ad: crf.Adapter, state: CacheState, window: Tuple[int, int]) -> Tuple[float, bool]:
         """KL(fresh || recovered) and top-1 agreement of the first-step distribution: the last row
@@ -119,19 +105,19 @@ class Trajectory:
             req = crf.Request(self.pt, 0, 0, n_tokens=self.n, tokens=self.tokens, final_hidden_out=self.fin)
         else:
             req = crf.Request(self.pt, b, b, n_tokens=self.n, hidden_in=state.H[b - 1], final_hidden_out=self.fin)
-        self.ctx.recompute_window(self.dm.crf, ad, state.pool, [req], self._workspace(ad, req, (b, b, True)))
-        self.ctx.kl(self.dm.crf, self.fresh_fin[None], self.fin[None], self.out_kl, self.cfg.vocab, self.kl_ws,
+        self.ctx.recompute_window(self.model, ad, state.pool, [req], self._workspace(ad, req, (b, b, True)))
+        self.ctx.kl(self.model, self.fresh_fin[None], self.fin[None], self.out_kl, self.dims["vocab"], self.kl_ws,
                     logits_out=self.logits)
         top1 = bool((self.logits[0].argmax() == self.logits[1].argmax()).item())
         return float(self.out_kl.item()), top1
 
-    def state_distance(self, vers: Versions, t: int, anchor: int, ws) -> float:
+    def state_distance(self, vers, t: int, anchor: int, ws) -> float:
         """||theta_t - theta_anchor|| over the whole adapter state, on the device."""
-        self.ctx.drift(self.dm.crf.dims_c, vers.adapter(t), [vers.adapter(anchor)] * self.N, self.drift_out, ws)
+        self.ctx.drift(self.model.dims_c, vers.adapter(t), [vers.adapter(anchor)] * self.N, self.drift_out, ws)
         return P.state_displacement(self.drift_out.cpu().tolist())
 
     # ------------------------------------------------------------------ calibration (Eq. 6-7)
-    def calibrate(self, vers: Versions, versions: int, base: CacheState, scratch: CacheState, drift_ws):
+    def calibrate(self, vers, versions: int, base: CacheState, scratch: CacheState, drift_ws):
         """Conditions (d_k, r, h*_k) for k = 1..versions of a calibration trajectory whose cache
         was built under version 0: h*_k is the first candidate window whose first-step state meets
         the acceptance rule against the fresh model of version k."""
@@ -178,38 +164,42 @@ def make_policy(method: str, n_layers: int, sens, thr) -> P.RecoveryPolicy:
     raise ValueError(method)
 
 
-def run(ctx, dm, cfg, lcfg, n: int, versions: int = 32, calib_versions: int = 8, layer: Optional[int] = None,
-        module: str = "v", std: float = 1e-2, methods: Sequence[str] = METHODS, device="cuda:0",
-        calib_seed: int = 101, eval_seed: int = 202, sensitivity: Optional[Sequence[float]] = None,
-        threshold: Optional[float] = None, base_version: int = 0) -> dict:
+def run(ctx, model: crf.Model, tokens: torch.Tensor, page_table: torch.Tensor, make_versions,
+        versions: int = 32, calib_versions: int = 8, layer: Optional[int] = None, module: str = "v",
+        methods: Sequence[str] = METHODS, device="cuda:0", calib_seed: int = 101, eval_seed: int = 202,
+        sensitivity: Optional[Sequence[float]] = None, threshold: Optional[float] = None) -> dict:
     """Calibrate on one trajectory (unless ``sensitivity`` and ``threshold`` are given), then replay
     another for every method; returns the summary with each method's per-version windows and KL.
-    Version 0 of both trajectories is the workload adapter's version ``base_version``."""
-    layer = cfg.n_layers // 2 if layer is None else layer
-    tr = Trajectory(ctx, dm, cfg, lcfg, n, layer, module, std, device)
-    base = CacheState(cfg, n, tr.num_pages, device)
+    ``make_versions(seed)`` returns that trajectory's versions: an object whose ``adapter(t)`` is
+    the ``crf.Adapter`` of version t (t = 0 the adapter every cache starts from) and differs from
+    version 0 only at (layer, module)."""
+    n_layers = model.dims["n_layers"]
+    layer = n_layers // 2 if layer is None else layer
+    n = int(tokens.shape[0])
+    tr = Trajectory(ctx, model, tokens, page_table, layer, module, device)
+    base = CacheState(model.dims, n, tr.num_pages, device)
     conds = []
     if sensitivity is None:
-        scratch = CacheState(cfg, n, tr.num_pages, device)
-        cal = Versions(cfg, lcfg, layer, module, std, calib_seed, device, base_version)
-        drift_ws = ctx.drift_workspace(dm.crf.dims_c, cal.base.crf.dims_c)
+        scratch = CacheState(model.dims, n, tr.num_pages, device)
+        cal = make_versions(calib_seed)
+        drift_ws = ctx.drift_workspace(model.dims_c, cal.adapter(0).dims_c)
         tr.prefill(cal.adapter(0), base)
         conds = tr.calibrate(cal, calib_versions, base, scratch, drift_ws)
-        sens = P.calibrate_sensitivity(conds, cfg.n_layers)
+        sens = P.calibrate_sensitivity(conds, n_layers)
         thr = drift_threshold(conds)
         del scratch, cal
     else:
         sens, thr = list(sensitivity), threshold
 
-    ev = Versions(cfg, lcfg, layer, module, std, eval_seed, device, base_version)
-    drift_ws = ctx.drift_workspace(dm.crf.dims_c, ev.base.crf.dims_c)
+    ev = make_versions(eval_seed)
+    drift_ws = ctx.drift_workspace(model.dims_c, ev.adapter(0).dims_c)
     tr.prefill(ev.adapter(0), base)
     states = {}
     for m in methods:
-        states[m] = CacheState(cfg, n, tr.num_pages, device)
+        states[m] = CacheState(model.dims, n, tr.num_pages, device)
         states[m].copy_from(base)
     del base
-    pols = {m: make_policy(m, cfg.n_layers, sens, thr) for m in methods}
+    pols = {m: make_policy(m, n_layers, sens, thr) for m in methods}
     stats = {m: {"maint_ms": 0.0, "kl": [], "top1": [], "frac": [], "windows": [],
                  "actions": {"reuse": 0, "bounded": 0, "suffix": 0}} for m in methods}
     ev_a, ev_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -238,7 +228,7 @@ def run(ctx, dm, cfg, lcfg, n: int, versions: int = 32, calib_versions: int = 8,
             s["top1"].append(top1)
             s["frac"].append(pol.fraction(w))
             s["windows"].append(list(w))
-            kind = "reuse" if w[1] <= w[0] else ("suffix" if w[1] == cfg.n_layers else "bounded")
+            kind = "reuse" if w[1] <= w[0] else ("suffix" if w[1] == n_layers else "bounded")
             s["actions"][kind] += 1
     ctx.check()
     out = {"calibration": {"versions": calib_versions if conds else 0, "seed": calib_seed,

@@ -20,7 +20,7 @@ import torch  # noqa: E402
 
 import synth  # noqa: E402
 import paper_2609_30884_gb300 as crf  # noqa: E402
-from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables  # noqa: E402
+from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables  # noqa: E402
 from oracle import cache as C  # noqa: E402
 from tests.gpu_util import (REL_KVH, oracle_adapter, oracle_model, oracle_pool, rel_frob,  # noqa: E402
                             request_kv, to_np)

@@ -19,7 +19,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceAdapter, DeviceModel, make_pool, split_page_tables
+from tests.harness import DeviceAdapter, DeviceModel, make_pool, split_page_tables
 from oracle import build as obuild, decoder as Dec
 from tests.gpu_util import (REL_KVH, bf16_layer_rows, free_slots, rel_frob, snapshot, to_np,
                             untouched_mask)

@@ -14,7 +14,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 
 pytestmark = pytest.mark.gpu
 

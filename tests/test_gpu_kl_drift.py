@@ -4,7 +4,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceAdapter, DeviceModel
+from tests.harness import DeviceAdapter, DeviceModel
 from oracle import cache as C, drift as odrift, fidelity
 from tests.gpu_util import DRIFT_REL, KL_ABS, oracle_adapter, oracle_model, rel_frob, to_np
 

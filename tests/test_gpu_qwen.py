@@ -23,7 +23,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 from oracle import build as obuild, cache as C, decoder as Dec, fidelity
 from tests.gpu_util import (KL_ABS, REL_KVH, bf16_round, free_slots, oracle_adapter, oracle_model,
                             oracle_pool, rel_frob, request_kv, snapshot, bf16_execution_recover,

@@ -10,7 +10,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 from oracle import cache as C, fidelity
 from tests.gpu_util import KL_ABS, oracle_adapter, oracle_model, to_np
 

@@ -14,7 +14,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceModel, pages_needed, split_page_tables
+from tests.harness import DeviceModel, Versions, pages_needed, split_page_tables
 from oracle import cache as C, drift as odrift, fidelity, policy as OP
 from oracle.decoder import LayerAdapter, lora_scale
 from tests.gpu_util import KL_ABS, oracle_model
@@ -88,7 +88,7 @@ def test_trajectory_matches_oracle_replay():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     import paper_2609_30884_gb300 as crf
-    import trajectory as T
+    from paper_2609_30884_gb300 import trajectory as T
 
     ads = [_oracle_adapter(t) for t in range(VERSIONS + 1)]
     d01 = math.sqrt(_state_sq(ads[0][1], ads[1][1]))
@@ -108,8 +108,11 @@ def test_trajectory_matches_oracle_replay():
     assert any(w[1] > w[0] for w in want["cachereforge"][0]) and any(w[1] == w[0] for w in want["cachereforge"][0])
 
     ctx = crf.Context(0)
-    got = T.run(ctx, dm, CFG, LC, N_TOK, versions=VERSIONS, layer=LAYER, module=MODULE, std=STD,
-                eval_seed=SEED, sensitivity=sens, threshold=thr, base_version=BASE)
+    got = T.run(ctx, dm.crf, synth.token_ids(CFG, N_TOK, device="cuda:0"),
+                split_page_tables([N_TOK], pages_needed(N_TOK), seed=1, device="cuda:0")[0],
+                lambda seed: Versions(CFG, LC, LAYER, MODULE, STD, seed, "cuda:0", BASE),
+                versions=VERSIONS, layer=LAYER, module=MODULE, eval_seed=SEED, sensitivity=sens,
+                threshold=thr)
     for m, (wins, kls, _) in want.items():
         g = got["methods"][m]
         assert g["windows"] == wins, (m, g["windows"], wins)

@@ -13,7 +13,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 from oracle import cache as C, drift as odrift, fidelity
 from tests.gpu_util import (DRIFT_REL, KL_ABS, REL_KVH, oracle_adapter, oracle_model, oracle_pool,
                             rel_frob, request_kv, snapshot, to_np, untouched_mask, free_slots)

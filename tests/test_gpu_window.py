@@ -4,7 +4,7 @@ import pytest
 import torch
 
 import synth
-from harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
+from tests.harness import DeviceAdapter, DeviceModel, make_pool, pages_needed, split_page_tables
 from oracle import cache as C
 from tests.gpu_util import (REL_KVH, free_slots, oracle_adapter, oracle_model, oracle_pool,
                             rel_frob, request_kv, snapshot, to_np, untouched_mask)
@@ -179,6 +179,7 @@ def test_full_prefill_matches_oracle_prefill(ctx, tiny):
     for l in range(cfg.n_layers):
         assert rel_frob(to_np(hs[l]), oreq.hidden[l]) <= REL_KVH
         assert rel_frob(request_kv(pool.k_pages[l], pt, n), request_kv(torch.from_numpy(opool.k[l]), pt, n)) <= REL_KVH
+        assert rel_frob(request_kv(pool.v_pages[l], pt, n), request_kv(torch.from_numpy(opool.v[l]), pt, n)) <= REL_KVH
     assert rel_frob(to_np(fin), x[-1]) <= REL_KVH
 
 

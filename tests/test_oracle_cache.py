@@ -47,15 +47,37 @@ def test_write_touches_only_request_slots():
     assert not pool.k[1][8, :, 3:].any()          # slots past the prefix end
 
 
-def test_window_full_equals_prefill(tiny):
+def test_prefill_equals_hand_unrolled_layer_loop(tiny):
+    """Fresh prefill against the decoder layers composed by hand from the embedding (Eq. S1:
+    H_l = F_l(H_{l-1}), C_l = G_l(H_{l-1}), H_{-1} = E[tokens]), with each layer's K/V read back
+    from page page_table[t // 16], slot t % 16 by direct indexing of the pool arrays."""
+    model, v0, _ = tiny
+    req = _req(n=83)
+    pool = _pool(16)
+    C.prefill(model, v0, pool, req)
+    x = model.embed[req.tokens].astype(np.float32)
+    np.testing.assert_array_equal(req.hidden[-1], x)
+    t = np.arange(req.n)
+    for l in range(CFG.n_layers):
+        x, k, v = D.decoder_layer(x, model.layers[l], v0.layers[l], model.dims)
+        np.testing.assert_array_equal(pool.k[l][req.page_table[t // 16], :, t % 16, :], k)
+        np.testing.assert_array_equal(pool.v[l][req.page_table[t // 16], :, t % 16, :], v)
+        np.testing.assert_array_equal(req.hidden[l], x)
+
+
+def test_split_windows_compose_to_prefill(tiny):
+    """Two windows [0, 2) and [2, N), the second restarting from the first's H_1, leave the same
+    cache and checkpoints as one fresh prefill: restart from a retained boundary state (Section 4.2)."""
     model, v0, _ = tiny
     r1, r2 = _req(), _req()
     p1, p2 = _pool(16), _pool(16)
     C.prefill(model, v0, p1, r1)
-    x = C.run_window(model, v0, p2, r2, 0, CFG.n_layers)
+    C.run_window(model, v0, p2, r2, 0, 2)
+    x = C.run_window(model, v0, p2, r2, 2, CFG.n_layers)
     for l in range(CFG.n_layers):
         np.testing.assert_array_equal(p1.k[l], p2.k[l])
         np.testing.assert_array_equal(p1.v[l], p2.v[l])
+        np.testing.assert_array_equal(r1.hidden[l], r2.hidden[l])
     np.testing.assert_array_equal(x, r1.hidden[CFG.n_layers - 1])
 
 
