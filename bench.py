@@ -348,7 +348,8 @@ def run_reference(args):
     value = n_rows / (ms / 1000.0)
     cores = blas_threads()
     sample = (f"oracle decoder layer {s} of {wl.name} over the first {n_rows} of "
-              f"{wl.n_tokens[0]} tokens per step (fp32 NumPy)")
+              f"{wl.n_tokens[0]} tokens per step (fp32 NumPy); an upper bound on the oracle's rate "
+              f"over the whole prefix, whose later rows attend to more keys")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
@@ -666,6 +667,45 @@ def run_drift_case(args):
     return 0
 
 
+def run_kl_only(args):
+    """crf_kl with the model's head alone (final norm + LM head GEMV + KL over --decode-rows row
+    pairs): the small profiling case of the head kernels (only the head weights on the device)."""
+    import torch
+    import synth
+    import paper_2609_30884_gb300 as crf
+    from tests.harness import DeviceModel
+
+    wl = workload_of(args)
+    cfg = wl.model
+    rows = max(1, args.decode_rows)
+    ctx = crf.Context(0)
+    dm = DeviceModel(cfg, "cuda:0", layers=[], with_head=True)
+    h_ref = synth.hidden_state(cfg, rows, "kl_ref", device="cuda:0")
+    h_cur = synth.hidden_state(cfg, rows, "kl_cur", device="cuda:0")
+    out = torch.empty(rows, dtype=torch.float32, device="cuda:0")
+    ws = ctx.kl_workspace(rows, cfg.vocab, cfg.hidden)
+    for _ in range(args.warmup):
+        ctx.kl(dm.crf, h_ref, h_cur, out, cfg.vocab, ws)
+    ctx.check()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        ctx.kl(dm.crf, h_ref, h_cur, out, cfg.vocab, ws)
+    b.record()
+    torch.cuda.synchronize()
+    ctx.check()
+    ms = a.elapsed_time(b) / args.steps
+    head_bytes = cfg.vocab * cfg.hidden * 2
+    peaks, src = load_peaks()
+    print(json.dumps({"case": "kl-only", "workload": f"{args.workload}: {wl.name}", "row_pairs": rows,
+                      "ms_per_call": round(ms, 4),
+                      "hbm": {"bytes": head_bytes, "achieved_gbs": round(head_bytes / (ms / 1000.0) / 1e9, 1),
+                              "frac": round(head_bytes / (ms / 1000.0) / 1e9 / peaks["hbm_gbs"], 4),
+                              "peak_source": src}}))
+    ctx.close()
+    return 0
+
+
 def synth_tokens(cfg, n):
     import synth
     return synth.token_ids(cfg, n, device="cuda:0")
@@ -698,13 +738,14 @@ def main():
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--case", default="step",
                     choices=["step", "window-only", "decode-only", "trajectory", "tail-influence", "decode",
-                             "drift"],
+                             "drift", "kl-only"],
                     help="window-only / decode-only: small profiling cases (window layers only / "
                          "the last layer and its first-step row); trajectory: the recovery policy "
                          "over a synthetic continual-adapter trajectory; tail-influence: the offline "
                          "N + 1 hybrid-pass sweep (the update and --versions as for trajectory)")
     ap.add_argument("--versions", type=int, default=32, help="trajectory: adapter updates replayed")
-    ap.add_argument("--decode-rows", type=int, default=8, help="decode: requests generating together")
+    ap.add_argument("--decode-rows", type=int, default=8,
+                    help="decode: requests generating together; kl-only: row pairs")
     ap.add_argument("--decode-steps", type=int, default=32, help="decode: timed generation steps")
     ap.add_argument("--calib-versions", type=int, default=8, help="trajectory: calibration updates")
     ap.add_argument("--update-layer", type=int, default=-1, help="trajectory: updated layer (-1: N // 2)")
@@ -727,6 +768,8 @@ def main():
         return run_decode_case(args)
     if args.case == "drift":
         return run_drift_case(args)
+    if args.case == "kl-only":
+        return run_kl_only(args)
     if args.warmup < 3 and args.impl == "crf":
         args.warmup = 3
     if args.impl == "reference":
@@ -930,7 +973,8 @@ def main():
         line["cpu_baseline"] = {
             "value": args.cpu_rows / secs, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
             "sample": (f"oracle decoder layer {s} over the first {args.cpu_rows} of {n} tokens "
-                       f"(fp32 NumPy), {secs:.1f} s")}
+                       f"(fp32 NumPy), {secs:.1f} s; an upper bound on the oracle's rate over the "
+                       f"whole prefix, whose later rows attend to more keys")}
     if rank == 0:
         print(json.dumps(line))
     ctx.close()

@@ -32,27 +32,31 @@
  *     live in the caller's workspace (see crf_workspace_size).
  *   - `stream` is a cudaStream_t (NULL = legacy default stream). Work is
  *     enqueued on it; results are valid once the stream has synchronised.
- *   - Every argument is validated on the host before anything is launched.
- *     A non-OK status from validation (CRF_EINVAL, CRF_ESHAPE,
- *     CRF_EUNSUPPORTED, CRF_ENOMEM) means nothing was enqueued and nothing
- *     was written. A CRF_ECUDA from a failed launch can leave the call's
- *     earlier kernels enqueued; their outputs are then undefined.
+ *   - Every argument the host can see is validated before anything is
+ *     launched. A non-OK status from that validation (CRF_EINVAL,
+ *     CRF_ESHAPE, CRF_EUNSUPPORTED, CRF_ENOMEM) means nothing was enqueued
+ *     and nothing was written. A CRF_ECUDA from a failed launch can leave the
+ *     call's earlier kernels enqueued; their outputs are then undefined.
  *     crf_last_error() returns a message in either case (thread-local).
+ *   - Page tables live in device memory and the host never reads them: no
+ *     call waits on its stream (crf_check alone synchronises). The first
+ *     kernel of crf_recompute_window and crf_decode_step checks every page
+ *     id (inside [0, num_pages), no page twice across the call's tables);
+ *     a failure makes every later kernel of that call return at once, so the
+ *     call writes nothing outside its workspace (pool pages, checkpoints,
+ *     final rows, logits, tokens), and the next crf_check returns CRF_EINVAL.
  *   - A context is used by one host thread at a time: its device status word
  *     and timing state are shared by its calls. Separate contexts may run
- *     concurrently. For the page
- *     ids, crf_recompute_window and crf_decode_step read each page table back
- *     to the host on `stream` and wait for it. That waits for the work already
- *     on `stream`, and it keeps these two calls out of CUDA graph capture.
+ *     concurrently.
  *   - A kernel that gives up on a bounded internal wait records it in the
  *     context; crf_check() reports it as CRF_ETIMEOUT. An asynchronous CUDA
  *     error is reported as CRF_ECUDA by the next call.
  *   - Ids read from device memory are checked where they are used. A token id
  *     outside [0, vocab) is read as token 0 and recorded; crf_check() then
- *     returns CRF_EINVAL. Page ids are checked on the host before launch; a
- *     library built with CRF_DEBUG defined (libcrf_debug.so) checks them again
- *     at every device-side use, reads or writes page 0 in place of a bad id
- *     and records it the same way.
+ *     returns CRF_EINVAL. A library built with CRF_DEBUG defined
+ *     (libcrf_debug.so) also checks every page id again at each device-side
+ *     use, reads or writes page 0 in place of a bad id and records it the
+ *     same way.
  *   - Tensors are row-major, bf16 unless stated. Weights are [out, in].
  */
 #ifndef CRF_H
@@ -176,9 +180,10 @@ CRF_API crf_status crf_destroy(crf_ctx* ctx);
 CRF_API const char* crf_last_error(void);
 
 /* Synchronise `stream`, then report what the kernels recorded since the last
- * check: a failed device-side bounds check (CRF_EINVAL, which takes
- * precedence) or an abandoned bounded wait (CRF_ETIMEOUT); else a pending
- * CUDA error (CRF_ECUDA). The record is cleared. */
+ * check: a rejected page table or a failed device-side bounds check
+ * (CRF_EINVAL, which takes precedence) or an abandoned bounded wait
+ * (CRF_ETIMEOUT); else a pending CUDA error (CRF_ECUDA). The record is
+ * cleared. */
 CRF_API crf_status crf_check(crf_ctx* ctx, void* stream);
 
 /* Failure-path self-test (no counterpart in the paper): launches one block on

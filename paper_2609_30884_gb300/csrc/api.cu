@@ -44,12 +44,12 @@ namespace {
 
 enum ProfKind : int {
   kPQkv, kPO, kPGateUp, kPDown, kPLoraDown, kPAttn, kPNorm, kPEmbed, kPRope, kPCopy,
-  kPDecode, kPLmHead, kPKl, kPDrift, kPNumKinds
+  kPDecode, kPLmHead, kPKl, kPDrift, kPCheck, kPNumKinds
 };
 const char* const kProfNames[kPNumKinds] = {
     "gemm_qkv_rope_paged", "gemm_o_resid", "gemm_gateup_swiglu", "gemm_down_resid",
     "gemm_lora_down", "attn_prefill_paged", "rmsnorm", "embed_gather", "rope_table", "row_copy",
-    "tail_decode", "lm_head", "kl_reduce", "drift_gram"};
+    "tail_decode", "lm_head", "kl_reduce", "drift_gram", "page_check"};
 
 // Brackets the launches issued in its lifetime with two events on `st` when
 // profiling is on; `kernels` is how many kernels those launches are.
@@ -168,6 +168,8 @@ struct Plan {
   int splits = 1;
   size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_bx, off_rope;
   size_t off_dx0, off_dec;  // decode: bf16 starting rows, fp32 scratch
+  size_t off_abort, off_ptab;  // the call's abort word; the page-check table (ptab_slots ints)
+  uint32_t ptab_slots = 2;
   size_t dec_bytes;
   size_t total;
 };
@@ -185,6 +187,13 @@ int module_rows_total(const Dims& D) {
 
 // decode attention partials: one per chunk of the longest prefix
 int dec_splits(int max_n) { return decode_attention_splits(max_n); }
+
+// Slots of the page-check table for `ids` page ids: a power of two, at least twice the ids.
+uint32_t ptab_slots_for(long ids) {
+  uint32_t s = 2;
+  while (s < 2 * ids) s <<= 1;
+  return s;
+}
 
 Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   Plan p;
@@ -216,6 +225,11 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_bx = take(static_cast<size_t>(module_rows_total(D)) * kBxCols * 2);
   p.off_rope = take(static_cast<size_t>(p.max_n) * (D.d / 2) * sizeof(float2));
   p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
+  long ids = 0;
+  for (int i = 0; i < n_req; ++i) ids += (reqs[i].n_tokens + kPage - 1) / kPage;
+  p.ptab_slots = ptab_slots_for(ids);
+  p.off_abort = take(sizeof(int));
+  p.off_ptab = take(static_cast<size_t>(p.ptab_slots) * sizeof(int));
   p.splits = dec_splits(p.max_n);
   // decode scratch per row, fp32: x, xn, x1, q, k, v, o, xa (3 slots), gu, m, attention partials
   const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 3 * kRankPad + 3 * D.f) * 4 +
@@ -264,6 +278,7 @@ struct LayerCtx {
   uint8_t* ws;
   const Plan* plan;
   float scale;
+  const int* abort;  // the call's abort word (set by the page-table check)
 };
 
 bool adapted(const crf_adapter* a, int m) { return (a->dims.module_mask >> m) & 1u; }
@@ -291,6 +306,7 @@ cudaError_t lora_down(const LayerCtx& c, int l, const void* X, int M, int K, con
   g.out = XA;
   g.ldo = kXaCols;
   g.status = c.ctx->status_dev;
+  g.abort = c.abort;
   return launch_gemm(g, nm * kRankPad, c.ctx->num_sms, c.st);
 }
 
@@ -379,6 +395,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.vpages = c.pool->v_pages[l];
     g.req = rt;
     g.status = c.ctx->status_dev;
+    g.abort = c.abort;
     ProfScope ps(c.ctx, kPQkv, c.st);
     CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
   }
@@ -397,6 +414,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     a.head_dim = D.d;
     a.req = rt;
     a.status = c.ctx->status_dev;
+    a.abort = c.abort;
     ProfScope ps(c.ctx, kPAttn, c.st);
     CRF_CUDA(launch_attention_tc(a, c.pool->num_pages, M, c.st));
   }
@@ -435,6 +453,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.resid = resid;
     g.ld_resid = D.h;
     g.status = c.ctx->status_dev;
+    g.abort = c.abort;
     ProfScope ps(c.ctx, m == CRF_MOD_O ? kPO : kPDown, c.st);
     return launch_gemm(g, 256, c.ctx->num_sms, c.st);
   };
@@ -479,6 +498,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.out = MLP;
     g.ldo = D.f;
     g.status = c.ctx->status_dev;
+    g.abort = c.abort;
     ProfScope ps(c.ctx, kPGateUp, c.st);
     CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
   }
@@ -580,6 +600,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
     }
     for (int r0 = 0; r0 < nr; r0 += 8) {
       GemvDesc g{};
+      g.abort = c.abort;
       g.nseg = nm;
       g.in_dim = in_dim;
       g.x = in + static_cast<size_t>(r0) * in_dim;
@@ -646,6 +667,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
       a.n_kv_heads = D.hkv;
       a.head_dim = D.d;
       a.splits = p.splits;
+      a.abort = c.abort;
       CRF_CUDA(launch_decode_attention(a, c.pool->num_pages, c.ctx->num_sms, c.ctx->status_dev, c.st));
       if (opt.write_kv) {
         RowPages pg{};
@@ -655,7 +677,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
         }
         pg.num_pages = c.pool->num_pages;
         CRF_CUDA(launch_kv_write_rows(k, v, c.pool->k_pages[l], c.pool->v_pages[l], pg, nr, D.hkv, D.d,
-                                      c.ctx->status_dev, c.st));
+                                      c.ctx->status_dev, c.abort, c.st));
       }
       CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
       CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
@@ -667,27 +689,40 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
   for (int i = 0; i < R; ++i)
     if (rows[i].out)
       CRF_CUDA(launch_f32_to_bf16(x + i * static_cast<size_t>(D.h),
-                                  static_cast<__nv_bfloat16*>(rows[i].out), D.h, c.st));
+                                  static_cast<__nv_bfloat16*>(rows[i].out), D.h, c.st, c.abort));
   return CRF_OK;
 }
 
-// Page ids are read back and checked on the host before every launch. Only a CRF_DEBUG build run
-// with CRF_DEBUG_DEVICE_CHECKS_ONLY=1 skips that read, so that its device-side checks alone
-// stand between a bad id and the pool (the way its tests exercise them).
-bool host_page_check() {
+// Page ids are checked on the device by the first kernel of every call that uses them. Only a
+// CRF_DEBUG build run with CRF_DEBUG_DEVICE_CHECKS_ONLY=1 skips that check, so that the per-use
+// checks of that build alone stand between a bad id and the pool (the way its tests exercise them).
+bool device_page_check() {
   if (!kDebugBuild) return true;
   const char* e = std::getenv("CRF_DEBUG_DEVICE_CHECKS_ONLY");
   return !(e && e[0] == '1');
 }
 
+// Opens a call on `st`: clears the call's abort word and checks every page id of the listed
+// tables (in [0, num_pages), no page twice). Enqueued work only: the host does not wait.
+crf_status open_call(crf_ctx* ctx, const PageCheck& pc, int num_pages, uint8_t* ws, size_t off_abort,
+                     size_t off_ptab, uint32_t ptab_slots, cudaStream_t st) {
+  int* abort = reinterpret_cast<int*>(ws + off_abort);
+  ProfScope ps(ctx, kPCheck, st, device_page_check() ? 1 : 0);
+  CRF_CUDA(cudaMemsetAsync(abort, 0, sizeof(int), st));
+  if (!device_page_check()) return CRF_OK;
+  int* table = reinterpret_cast<int*>(ws + off_ptab);
+  CRF_CUDA(cudaMemsetAsync(table, 0xff, static_cast<size_t>(ptab_slots) * sizeof(int), st));
+  CRF_CUDA(launch_validate_pages(pc, num_pages, table, ptab_slots - 1, abort, ctx->status_dev, st));
+  return CRF_OK;
+}
+
 crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const crf_adapter* cur,
                              const crf_kv_pool* pool, const crf_request* reqs, int n_req,
-                             const Dims& D, cudaStream_t st) {
+                             const Dims& D) {
   if (n_req < 1 || n_req > CRF_MAX_REQUESTS)
     return fail(CRF_EINVAL, "n_req %d outside [1, %d]", n_req, CRF_MAX_REQUESTS);
   if (!pool || !pool->k_pages || !pool->v_pages || pool->num_pages < 1)
     return fail(CRF_EINVAL, "kv pool missing");
-  std::vector<char> seen(static_cast<size_t>(pool->num_pages), 0);
   for (int i = 0; i < n_req; ++i) {
     const crf_request& r = reqs[i];
     if (r.n_tokens < 1) return fail(CRF_EINVAL, "request %d: n_tokens must be >= 1", i);
@@ -713,18 +748,6 @@ crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const c
       if (!pool->k_pages[l] || !pool->v_pages[l] || !aligned16(pool->k_pages[l]) ||
           !aligned16(pool->v_pages[l]))
         return fail(CRF_EINVAL, "kv pool layer %d null or misaligned", l);
-    // page ids: in range and not shared between requests
-    if (!host_page_check()) continue;
-    const int np = (r.n_tokens + kPage - 1) / kPage;
-    std::vector<int32_t> pt(np);
-    CRF_CUDA(cudaMemcpyAsync(pt.data(), r.page_table, np * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
-    CRF_CUDA(cudaStreamSynchronize(st));
-    for (int j = 0; j < np; ++j) {
-      if (pt[j] < 0 || pt[j] >= pool->num_pages)
-        return fail(CRF_EINVAL, "request %d: page id %d out of range [0,%d)", i, pt[j], pool->num_pages);
-      if (seen[pt[j]]) return fail(CRF_EINVAL, "request %d: page %d used twice", i, pt[j]);
-      seen[pt[j]] = 1;
-    }
   }
   (void)ctx;
   return CRF_OK;
@@ -735,7 +758,7 @@ crf_status validate_requests(const crf_ctx* ctx, const crf_model* model, const c
 struct StepPlan {
   Plan p;
   size_t off_angles, off_norm, off_logits, total;
-};
+};  // p.off_abort / p.off_ptab / p.ptab_slots: the page check of the rows' tables
 
 StepPlan make_step_plan(const Dims& D, const crf_decode_row* rows, int n) {
   StepPlan sp;
@@ -758,30 +781,22 @@ StepPlan make_step_plan(const Dims& D, const crf_decode_row* rows, int n) {
   sp.off_angles = take(static_cast<size_t>(n) * (D.d / 2) * sizeof(float2));
   sp.off_norm = take(static_cast<size_t>(n) * D.h * 4);
   sp.off_logits = take(static_cast<size_t>(n) * D.V * 4);
+  long ids = 0;
+  for (int i = 0; i < n; ++i) ids += rows[i].pos / kPage + 1;
+  p.ptab_slots = ptab_slots_for(ids);
+  p.off_abort = take(sizeof(int));
+  p.off_ptab = take(static_cast<size_t>(p.ptab_slots) * sizeof(int));
   sp.total = p.total = o;
   return sp;
 }
 
-crf_status validate_decode_rows(const crf_kv_pool* pool, const crf_decode_row* rows, int n,
-                                cudaStream_t st) {
+crf_status validate_decode_rows(const crf_kv_pool* pool, const crf_decode_row* rows, int n) {
   if (n < 1 || n > CRF_MAX_REQUESTS) return fail(CRF_EINVAL, "n_rows %d outside [1, %d]", n, CRF_MAX_REQUESTS);
   if (!pool || !pool->k_pages || !pool->v_pages || pool->num_pages < 1) return fail(CRF_EINVAL, "kv pool missing");
-  std::vector<char> seen(static_cast<size_t>(pool->num_pages), 0);
   for (int i = 0; i < n; ++i) {
     const crf_decode_row& r = rows[i];
     if (r.pos < 0) return fail(CRF_EINVAL, "row %d: negative position", i);
     if (!r.page_table || !r.token) return fail(CRF_EINVAL, "row %d: page_table or token is null", i);
-    if (!host_page_check()) continue;
-    const int np = r.pos / kPage + 1;
-    std::vector<int32_t> pt(np);
-    CRF_CUDA(cudaMemcpyAsync(pt.data(), r.page_table, np * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
-    CRF_CUDA(cudaStreamSynchronize(st));
-    for (int j = 0; j < np; ++j) {
-      if (pt[j] < 0 || pt[j] >= pool->num_pages)
-        return fail(CRF_EINVAL, "row %d: page id %d out of range [0,%d)", i, pt[j], pool->num_pages);
-      if (seen[pt[j]]) return fail(CRF_EINVAL, "row %d: page %d used twice", i, pt[j]);
-      seen[pt[j]] = 1;
-    }
   }
   return CRF_OK;
 }
@@ -841,6 +856,9 @@ crf_status crf_check(crf_ctx* ctx, void* stream) {
   CRF_CUDA(cudaMemcpy(&status, ctx->status_dev, sizeof(int), cudaMemcpyDeviceToHost));
   if (status) {
     CRF_CUDA(cudaMemset(ctx->status_dev, 0, sizeof(int)));
+    if (status & kStatusPages)
+      return fail(CRF_EINVAL, "a page table held an id outside the pool or a page twice; that call wrote "
+                  "nothing outside its workspace (status 0x%x)", status);
     if (status & kStatusBounds)
       return fail(CRF_EINVAL, "a device-side bounds check failed: a token id outside the vocabulary%s "
                   "(status 0x%x)", kDebugBuild ? " or a page id outside the pool" : "", status);
@@ -885,7 +903,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
   CRF_CUDA(cudaSetDevice(ctx->device));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const Dims D = dims_of(model->dims);
-  s = validate_requests(ctx, model, cur, pool, reqs, n_req, D, st);
+  s = validate_requests(ctx, model, cur, pool, reqs, n_req, D);
   if (s != CRF_OK) return s;
   const Plan plan = make_plan(D, reqs, n_req);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255))
@@ -904,6 +922,18 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
   c.ws = ws;
   c.plan = &plan;
   c.scale = cur->dims.alpha / cur->dims.rank;
+  c.abort = reinterpret_cast<const int*>(ws + plan.off_abort);
+  {
+    PageCheck pc{};
+    pc.n = n_req;
+    pc.first[0] = 0;
+    for (int i = 0; i < n_req; ++i) {
+      pc.pt[i] = reqs[i].page_table;
+      pc.first[i + 1] = pc.first[i] + (reqs[i].n_tokens + kPage - 1) / kPage;
+    }
+    s = open_call(ctx, pc, pool->num_pages, ws, plan.off_abort, plan.off_ptab, plan.ptab_slots, st);
+    if (s != CRF_OK) return s;
+  }
 
   {
     ProfScope ps(ctx, kPRope, st);
@@ -994,11 +1024,12 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
     if (s != CRF_OK) return s;
     for (int k = 0; k < rt.n; ++k) {
       const int i = act[k];
-      ProfScope ps(ctx, kPCopy, st, 0);
+      const bool copy_out = !single && reqs[i].hidden_out;
+      ProfScope ps(ctx, kPCopy, st, copy_out ? 1 : 0);
       curp[i] = X_out + static_cast<size_t>(rt.row0[k]) * D.h;
-      if (!single && reqs[i].hidden_out)
-        CRF_CUDA(cudaMemcpyAsync(reqs[i].hidden_out[l - reqs[i].s], curp[i],
-                                 reqs[i].n_tokens * row_bytes, cudaMemcpyDeviceToDevice, st));
+      if (copy_out)
+        CRF_CUDA(launch_copy_bf16(static_cast<__nv_bfloat16*>(reqs[i].hidden_out[l - reqs[i].s]), curp[i],
+                                  static_cast<size_t>(reqs[i].n_tokens) * D.h, c.abort, st));
       if (l == reqs[i].e - 1 && reqs[i].final_hidden_out)
         CRF_CUDA(cudaMemcpyAsync(dx0 + static_cast<size_t>(i) * D.h,
                                  curp[i] + static_cast<size_t>(reqs[i].n_tokens - 1) * D.h, row_bytes,
@@ -1025,8 +1056,8 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
       }
     }
     if (r.e == D.N) {
-      ProfScope ps(ctx, kPCopy, st, 0);
-      CRF_CUDA(cudaMemcpyAsync(r.final_hidden_out, start, row_bytes, cudaMemcpyDeviceToDevice, st));
+      ProfScope ps(ctx, kPCopy, st, 1);
+      CRF_CUDA(launch_copy_bf16(static_cast<__nv_bfloat16*>(r.final_hidden_out), start, D.h, c.abort, st));
     } else {
       dec.push_back({r.e, r.n_tokens - 1, r.page_table, start, r.final_hidden_out});
     }
@@ -1075,7 +1106,7 @@ crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const crf_adapt
     if (!pool || !pool->k_pages || !pool->v_pages || !pool->k_pages[l] || !pool->v_pages[l] ||
         !aligned16(pool->k_pages[l]) || !aligned16(pool->v_pages[l]))
       return fail(CRF_EINVAL, "kv pool layer %d null or misaligned", l);
-  s = validate_decode_rows(pool, rows, n_rows, st);
+  s = validate_decode_rows(pool, rows, n_rows);
   if (s != CRF_OK) return s;
   const StepPlan sp = make_step_plan(D, rows, n_rows);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255))
@@ -1093,6 +1124,18 @@ crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const crf_adapt
   c.ws = ws;
   c.plan = &sp.p;
   c.scale = cur->dims.alpha / cur->dims.rank;
+  c.abort = reinterpret_cast<const int*>(ws + sp.p.off_abort);
+  {
+    PageCheck pc{};
+    pc.n = n_rows;
+    pc.first[0] = 0;
+    for (int i = 0; i < n_rows; ++i) {
+      pc.pt[i] = rows[i].page_table;
+      pc.first[i + 1] = pc.first[i] + rows[i].pos / kPage + 1;
+    }
+    s = open_call(ctx, pc, pool->num_pages, ws, sp.p.off_abort, sp.p.off_ptab, sp.p.ptab_slots, st);
+    if (s != CRF_OK) return s;
+  }
   RowPositions rp{};
   std::vector<DecodeRow> dec;
   for (int i = 0; i < n_rows; ++i) {
@@ -1122,8 +1165,8 @@ crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const crf_adapt
     ProfScope ps(ctx, kPLmHead, st, 3);
     CRF_CUDA(launch_rmsnorm_f32(x, static_cast<const __nv_bfloat16*>(model->final_norm), hn, n_rows, D.h, D.eps, st));
     CRF_CUDA(launch_lm_head(static_cast<const __nv_bfloat16*>(model->lm_head), hn, n_rows, D.V, D.h, z,
-                            ctx->num_sms, st));
-    CRF_CUDA(launch_argmax_rows(z, n_rows, D.V, next_tokens, st));
+                            ctx->num_sms, st, c.abort));
+    CRF_CUDA(launch_argmax_rows(z, n_rows, D.V, next_tokens, st, c.abort));
   }
   return CRF_OK;
 }

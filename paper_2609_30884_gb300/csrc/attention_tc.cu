@@ -69,6 +69,7 @@ struct AttnTcArgs {
   int total_items;
   ReqTable req;
   int* status;
+  const int* abort;
 };
 
 struct AttnWork {
@@ -198,7 +199,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1) attn_tc_kernel(const __grid_c
   __shared__ volatile int abort_flag;
 
   AttnWork w;
-  if (!attn_work(a, blockIdx.x, w)) return;
+  if (call_aborted(a.abort) || !attn_work(a, blockIdx.x, w)) return;
   const int n = a.req.len[w.req];
   const int row0 = a.req.row0[w.req];
   const int32_t* pt = a.req.page_table[w.req];
@@ -527,6 +528,7 @@ cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows
   a.group = d.n_q_heads / d.n_kv_heads;
   a.req = d.req;
   a.status = d.status;
+  a.abort = d.abort;
   a.total_items = 0;
   for (int i = 0; i < d.req.n; ++i)
     a.total_items += ((d.req.len[i] + 2 * kM - 1) / (2 * kM)) * d.n_q_heads;

@@ -11,7 +11,13 @@
 namespace crf {
 
 // Status bits a kernel may set in the context's device status word.
-enum : int { kStatusTimeout = 1, kStatusBounds = 2 };
+enum : int { kStatusTimeout = 1, kStatusBounds = 2, kStatusPages = 4 };
+
+// The per-call abort word: set by the page-table check that opens a call when a page id is out of
+// the pool or a page appears twice. Every later kernel of the call that reads pages or writes
+// memory outside the call's workspace tests it first and returns at once, so a rejected call
+// writes nothing outside its workspace. Null where a launch has no such word.
+__device__ __forceinline__ bool call_aborted(const int* abort) { return abort != nullptr && *abort != 0; }
 
 #ifdef CRF_DEBUG
 constexpr bool kDebugBuild = true;
@@ -33,9 +39,10 @@ __device__ __forceinline__ int checked_token(int tok, int vocab, int* status) {
 // Device-side bounds check on a page id read from a page table. In a build
 // with CRF_DEBUG defined, an id outside [0, num_pages) sets kStatusBounds and
 // comes back as page 0, so the copy that uses it stays inside the pool and
-// every barrier still completes; the host reports the bit. The host already
-// validates every page table before launch, so in the release build the
-// check compiles away and the id is returned unchanged.
+// every barrier still completes; the host reports the bit. In every build the
+// page-table check that opens the call has already rejected bad ids (the call's
+// abort word), so in the release build this check compiles away and the id is
+// returned unchanged.
 __device__ __forceinline__ int checked_page(int page, int num_pages, int* status) {
 #ifdef CRF_DEBUG
   if (page < 0 || page >= num_pages) {

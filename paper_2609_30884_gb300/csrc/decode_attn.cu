@@ -71,6 +71,7 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
   constexpr int QHALF = 16 * 128;        // one 64-column half of the 16-row Q tile
   const DecodeAttnDesc& p = a.d;
   griddep_begin();  // q, k, v of the rows come from the kernel before
+  if (call_aborted(p.abort)) return;
   // block -> (row, kv head, its chunks c_beg .. c_end - 1, partial slot)
   int r = -1, g = 0, slot = 0, c_beg = 0, c_end = 0;
   {

@@ -36,7 +36,7 @@ namespace {
 
 constexpr int kDtThreads = 256;
 constexpr int kDtRows = 128;   // long-dimension rows per step: 8 warps x 16
-constexpr int kDtStages = 3;
+constexpr int kDtStages = 4;   // three steps in flight while one is multiplied
 constexpr int kDtCtasPerSm = 3;
 constexpr int kDtMaxItems = 224;
 constexpr int kDtMaxSegs = 2 * kDtMaxItems;
@@ -48,8 +48,9 @@ struct DriftTcArgs {
   int n_items, n_segs, total_steps, grid, rank;
 };
 
-template <int RP>
+template <int R>
 struct DtShape {
+  static constexpr int RP = R < 8 ? 8 : R;                      // features per part (zero padded)
   static constexpr int kBStride = RP == 16 ? 48 : 16;          // bytes per B row in a stage
   static constexpr int kBVersion = kDtRows * kBStride;          // one version of the B side
   static constexpr int kAVersion = RP * kDtAStride;             // one version of the A side
@@ -57,16 +58,23 @@ struct DtShape {
   static constexpr int kBlocks = RP == 16 ? 3 : 2;              // 16-feature blocks of [hi|lo|base]
   static constexpr int kPairs = kBlocks * (kBlocks + 1) / 2;    // block-upper triangle
   static constexpr int kSlotFloats = kPairs * 256;
+  // copies per step and version: B side in chunks of min(16, 2R) bytes per row; A side in 16-byte
+  // chunks of R rows
+  static constexpr int kBChunkBytes = 2 * R < 16 ? 2 * R : 16;
+  static constexpr int kBChunksPerRow = 2 * R / kBChunkBytes;
+  static constexpr int kBCopies = 2 * kDtRows * kBChunksPerRow;
+  static constexpr int kACopies = 2 * R * (kDtRows / 8);
+  static constexpr int kBPerThread = (kBCopies + kDtThreads - 1) / kDtThreads;
+  static constexpr int kAPerThread = (kACopies + kDtThreads - 1) / kDtThreads;
 };
 
-__device__ __forceinline__ void cp_async(uint32_t dst, const void* src, int bytes, bool valid) {
-  // bytes is 8 or 16; an invalid source copies nothing and fills the destination with zeros
-  if (bytes == 16)
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
-                 : "memory");
-  else
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(valid ? 8 : 0)
-                 : "memory");
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async8(uint32_t dst, const void* src, bool valid) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(valid ? 8 : 0)
+               : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
@@ -79,71 +87,104 @@ __device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t&
   asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
 }
 
-// (hi, lo) of the exact fp32 differences of two bf16 pairs, and the pairs themselves
+// (hi, lo) of the exact fp32 differences of two bf16 pairs
 __device__ __forceinline__ void split_diff(uint32_t a, uint32_t b, uint32_t& hi, uint32_t& lo) {
   const float d0 = bf16_lo(a) - bf16_lo(b), d1 = bf16_hi(a) - bf16_hi(b);
   hi = pack_bf16(d0, d1);
   lo = pack_bf16(d0 - bf16_lo(hi), d1 - bf16_hi(hi));
 }
 
-// Step x of the grid-wide sequence: its segment, side and first long-dimension row.
-struct StepRef {
-  const DriftItem* it;
-  int side, row0, len;
+// This thread's copies of a step, fixed for the whole kernel: for copy u, the version, the row
+// (B side: long-dimension row; A side: rank row k), the chunk and the stage offset.
+template <int R>
+struct CopyPlan {
+  using S = DtShape<R>;
+  int b_row[S::kBPerThread], b_src[S::kBPerThread];  // b_src: element offset within the row block
+  uint32_t b_dst[S::kBPerThread];
+  int a_col[S::kAPerThread], a_k[S::kAPerThread];
+  uint32_t a_dst[S::kAPerThread];
+  bool b_v1[S::kBPerThread], a_v1[S::kAPerThread], b_on[S::kBPerThread], a_on[S::kAPerThread];
+
+  __device__ __forceinline__ void init(int tid) {
+#pragma unroll
+    for (int u = 0; u < S::kBPerThread; ++u) {
+      const int i = tid + u * kDtThreads;
+      const int v = i / (kDtRows * S::kBChunksPerRow), rem = i % (kDtRows * S::kBChunksPerRow);
+      const int row = rem / S::kBChunksPerRow, ch = rem % S::kBChunksPerRow;
+      b_on[u] = i < S::kBCopies;
+      b_v1[u] = v == 0;
+      b_row[u] = row;
+      b_src[u] = row * R + ch * (S::kBChunkBytes / 2);
+      b_dst[u] = v * S::kBVersion + row * S::kBStride + ch * 16;
+    }
+#pragma unroll
+    for (int u = 0; u < S::kAPerThread; ++u) {
+      const int i = tid + u * kDtThreads;
+      const int v = i / (R * (kDtRows / 8)), rem = i % (R * (kDtRows / 8));
+      const int k = rem / (kDtRows / 8), ch = rem % (kDtRows / 8);
+      a_on[u] = i < S::kACopies;
+      a_v1[u] = v == 0;
+      a_k[u] = k;
+      a_col[u] = ch * 8;
+      a_dst[u] = v * S::kAVersion + k * kDtAStride + ch * 16;
+    }
+  }
 };
 
-__device__ __forceinline__ int seg_of(const DriftTcArgs& a, int x, int seg) {
-  while (seg + 1 < a.n_segs && x >= a.seg_step0[seg + 1]) ++seg;
-  return seg;
-}
+// The item a run of steps belongs to, cached while the run stays in one segment.
+struct SegCache {
+  int seg = -1, side = 0, len = 0, step0 = 0, next0 = 0;
+  const __nv_bfloat16 *p1 = nullptr, *p0 = nullptr;  // version 1 / version 0 of this side
 
-__device__ __forceinline__ StepRef step_ref(const DriftTcArgs& a, int x, int seg) {
-  StepRef s;
-  s.it = &a.items[seg >> 1];
-  s.side = seg & 1;
-  s.row0 = (x - a.seg_step0[seg]) * kDtRows;
-  s.len = s.side == 0 ? s.it->out_dim : s.it->in_dim;
-  return s;
-}
+  __device__ __forceinline__ void at(const DriftTcArgs& a, int x) {
+    if (seg >= 0 && x < next0) return;
+    int s = seg < 0 ? 0 : seg;
+    while (s + 1 < a.n_segs && x >= a.seg_step0[s + 1]) ++s;
+    seg = s;
+    side = s & 1;
+    const DriftItem& it = a.items[s >> 1];
+    len = side == 0 ? it.out_dim : it.in_dim;
+    step0 = a.seg_step0[s];
+    next0 = a.seg_step0[s + 1];
+    p1 = side == 0 ? it.B1 : it.A1;
+    p0 = side == 0 ? it.B0 : it.A0;
+  }
+};
 
-// Issue the copies of one step into a stage: version 1 (current) then version 0 (anchor).
-template <int RP>
-__device__ __forceinline__ void load_step(const StepRef& s, int rank, uint32_t stage) {
-  using S = DtShape<RP>;
-  const int tid = threadIdx.x;
-  if (s.side == 0) {
-    // B [out, r]: row o holds r contiguous bf16; chunks of 16 bytes (8 bytes when r = 4)
-    const int cbytes = rank >= 8 ? 16 : 8;
-    const int cpr = rank * 2 / cbytes;  // chunks per row
-    const int total = 2 * kDtRows * cpr;
-    for (int i = tid; i < total; i += kDtThreads) {
-      const int v = i / (kDtRows * cpr), rem = i - v * kDtRows * cpr;
-      const int row = rem / cpr, ch = rem - row * cpr;
-      const int o = s.row0 + row;
-      const bool ok = o < s.len;
-      const __nv_bfloat16* base = v == 0 ? s.it->B1 : s.it->B0;
-      const __nv_bfloat16* src = base + (ok ? static_cast<size_t>(o) * rank + ch * (cbytes / 2) : 0);
-      cp_async(stage + v * S::kBVersion + row * S::kBStride + ch * 16, src, cbytes, ok);
+// Issue the copies of step x (version 1 then version 0) into a stage.
+template <int R>
+__device__ __forceinline__ void load_step(const CopyPlan<R>& cp, const SegCache& sc, int x, uint32_t stage) {
+  using S = DtShape<R>;
+  const int row0 = (x - sc.step0) * kDtRows;
+  if (sc.side == 0) {
+    const size_t blk = static_cast<size_t>(row0) * R;
+#pragma unroll
+    for (int u = 0; u < S::kBPerThread; ++u) {
+      if (!cp.b_on[u]) continue;
+      const bool ok = row0 + cp.b_row[u] < sc.len;
+      const __nv_bfloat16* src = (cp.b_v1[u] ? sc.p1 : sc.p0) + (ok ? blk + cp.b_src[u] : 0);
+      if constexpr (S::kBChunkBytes == 16)
+        cp_async16(stage + cp.b_dst[u], src, ok);
+      else
+        cp_async8(stage + cp.b_dst[u], src, ok);
     }
   } else {
-    // A [r, in]: rows k < r, 128 columns from row0 in 16-byte chunks (in % 8 == 0)
-    const int total = 2 * rank * (kDtRows / 8);
-    for (int i = tid; i < total; i += kDtThreads) {
-      const int v = i / (rank * (kDtRows / 8)), rem = i - v * rank * (kDtRows / 8);
-      const int k = rem / (kDtRows / 8), ch = rem - k * (kDtRows / 8);
-      const int c = s.row0 + ch * 8;
-      const bool ok = c < s.len;
-      const __nv_bfloat16* base = v == 0 ? s.it->A1 : s.it->A0;
-      const __nv_bfloat16* src = base + (ok ? static_cast<size_t>(k) * s.len + c : 0);
-      cp_async(stage + v * S::kAVersion + k * kDtAStride + ch * 16, src, 16, ok);
+#pragma unroll
+    for (int u = 0; u < S::kAPerThread; ++u) {
+      if (!cp.a_on[u]) continue;
+      const int c = row0 + cp.a_col[u];
+      const bool ok = c < sc.len;  // the input width is a multiple of 8: a chunk is in or out
+      const __nv_bfloat16* src = (cp.a_v1[u] ? sc.p1 : sc.p0) + (ok ? static_cast<size_t>(cp.a_k[u]) * sc.len + c : 0);
+      cp_async16(stage + cp.a_dst[u], src, ok);
     }
   }
 }
 
 // This warp's 16-row slice of a staged step into its Gram accumulators.
-template <int RP>
-__device__ __forceinline__ void mma_step(int side, uint32_t stage, float (&acc)[DtShape<RP>::kPairs][2][4]) {
-  using S = DtShape<RP>;
+template <int R>
+__device__ __forceinline__ void mma_step(int side, uint32_t stage, float (&acc)[DtShape<R>::kPairs][2][4]) {
+  using S = DtShape<R>;
+  constexpr int RP = S::RP;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m = lane >> 3, i = lane & 7;
   uint32_t f1[4], f0[4];  // fragments of version 1 and version 0: {m0, m1, m2, m3} (RP = 8: m0, m2)
@@ -198,12 +239,12 @@ __device__ __forceinline__ void mma_step(int side, uint32_t stage, float (&acc)[
     }
 }
 
-template <int RP>
+template <int R>
 __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
     drift_tc_kernel(const __grid_constant__ DriftTcArgs a, float* __restrict__ slots) {
-  using S = DtShape<RP>;
+  using S = DtShape<R>;
   extern __shared__ __align__(128) uint8_t dt_smem[];
-  float* red = reinterpret_cast<float*>(dt_smem + kDtStages * S::kStage);  // [32][kPairs * 8]
+  float* red = reinterpret_cast<float*>(dt_smem + kDtStages * S::kStage);  // [kPairs * 8][32]
   const uint32_t stage0 = smem_u32(dt_smem);
   const int b = blockIdx.x;
   const int x0 = static_cast<int>((static_cast<long long>(b) * a.total_steps) / a.grid);
@@ -214,6 +255,8 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
     reinterpret_cast<uint4*>(dt_smem)[i] = make_uint4(0u, 0u, 0u, 0u);
   __syncthreads();
 
+  CopyPlan<R> cp;
+  cp.init(threadIdx.x);
   float acc[S::kPairs][2][4];
 #pragma unroll
   for (int p = 0; p < S::kPairs; ++p)
@@ -222,29 +265,26 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
 #pragma unroll
       for (int v = 0; v < 4; ++v) acc[p][h][v] = 0.f;
 
-  int lseg = seg_of(a, x0, 0);  // segment of the next step to load
+  SegCache lc, sc;  // the next step to load, the step multiplied
   int lx = x0;
   auto issue = [&]() {
     if (lx < x1) {
-      lseg = seg_of(a, lx, lseg);
-      load_step<RP>(step_ref(a, lx, lseg), a.rank, stage0 + ((lx - x0) % kDtStages) * S::kStage);
+      lc.at(a, lx);
+      load_step<R>(cp, lc, lx, stage0 + ((lx - x0) % kDtStages) * S::kStage);
     }
     cp_async_commit();  // empty groups keep the count uniform
     ++lx;
   };
-  issue();
-  issue();
-  int seg = seg_of(a, x0, 0);
+  for (int k = 0; k < kDtStages - 1; ++k) issue();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int x = x0; x < x1; ++x) {
-    issue();
-    cp_async_wait<kDtStages - 1>();
-    __syncthreads();
-    seg = seg_of(a, x, seg);
-    mma_step<RP>(seg & 1, stage0 + ((x - x0) % kDtStages) * S::kStage, acc);
-    const bool flush = x + 1 == x1 || x + 1 >= a.seg_step0[seg + 1];
-    if (flush) {
+    cp_async_wait<kDtStages - 2>();  // this thread's copies of step x have landed
+    __syncthreads();                 // everyone's have, and step x - 1's stage is free again
+    issue();                         // step x + kDtStages - 1 into that stage
+    sc.at(a, x);
+    mma_step<R>(sc.side, stage0 + ((x - x0) % kDtStages) * S::kStage, acc);
+    if (x + 1 == x1 || x + 1 >= sc.next0) {
       // the warps' partial Grams summed in warp order, then written as one slot
-      const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
       for (int w = 0; w < kDtThreads / 32; ++w) {
         if (warp == w) {
 #pragma unroll
@@ -253,18 +293,18 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
             for (int h = 0; h < 2; ++h)
 #pragma unroll
               for (int v = 0; v < 4; ++v) {
-                float* r = red + lane * (S::kPairs * 8) + p * 8 + h * 4 + v;
+                float* r = red + (p * 8 + h * 4 + v) * 32 + lane;
                 *r = (w == 0 ? 0.f : *r) + acc[p][h][v];
               }
         }
         __syncthreads();
       }
-      float* out = slots + static_cast<size_t>(b + seg) * S::kSlotFloats;
+      float* out = slots + static_cast<size_t>(b + sc.seg) * S::kSlotFloats;
       for (int e = threadIdx.x; e < S::kSlotFloats; e += kDtThreads) {
         const int p = e >> 8, rr = (e >> 4) & 15, cc = e & 15;
         const int ln = (rr & 7) * 4 + ((cc & 7) >> 1);
         const int v = (rr >> 3) * 2 + (cc & 1);
-        out[e] = red[ln * (S::kPairs * 8) + p * 8 + (cc >> 3) * 4 + v];
+        out[e] = red[(p * 8 + (cc >> 3) * 4 + v) * 32 + ln];
       }
 #pragma unroll
       for (int p = 0; p < S::kPairs; ++p)
@@ -272,19 +312,18 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
         for (int h = 0; h < 2; ++h)
 #pragma unroll
           for (int v = 0; v < 4; ++v) acc[p][h][v] = 0.f;
+      __syncthreads();  // `red` is read before the next flush overwrites it
     }
-    __syncthreads();  // the stage read here is refilled two steps on; `red` is reused at the next flush
   }
   cp_async_wait<0>();
 }
 
-// One block per item: the segment's slots summed in CTA order, then tr(GB GA) and the
-// parameter distance from the [hi | lo | base] Grams, in fp64.
-template <int RP>
+template <int R>
 __global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_constant__ DriftTcArgs a,
                                                              const float* __restrict__ slots,
                                                              float* __restrict__ out_sq) {
-  using S = DtShape<RP>;
+  using S = DtShape<R>;
+  constexpr int RP = S::RP;
   __shared__ float g[2][S::kSlotFloats];
   __shared__ double red[2][8];
   const int item = blockIdx.x;
@@ -317,7 +356,7 @@ __global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_consta
   };
   auto db = [&](int s, int i, int j) { return G(s, i, 2 * RP + j) + G(s, RP + i, 2 * RP + j); };
   auto bb = [&](int s, int i, int j) { return G(s, 2 * RP + i, 2 * RP + j); };
-  const int r = a.rank, r2 = 2 * a.rank;
+  constexpr int r = R, r2 = 2 * R;
   double t = 0.0, par = 0.0;
   for (int idx = threadIdx.x; idx < r2 * r2; idx += 256) {
     const int p = idx / r2, q = idx - p * r2;
@@ -355,20 +394,20 @@ __global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_consta
   }
 }
 
-template <int RP>
-cudaError_t launch_rp(const DriftTcArgs& a, float* slots, float* out_sq, cudaStream_t stream) {
-  using S = DtShape<RP>;
+template <int R>
+cudaError_t launch_rank(const DriftTcArgs& a, float* slots, float* out_sq, cudaStream_t stream) {
+  using S = DtShape<R>;
   constexpr int smem = kDtStages * S::kStage + 32 * S::kPairs * 8 * 4;
   static PerDevice once;
   int dev = 0;
   if (once.pending(&dev)) {
     const cudaError_t e =
-        cudaFuncSetAttribute(drift_tc_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(drift_tc_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     once.done(dev);
   }
-  drift_tc_kernel<RP><<<a.grid, kDtThreads, smem, stream>>>(a, slots);
-  drift_tc_final_kernel<RP><<<a.n_items, 256, 0, stream>>>(a, slots, out_sq);
+  drift_tc_kernel<R><<<a.grid, kDtThreads, smem, stream>>>(a, slots);
+  drift_tc_final_kernel<R><<<a.n_items, 256, 0, stream>>>(a, slots, out_sq);
   return cudaGetLastError();
 }
 
@@ -406,8 +445,9 @@ cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, float* s
     const int want = kDtCtasPerSm * num_sms;
     a.grid = steps < want ? steps : want;
     if (a.grid < 1) continue;
-    const cudaError_t e = rank == 16 ? launch_rp<16>(a, slots, out_sq, stream)
-                                     : launch_rp<8>(a, slots, out_sq, stream);
+    const cudaError_t e = rank == 16 ? launch_rank<16>(a, slots, out_sq, stream)
+                          : rank == 8 ? launch_rank<8>(a, slots, out_sq, stream)
+                                      : launch_rank<4>(a, slots, out_sq, stream);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

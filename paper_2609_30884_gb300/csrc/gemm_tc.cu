@@ -68,6 +68,7 @@ struct GemmArgs {
   __nv_bfloat16* vpages;
   ReqTable req;
   int* status;
+  const int* abort;
 };
 
 struct Tile {
@@ -332,6 +333,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   __shared__ __align__(8) uint64_t drain_bar;
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_flag;
+  // a rejected call: every CTA of every cluster sees the same word and leaves before any set-up
+  if (call_aborted(a.abort)) return;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -719,6 +722,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
   a.vpages = static_cast<__nv_bfloat16*>(d.vpages);
   a.req = d.req;
   a.status = d.status;
+  a.abort = d.abort;
   if (a.total_tiles == 0) return cudaSuccess;
   if (pair == 2) return launch_impl<256, 6, 2>(a, num_sms, stream);
   switch (bn) {

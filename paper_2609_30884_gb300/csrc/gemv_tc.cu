@@ -53,6 +53,7 @@ __global__ void __launch_bounds__(kWarps * 32) gemv_tc_kernel(const __grid_const
     if (jb0 < jb1) prefetch_l2_range(sg.W + (size_t)jb0 * d.in_dim, (size_t)(jb1 - jb0) * d.in_dim * 2);
   }
   griddep_begin();  // x, xa and the residual come from the kernels before
+  if (call_aborted(d.abort)) return;
   const int j0 = (tb + tl) * 16;
   const int g = lane >> 2, c = lane & 3;
   const int K = d.in_dim;

@@ -123,6 +123,7 @@ struct GemmDesc {
   void* vpages;
   ReqTable req;
   int* status;
+  const int* abort;       // per-call abort word (call_aborted), or null
 };
 
 // Launch the tcgen05 GEMM. bn: 256 for projections (CTA pairs with 256-row tiles); 16/32/48 for
@@ -161,6 +162,7 @@ struct AttnDesc {
   int n_q_heads, n_kv_heads, head_dim;
   ReqTable req;
   int* status;
+  const int* abort;
 };
 // tcgen05, S and O in TMEM: num_pages of the pool, total_rows of q (for the TMA maps).
 cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows,
@@ -186,6 +188,7 @@ struct GemvDesc {
   int rows;        // 1..8
   int rank;
   int prefetch;    // set by the launcher: prefetch the block's weight rows into L2 before the wait
+  const int* abort;  // per-call abort word, or null
 };
 // Tensor-core GEMV (mma.sync, rows as a bf16 hi/lo pair); launch_gemv uses it when the call's
 // rows (total_rows, the rows of all chunks one caller splits into launches of <= 8; 0 = d.rows)
@@ -220,6 +223,7 @@ struct DecodeAttnDesc {
   float* part;             // scratch [rows, Hq, splits, d + 2]
   int rows, n_q_heads, n_kv_heads, head_dim, splits, max_pos;
   int chunks_per_block;    // set by launch_decode_attention
+  const int* abort;        // per-call abort word, or null
 };
 // Decode attention streamed in 128-position chunks (TMA-staged pages, one block per SM walking
 // a run of chunks of one row and kv head) + merge of the blocks' partials. `splits` in the
@@ -253,21 +257,36 @@ struct RowPages {
 // Rows' fp32 k, v [rows, hkv * head_dim] into their page slot (page_table[pos / 16], pos % 16).
 cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, void* vpages,
                                  const RowPages& rp, int rows, int hkv, int head_dim, int* status,
-                                 cudaStream_t stream);
+                                 const int* abort, cudaStream_t stream);
 // out[r] = argmax of logits row r (lowest index among equal maxima).
 // One block whose wait on an mbarrier nothing arrives on runs out after the bounded-wait limit
 // and raises kStatusTimeout in *status (the failure path, exercised without a fault).
 cudaError_t launch_wait_selftest(int* status, cudaStream_t stream);
 cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
-                               cudaStream_t stream);
+                               cudaStream_t stream, const int* abort = nullptr);
 cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
                                     cudaStream_t stream);
-cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream);
+cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream,
+                               const int* abort = nullptr);
+// dst[0 .. n) = src[0 .. n) (bf16), unless the call's abort word is set.
+cudaError_t launch_copy_bf16(__nv_bfloat16* dst, const __nv_bfloat16* src, size_t n, const int* abort,
+                             cudaStream_t stream);
+// The page-table check that opens crf_recompute_window and crf_decode_step: every id of every
+// table in [0, num_pages) and no page twice across the tables. A failure sets *abort and raises
+// kStatusPages in *status. `table` is scratch of (mask + 1) ints, mask + 1 a power of two at
+// least twice the ids checked, filled with -1 (0xff bytes) before the launch.
+struct PageCheck {
+  const int32_t* pt[kMaxReq];
+  int first[kMaxReq + 1];  // prefix of the tables' id counts
+  int n;
+};
+cudaError_t launch_validate_pages(const PageCheck& pc, int num_pages, int* table, uint32_t mask, int* abort,
+                                  int* status, cudaStream_t stream);
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStream_t stream);
 
 // LM head + KL: logits [2*rows, V] (ref rows first) from final-normed hidden rows.
 cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,
-                           float* logits, int num_sms, cudaStream_t stream);
+                           float* logits, int num_sms, cudaStream_t stream, const int* abort = nullptr);
 // KL per row from fp32 logits; part: scratch [rows][splits][5].
 cudaError_t launch_kl(const float* zref, const float* zcur, int rows, int vocab, float* out,
                       float* part, int splits, cudaStream_t stream);

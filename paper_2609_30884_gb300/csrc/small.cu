@@ -138,6 +138,7 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const __grid_cons
     if (jb0 < jb1) prefetch_l2_range(sg.W + (size_t)jb0 * d.in_dim, (size_t)(jb1 - jb0) * d.in_dim * 2);
   }
   griddep_begin();  // x, xa and the residual come from the kernels before
+  if (call_aborted(d.abort)) return;
   const int g = gb + gl;
   const int j0 = g * OPW;
   const int n8 = d.in_dim / 8;
@@ -310,9 +311,46 @@ __global__ void swiglu_split_f32_kernel(const float* g, const float* u, float* m
   if (i < n) m[i] = g[i] / (1.f + __expf(-g[i])) * u[i];
 }
 
-__global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int n) {
+__global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int n, const int* abort) {
+  if (call_aborted(abort)) return;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) y[i] = __float2bfloat16_rn(x[i]);
+}
+
+__global__ void copy_bf16_kernel(__nv_bfloat16* __restrict__ dst, const __nv_bfloat16* __restrict__ src,
+                                 size_t n, const int* abort) {
+  if (call_aborted(abort)) return;
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x)
+    dst[i] = src[i];
+}
+
+// One thread per page id: outside [0, num_pages), or already in the open-addressing table
+// (linear probing, at most mask + 1 probes), rejects the call.
+__global__ void validate_pages_kernel(const PageCheck pc, int num_pages, int* table, uint32_t mask,
+                                      int* abort, int* status) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= pc.first[pc.n]) return;
+  int i = 0;
+  while (i + 1 < pc.n && idx >= pc.first[i + 1]) ++i;
+  const int id = pc.pt[i][idx - pc.first[i]];
+  bool bad = id < 0 || id >= num_pages;
+  if (!bad) {
+    uint32_t h = (static_cast<uint32_t>(id) * 0x9E3779B1u) & mask;
+    for (uint32_t probe = 0; probe <= mask; ++probe) {
+      const int prev = atomicCAS(table + h, -1, id);
+      if (prev == -1) break;
+      if (prev == id) {
+        bad = true;
+        break;
+      }
+      h = (h + 1) & mask;
+    }
+  }
+  if (bad) {
+    atomicExch(abort, 1);
+    atomicOr(status, kStatusPages);
+  }
 }
 __global__ void bf16_to_f32_kernel(const __nv_bfloat16* x, float* y, int n) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -577,8 +615,9 @@ __global__ void embed_rows_f32_kernel(const __nv_bfloat16* __restrict__ embed, c
 // The rows' fp32 k, v [rows, Hkv * d] into slot pos % 16 of page page_table[pos / 16], bf16.
 __global__ void kv_write_rows_kernel(const float* __restrict__ k, const float* __restrict__ v,
                                      __nv_bfloat16* kpages, __nv_bfloat16* vpages, const RowPages rp,
-                                     int hkv, int d, int* status) {
+                                     int hkv, int d, int* status, const int* abort) {
   griddep_begin();  // k, v come from the kernels before
+  if (call_aborted(abort)) return;
   const int r = blockIdx.y;
   const int pos = rp.pos[r];
   const int page = checked_page(rp.page_table[r][pos / kPage], rp.num_pages,
@@ -593,7 +632,9 @@ __global__ void kv_write_rows_kernel(const float* __restrict__ k, const float* _
 
 // out[r] = argmax_i logits[r, i], the lowest index among equal maxima.
 // One block per row; 16-byte loads, four in flight per thread before their compares.
-__global__ void argmax_rows_kernel(const float* __restrict__ logits, int vocab, int32_t* out) {
+__global__ void argmax_rows_kernel(const float* __restrict__ logits, int vocab, int32_t* out,
+                                   const int* abort) {
+  if (call_aborted(abort)) return;
   const int r = blockIdx.x;
   const float* z = logits + (size_t)r * vocab;
   float best = -INFINITY;
@@ -679,17 +720,34 @@ cudaError_t launch_embed_rows_f32(const __nv_bfloat16* embed, const TokenRows& t
 
 cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, void* vpages,
                                  const RowPages& rp, int rows, int hkv, int head_dim, int* status,
-                                 cudaStream_t stream) {
+                                 const int* abort, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
   return launch_kernel(kv_write_rows_kernel, dim3(cdiv(hkv * head_dim, 256), rows), dim3(256), 0, stream, k, v,
                        static_cast<__nv_bfloat16*>(kpages), static_cast<__nv_bfloat16*>(vpages), rp, hkv,
-                       head_dim, status);
+                       head_dim, status, abort);
 }
 
 cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
-                               cudaStream_t stream) {
+                               cudaStream_t stream, const int* abort) {
   if (rows == 0) return cudaSuccess;
-  argmax_rows_kernel<<<rows, 1024, 0, stream>>>(logits, vocab, out);
+  argmax_rows_kernel<<<rows, 1024, 0, stream>>>(logits, vocab, out, abort);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_copy_bf16(__nv_bfloat16* dst, const __nv_bfloat16* src, size_t n, const int* abort,
+                             cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  const size_t want = (n + 255) / 256;
+  copy_bf16_kernel<<<static_cast<unsigned>(want < 4096 ? want : 4096), 256, 0, stream>>>(dst, src, n, abort);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_validate_pages(const PageCheck& pc, int num_pages, int* table, uint32_t mask, int* abort,
+                                  int* status, cudaStream_t stream) {
+  const int total = pc.first[pc.n];
+  if (total == 0) return cudaSuccess;
+  if (static_cast<uint32_t>(total) > (mask + 1u) / 2u) return cudaErrorInvalidValue;
+  validate_pages_kernel<<<cdiv(total, 256), 256, 0, stream>>>(pc, num_pages, table, mask, abort, status);
   return cudaGetLastError();
 }
 
@@ -708,9 +766,10 @@ cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, in
   return launch_kernel(swiglu_split_f32_kernel, dim3(cdiv(n, 256)), dim3(256), 0, stream, g, u, m, n);
 }
 
-cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream) {
+cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream,
+                               const int* abort) {
   if (n == 0) return cudaSuccess;
-  f32_to_bf16_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, y, n);
+  f32_to_bf16_kernel<<<cdiv(n, 256), 256, 0, stream>>>(x, y, n, abort);
   return cudaGetLastError();
 }
 cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStream_t stream) {
@@ -720,9 +779,10 @@ cudaError_t launch_bf16_to_f32(const __nv_bfloat16* x, float* y, int n, cudaStre
 }
 
 cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int vocab, int hidden,
-                           float* logits, int num_sms, cudaStream_t stream) {
+                           float* logits, int num_sms, cudaStream_t stream, const int* abort) {
   for (int r0 = 0; r0 < rows; r0 += kGemvMaxRows) {
     GemvDesc d{};
+    d.abort = abort;
     d.seg[0].W = W;
     d.seg[0].out_dim = vocab;
     d.seg[0].y = logits + (size_t)r0 * vocab;

@@ -1,5 +1,5 @@
 """Run in a child process by tests/test_gpu_bounds.py with CRF_LIB_VARIANT=debug and
-CRF_DEBUG_DEVICE_CHECKS_ONLY=1: the CRF_DEBUG library, whose host-side page-table read is skipped,
+CRF_DEBUG_DEVICE_CHECKS_ONLY=1: the CRF_DEBUG library, whose page-table check at the start of each call is skipped,
 so its device-side checks alone meet the bad page ids below.
 
 1. A valid two-request prefill matches the oracle and records nothing (no false positives).

@@ -12,6 +12,12 @@ from oracle.decoder import LayerAdapter
 REL_KVH = 1e-2       # per-layer relative Frobenius error of K/V pages and hidden states
 KL_ABS = 1e-3        # absolute KL error
 DRIFT_REL = 1e-4     # relative drift error
+# Where a layer's own conditioning keeps every bf16-storage implementation above REL_KVH, the
+# bar is this factor times the distance that the same layer moves when the oracle's steps store
+# their intermediate tensors in bf16 at the points the path does (``bf16_storage_layer``): the
+# two round at the same points and differ only in fp32 accumulation order, which decides a few
+# roundings differently (measured ratio GPU / storage model on whole layers: 0.9-1.1).
+STORAGE_FACTOR = 1.25
 
 
 def to_np(t: torch.Tensor) -> np.ndarray:
@@ -82,71 +88,99 @@ def bf16_round(a) -> np.ndarray:
     return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).bfloat16().float().numpy()
 
 
-def _bf16_proj(xin, P, A, m, bias):
-    """One adapted projection as a bf16 tensor pipeline runs it (op outputs rounded to bf16)."""
-    R = bf16_round
-    y = xin @ P.W[m].T
-    if bias and m in P.bias:
-        y = y + P.bias[m]
-    y = R(y)
-    if m in A.AB:
-        Am, Bm = A.AB[m]
-        y = R(y + R(A.scale * R(R(xin @ Am.T) @ Bm.T)))
-    return y
+def _storage_proj(xin, P, A, m, bias):
+    Am, Bm = A.AB.get(m, (None, None))
+    return Dec.lora_linear(xin, P.W[m], Am, Bm, A.scale, P.bias.get(m) if bias else None)
 
 
-def bf16_layer_rows(x, P, A, dims, rows):
-    """Layer output at `rows` (attention over all positions <= row) run as a bf16 tensor pipeline."""
+def _storage_qkv(x, P, A, dims):
+    """q, K, V of every position as the path stores them (bf16), from the bf16 normalised input."""
     R = bf16_round
     n = x.shape[0]
-    x = R(x)
+    d = dims.head_dim
     xn = R(Dec.rmsnorm(x, P.ln1, dims.rms_eps))
-    cos, sin = Dec.rope_angles(np.arange(n), dims.head_dim, dims.rope_theta)
-    q = R(Dec.apply_rope(_bf16_proj(xn, P, A, "q", True).reshape(n, dims.n_q_heads, dims.head_dim), cos, sin))
-    k = R(Dec.apply_rope(_bf16_proj(xn, P, A, "k", True).reshape(n, dims.n_kv_heads, dims.head_dim), cos, sin))
-    v = _bf16_proj(xn, P, A, "v", True).reshape(n, dims.n_kv_heads, dims.head_dim)
-    out = []
-    for t in rows:
-        o = R(Dec.single_query_attention(q[t], k[:t + 1], v[:t + 1])).reshape(1, -1)
-        x1 = R(x[t:t + 1] + _bf16_proj(o, P, A, "o", False))
-        xn2 = R(Dec.rmsnorm(x1, P.ln2, dims.rms_eps))
-        m = R(R(Dec.silu(_bf16_proj(xn2, P, A, "gate", False))) * _bf16_proj(xn2, P, A, "up", False))
-        out.append(R(x1 + _bf16_proj(m, P, A, "down", False))[0])
-    return np.stack(out)
+    cos, sin = Dec.rope_angles(np.arange(n), d, dims.rope_theta)
+    q = R(Dec.apply_rope(_storage_proj(xn, P, A, "q", True).reshape(n, dims.n_q_heads, d), cos, sin))
+    k = R(Dec.apply_rope(_storage_proj(xn, P, A, "k", True).reshape(n, dims.n_kv_heads, d), cos, sin))
+    v = R(_storage_proj(xn, P, A, "v", True).reshape(n, dims.n_kv_heads, d))
+    return q, k, v
 
 
-def bf16_execution_recover(om, oa, pool, req, s, e, restart):
-    """The window recovery executed the way a bf16 tensor pipeline runs it.
-
-    The paper computes in bfloat16 throughout (Section 5.1): every op's output tensor is bf16
-    while arithmetic inside an op accumulates in fp32. This runs the oracle's steps that way
-    (projections, LoRA factors, RoPE outputs, attention output, residual sums, norms, the MLP
-    activation and the cache K/V all rounded to bf16 as they are produced); the last row then
-    continues through the tail in fp32, as the decode path does. Its distance from the plain fp32
-    oracle measures how strongly the problem at hand amplifies bf16 rounding (large when deep-layer
-    adapters dominate and attention is near one-hot). Returns (per-layer K, V, H dicts, final row).
-    """
+def _storage_post(x, o, P, A, dims):
+    """Output projection, residual, MLP and residual of rows whose attention output is o (bf16 stores)."""
     R = bf16_round
-    dims = om.dims
-    n = req.n
-    proj = _bf16_proj
+    o = R(o.reshape(x.shape[0], -1))
+    x1 = R(x + _storage_proj(o, P, A, "o", False))
+    xn2 = R(Dec.rmsnorm(x1, P.ln2, dims.rms_eps))
+    m = R(Dec.silu(_storage_proj(xn2, P, A, "gate", False)) * _storage_proj(xn2, P, A, "up", False))
+    return R(x1 + _storage_proj(m, P, A, "down", False))
 
-    cos, sin = Dec.rope_angles(np.arange(n), dims.head_dim, dims.rope_theta)
-    x = R(restart)
-    ks, vs, hs = {}, {}, {}
-    for l in range(s, e):
-        P, A = om.layers[l], oa.layers[l]
-        xn = R(Dec.rmsnorm(x, P.ln1, dims.rms_eps))
-        q = proj(xn, P, A, "q", True).reshape(n, dims.n_q_heads, dims.head_dim)
-        k = proj(xn, P, A, "k", True).reshape(n, dims.n_kv_heads, dims.head_dim)
-        v = proj(xn, P, A, "v", True).reshape(n, dims.n_kv_heads, dims.head_dim)
-        q, k = R(Dec.apply_rope(q, cos, sin)), R(Dec.apply_rope(k, cos, sin))
-        o = R(Dec.causal_gqa_attention(q, k, v))
-        x1 = R(x + proj(o.reshape(n, -1), P, A, "o", False))
-        xn2 = R(Dec.rmsnorm(x1, P.ln2, dims.rms_eps))
-        mlp = R(R(Dec.silu(proj(xn2, P, A, "gate", False))) * proj(xn2, P, A, "up", False))
-        x = R(x1 + proj(mlp, P, A, "down", False))
-        pool.write(l, req.page_table, k, v)
-        ks[l], vs[l], hs[l] = k, v, x
-    final = C.tail_decode(om, oa, pool, req, e, x[-1])
-    return ks, vs, hs, final
+
+def _storage_attention_rows(q, k, v, rows, grp):
+    """Attention of query rows t over keys 0..t with the softmax weights rounded to bf16 before the
+    P.V product and normalised by the sum of the unrounded weights (fp64)."""
+    d = q.shape[-1]
+    scale = np.float32(1.0 / np.sqrt(d))
+    out = np.empty((len(rows), q.shape[1], d), np.float32)
+    for j, t in enumerate(rows):
+        for h in range(q.shape[1]):
+            g = h // grp
+            sc = (k[:t + 1, g] @ q[t, h]) * scale
+            p = np.exp(sc - sc.max())
+            out[j, h] = (bf16_round(p) @ v[:t + 1, g]) / np.float32(p.sum(dtype=np.float64))
+    return out
+
+
+def bf16_storage_rows(x, P, A, dims, rows):
+    """``bf16_storage_layer`` evaluated at the given rows only (H at ``rows``; K and V of every
+    position, which those rows attend to)."""
+    x = np.asarray(x, np.float32)
+    q, k, v = _storage_qkv(x, P, A, dims)
+    o = _storage_attention_rows(q, k, v, rows, dims.n_q_heads // dims.n_kv_heads)
+    return _storage_post(x[rows], o, P, A, dims), k, v
+
+
+def bf16_storage_layer(x, P, A, dims, chunk: int = 512):
+    """One decoder layer (the oracle's steps and arithmetic: fp32 products, fp32 softmax with fp64
+    sums) with every tensor that the recomputation path keeps in memory between its kernels
+    rounded to bf16 once: the normalised inputs, q and the cached K and V (after rotation), the
+    softmax weights entering the P.V product (normalised by the sum of the unrounded weights),
+    the attention output, the residual after attention, the MLP activation and the layer output.
+    This is the declared precision of the path (bf16 storage, fp32 accumulation) applied to the
+    oracle; its distance from the fp32 oracle is how far that precision alone moves a layer.
+    Returns (H, K, V) like ``decoder.decoder_layer``."""
+    x = np.asarray(x, np.float32)
+    n = x.shape[0]
+    q, k, v = _storage_qkv(x, P, A, dims)
+    grp = dims.n_q_heads // dims.n_kv_heads
+    scale = np.float32(1.0 / np.sqrt(dims.head_dim))
+    o = np.empty_like(q)
+    for h in range(dims.n_q_heads):
+        g = h // grp
+        for i0 in range(0, n, chunk):
+            i1 = min(n, i0 + chunk)
+            sc = (q[i0:i1, h] @ k[:i1, g].T) * scale
+            sc[np.arange(i1)[None, :] > np.arange(i0, i1)[:, None]] = -np.inf
+            p = np.exp(sc - sc.max(axis=-1, keepdims=True))
+            den = p.sum(axis=-1, keepdims=True, dtype=np.float64).astype(np.float32)
+            o[i0:i1, h] = (bf16_round(p) @ v[:i1, g]) / den
+    return _storage_post(x, o, P, A, dims), k, v
+
+
+def local_layer_report(x_in, P, A, dims, got_h, got_k, got_v, tag, plain: bool = False):
+    """The GPU's layer outputs (H, and the request's K/V of that layer, every position) against the
+    oracle's layer run on the GPU's own input for that layer (its bf16 restart state or previous
+    window output), so each layer is judged on its own arithmetic. Returns
+    [(name, err, bar, storage distance)]: the bar is REL_KVH, or, unless ``plain``, STORAGE_FACTOR
+    times the bf16-storage model's distance on the same input when that is larger."""
+    want_h, want_k, want_v = Dec.decoder_layer(x_in, P, A, dims)
+    if plain:
+        dist = {"h": 0.0, "k": 0.0, "v": 0.0}
+    else:
+        sh, sk, sv = bf16_storage_layer(x_in, P, A, dims)
+        dist = {"h": rel_frob(sh, want_h), "k": rel_frob(sk, want_k), "v": rel_frob(sv, want_v)}
+    out = []
+    for name, got, want in (("h", got_h, want_h), ("k", got_k, want_k), ("v", got_v, want_v)):
+        out.append((f"{name}{tag}", rel_frob(got, want), max(REL_KVH, STORAGE_FACTOR * dist[name]),
+                    dist[name]))
+    return out

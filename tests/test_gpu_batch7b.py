@@ -5,13 +5,13 @@ its own window, one shared pool with a randomly permuted page table.
   checkpoints to running every request alone (each row is computed the same way whatever else
   shares its tile or launch); the first-step rows agree to bf16 rounding (their GEMV kernel
   depends on how many rows share a weight pass).
-* Against the oracle, per request, on what it computes one by one at this size: K and V of every
-  position of the request's first window layer, and that layer's output at sampled rows, held to
-  1e-2 plus twice the largest distance that rounding-sized changes move the same rows (a bf16
-  tensor pipeline, and seeded relative perturbations of q and K at most 2^-8). Deep layers of
-  an adapter several versions old are adapter-dominated: attention scores have a spread of ~1e3
-  and top-2 gaps of a few units, so a rounding-sized change flips which key a head attends to.
-  Windows starting at layer 3 or below are well conditioned and also meet the plain 1e-2 bar.
+* Against the oracle, per request, on what it computes at this size: K and V of every position of
+  the request's first window layer, and that layer's output at 48 rows spread over the prefix,
+  held to 1e-2 or 1.25x the distance the oracle's layer moves at the same rows when it stores its
+  intermediates in bf16 where the path does, whichever is larger. Deep layers of an adapter
+  several versions old are adapter-dominated: attention scores have a spread of ~1e3 and top-2
+  gaps of a few units, so a rounding-sized change flips which key a head attends to. Windows
+  starting at layer 3 or below are well conditioned and meet the plain 1e-2 bar.
 * Slots no request owns, and layers outside every window, stay bit-identical.
 """
 import numpy as np
@@ -21,8 +21,8 @@ import torch
 import synth
 from tests.harness import DeviceAdapter, DeviceModel, make_pool, split_page_tables
 from oracle import build as obuild, decoder as Dec
-from tests.gpu_util import (REL_KVH, bf16_layer_rows, free_slots, rel_frob, snapshot, to_np,
-                            untouched_mask)
+from tests.gpu_util import (REL_KVH, STORAGE_FACTOR, bf16_storage_rows, free_slots, rel_frob, snapshot,
+                            to_np, untouched_mask)
 
 pytestmark = pytest.mark.gpu
 
@@ -101,35 +101,23 @@ def test_batch7b_equals_single_and_oracle(ctx):
         tok, h_in, h_out, _ = keep[i]
         x = to_np(h_in) if s > 0 else to_np(dm.embed[tok.long()])
         q_all, k_all, v_all = Dec.qkv(x, P_l, A_l, dims, np.arange(n))
-        assert rel_frob(to_np(request_kv_t(got_k[s], pts[i], n)), k_all) <= REL_KVH, i
-        assert rel_frob(to_np(request_kv_t(got_v[s], pts[i], n)), v_all) <= REL_KVH, i
-        rows = np.unique(np.array([0, 15, 16, n // 2, n - 2, n - 1]))
+        rows = np.unique(np.concatenate([[0, 15, 16, n - 2, n - 1], np.linspace(32, n - 3, 43).astype(int)]))
+        st_h, st_k, st_v = bf16_storage_rows(x, P_l, A_l, dims, rows)
         want = []
         for t in rows:
             o = Dec.single_query_attention(q_all[t], k_all[:t + 1], v_all[:t + 1])
             want.append(Dec.post_attention(x[t:t + 1], o[None], P_l, A_l, dims)[0])
         want = np.stack(want)
         got = to_np(h_out[0])[rows]
-        # conditioning: the same rows run as a bf16 tensor pipeline, and with q and K moved by
-        # seeded relative perturbations of bf16 rounding size (at most 2^-8)
-        alts = [bf16_layer_rows(x, P_l, A_l, dims, rows)]
-        rng = np.random.default_rng(1000 + i)
-        for _ in range(8):
-            out = []
-            for t in rows:
-                qq = q_all[t] * (1 + rng.uniform(-2.0 ** -8, 2.0 ** -8, q_all[t].shape))
-                kk = k_all[:t + 1] * (1 + rng.uniform(-2.0 ** -8, 2.0 ** -8, k_all[:t + 1].shape))
-                o = Dec.single_query_attention(qq, kk, v_all[:t + 1])
-                out.append(Dec.post_attention(x[t:t + 1], o[None], P_l, A_l, dims)[0])
-            alts.append(np.stack(out))
-        err = rel_frob(got, want)
-        sens = max(rel_frob(a, want) for a in alts)
-        per_row = [round(rel_frob(got[j], want[j]), 4) for j in range(len(rows))]
-        print(f"request {i} n={n} window [{s},{e}): h err {err:.4f}, rounding-scale spread {sens:.4f}; "
-              f"rows {rows.tolist()} err {per_row}")
-        assert err <= REL_KVH + 2 * sens, (i, err, sens)
-        if s <= 3:   # the shallowest windows are well conditioned: the plain bar
-            assert err <= REL_KVH, (i, err)
+        report = [("k", rel_frob(to_np(request_kv_t(got_k[s], pts[i], n)), k_all), rel_frob(st_k, k_all)),
+                  ("v", rel_frob(to_np(request_kv_t(got_v[s], pts[i], n)), v_all), rel_frob(st_v, v_all)),
+                  ("h", rel_frob(got, want), rel_frob(st_h, want))]
+        print(f"request {i} n={n} window [{s},{e}) first layer (name, err, bf16-storage distance):",
+              [(a, round(b, 5), round(c, 5)) for a, b, c in report])
+        for name, err, dist in report:
+            assert err <= max(REL_KVH, STORAGE_FACTOR * dist), (i, name, err, dist)
+            if s <= 3:   # the shallowest windows are well conditioned: the plain bar
+                assert err <= REL_KVH, (i, name, err)
 
 
 def request_kv_t(pool_layer, page_table, n):

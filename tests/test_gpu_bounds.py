@@ -2,10 +2,11 @@
 as an address, replaced by a safe one (token 0, page 0), recorded in the context's status word and
 reported by crf_check as CRF_EINVAL; the report is cleared and the context keeps working.
 
-Token ids are checked in every build. Page ids are checked on the host before launch; the library
-built with CRF_DEBUG (libcrf_debug.so) re-checks them at every device-side use, and with
-CRF_DEBUG_DEVICE_CHECKS_ONLY=1 it skips the host read so that those device checks alone meet the
-bad ids. That build runs in a child process (tests/debug_bounds_child.py)."""
+Token ids are checked in every build. Page ids are checked by the first kernel of every call
+(which rejects the whole call); the library built with CRF_DEBUG (libcrf_debug.so) re-checks them
+at every device-side use, and with CRF_DEBUG_DEVICE_CHECKS_ONLY=1 it skips that first check so that
+the per-use checks alone meet the bad ids. That build runs in a child process
+(tests/debug_bounds_child.py)."""
 import os
 import subprocess
 import sys

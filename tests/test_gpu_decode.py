@@ -111,10 +111,23 @@ def test_decode_step_rejects_bad_arguments():
     tok = torch.zeros(2, dtype=torch.int32, device="cuda")
     nxt = torch.empty(2, dtype=torch.int32, device="cuda")
     ws = ctx.decode_workspace(dm.crf, ad.crf, [20, 20], [pt, pt], tok)
-    with pytest.raises(CrfError):   # the same page in two rows
-        ctx.decode_step(dm.crf, ad.crf, pool, [20, 20], [pt, pt], tok, nxt, ws)
+    bk, bv = [t.clone() for t in pool.k_pages], [t.clone() for t in pool.v_pages]
     bad = torch.tensor([0, 99], dtype=torch.int32, device="cuda")
-    with pytest.raises(CrfError):   # a page id past the pool
-        ctx.decode_step(dm.crf, ad.crf, pool, [20], [bad], tok[:1], nxt[:1], ws)
-    with pytest.raises(CrfError):   # workspace too small
+    logits = torch.full((2, cfg.vocab), 7.0, dtype=torch.float32, device="cuda")
+    nxt.fill_(-5)
+    # page tables are checked by the step's first kernel: the same page in two rows, or an id past
+    # the pool, makes the step write nothing (pages, logits, tokens) and crf_check report EINVAL
+    for pos, pts, t in (([20, 20], [pt, pt], tok), ([20], [bad], tok[:1])):
+        ctx.decode_step(dm.crf, ad.crf, pool, pos, pts, t, nxt[:len(pos)], ws, logits=logits[:len(pos)])
+        with pytest.raises(CrfError) as ei:
+            ctx.check()
+        assert ei.value.status == crf.abi.EINVAL
+        assert all(torch.equal(a, b) for a, b in zip(pool.k_pages, bk))
+        assert all(torch.equal(a, b) for a, b in zip(pool.v_pages, bv))
+        assert torch.all(logits == 7.0) and torch.all(nxt == -5)
+    with pytest.raises(CrfError):   # workspace too small: refused before anything is enqueued
         ctx.decode_step(dm.crf, ad.crf, pool, [20], [pt], tok[:1], nxt[:1], ws[:256])
+    # a valid step on the same workspace afterwards
+    ctx.decode_step(dm.crf, ad.crf, pool, [20], [pt], tok[:1], nxt[:1], ws, logits=logits[:1])
+    ctx.check()
+    assert not torch.all(logits[0] == 7.0) and int(nxt[0]) >= 0

@@ -184,6 +184,7 @@ def test_full_prefill_matches_oracle_prefill(ctx, tiny):
 
 
 def test_invalid_arguments_rejected(ctx, tiny):
+    """Host-checkable arguments are refused before anything is enqueued (CRF_EINVAL / CRF_ENOMEM)."""
     cfg, lc, dm, cur, _, _ = tiny
     import paper_2609_30884_gb300 as crf
     n = 64
@@ -198,8 +199,6 @@ def test_invalid_arguments_rejected(ctx, tiny):
         crf.Request(pt, 1, 5, hidden_in=h),                      # e > N
         crf.Request(pt, 1, 2, n_tokens=n),                       # missing hidden_in
         crf.Request(pt, 2, 2, hidden_in=h),                      # empty window, no final out
-        crf.Request(torch.full_like(pt, P), 1, 2, hidden_in=h),  # page id out of range
-        crf.Request(torch.zeros_like(pt), 1, 2, hidden_in=h),    # duplicate pages
     ]
     for r in bad:
         with pytest.raises(crf.CrfError) as ei:
@@ -210,3 +209,44 @@ def test_invalid_arguments_rejected(ctx, tiny):
     assert ei.value.status == crf.abi.ENOMEM
     torch.cuda.synchronize()
     assert all(torch.equal(a, b) for a, b in zip(pool.k_pages, bk))
+
+
+def test_bad_page_tables_rejected_on_device(ctx, tiny):
+    """Page ids are checked by the first kernel of the call, without a host round trip: an id
+    outside the pool, a page used twice within a request or shared by two requests, makes the
+    call write nothing outside its workspace (pool, checkpoints, final rows) and crf_check report
+    CRF_EINVAL once; the next call with valid tables runs normally."""
+    cfg, lc, dm, cur, om, oa = tiny
+    import paper_2609_30884_gb300 as crf
+    n = 64
+    P = 2 * pages_needed(n)
+    pool = make_pool(cfg, P, fill="random", seed=4)
+    pt0, pt1 = split_page_tables([n, n], P, seed=2)
+    h = synth.hidden_state(cfg, n, device="cuda")
+    ws = torch.empty(1 << 24, dtype=torch.uint8, device="cuda")
+    bk, bv = snapshot(pool)
+    hout = [torch.full((n, cfg.hidden), 3.0, dtype=torch.bfloat16, device="cuda")]
+    fin = torch.full((cfg.hidden,), 5.0, dtype=torch.bfloat16, device="cuda")
+    shared = pt1.clone()
+    shared[1] = pt0[2]
+    cases = [
+        [crf.Request(torch.full_like(pt0, P), 1, 2, hidden_in=h, hidden_out=hout, final_hidden_out=fin)],
+        [crf.Request(torch.full_like(pt0, -1), 1, 2, hidden_in=h, hidden_out=hout)],
+        [crf.Request(torch.zeros_like(pt0), 1, 2, hidden_in=h, hidden_out=hout, final_hidden_out=fin)],
+        [crf.Request(pt0, 1, 2, hidden_in=h, hidden_out=hout),
+         crf.Request(shared, 1, 3, hidden_in=h, final_hidden_out=fin)],
+        [crf.Request(torch.full_like(pt0, P), 3, 4, hidden_in=h, final_hidden_out=fin)],   # last layer
+    ]
+    for reqs in cases:
+        ctx.recompute_window(dm.crf, cur.crf, pool, reqs, ws)    # enqueued: nothing waits here
+        with pytest.raises(crf.CrfError) as ei:
+            ctx.check()
+        assert ei.value.status == crf.abi.EINVAL
+        ctx.check()                                                # reported once
+        assert all(torch.equal(a, b) for a, b in zip(pool.k_pages, bk))
+        assert all(torch.equal(a, b) for a, b in zip(pool.v_pages, bv))
+        assert torch.all(hout[0] == 3.0) and torch.all(fin == 5.0)
+    # the same workspace then serves a valid call
+    _run(ctx, dm, cur, pool, [crf.Request(pt0, 1, 2, hidden_in=h, hidden_out=hout, final_hidden_out=fin)])
+    assert not torch.equal(pool.k_pages[1], bk[1])
+    assert not torch.all(hout[0] == 3.0)
