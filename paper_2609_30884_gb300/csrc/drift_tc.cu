@@ -17,12 +17,12 @@
 // RP = max(r, 8) features per part (zeros), and the kernel accumulates the block-upper triangle
 // of its Gram (16 x 16 blocks).
 //
-// Work split: the long dimension of every (item, side) segment is cut into 128-row steps; the
+// Work split: the long dimension of every (item, side) segment is cut into 256-row steps; the
 // steps of all segments are laid end to end and a persistent grid of G CTAs takes equal
 // consecutive ranges of them (stream-K). A CTA stages each step's rows of both versions with
-// cp.async (three stages in flight, no registers held), builds the hi/lo/base fragments in
-// registers from ldmatrix loads (transposed for the B side, whose rows are [r] wide), and its 8
-// warps each accumulate one 16-row slice. When its range leaves a segment (or ends) the CTA sums
+// cp.async (two steps in flight while one is multiplied, no registers held), builds the
+// hi/lo/base fragments in registers from ldmatrix loads (transposed for the B side, whose rows
+// are [r] wide), and its 8 warps each accumulate two 16-row slices. When its range leaves a segment (or ends) the CTA sums
 // its warps in a fixed order and writes one partial Gram to slot (b + seg), unique because a
 // CTA's segments follow the previous CTA's. The final kernel sums each segment's slots in CTA
 // order and forms tr(GB GA) and the parameter distance in fp64. The result does not depend on
@@ -35,9 +35,10 @@ namespace crf {
 namespace {
 
 constexpr int kDtThreads = 256;
-constexpr int kDtRows = 128;   // long-dimension rows per step: 8 warps x 16
-constexpr int kDtStages = 4;   // three steps in flight while one is multiplied
-constexpr int kDtCtasPerSm = 3;
+constexpr int kDtRows = 256;   // long-dimension rows per step: 8 warps x 2 slices x 16
+constexpr int kDtSlices = kDtRows / 128;  // 16-row slices per warp and step
+constexpr int kDtStages = 3;   // two steps in flight while one is multiplied
+constexpr int kDtCtasPerSm = 2;
 constexpr int kDtMaxItems = 224;
 constexpr int kDtMaxSegs = 2 * kDtMaxItems;
 constexpr int kDtAStride = kDtRows * 2 + 16;  // bytes per A row in a stage (+16: no bank conflicts)
@@ -56,7 +57,9 @@ struct DtShape {
   static constexpr int kAVersion = RP * kDtAStride;             // one version of the A side
   static constexpr int kStage = 2 * (kBVersion > kAVersion ? kBVersion : kAVersion);
   static constexpr int kBlocks = RP == 16 ? 3 : 2;              // 16-feature blocks of [hi|lo|base]
-  static constexpr int kPairs = kBlocks * (kBlocks + 1) / 2;    // block-upper triangle
+  // block pairs (I <= J) accumulated: the block-upper triangle, except lo x lo for RP = 16 (its
+  // entries are below 2^-18 of hi x hi, far under the drift tolerance)
+  static constexpr int kPairs = RP == 16 ? 5 : 3;
   static constexpr int kSlotFloats = kPairs * 256;
   // copies per step and version: B side in chunks of min(16, 2R) bytes per row; A side in 16-byte
   // chunks of R rows
@@ -67,6 +70,16 @@ struct DtShape {
   static constexpr int kBPerThread = (kBCopies + kDtThreads - 1) / kDtThreads;
   static constexpr int kAPerThread = (kACopies + kDtThreads - 1) / kDtThreads;
 };
+
+// (I, J) of accumulated pair p, and the pair of (I, J) (-1: not accumulated, reads as zero)
+template <int RP>
+__host__ __device__ constexpr int pair_I(int p) { return RP == 16 ? (p < 3 ? 0 : (p == 3 ? 1 : 2)) : (p < 2 ? 0 : 1); }
+template <int RP>
+__host__ __device__ constexpr int pair_J(int p) { return RP == 16 ? (p < 3 ? p : 2) : (p < 2 ? p : 1); }
+template <int RP>
+__host__ __device__ constexpr int pair_of(int I, int J) {
+  return RP == 16 ? (I == 0 ? J : (I == 1 ? (J == 2 ? 3 : -1) : 4)) : (I == 0 ? J : 2);
+}
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
@@ -87,49 +100,26 @@ __device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t&
   asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
 }
 
-// (hi, lo) of the exact fp32 differences of two bf16 pairs
-__device__ __forceinline__ void split_diff(uint32_t a, uint32_t b, uint32_t& hi, uint32_t& lo) {
-  const float d0 = bf16_lo(a) - bf16_lo(b), d1 = bf16_hi(a) - bf16_hi(b);
-  hi = pack_bf16(d0, d1);
-  lo = pack_bf16(d0 - bf16_lo(hi), d1 - bf16_hi(hi));
+__device__ __forceinline__ uint32_t bf2_sub(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+__device__ __forceinline__ uint32_t bf2_add(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("add.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
 }
 
-// This thread's copies of a step, fixed for the whole kernel: for copy u, the version, the row
-// (B side: long-dimension row; A side: rank row k), the chunk and the stage offset.
-template <int R>
-struct CopyPlan {
-  using S = DtShape<R>;
-  int b_row[S::kBPerThread], b_src[S::kBPerThread];  // b_src: element offset within the row block
-  uint32_t b_dst[S::kBPerThread];
-  int a_col[S::kAPerThread], a_k[S::kAPerThread];
-  uint32_t a_dst[S::kAPerThread];
-  bool b_v1[S::kBPerThread], a_v1[S::kAPerThread], b_on[S::kBPerThread], a_on[S::kAPerThread];
-
-  __device__ __forceinline__ void init(int tid) {
-#pragma unroll
-    for (int u = 0; u < S::kBPerThread; ++u) {
-      const int i = tid + u * kDtThreads;
-      const int v = i / (kDtRows * S::kBChunksPerRow), rem = i % (kDtRows * S::kBChunksPerRow);
-      const int row = rem / S::kBChunksPerRow, ch = rem % S::kBChunksPerRow;
-      b_on[u] = i < S::kBCopies;
-      b_v1[u] = v == 0;
-      b_row[u] = row;
-      b_src[u] = row * R + ch * (S::kBChunkBytes / 2);
-      b_dst[u] = v * S::kBVersion + row * S::kBStride + ch * 16;
-    }
-#pragma unroll
-    for (int u = 0; u < S::kAPerThread; ++u) {
-      const int i = tid + u * kDtThreads;
-      const int v = i / (R * (kDtRows / 8)), rem = i % (R * (kDtRows / 8));
-      const int k = rem / (kDtRows / 8), ch = rem % (kDtRows / 8);
-      a_on[u] = i < S::kACopies;
-      a_v1[u] = v == 0;
-      a_k[u] = k;
-      a_col[u] = ch * 8;
-      a_dst[u] = v * S::kAVersion + k * kDtAStride + ch * 16;
-    }
-  }
-};
+// hi = bf16(a - b) and lo = (a - b) - hi, exactly, for two bf16 pairs: Knuth's TwoSum of a and -b
+// in bf16 arithmetic with round-to-nearest (the rounding error of a sum is itself representable,
+// and these six operations recover it without a wider format).
+__device__ __forceinline__ void split_diff(uint32_t a, uint32_t b, uint32_t& hi, uint32_t& lo) {
+  hi = bf2_sub(a, b);
+  const uint32_t bv = bf2_sub(hi, a);   // the part of -b that hi holds
+  const uint32_t av = bf2_sub(hi, bv);  // the part of a that hi holds
+  lo = bf2_sub(bf2_sub(a, av), bf2_add(b, bv));
+}
 
 // The item a run of steps belongs to, cached while the run stays in one segment.
 struct SegCache {
@@ -151,62 +141,74 @@ struct SegCache {
   }
 };
 
-// Issue the copies of step x (version 1 then version 0) into a stage.
+// Issue the copies of step x (version 1 then version 0) into a stage. Copy i of the step goes
+// to thread i % 256: for the B side version i / (rows * chunks per row), then row and chunk; for
+// the A side version, rank row and 16-byte chunk.
 template <int R>
-__device__ __forceinline__ void load_step(const CopyPlan<R>& cp, const SegCache& sc, int x, uint32_t stage) {
+__device__ __forceinline__ void load_step(const SegCache& sc, int x, uint32_t stage) {
   using S = DtShape<R>;
+  const int tid = threadIdx.x;
   const int row0 = (x - sc.step0) * kDtRows;
   if (sc.side == 0) {
     const size_t blk = static_cast<size_t>(row0) * R;
 #pragma unroll
     for (int u = 0; u < S::kBPerThread; ++u) {
-      if (!cp.b_on[u]) continue;
-      const bool ok = row0 + cp.b_row[u] < sc.len;
-      const __nv_bfloat16* src = (cp.b_v1[u] ? sc.p1 : sc.p0) + (ok ? blk + cp.b_src[u] : 0);
+      const int i = tid + u * kDtThreads;
+      if (S::kBCopies % kDtThreads != 0 && i >= S::kBCopies) continue;
+      const int v = i / (kDtRows * S::kBChunksPerRow), rem = i % (kDtRows * S::kBChunksPerRow);
+      const int row = rem / S::kBChunksPerRow, ch = rem % S::kBChunksPerRow;
+      const bool ok = row0 + row < sc.len;
+      const __nv_bfloat16* src =
+          (v == 0 ? sc.p1 : sc.p0) + (ok ? blk + row * R + ch * (S::kBChunkBytes / 2) : 0);
+      const uint32_t dst = stage + v * S::kBVersion + row * S::kBStride + ch * 16;
       if constexpr (S::kBChunkBytes == 16)
-        cp_async16(stage + cp.b_dst[u], src, ok);
+        cp_async16(dst, src, ok);
       else
-        cp_async8(stage + cp.b_dst[u], src, ok);
+        cp_async8(dst, src, ok);
     }
   } else {
 #pragma unroll
     for (int u = 0; u < S::kAPerThread; ++u) {
-      if (!cp.a_on[u]) continue;
-      const int c = row0 + cp.a_col[u];
+      const int i = tid + u * kDtThreads;
+      if (S::kACopies % kDtThreads != 0 && i >= S::kACopies) continue;
+      const int v = i / (R * (kDtRows / 8)), rem = i % (R * (kDtRows / 8));
+      const int k = rem / (kDtRows / 8), ch = rem % (kDtRows / 8);
+      const int c = row0 + ch * 8;
       const bool ok = c < sc.len;  // the input width is a multiple of 8: a chunk is in or out
-      const __nv_bfloat16* src = (cp.a_v1[u] ? sc.p1 : sc.p0) + (ok ? static_cast<size_t>(cp.a_k[u]) * sc.len + c : 0);
-      cp_async16(stage + cp.a_dst[u], src, ok);
+      const __nv_bfloat16* src = (v == 0 ? sc.p1 : sc.p0) + (ok ? static_cast<size_t>(k) * sc.len + c : 0);
+      cp_async16(stage + v * S::kAVersion + k * kDtAStride + ch * 16, src, ok);
     }
   }
 }
 
 // This warp's 16-row slice of a staged step into its Gram accumulators.
 template <int R>
-__device__ __forceinline__ void mma_step(int side, uint32_t stage, float (&acc)[DtShape<R>::kPairs][2][4]) {
+__device__ __forceinline__ void mma_slice(int side, uint32_t stage, int row0,
+                                          float (&acc)[DtShape<R>::kPairs][2][4]) {
   using S = DtShape<R>;
   constexpr int RP = S::RP;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31;
   const int m = lane >> 3, i = lane & 7;
   uint32_t f1[4], f0[4];  // fragments of version 1 and version 0: {m0, m1, m2, m3} (RP = 8: m0, m2)
   if (side == 0) {
     // X[o][f] rows: matrix m covers rows k0 + (m >> 1) * 8 .. and features (m & 1) * 8 ..
     if constexpr (RP == 16) {
-      const uint32_t off = (warp * 16 + (m >> 1) * 8 + i) * S::kBStride + (m & 1) * 16;
+      const uint32_t off = (row0 + (m >> 1) * 8 + i) * S::kBStride + (m & 1) * 16;
       ldsm_x4_t(stage + off, f1[0], f1[1], f1[2], f1[3]);
       ldsm_x4_t(stage + S::kBVersion + off, f0[0], f0[1], f0[2], f0[3]);
     } else {
-      const uint32_t off = (warp * 16 + (m & 1) * 8 + i) * S::kBStride;
+      const uint32_t off = (row0 + (m & 1) * 8 + i) * S::kBStride;
       ldsm_x2_t(stage + off, f1[0], f1[2]);
       ldsm_x2_t(stage + S::kBVersion + off, f0[0], f0[2]);
     }
   } else {
     // Xt[f][c] rows: matrix m covers features (m & 1) * 8 .. and columns k0 + (m >> 1) * 8 ..
     if constexpr (RP == 16) {
-      const uint32_t off = ((m & 1) * 8 + i) * kDtAStride + (warp * 16 + (m >> 1) * 8) * 2;
+      const uint32_t off = ((m & 1) * 8 + i) * kDtAStride + (row0 + (m >> 1) * 8) * 2;
       ldsm_x4(stage + off, f1[0], f1[1], f1[2], f1[3]);
       ldsm_x4(stage + S::kAVersion + off, f0[0], f0[1], f0[2], f0[3]);
     } else {
-      const uint32_t off = i * kDtAStride + (warp * 16 + (m & 1) * 8) * 2;
+      const uint32_t off = i * kDtAStride + (row0 + (m & 1) * 8) * 2;
       ldsm_x2(stage + off, f1[0], f1[2]);
       ldsm_x2(stage + S::kAVersion + off, f0[0], f0[2]);
     }
@@ -229,14 +231,20 @@ __device__ __forceinline__ void mma_step(int side, uint32_t stage, float (&acc)[
       blk[1][r + 1] = 0u;
     }
   }
-  int p = 0;
 #pragma unroll
-  for (int I = 0; I < S::kBlocks; ++I)
+  for (int p = 0; p < S::kPairs; ++p) {
+    const int I = pair_I<RP>(p), J = pair_J<RP>(p);
+    mma16816(acc[p][0], blk[I], blk[J][0], blk[J][2]);
+    mma16816(acc[p][1], blk[I], blk[J][1], blk[J][3]);
+  }
+}
+
+// This warp's slices of a staged step.
+template <int R>
+__device__ __forceinline__ void mma_step(int side, uint32_t stage, float (&acc)[DtShape<R>::kPairs][2][4]) {
+  const int warp = threadIdx.x >> 5;
 #pragma unroll
-    for (int J = I; J < S::kBlocks; ++J, ++p) {
-      mma16816(acc[p][0], blk[I], blk[J][0], blk[J][2]);
-      mma16816(acc[p][1], blk[I], blk[J][1], blk[J][3]);
-    }
+  for (int sl = 0; sl < kDtSlices; ++sl) mma_slice<R>(side, stage, (warp * kDtSlices + sl) * 16, acc);
 }
 
 template <int R>
@@ -255,8 +263,6 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
     reinterpret_cast<uint4*>(dt_smem)[i] = make_uint4(0u, 0u, 0u, 0u);
   __syncthreads();
 
-  CopyPlan<R> cp;
-  cp.init(threadIdx.x);
   float acc[S::kPairs][2][4];
 #pragma unroll
   for (int p = 0; p < S::kPairs; ++p)
@@ -270,7 +276,7 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
   auto issue = [&]() {
     if (lx < x1) {
       lc.at(a, lx);
-      load_step<R>(cp, lc, lx, stage0 + ((lx - x0) % kDtStages) * S::kStage);
+      load_step<R>(lc, lx, stage0 + ((lx - x0) % kDtStages) * S::kStage);
     }
     cp_async_commit();  // empty groups keep the count uniform
     ++lx;
@@ -318,13 +324,18 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
   cp_async_wait<0>();
 }
 
+// One block per item: the segment's slots summed in CTA order, GB and GA assembled from the
+// [hi | lo | base] Grams (fp32: sums of at most four entries), then tr(GB GA) and the parameter
+// distance in fp64.
 template <int R>
 __global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_constant__ DriftTcArgs a,
                                                              const float* __restrict__ slots,
                                                              float* __restrict__ out_sq) {
   using S = DtShape<R>;
   constexpr int RP = S::RP;
+  constexpr int r2 = 2 * R;
   __shared__ float g[2][S::kSlotFloats];
+  __shared__ float gb[r2][r2 + 1], ga[r2][r2 + 1];
   __shared__ double red[2][8];
   const int item = blockIdx.x;
   for (int side = 0; side < 2; ++side) {
@@ -333,21 +344,34 @@ __global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_consta
     const int b_lo = static_cast<int>(((s0 + 1) * a.grid - 1) / a.total_steps);
     const int b_hi = static_cast<int>(((s1 + 1) * a.grid - 1) / a.total_steps);
     for (int e = threadIdx.x; e < S::kSlotFloats; e += 256) {
+      const float* p = slots + static_cast<size_t>(b_lo + seg) * S::kSlotFloats + e;
       float v = 0.f;
-      for (int bb = b_lo; bb <= b_hi; ++bb) v += slots[static_cast<size_t>(bb + seg) * S::kSlotFloats + e];
+      int bb = b_lo;
+      for (; bb + 4 <= b_hi + 1; bb += 4, p += 4 * S::kSlotFloats) {  // four loads in flight
+        const float x0 = p[0], x1 = p[S::kSlotFloats], x2 = p[2 * S::kSlotFloats],
+                    x3 = p[3 * S::kSlotFloats];
+        v += x0;
+        v += x1;
+        v += x2;
+        v += x3;
+      }
+      for (; bb <= b_hi; ++bb, p += S::kSlotFloats) v += *p;
       g[side][e] = v;
     }
   }
   __syncthreads();
-  // entry (f1, f2) of a side's symmetric feature Gram from its block-upper triangle
-  auto G = [&](int side, int f1, int f2) -> double {
+  // entry (f1, f2) of a side's symmetric feature Gram from its accumulated block pairs
+  auto G = [&](int side, int f1, int f2) -> float {
     int I = f1 >> 4, J = f2 >> 4;
     if (I > J) {
-      const int t = f1; f1 = f2; f2 = t;
-      I = f1 >> 4; J = f2 >> 4;
+      const int t = f1;
+      f1 = f2;
+      f2 = t;
+      I = f1 >> 4;
+      J = f2 >> 4;
     }
-    const int p = I * S::kBlocks - I * (I - 1) / 2 + (J - I);
-    return static_cast<double>(g[side][p * 256 + (f1 & 15) * 16 + (f2 & 15)]);
+    const int p = pair_of<RP>(I, J);
+    return p < 0 ? 0.f : g[side][p * 256 + (f1 & 15) * 16 + (f2 & 15)];
   };
   // <d_i, d_j>, <d_i, base_j>, <base_i, base_j> with d = hi + lo; features hi_i = i,
   // lo_i = RP + i, base_i = 2 RP + i
@@ -356,23 +380,20 @@ __global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_consta
   };
   auto db = [&](int s, int i, int j) { return G(s, i, 2 * RP + j) + G(s, RP + i, 2 * RP + j); };
   auto bb = [&](int s, int i, int j) { return G(s, 2 * RP + i, 2 * RP + j); };
-  constexpr int r = R, r2 = 2 * R;
+  for (int idx = threadIdx.x; idx < r2 * r2; idx += 256) {
+    const int p = idx / r2, q = idx % r2;
+    // GB over [B1 - B0 | B0]; GA over [A1 ; A1 - A0]: base first on the A side
+    gb[p][q] = p < R ? (q < R ? dd(0, p, q) : db(0, p, q - R)) : (q < R ? db(0, q, p - R) : bb(0, p - R, q - R));
+    ga[p][q] = p < R ? (q < R ? bb(1, p, q) : db(1, q - R, p)) : (q < R ? db(1, p - R, q) : dd(1, p - R, q - R));
+  }
+  __syncthreads();
   double t = 0.0, par = 0.0;
   for (int idx = threadIdx.x; idx < r2 * r2; idx += 256) {
-    const int p = idx / r2, q = idx - p * r2;
-    // GB over [B1 - B0 | B0]; GA over [A1 ; A1 - A0]: base first on the A side
-    double gb, ga;
-    if (p < r && q < r) gb = dd(0, p, q);
-    else if (p < r) gb = db(0, p, q - r);
-    else if (q < r) gb = db(0, q, p - r);
-    else gb = bb(0, p - r, q - r);
-    if (p < r && q < r) ga = bb(1, p, q);
-    else if (p < r) ga = db(1, q - r, p);
-    else if (q < r) ga = db(1, p - r, q);
-    else ga = dd(1, p - r, q - r);
-    t += gb * ga;  // both Grams are symmetric: tr(GB GA) = sum_pq GB[p][q] GA[p][q]
-    if (p == q && p < r) par += dd(0, p, p) + dd(1, p, p);
+    const int p = idx / r2, q = idx % r2;
+    t += static_cast<double>(gb[p][q]) * static_cast<double>(ga[p][q]);  // both symmetric
   }
+  if (threadIdx.x < R)
+    par = static_cast<double>(gb[threadIdx.x][threadIdx.x]) + static_cast<double>(ga[R + threadIdx.x][R + threadIdx.x]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     t += __shfl_xor_sync(0xffffffffu, t, o);
