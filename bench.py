@@ -44,7 +44,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu --set full
 # capture of the kernel as it now stands, at the full launch size of the 7B-shape 16K workload
 # (profiles/gemm_gateup_swiglu_7b16k.md). An entry is removed whenever its kernel changes.
-NCU_TRAFFIC_BYTES = {"gemm_gateup_swiglu": 2.957646e9 + 0.614966e9}
+NCU_TRAFFIC_BYTES = {}
 
 
 def load_peaks():
@@ -141,25 +141,22 @@ def job_throughput(units_per_rank: float, steps: int, world: int, max_ms: float)
 
 # ----------------------------------------------------------------------------- workload
 def algorithmic_work(cfg, lc, n):
-    """Algorithmic FLOPs per kernel kind for one recomputed layer over n tokens (and bytes)."""
+    """Algorithmic FLOPs per kernel kind for one recomputed layer over n tokens (and bytes).
+
+    Each projection counts its base product, the adapter's down products x A^T (2 n r in per
+    adapted module) and its up products (2 n r out), all computed in the same launch.
+    """
     h, f, qd, kvd, r = cfg.hidden, cfg.ffn, cfg.n_q_heads * cfg.head_dim, cfg.n_kv_heads * cfg.head_dim, lc.rank
     ad = lambda m: m in lc.modules
-    up = lambda m, out: 2 * n * r * out if ad(m) else 0
+    lora = lambda m, i, out: 2 * n * r * (i + out) if ad(m) else 0
     flops = {
-        "gemm_qkv_rope_paged": 2 * n * h * (qd + 2 * kvd) + up("q", qd) + up("k", kvd) + up("v", kvd),
-        "gemm_o_resid": 2 * n * qd * h + up("o", h),
-        "gemm_gateup_swiglu": 2 * n * h * 2 * f + up("gate", f) + up("up", f),
-        "gemm_down_resid": 2 * n * f * h + up("down", h),
+        "gemm_qkv_rope_paged": 2 * n * h * (qd + 2 * kvd) + lora("q", h, qd) + lora("k", h, kvd) + lora("v", h, kvd),
+        "gemm_o_resid": 2 * n * qd * h + lora("o", qd, h),
+        "gemm_gateup_swiglu": 2 * n * h * 2 * f + lora("gate", h, f) + lora("up", h, f),
+        "gemm_down_resid": 2 * n * f * h + lora("down", f, h),
         "attn_prefill_paged": 4 * cfg.n_q_heads * cfg.head_dim * n * (n + 1) // 2,
     }
-    byts = {"rmsnorm": 2 * (2 * n * h * 2),   # two norms, read + write bf16
-            # down products x A^T (2 n r in_m FLOP, HBM-bound): each distinct input read once
-            # (the q/k/v and the gate/up modules share theirs), a bf16 hi/lo pair of r columns
-            # written per adapted module
-            "gemm_lora_down": 2 * n * (h * any(ad(m) for m in ("q", "k", "v"))
-                                       + h * any(ad(m) for m in ("gate", "up"))
-                                       + qd * ad("o") + f * ad("down"))
-                              + n * 2 * r * 2 * sum(ad(m) for m in ("q", "k", "v", "o", "gate", "up", "down"))}
+    byts = {"rmsnorm": 2 * (2 * n * h * 2)}   # two norms, read + write bf16
     return flops, byts
 
 

@@ -4,9 +4,10 @@
 // Executable restart (Section 4.2): for each layer l of the union of the
 // requests' windows, the rows of every request whose window covers l form one
 // activation matrix, and the layer runs as
-//   rmsnorm -> [LoRA down] -> QKV GEMM (+LoRA up, bias, RoPE, q out, K/V to pages)
-//   -> causal GQA attention over the pages -> [LoRA down] -> O GEMM (+residual)
-//   -> rmsnorm -> [LoRA down] -> gate|up GEMM (+SwiGLU) -> [LoRA down] -> down GEMM (+residual)
+//   rmsnorm -> QKV GEMM (+LoRA down and up, bias, RoPE, q out, K/V to pages)
+//   -> causal GQA attention over the pages -> O GEMM (+LoRA, residual)
+//   -> rmsnorm -> gate|up GEMM (+LoRA, SwiGLU) -> down GEMM (+LoRA, residual)
+// where each GEMM launch computes its own unmerged adapter term (Eq. S3).
 // Then the last prefix row of each request that asks for it continues through
 // layers e..N-1 against the historical cache (first-step state, Section S2.1).
 #include "../../include/crf.h"
@@ -43,12 +44,12 @@ struct crf_ctx {
 namespace {
 
 enum ProfKind : int {
-  kPQkv, kPO, kPGateUp, kPDown, kPLoraDown, kPAttn, kPNorm, kPEmbed, kPRope, kPCopy,
+  kPQkv, kPO, kPGateUp, kPDown, kPAttn, kPNorm, kPEmbed, kPRope, kPCopy,
   kPDecode, kPLmHead, kPKl, kPDrift, kPCheck, kPNumKinds
 };
 const char* const kProfNames[kPNumKinds] = {
     "gemm_qkv_rope_paged", "gemm_o_resid", "gemm_gateup_swiglu", "gemm_down_resid",
-    "gemm_lora_down", "attn_prefill_paged", "rmsnorm", "embed_gather", "rope_table", "row_copy",
+    "attn_prefill_paged", "rmsnorm", "embed_gather", "rope_table", "row_copy",
     "tail_decode", "lm_head", "kl_reduce", "drift_gram", "page_check"};
 
 // Brackets the launches issued in its lifetime with two events on `st` when
@@ -166,24 +167,16 @@ struct Plan {
   int max_n = 0;
   int dec_rows = 0;   // requests asking for the first-step state
   int splits = 1;
-  size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_bx, off_rope;
+  size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_rope;
   size_t off_dx0, off_dec;  // decode: bf16 starting rows, fp32 scratch
   size_t off_abort, off_ptab;  // the call's abort word; the page-check table (ptab_slots ints)
+  // the projections' XA ready words: 4 launches x ceil(M / 256) row blocks per layer, laid out
+  // after the abort word so one clear at the start of the call covers both
+  size_t flag_words = 0;
   uint32_t ptab_slots = 2;
   size_t dec_bytes;
   size_t total;
 };
-
-// output rows of module m (q, k, v, o, gate, up, down) and their sum
-int module_rows(const Dims& D, int m) {
-  const int r[7] = {D.qd, D.kvd, D.kvd, D.h, D.f, D.f, D.h};
-  return r[m];
-}
-int module_rows_total(const Dims& D) {
-  int t = 0;
-  for (int m = 0; m < 7; ++m) t += module_rows(D, m);
-  return t;
-}
 
 // decode attention partials: one per chunk of the longest prefix
 int dec_splits(int max_n) { return decode_attention_splits(max_n); }
@@ -222,13 +215,19 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_o = take(M * D.qd * 2);
   p.off_mlp = take(M * D.f * 2);
   p.off_xa = take(M * kXaCols * 2);
-  p.off_bx = take(static_cast<size_t>(module_rows_total(D)) * kBxCols * 2);
   p.off_rope = take(static_cast<size_t>(p.max_n) * (D.d / 2) * sizeof(float2));
   p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
   long ids = 0;
   for (int i = 0; i < n_req; ++i) ids += (reqs[i].n_tokens + kPage - 1) / kPage;
   p.ptab_slots = ptab_slots_for(ids);
-  p.off_abort = take(sizeof(int));
+  int layers = 0;
+  for (int l = 0; l < D.N; ++l) {
+    bool any = false;
+    for (int i = 0; i < n_req; ++i) any |= reqs[i].s <= l && l < reqs[i].e;
+    layers += any ? 1 : 0;
+  }
+  p.flag_words = static_cast<size_t>(layers) * 4 * ((p.M + 255) / 256);
+  p.off_abort = take((1 + p.flag_words) * sizeof(int));
   p.off_ptab = take(static_cast<size_t>(p.ptab_slots) * sizeof(int));
   p.splits = dec_splits(p.max_n);
   // decode scratch per row, fp32: x, xn, x1, q, k, v, o, xa (3 slots), gu, m, attention partials
@@ -279,36 +278,10 @@ struct LayerCtx {
   const Plan* plan;
   float scale;
   const int* abort;  // the call's abort word (set by the page-table check)
+  int* xa_flags;     // this layer's XA ready words (4 projections x row blocks), zero
 };
 
 bool adapted(const crf_adapter* a, int m) { return (a->dims.module_mask >> m) & 1u; }
-
-// LoRA down product of `X` for the listed modules into XA (16 columns per module).
-cudaError_t lora_down(const LayerCtx& c, int l, const void* X, int M, int K, const int* mods, int nm,
-                      __nv_bfloat16* XA) {
-  ProfScope ps(c.ctx, kPLoraDown, c.st);
-  GemmDesc g;
-  std::memset(&g, 0, sizeof(g));
-  g.A = X;
-  g.M = M;
-  g.K = K;
-  g.lda = K;
-  g.ngroups = 1;
-  g.nseg = nm;
-  for (int s = 0; s < nm; ++s) {
-    g.B[s] = c.ad->A[l * 7 + mods[s]];
-    g.B_rows[s] = c.ad->dims.rank;
-    g.ldb[s] = K;
-  }
-  g.group_cols[0] = nm * kRankPad;
-  g.epi = kEpiScaleBf16;
-  g.scale = c.scale;
-  g.out = XA;
-  g.ldo = kXaCols;
-  g.status = c.ctx->status_dev;
-  g.abort = c.abort;
-  return launch_gemm(g, nm * kRankPad, c.ctx->num_sms, c.st);
-}
 
 crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_bfloat16* X_out,
                      int M, const ReqTable& rt) {
@@ -323,30 +296,25 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
   auto* MLP = reinterpret_cast<__nv_bfloat16*>(ws + p.off_mlp);
   auto* XA = reinterpret_cast<__nv_bfloat16*>(ws + p.off_xa);
   auto* rope = reinterpret_cast<const float2*>(ws + p.off_rope);
-  const int rank = c.ad->dims.rank;
-
-  // BX = [B | B] rows of every module of layer l under its XA slot (up follows gate when both
-  // are adapted, so one K block carries the stacked gate|up pair)
-  __nv_bfloat16* BX[7];
-  {
-    auto* bx = reinterpret_cast<__nv_bfloat16*>(ws + p.off_bx);
-    BextDesc bd{};
-    bool any = false;
-    for (int m = 0; m < 7; ++m) {
-      BX[m] = bx;
-      bd.B[m] = adapted(c.ad, m) ? static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + m]) : nullptr;
-      bd.out[m] = bx;
-      bd.rows[m] = module_rows(D, m);
-      bd.col_off[m] = (m == CRF_MOD_UP && adapted(c.ad, CRF_MOD_GATE)) ? 32 : 0;
-      bx += static_cast<size_t>(bd.rows[m]) * kBxCols;
-      any |= adapted(c.ad, m);
+  // one ready word per 256-row block for each of the layer's four projection launches
+  int* flags = c.xa_flags;
+  const int flag_stride = (p.M + 255) / 256;
+  // the unmerged adapter of the listed modules, slots in list order (Eq. S3)
+  auto set_lora = [&](GemmDesc& g, const int* mods, int nm, int* slot_of) {
+    g.n_slots = 0;
+    for (int s = 0; s < nm; ++s) {
+      slot_of[s] = -1;
+      if (!adapted(c.ad, mods[s])) continue;
+      slot_of[s] = g.n_slots;
+      g.LA[g.n_slots++] = c.ad->A[l * 7 + mods[s]];
     }
-    bd.n = 7;
-    if (any) {
-      ProfScope ps(c.ctx, kPLoraDown, c.st);
-      CRF_CUDA(launch_lora_bext(bd, rank, c.st));
-    }
-  }
+    if (!g.n_slots) return;
+    g.XA = XA;
+    g.rank = c.ad->dims.rank;
+    g.scale = c.scale;
+    g.xa_flags = flags;
+    flags += flag_stride;
+  };
 
   // 1. RMSNorm before attention
   {
@@ -356,10 +324,6 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
 
   // 2-3. q/k/v projections (+ LoRA, bias, RoPE; K/V into the pages of layer l)
   {
-    int mods[3], nm = 0;
-    for (int m = 0; m < 3; ++m)
-      if (adapted(c.ad, m)) mods[nm++] = m;
-    if (nm) CRF_CUDA(lora_down(c, l, XN, M, D.h, mods, nm, XA));
     GemmDesc g;
     std::memset(&g, 0, sizeof(g));
     g.A = XN;
@@ -368,23 +332,24 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.lda = D.h;
     g.ngroups = 3;
     g.nseg = 1;
+    const int mods[3] = {CRF_MOD_Q, CRF_MOD_K, CRF_MOD_V};
+    int slot[3];
+    set_lora(g, mods, 3, slot);
     const int rows[3] = {D.qd, D.kvd, D.kvd};
-    int slot = 0;
     for (int m = 0; m < 3; ++m) {
       g.B[m] = w.W[m];
       g.B_rows[m] = rows[m];
       g.ldb[m] = D.h;
       g.group_cols[m] = rows[m];
-      if (adapted(c.ad, m)) {
-        g.BX[m] = BX[m];
+      if (slot[m] >= 0) {
+        g.BL[m] = c.ad->B[l * 7 + m];
+        g.bl_slot[m] = slot[m];
         g.ext_on[m] = 1;
         g.ext_steps[m] = 2;
-        g.xa_base[m] = 32 * slot++;
+        g.xa_base[m] = 32 * slot[m];
       }
       g.bias[m] = D.bias ? w.bias[m] : nullptr;
     }
-    g.XA = XA;
-    g.ldxa = kXaCols;
     g.epi = kEpiQkv;
     g.rope = rope;
     g.head_dim = D.d;
@@ -397,7 +362,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.status = c.ctx->status_dev;
     g.abort = c.abort;
     ProfScope ps(c.ctx, kPQkv, c.st);
-    CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
+    CRF_CUDA(launch_gemm(g, c.ctx->num_sms, c.st));
   }
 
   // 4. causal GQA attention over the pages of layer l
@@ -421,12 +386,6 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
 
   // 5-6. output projection + residual: X1 = X_in + O W_o^T (+ LoRA)
   auto proj_resid = [&](int m, const void* A, int K, const void* resid, void* out) -> cudaError_t {
-    const bool lo = adapted(c.ad, m);
-    if (lo) {
-      const int mods[1] = {m};
-      cudaError_t e = lora_down(c, l, A, M, K, mods, 1, XA);
-      if (e != cudaSuccess) return e;
-    }
     GemmDesc g;
     std::memset(&g, 0, sizeof(g));
     g.A = A;
@@ -439,10 +398,11 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.B_rows[0] = D.h;
     g.ldb[0] = K;
     g.group_cols[0] = D.h;
-    if (lo) {
-      g.XA = XA;
-      g.ldxa = kXaCols;
-      g.BX[0] = BX[m];
+    int slot[1];
+    set_lora(g, &m, 1, slot);
+    if (slot[0] >= 0) {
+      g.BL[0] = c.ad->B[l * 7 + m];
+      g.bl_slot[0] = 0;
       g.ext_on[0] = 1;
       g.ext_steps[0] = 2;
       g.xa_base[0] = 0;
@@ -455,7 +415,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.status = c.ctx->status_dev;
     g.abort = c.abort;
     ProfScope ps(c.ctx, m == CRF_MOD_O ? kPO : kPDown, c.st);
-    return launch_gemm(g, 256, c.ctx->num_sms, c.st);
+    return launch_gemm(g, c.ctx->num_sms, c.st);
   };
   CRF_CUDA(proj_resid(CRF_MOD_O, O, D.qd, X_in, X1));
 
@@ -467,10 +427,6 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
 
   // 8-9. gate|up projections with SwiGLU epilogue
   {
-    int mods[2], nm = 0;
-    for (int m = CRF_MOD_GATE; m <= CRF_MOD_UP; ++m)
-      if (adapted(c.ad, m)) mods[nm++] = m;
-    if (nm) CRF_CUDA(lora_down(c, l, XN, M, D.h, mods, nm, XA));
     GemmDesc g;
     std::memset(&g, 0, sizeof(g));
     g.A = XN;
@@ -479,28 +435,32 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     g.lda = D.h;
     g.ngroups = 1;
     g.nseg = 2;
+    const int mods[2] = {CRF_MOD_GATE, CRF_MOD_UP};
+    int slot[2];
+    set_lora(g, mods, 2, slot);
     for (int s = 0; s < 2; ++s) {
-      const int m = CRF_MOD_GATE + s;
-      g.B[s] = w.W[m];
+      g.B[s] = w.W[mods[s]];
       g.B_rows[s] = D.f;
       g.ldb[s] = D.h;
-      g.BX[s] = BX[m];  // all-zero rows for a module without adapter
+      if (slot[s] >= 0) {
+        g.BL[s] = c.ad->B[l * 7 + mods[s]];
+        g.bl_slot[s] = slot[s];
+      }
     }
-    if (nm) {
+    if (g.n_slots) {
+      // one K block carries both slots; each segment's B rows sit under its own slot only
       g.ext_on[0] = 1;
-      g.ext_steps[0] = 2 * nm;
+      g.ext_steps[0] = 2 * g.n_slots;
       g.xa_base[0] = 0;
     }
     g.group_cols[0] = D.f;
-    g.XA = XA;
-    g.ldxa = kXaCols;
     g.epi = kEpiSwiGLU;
     g.out = MLP;
     g.ldo = D.f;
     g.status = c.ctx->status_dev;
     g.abort = c.abort;
     ProfScope ps(c.ctx, kPGateUp, c.st);
-    CRF_CUDA(launch_gemm(g, 256, c.ctx->num_sms, c.st));
+    CRF_CUDA(launch_gemm(g, c.ctx->num_sms, c.st));
   }
 
   // 10-11. down projection + residual: X_out = X1 + MLP W_d^T (+ LoRA)
@@ -702,13 +662,14 @@ bool device_page_check() {
   return !(e && e[0] == '1');
 }
 
-// Opens a call on `st`: clears the call's abort word and checks every page id of the listed
-// tables (in [0, num_pages), no page twice). Enqueued work only: the host does not wait.
+// Opens a call on `st`: clears the call's abort word and the `flag_words` ready words after it,
+// and checks every page id of the listed tables (in [0, num_pages), no page twice). Enqueued
+// work only: the host does not wait.
 crf_status open_call(crf_ctx* ctx, const PageCheck& pc, int num_pages, uint8_t* ws, size_t off_abort,
-                     size_t off_ptab, uint32_t ptab_slots, cudaStream_t st) {
+                     size_t flag_words, size_t off_ptab, uint32_t ptab_slots, cudaStream_t st) {
   int* abort = reinterpret_cast<int*>(ws + off_abort);
   ProfScope ps(ctx, kPCheck, st, device_page_check() ? 1 : 0);
-  CRF_CUDA(cudaMemsetAsync(abort, 0, sizeof(int), st));
+  CRF_CUDA(cudaMemsetAsync(abort, 0, (1 + flag_words) * sizeof(int), st));
   if (!device_page_check()) return CRF_OK;
   int* table = reinterpret_cast<int*>(ws + off_ptab);
   CRF_CUDA(cudaMemsetAsync(table, 0xff, static_cast<size_t>(ptab_slots) * sizeof(int), st));
@@ -931,7 +892,8 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
       pc.pt[i] = reqs[i].page_table;
       pc.first[i + 1] = pc.first[i] + (reqs[i].n_tokens + kPage - 1) / kPage;
     }
-    s = open_call(ctx, pc, pool->num_pages, ws, plan.off_abort, plan.off_ptab, plan.ptab_slots, st);
+    s = open_call(ctx, pc, pool->num_pages, ws, plan.off_abort, plan.flag_words, plan.off_ptab,
+                  plan.ptab_slots, st);
     if (s != CRF_OK) return s;
   }
 
@@ -954,6 +916,7 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
       lmin = std::min(lmin, reqs[i].s);
       lmax = std::max(lmax, reqs[i].e);
     }
+  int layer_seq = 0;  // layers run so far: each owns a slice of the ready words
   for (int l = lmin; l < lmax; ++l) {
     std::vector<int> act;
     for (int i = 0; i < n_req; ++i)
@@ -1020,6 +983,8 @@ crf_status crf_recompute_window(crf_ctx* ctx, const crf_model* model, const crf_
       int b = in_buf >= 0 ? 1 - in_buf : 0;
       X_out = G[b];
     }
+    c.xa_flags = reinterpret_cast<int*>(ws + plan.off_abort) + 1 +
+                 static_cast<size_t>(layer_seq++) * 4 * ((plan.M + 255) / 256);
     s = run_layer(c, l, X_in, X_out, M, rt);
     if (s != CRF_OK) return s;
     for (int k = 0; k < rt.n; ++k) {
@@ -1133,7 +1098,7 @@ crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const crf_adapt
       pc.pt[i] = rows[i].page_table;
       pc.first[i + 1] = pc.first[i] + rows[i].pos / kPage + 1;
     }
-    s = open_call(ctx, pc, pool->num_pages, ws, sp.p.off_abort, sp.p.off_ptab, sp.p.ptab_slots, st);
+    s = open_call(ctx, pc, pool->num_pages, ws, sp.p.off_abort, 0, sp.p.off_ptab, sp.p.ptab_slots, st);
     if (s != CRF_OK) return s;
   }
   RowPositions rp{};

@@ -1,28 +1,33 @@
-// Persistent tcgen05 GEMM for sm_103a with fused LoRA-up and fused epilogues.
+// Persistent tcgen05 GEMM for sm_103a with the unmerged LoRA product and fused epilogues.
 //
-//   D[BM*PAIR x BN] = A[BM*PAIR x K] * B[BN x K]^T  (+ XA[. x 64] * BX[BN x 64]^T)
+//   D[256 x 256] = A[256 x K] * B[256 x K]^T  (+ XA[256 x 64] * BL^T)
 //
-// PAIR = 2 (the projection GEMMs): a cluster of two CTAs on one TPC works on a
-// 256 x 256 tile with cta_group::2 MMAs. Each CTA stages its own 128 rows of A
-// and its own half of the B rows, so the operand bytes each SM pulls through L2
-// per FLOP are two thirds of the single-CTA 128 x 256 tile's. The even CTA
-// issues the MMAs; both CTAs hold 128 accumulator lanes in their own TMEM and
-// drain them through the same epilogue. PAIR = 1: one CTA per tile (the narrow
-// LoRA-down products).
+// A cluster of two CTAs on one TPC works on a 256 x 256 tile with cta_group::2 MMAs. Each CTA
+// stages its own 128 rows of A and its own half of the B rows, so the operand bytes each SM
+// pulls through L2 per FLOP are two thirds of the single-CTA 128 x 256 tile's. The even CTA
+// issues the MMAs; both CTAs hold 128 accumulator lanes in their own TMEM and drain them through
+// the same epilogue.
 //
-// Per CTA: warp 0 issues TMA loads into a STAGES-deep shared-memory ring, warp 1
-// owns TMEM (two accumulators, so the epilogue of tile i overlaps the main loop
-// of tile i+1) and, in the MMA-issuing CTA, issues tcgen05.mma from one thread;
-// warps 2..5 drain the accumulator (one TMEM lane = one output row per thread)
-// through the fused epilogue. Operands are bf16, K-major, staged with 128-byte
-// swizzle; accumulation is fp32 in TMEM.
+// Per CTA: warp 0 loads operands into a STAGES-deep shared-memory ring (TMA, issued by one lane),
+// warp 1 owns TMEM (two accumulators, so the epilogue of tile i overlaps the main loop of tile
+// i+1) and, in the MMA-issuing CTA, issues tcgen05.mma from one thread; warps 2..5 drain the
+// accumulator (one TMEM lane = one output row per thread) through the fused epilogue. Operands
+// are bf16, K-major, staged with 128-byte swizzle; accumulation is fp32 in TMEM.
 //
-// The unmerged adapter term (alpha/r) (x A^T) B^T of every adapted projection
-// (Eq. S3 with W = W0 + (alpha/r) B A) enters as one extra 64-wide K block per
-// tile: A side = the scaled down product of the tile's rows stored as a bf16
-// pair [hi | lo] per module (16 + 16 columns), B side = rows of BX = [B | B]
-// placed under that module's columns (zeros elsewhere), so one K block serves
-// up to two stacked modules and the two halves of a pair alike.
+// The adapter term (alpha/r) (x A^T) B^T of every adapted projection (Eq. S3, W = W0 + (alpha/r)
+// B A kept unmerged) is computed in the same launch:
+//  - down tiles, one per 256-row block of A, form x A^T for the GEMM's adapted modules (N = 16
+//    per module, B operand = the LoRA A rows) and store it, scaled, as a bf16 pair [hi | lo]
+//    per module (16 + 16 columns of the XA buffer), then count themselves done in the row
+//    block's ready word;
+//  - every output tile of an adapted module adds one 64-wide K block: A side = the XA columns
+//    of its row block (loaded once the ready word shows both CTAs of the down tile done), B side
+//    = the module's B rows, written into the stage by the loading warp under the K steps of the
+//    module's own slot (zeros under the other slot), so one K block serves two stacked modules
+//    and the two halves of a pair alike.
+// Down tiles are ordered one wave ahead of the first output tiles of their row block, so those
+// rarely wait; the wait is bounded like every other. The XA rows a down tile reads in are the
+// A rows its row block's output tiles read next, so they come from L2.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -44,7 +49,7 @@ struct GemmArgs {
   CUtensorMap tmA;
   CUtensorMap tmB[3];
   CUtensorMap tmXA;
-  CUtensorMap tmBX[3];
+  CUtensorMap tmLA[3];  // LoRA A of XA slot j: the down tiles' B operand
   int M, K, num_kb;
   int ngroups, nseg;
   int group_tiles[3];
@@ -53,6 +58,15 @@ struct GemmArgs {
   int ext_steps[3];   // per group: K = 16 steps of that block that carry data
   int xa_base[3];     // per group: first XA column of that block
   int row_tiles, total_n, total_tiles;
+  int n_slots;        // adapted modules (XA slots); 0: no down tiles
+  int down_n;         // N of a down tile: 16 per slot, two CTA halves of 16 x slots_per_cta
+  int down_lead;      // down tiles placed ahead of the first output tiles of their row block
+  const __nv_bfloat16* BL[3];  // adapter B of map index i, [b_rows[i], rank], or null
+  int bl_slot[3];
+  int b_rows[3];
+  int rank;
+  __nv_bfloat16* xa;
+  int* xa_flags;
   int epi;
   float scale;
   __nv_bfloat16* out;
@@ -73,15 +87,45 @@ struct GemmArgs {
 
 struct Tile {
   int m_blk, g, n_loc;
+  bool down;  // the row block's LoRA down product
 };
 
+// Output tiles run in bands of kRasterGroup column tiles over every row block (the band's B
+// rows stay in L2). With down tiles, band 0 carries them: the first `lead` down tiles, then per
+// row block m the down tile of m + lead followed by m's band-0 output tiles.
 __device__ __forceinline__ Tile decode_tile(int t, const GemmArgs& a) {
+  Tile r;
+  r.down = false;
+  r.g = 0;
+  r.n_loc = 0;
+  if (a.n_slots > 0) {
+    const int w0 = min(kRasterGroup, a.total_n);
+    const int lead = min(a.down_lead, a.row_tiles);
+    if (t < lead) {
+      r.down = true;
+      r.m_blk = t;
+      return r;
+    }
+    int u = t - lead;
+    const int g1 = a.row_tiles - lead;  // row blocks whose band-0 tiles follow a down tile
+    if (u < g1 * (w0 + 1)) {
+      r.m_blk = u / (w0 + 1);
+      const int i = u - r.m_blk * (w0 + 1);
+      if (i == 0) {
+        r.down = true;
+        r.m_blk += lead;
+        return r;
+      }
+      t = r.m_blk * w0 + (i - 1);  // the plain order's index of output tile (m, i - 1)
+    } else {
+      t = u - g1;  // the remaining band-0 tiles, then the later bands, in plain order
+    }
+  }
   const int band_tiles = a.row_tiles * kRasterGroup;
   const int band = t / band_tiles;
   const int idx = t - band * band_tiles;
   const int n0 = band * kRasterGroup;
   const int width = min(kRasterGroup, a.total_n - n0);
-  Tile r;
   r.m_blk = idx / width;
   int n = n0 + (idx - r.m_blk * width);
   int g = 0;
@@ -154,17 +198,16 @@ __device__ __forceinline__ bool row_lookup(const ReqTable& rt, int row, int& pos
   return false;
 }
 
-template <int BN>
+template <int BN, int EPI>
 __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl, uint32_t tacc,
                                               int row) {
   const bool row_ok = row < a.M;
   uint32_t r0[16], r1[16];
   float v[16], w[16];
 
-  if (a.epi == kEpiScaleBf16 || a.epi == kEpiResid) {
+  if constexpr (EPI == kEpiResid) {
     const int col0 = tl.n_loc * BN;
     const int ncols = a.group_cols[tl.g];
-    const bool resid = a.epi == kEpiResid;
     // residual chunk c + 16 is requested while chunk c is drained: its load latency overlaps
     auto load_resid = [&](int col, float (&dst)[16]) {
       const int n = min(16, ncols - col);
@@ -177,32 +220,18 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
       }
     };
     float wn[16];
-    if (resid && row_ok && col0 < ncols) load_resid(col0, w);
+    if (row_ok && col0 < ncols) load_resid(col0, w);
 #pragma unroll 1
     for (int c = 0; c < BN; c += 16) {
       tmem_ld16(tacc + c, r0);
-      const bool more = resid && row_ok && c + 16 < BN && col0 + c + 16 < ncols;
+      const bool more = row_ok && c + 16 < BN && col0 + c + 16 < ncols;
       if (more) load_resid(col0 + c + 16, wn);
       tmem_ld_wait();
       const int col = col0 + c;
       if (!row_ok || col >= ncols) continue;
-      const int n = min(16, ncols - col);
-      if (a.epi == kEpiScaleBf16) {
-        // hi = bf16(v), lo = bf16(v - hi): the pair carries the product to ~16 mantissa bits.
-        // Module slot j = col / 16 keeps hi at columns 32j.. and lo at 32j + 16..
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          v[j] = __uint_as_float(r0[j]) * a.scale;
-          w[j] = v[j] - __bfloat162float(__float2bfloat16_rn(v[j]));
-        }
-        store_bf16_n(a.out + (size_t)row * a.ldo + 2 * col + 16, w, n);
-        store_bf16_n(a.out + (size_t)row * a.ldo + 2 * col, v, n);
-        continue;
-      } else {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = w[j] + __uint_as_float(r0[j]);
-      }
-      store_bf16_n(a.out + (size_t)row * a.ldo + col, v, n);
+      for (int j = 0; j < 16; ++j) v[j] = w[j] + __uint_as_float(r0[j]);
+      store_bf16_n(a.out + (size_t)row * a.ldo + col, v, min(16, ncols - col));
       if (more) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) w[j] = wn[j];
@@ -211,7 +240,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
     return;
   }
 
-  if (a.epi == kEpiSwiGLU) {
+  if constexpr (EPI == kEpiSwiGLU) {
     constexpr int HALF = BN / 2;
     const int f0 = tl.n_loc * HALF;
     const int ffn = a.group_cols[0];
@@ -233,89 +262,282 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
     return;
   }
 
-  // kEpiQkv: group 0 = q, 1 = k, 2 = v; tiles are head-aligned (BN % head_dim == 0).
-  const int d = a.head_dim;
-  const int half = d >> 1;
-  int pos = 0;
-  const int32_t* pt = nullptr;
-  const bool have = row_ok && row_lookup(a.req, row, pos, pt);
-  const int g = tl.g;
-  const __nv_bfloat16* bias = a.bias[g];
-  __nv_bfloat16* dst_row = nullptr;
-  size_t head_stride = 0;
-  if (have) {
-    if (g == 0) {
-      dst_row = a.qbuf + (size_t)row * a.ldq;
-      head_stride = d;
-    } else {
-      const int page = checked_page(pt[pos / kPage], a.req.num_pages, a.status);
-      __nv_bfloat16* base = (g == 1) ? a.kpages : a.vpages;
-      dst_row = base + ((size_t)page * a.n_kv_heads * kPage + (pos % kPage)) * d;
-      head_stride = (size_t)kPage * d;
-    }
-  }
-  // Chunks of 16 rotation pairs outermost: a chunk's cos/sin (one row of the angle table,
-  // shared by every head of the tile) is loaded once, and the next chunk's is requested
-  // while this one is applied, so the table's load latency overlaps the TMEM drain.
-  const bool rot = have && g < 2;
-  const float4* rope4 = reinterpret_cast<const float4*>(a.rope + (size_t)pos * half);
-  float4 cs[8], csn[8];
-  if (rot) {
-#pragma unroll
-    for (int k = 0; k < 8; ++k) cs[k] = rope4[k];
-  }
-#pragma unroll 1
-  for (int i0 = 0; i0 < half; i0 += 16) {
-    const bool more = rot && i0 + 16 < half;
-    if (more) {
-#pragma unroll
-      for (int k = 0; k < 8; ++k) csn[k] = rope4[(i0 + 16) / 2 + k];
-    }
-#pragma unroll 1
-    for (int hh = 0; hh < BN / d; ++hh) {
-      const int head = (tl.n_loc * BN) / d + hh;
-      const int gcol = head * d;
-      tmem_ld16(tacc + hh * d + i0, r0);
-      tmem_ld16(tacc + hh * d + half + i0, r1);
-      tmem_ld_wait();
-      if (!have || gcol >= a.group_cols[g]) continue;
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        v[j] = __uint_as_float(r0[j]);
-        w[j] = __uint_as_float(r1[j]);
+  if constexpr (EPI == kEpiQkv) {
+    // kEpiQkv: group 0 = q, 1 = k, 2 = v; tiles are head-aligned (BN % head_dim == 0).
+    const int d = a.head_dim;
+    const int half = d >> 1;
+    int pos = 0;
+    const int32_t* pt = nullptr;
+    const bool have = row_ok && row_lookup(a.req, row, pos, pt);
+    const int g = tl.g;
+    const __nv_bfloat16* bias = a.bias[g];
+    __nv_bfloat16* dst_row = nullptr;
+    size_t head_stride = 0;
+    if (have) {
+      if (g == 0) {
+        dst_row = a.qbuf + (size_t)row * a.ldq;
+        head_stride = d;
+      } else {
+        const int page = checked_page(pt[pos / kPage], a.req.num_pages, a.status);
+        __nv_bfloat16* base = (g == 1) ? a.kpages : a.vpages;
+        dst_row = base + ((size_t)page * a.n_kv_heads * kPage + (pos % kPage)) * d;
+        head_stride = (size_t)kPage * d;
       }
-      if (bias) {
-        float b0[16], b1[16];
-        load16_bf16(bias + gcol + i0, b0);
-        load16_bf16(bias + gcol + half + i0, b1);
-#pragma unroll
+    }
+    // Chunks of 16 rotation pairs outermost: a chunk's cos/sin (one row of the angle table,
+    // shared by every head of the tile) is loaded once, and the next chunk's is requested
+    // while this one is applied, so the table's load latency overlaps the TMEM drain.
+    const bool rot = have && g < 2;
+    const float4* rope4 = reinterpret_cast<const float4*>(a.rope + (size_t)pos * half);
+    float4 cs[8], csn[8];
+    if (rot) {
+  #pragma unroll
+      for (int k = 0; k < 8; ++k) cs[k] = rope4[k];
+    }
+  #pragma unroll 1
+    for (int i0 = 0; i0 < half; i0 += 16) {
+      const bool more = rot && i0 + 16 < half;
+      if (more) {
+  #pragma unroll
+        for (int k = 0; k < 8; ++k) csn[k] = rope4[(i0 + 16) / 2 + k];
+      }
+  #pragma unroll 1
+      for (int hh = 0; hh < BN / d; ++hh) {
+        const int head = (tl.n_loc * BN) / d + hh;
+        const int gcol = head * d;
+        tmem_ld16(tacc + hh * d + i0, r0);
+        tmem_ld16(tacc + hh * d + half + i0, r1);
+        tmem_ld_wait();
+        if (!have || gcol >= a.group_cols[g]) continue;
+  #pragma unroll
         for (int j = 0; j < 16; ++j) {
-          v[j] += b0[j];
-          w[j] += b1[j];
+          v[j] = __uint_as_float(r0[j]);
+          w[j] = __uint_as_float(r1[j]);
         }
-      }
-      if (g < 2) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const float c = (j & 1) ? cs[j >> 1].z : cs[j >> 1].x;
-          const float sn = (j & 1) ? cs[j >> 1].w : cs[j >> 1].y;
-          const float x1 = v[j], x2 = w[j];
-          v[j] = x1 * c - x2 * sn;
-          w[j] = x2 * c + x1 * sn;
+        if (bias) {
+          float b0[16], b1[16];
+          load16_bf16(bias + gcol + i0, b0);
+          load16_bf16(bias + gcol + half + i0, b1);
+  #pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            v[j] += b0[j];
+            w[j] += b1[j];
+          }
         }
+        if (g < 2) {
+  #pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float c = (j & 1) ? cs[j >> 1].z : cs[j >> 1].x;
+            const float sn = (j & 1) ? cs[j >> 1].w : cs[j >> 1].y;
+            const float x1 = v[j], x2 = w[j];
+            v[j] = x1 * c - x2 * sn;
+            w[j] = x2 * c + x1 * sn;
+          }
+        }
+        __nv_bfloat16* dst = dst_row + head * head_stride;
+        store16_bf16(dst + i0, v);
+        store16_bf16(dst + half + i0, w);
       }
-      __nv_bfloat16* dst = dst_row + head * head_stride;
-      store16_bf16(dst + i0, v);
-      store16_bf16(dst + half + i0, w);
-    }
-    if (more) {
-#pragma unroll
-      for (int k = 0; k < 8; ++k) cs[k] = csn[k];
+      if (more) {
+  #pragma unroll
+        for (int k = 0; k < 8; ++k) cs[k] = csn[k];
+      }
     }
   }
 }
 
-template <int BN, int STAGES, int PAIR>
+// Down tile: slot j of the accumulator (columns 16j .. 16j + 15) is x A_j^T for this thread's
+// row; stored scaled as hi = bf16(v) at XA columns 32j.. and lo = bf16(v - hi) at 32j + 16..,
+// which carry the product to about 16 mantissa bits.
+__device__ __forceinline__ void epilogue_down(const GemmArgs& a, uint32_t tacc, int row) {
+  uint32_t r0[16];
+  float v[16], w[16];
+#pragma unroll 1
+  for (int j = 0; j < a.n_slots; ++j) {
+    tmem_ld16(tacc + 16 * j, r0);
+    tmem_ld_wait();
+    if (row >= a.M) continue;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      v[i] = __uint_as_float(r0[i]) * a.scale;
+      w[i] = v[i] - __bfloat162float(__float2bfloat16_rn(v[i]));
+    }
+    store16_bf16(a.xa + (size_t)row * kXaCols + 32 * j, v);
+    store16_bf16(a.xa + (size_t)row * kXaCols + 32 * j + 16, w);
+  }
+}
+
+// Bounded wait until *flag >= target (acquire at GPU scope). Gives up like mbar_wait.
+__device__ __forceinline__ bool flag_wait(const int* flag, int target, volatile int* abort_flag, int* status) {
+  unsigned long long t0 = 0;
+  for (uint32_t it = 0;; ++it) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(flag) : "memory");
+    if (v >= target) return true;
+    if (*abort_flag) return false;
+    if ((it & 15u) == 0) {
+      const unsigned long long now = globaltimer_ns();
+      if (t0 == 0) {
+        t0 = now;
+      } else if (now - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        if (status) atomicOr(status, kStatusTimeout);
+        return false;
+      }
+    }
+    __nanosleep(128);
+  }
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// The B side of an output tile's LoRA K block, written by the 128 epilogue threads into the
+// stage (128 rows x 128 bytes, 128-byte swizzle), one row each: row i is adapter B row y0 + i of
+// map index src, 16-byte unit c (K = 8c .. 8c + 7 of the block) holds B[row, 8 (c & 1) ..] when
+// K step c / 2 belongs to src's XA slot, zeros otherwise and past the rank or the matrix.
+__device__ __forceinline__ void load_lora_b(const GemmArgs& a, int src, int y, uint4& lo, uint4& hi) {
+  const __nv_bfloat16* B = a.BL[src];
+  const int rank = a.rank;
+  lo = make_uint4(0u, 0u, 0u, 0u);
+  hi = lo;
+  if (!B || y >= a.b_rows[src]) return;
+  const __nv_bfloat16* br = B + (size_t)y * rank;
+  if (rank >= 16) {
+    lo = reinterpret_cast<const uint4*>(br)[0];
+    hi = reinterpret_cast<const uint4*>(br)[1];
+  } else if (rank == 8) {
+    lo = reinterpret_cast<const uint4*>(br)[0];
+  } else {
+    const uint2 v = reinterpret_cast<const uint2*>(br)[0];
+    lo.x = v.x;
+    lo.y = v.y;
+  }
+}
+
+__device__ __forceinline__ void store_lora_b(const GemmArgs& a, int src, int xa_base, int steps, uint4 lo, uint4 hi,
+                                             uint8_t* sb, int i) {
+  const bool has = a.BL[src] != nullptr;
+  const int slot = a.bl_slot[src];
+  const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+  uint8_t* row = sb + i * 128;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    if (c >= 2 * steps) break;
+    const bool mine = has && xa_base / 32 + (c >> 2) == slot;
+    *reinterpret_cast<uint4*>(row + ((c ^ (i & 7)) << 4)) = mine ? ((c & 1) ? hi : lo) : zero;
+  }
+}
+
+// Producer ring position (stage, phase) and whether every wait so far succeeded.
+struct Ring {
+  int stage;
+  uint32_t phase;
+  int ok;
+};
+
+template <int STAGES>
+__device__ __forceinline__ void ring_next(Ring& r) {
+  if (++r.stage == STAGES) {
+    r.stage = 0;
+    r.phase ^= 1;
+  }
+}
+
+// Copies of a down tile: per K block the row block's x rows and the LoRA A rows of this CTA's
+// half of the tile's N (16 rows per XA slot; CTA r takes slots [r * spc, r * spc + spc)).
+template <int STAGES, int PAIR, int A_BYTES, int STAGE_BYTES>
+__device__ __noinline__ Ring load_down_tile(const GemmArgs& a, int m0, uint32_t rank, bool leader, uint8_t* smem,
+                                            uint64_t* full_bar, uint64_t* empty_bar, int* armed_parity,
+                                            volatile int* abort_flag, Ring ring) {
+  const int spc = a.down_n / (16 * PAIR);
+  const int s0 = static_cast<int>(rank) * spc, s1 = min(a.n_slots, s0 + spc);
+  const uint32_t bytes = PAIR * A_BYTES + a.n_slots * 16 * BK * 2;
+  for (int kb = 0; kb < a.num_kb; ++kb) {
+    if (!mbar_wait(&empty_bar[ring.stage], ring.phase ^ 1, abort_flag, a.status)) {
+      ring.ok = 0;
+      return ring;
+    }
+    uint8_t* sa = smem + ring.stage * STAGE_BYTES;
+    uint8_t* sb = sa + A_BYTES;
+    if (leader) {
+      mbar_arrive_expect_tx(&full_bar[ring.stage], bytes);
+      armed_parity[ring.stage] = ring.phase;
+    }
+    if constexpr (PAIR == 2) {
+      const uint32_t bar = mapa_shared(&full_bar[ring.stage], 0);
+      tma_load_2d_pair(sa, &a.tmA, bar, kb * BK, m0);
+      for (int j = s0; j < s1; ++j) tma_load_2d_pair(sb + (j - s0) * 16 * BK * 2, &a.tmLA[j], bar, kb * BK, 0);
+    } else {
+      tma_load_2d(sa, &a.tmA, &full_bar[ring.stage], kb * BK, m0);
+      for (int j = s0; j < s1; ++j)
+        tma_load_2d(sb + (j - s0) * 16 * BK * 2, &a.tmLA[j], &full_bar[ring.stage], kb * BK, 0);
+    }
+    ring_next<STAGES>(ring);
+  }
+  return ring;
+}
+
+// The LoRA stage of an output tile: once the stage is free, let the epilogue warps write the B
+// rows (bl_go), wait until both CTAs of the row block's down tile have stored its XA rows, and
+// copy those rows (the A side of the K block).
+template <int STAGES, int PAIR, int A_BYTES, int STAGE_BYTES>
+__device__ __noinline__ Ring load_lora_stage(const GemmArgs& a, const Tile& tl, int m0, bool leader, uint8_t* smem,
+                                             uint64_t* full_bar, uint64_t* empty_bar, uint64_t* bl_go,
+                                             int* armed_parity, volatile int* abort_flag, Ring ring) {
+  if (!mbar_wait(&empty_bar[ring.stage], ring.phase ^ 1, abort_flag, a.status)) {
+    ring.ok = 0;
+    return ring;
+  }
+  mbar_arrive(&bl_go[ring.stage]);
+  if (!flag_wait(a.xa_flags + tl.m_blk, 4 * PAIR, abort_flag, a.status)) {
+    ring.ok = 0;
+    return ring;
+  }
+  fence_proxy_async_global();  // the TMA copy below reads what the down tile's stores wrote
+  uint8_t* sa = smem + ring.stage * STAGE_BYTES;
+  if (leader) {
+    mbar_arrive_expect_tx(&full_bar[ring.stage], PAIR * A_BYTES);
+    armed_parity[ring.stage] = ring.phase;
+  }
+  if constexpr (PAIR == 2)
+    tma_load_2d_pair(sa, &a.tmXA, mapa_shared(&full_bar[ring.stage], 0), a.xa_base[tl.g], m0);
+  else
+    tma_load_2d(sa, &a.tmXA, &full_bar[ring.stage], a.xa_base[tl.g], m0);
+  ring_next<STAGES>(ring);
+  return ring;
+}
+
+// Between two epilogues, the epilogue warps write an output tile's LoRA B rows (one row per
+// thread) into its LoRA stage `st` once the producer has that stage free (bl_go), and count
+// themselves on the MMA-issuing CTA's bl_bar. False when the wait gave up.
+template <int STAGES, int PAIR, int A_BYTES, int STAGE_BYTES, int BN, int CTA_ROWS>
+__device__ __noinline__ bool write_lora_stage(const GemmArgs& a, const Tile& tl, uint32_t rank, int st, int b_row,
+                                              int lane, uint8_t* smem, uint64_t* bl_go, uint64_t* bl_bar,
+                                              uint32_t* go_parity, volatile int* abort_flag) {
+  const int nseg = a.nseg;
+  const int g0 = nseg == 1 ? tl.g : tl.g + static_cast<int>(rank) * (nseg / PAIR);
+  const int yb = nseg == 1 ? tl.n_loc * BN + static_cast<int>(rank) * CTA_ROWS : tl.n_loc * (BN / nseg);
+  uint4 lo, hi;
+  load_lora_b(a, g0, yb + b_row, lo, hi);
+  bool w = true;
+  if (lane == 0) w = mbar_wait(&bl_go[st], (*go_parity >> st) & 1u, abort_flag, a.status);
+  if (!__shfl_sync(0xffffffffu, w ? 1 : 0, 0)) return false;
+  *go_parity ^= 1u << st;
+  store_lora_b(a, g0, a.xa_base[tl.g], a.ext_steps[tl.g], lo, hi, smem + st * STAGE_BYTES + A_BYTES, b_row);
+  fence_proxy_async_smem();  // the tensor core reads these stores
+  __syncwarp();
+  if (lane == 0) {
+    if constexpr (PAIR == 2)
+      mbar_arrive_cluster(mapa_shared(&bl_bar[st], 0));
+    else
+      mbar_arrive(&bl_bar[st]);
+  }
+  return true;
+}
+
+template <int BN, int STAGES, int PAIR, int EPI>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
   constexpr int CTA_ROWS = BN / PAIR;  // B rows staged by this CTA
   constexpr int A_BYTES = BM * BK * 2;
@@ -331,6 +553,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   __shared__ __align__(8) uint64_t tfull_bar[2];
   __shared__ __align__(8) uint64_t tempty_bar[2];
   __shared__ __align__(8) uint64_t drain_bar;
+  __shared__ __align__(8) uint64_t bl_bar[STAGES];  // LoRA B rows written (each epilogue warp of both CTAs)
+  __shared__ __align__(8) uint64_t bl_go[STAGES];   // LoRA stage free for the B rows (producer)
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_flag;
   // a rejected call: every CTA of every cluster sees the same word and leaves before any set-up
@@ -347,6 +571,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
+      mbar_init(&bl_bar[s], 4 * PAIR);
+      mbar_init(&bl_go[s], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);
@@ -359,6 +585,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&a.tmA);
     for (int i = 0; i < 3; ++i) tma_prefetch_desc(&a.tmB[i]);
+    if (a.n_slots > 0) {
+      tma_prefetch_desc(&a.tmXA);
+      for (int i = 0; i < a.n_slots; ++i) tma_prefetch_desc(&a.tmLA[i]);
+    }
   }
   if (warp == 1) {
     if constexpr (PAIR == 2) {
@@ -376,17 +606,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer (every CTA)
+    // The per-stage loop of the output tiles stays minimal (one thread, on the critical path of
+    // every stage); down tiles and the LoRA stage go through out-of-line helpers.
     if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0;
+      Ring ring{0, 0u, 1};
       int armed_parity[STAGES];
       for (int s = 0; s < STAGES; ++s) armed_parity[s] = -1;
-      bool ok = true;
-      for (int t = unit; t < a.total_tiles && ok; t += n_units) {
+      for (int t = unit; t < a.total_tiles && ring.ok; t += n_units) {
         const Tile tl = decode_tile(t, a);
         const int m0 = tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM;
+        if (tl.down) {
+          ring = load_down_tile<STAGES, PAIR, A_BYTES, STAGE_BYTES>(a, m0, rank, leader, smem, full_bar, empty_bar,
+                                                                   armed_parity, &abort_flag, ring);
+          continue;
+        }
         const bool ext_tile = a.ext_on[tl.g] != 0;
-        const int nkb = a.num_kb + (ext_tile ? 1 : 0);
         const int nseg = a.nseg;
         const int seg_rows = BN / nseg;
         const int per = nseg / PAIR;
@@ -395,10 +629,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         const int nb = nseg == 1 ? 1 : per;
         const int yb = nseg == 1 ? tl.n_loc * BN + static_cast<int>(rank) * CTA_ROWS : tl.n_loc * seg_rows;
         const int b_step = nseg == 1 ? 0 : seg_rows * BK * 2;
-        const int xa_ext = a.xa_base[tl.g];
-        for (int kb = 0; kb < nkb; ++kb) {
+        int stage = ring.stage;
+        uint32_t phase = ring.phase;
+        for (int kb = 0; kb < a.num_kb; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1, &abort_flag, a.status)) {
-            ok = false;
+            ring.ok = 0;
             break;
           }
           uint8_t* sa = smem + stage * STAGE_BYTES;
@@ -408,26 +643,27 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             mbar_arrive_expect_tx(&full_bar[stage], PAIR * STAGE_BYTES);
             armed_parity[stage] = phase;
           }
-          const bool ext = kb == a.num_kb;
-          const CUtensorMap* mA = ext ? &a.tmXA : &a.tmA;
-          const CUtensorMap* mB = ext ? &a.tmBX[g0] : &a.tmB[g0];
-          const int xa = ext ? xa_ext : kb * BK;
-          const int xb = ext ? 0 : kb * BK;
+          const CUtensorMap* mB = &a.tmB[g0];
           if constexpr (PAIR == 2) {
             const uint32_t bar = mapa_shared(&full_bar[stage], 0);
-            tma_load_2d_pair(sa, mA, bar, xa, m0);
-            for (int j = 0; j < nb; ++j) tma_load_2d_pair(sb + j * b_step, mB + j, bar, xb, yb);
+            tma_load_2d_pair(sa, &a.tmA, bar, kb * BK, m0);
+            for (int j = 0; j < nb; ++j) tma_load_2d_pair(sb + j * b_step, mB + j, bar, kb * BK, yb);
           } else {
-            tma_load_2d(sa, mA, &full_bar[stage], xa, m0);
-            for (int j = 0; j < nb; ++j) tma_load_2d(sb + j * b_step, mB + j, &full_bar[stage], xb, yb);
+            tma_load_2d(sa, &a.tmA, &full_bar[stage], kb * BK, m0);
+            for (int j = 0; j < nb; ++j) tma_load_2d(sb + j * b_step, mB + j, &full_bar[stage], kb * BK, yb);
           }
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
           }
         }
+        ring.stage = stage;
+        ring.phase = phase;
+        if (ring.ok && ext_tile)
+          ring = load_lora_stage<STAGES, PAIR, A_BYTES, STAGE_BYTES>(a, tl, m0, leader, smem, full_bar, empty_bar, bl_go,
+                                                      armed_parity, &abort_flag, ring);
       }
-      if (!ok) {
+      if (!ring.ok) {
         if (leader) {
           // Let every copy already issued land before the CTA can exit.
           for (int s = 0; s < STAGES; ++s)
@@ -451,7 +687,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       int it = 0;
       bool ok = true;
       bool issued = false;
-      const uint32_t idesc = idesc_bf16_f32(BM * PAIR, BN);
+      const uint32_t idesc_tile = idesc_bf16_f32(BM * PAIR, BN);
+      const uint32_t idesc_down = idesc_bf16_f32(BM * PAIR, a.n_slots > 0 ? a.down_n : 32);
+      uint32_t bl_parity = 0;  // bit s: phase of bl_bar[s] to wait for next
       for (int t = unit; t < a.total_tiles && ok; t += n_units, ++it) {
         const Tile tl = decode_tile(t, a);
         const int acc = it & 1;
@@ -462,7 +700,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        const int ext_steps = a.ext_on[tl.g] ? a.ext_steps[tl.g] : 0;
+        const int ext_steps = !tl.down && a.ext_on[tl.g] ? a.ext_steps[tl.g] : 0;
+        const uint32_t idesc = tl.down ? idesc_down : idesc_tile;
         auto mma = [&](uint64_t ad, uint64_t bd, uint32_t accum) {
           if constexpr (PAIR == 2)
             mma_bf16_ss_pair(d_tmem, ad, bd, idesc, accum);
@@ -492,9 +731,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           release();
         }
         if (ok && ext_steps > 0) {
-          if (!mbar_wait(&full_bar[stage], phase, &abort_flag, a.status)) {
+          // the XA copies have landed and both CTAs have written their LoRA B rows
+          if (!mbar_wait(&full_bar[stage], phase, &abort_flag, a.status) ||
+              !mbar_wait<PAIR == 2>(&bl_bar[stage], (bl_parity >> stage) & 1u, &abort_flag, a.status)) {
             ok = false;
           } else {
+            bl_parity ^= 1u << stage;
             tc_fence_after();
             const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
             const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
@@ -516,20 +758,34 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     // ------------------------------------------------------------ epilogue (warps 2..5, every CTA)
     const int quarter = warp & 3;  // TMEM lane quarter this warp may access
     const int row_in_cta = quarter * 32 + lane;
+    const int b_row = (warp - 2) * 32 + lane;  // LoRA B row this thread writes
     uint32_t tempty_addr[2];
     for (int i = 0; i < 2; ++i)
       tempty_addr[i] = PAIR == 2 ? mapa_shared(&tempty_bar[i], 0) : smem_u32(&tempty_bar[i]);
+    int pos = 0;             // producer stages used by the tiles before this one
+    uint32_t go_parity = 0;  // bit s: phase of bl_go[s] to wait for next
     int it = 0;
     for (int t = unit; t < a.total_tiles; t += n_units, ++it) {
       const Tile tl = decode_tile(t, a);
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
+      const bool ext_tile = !tl.down && a.ext_on[tl.g] != 0;
+      if (ext_tile &&
+          !write_lora_stage<STAGES, PAIR, A_BYTES, STAGE_BYTES, BN, CTA_ROWS>(a, tl, rank, (pos + a.num_kb) % STAGES,
+                                                                            b_row, lane, smem, bl_go, bl_bar,
+                                                                            &go_parity, &abort_flag))
+        break;
+      pos += tl.down ? a.num_kb : a.num_kb + (ext_tile ? 1 : 0);
       // warp-uniform outcome: the TMEM loads of the epilogue are warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait(&tfull_bar[acc], acc_phase, &abort_flag, a.status)))
         break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<BN>(a, tl, tacc, tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM + row_in_cta);
+      const int row = tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM + row_in_cta;
+      if (tl.down)
+        epilogue_down(a, tacc, row);
+      else
+        epilogue_tile<BN, EPI>(a, tl, tacc, row);
       // the accumulator is free once this warp's TMEM loads have completed (tcgen05.wait::ld in
       // the epilogue); the tile's global stores need not be visible first, so the arrival on
       // the MMA-issuing CTA's barrier is relaxed
@@ -537,6 +793,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       __syncwarp();
       if (lane == 0) {
         if constexpr (PAIR == 2) mbar_arrive_cluster_relaxed(tempty_addr[acc]); else mbar_arrive(&tempty_bar[acc]);
+      }
+      if (tl.down) {
+        // publish this warp's XA rows: GPU-scope fence, then count the warp in the block's word
+        // (4 warps x both CTAs); the readers load them with TMA after an acquire
+        __threadfence();
+        fence_proxy_async_global();
+        __syncwarp();
+        if (lane == 0) atomicAdd(a.xa_flags + tl.m_blk, 1);
       }
     }
   }
@@ -583,10 +847,10 @@ bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int ld, int 
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, int PAIR>
-cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) {
+template <int BN, int STAGES, int PAIR, int EPI>
+cudaError_t launch_impl(GemmArgs& args, int num_sms, cudaStream_t stream) {
   constexpr int smem = STAGES * (BM * BK * 2 + (BN / PAIR) * BK * 2) + 1024;
-  auto kern = gemm_tc_kernel<BN, STAGES, PAIR>;
+  auto kern = gemm_tc_kernel<BN, STAGES, PAIR, EPI>;
   // the attributes and the co-resident cluster count are per device
   static PerDevice once;
   static std::atomic<int> units_of[64];
@@ -596,41 +860,39 @@ cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) 
   } else {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    if (PAIR == 2) {
-      e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
-      cudaLaunchConfig_t cfg = {};
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = 2;
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.gridDim = dim3(num_sms);
-      cfg.blockDim = dim3(kThreads);
-      cfg.dynamicSmemBytes = smem;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      int clusters = 0;
-      e = cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg);
-      if (e != cudaSuccess) return e;
-      max_units = std::max(1, std::min(clusters, num_sms / 2));
-    } else {
-      max_units = num_sms;
-    }
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = PAIR;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(num_sms);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    e = cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg);
+    if (e != cudaSuccess) return e;
+    max_units = std::max(1, std::min(clusters, num_sms / PAIR));
     if (dev >= 0 && dev < 64) units_of[dev].store(max_units, std::memory_order_relaxed);
     once.done(dev);
   }
+  // every unit of the grid is resident at once (one CTA per SM): a tile that waits for its row
+  // block's down tile never waits on a unit that has not started
   const int units = std::max(1, std::min(max_units, args.total_tiles));
-  if (PAIR == 1) {
-    kern<<<units, kThreads, smem, stream>>>(args);
-    return cudaGetLastError();
-  }
+  // down tiles one wave of units ahead of their row block's first output tiles
+  const int w0 = std::min(kRasterGroup, args.total_n);
+  args.down_lead = (units + w0) / (w0 + 1);
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.x = PAIR;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.gridDim = dim3(2 * units);
+  cfg.gridDim = dim3(PAIR * units);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
@@ -641,12 +903,11 @@ cudaError_t launch_impl(const GemmArgs& args, int num_sms, cudaStream_t stream) 
 
 }  // namespace
 
-cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream) {
+cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t stream) {
+  constexpr int bn = 256, pair = 2;
   GemmArgs a;
   std::memset(&a, 0, sizeof(a));
-  // the 256-wide projection tiles run on CTA pairs; the narrow LoRA-down tiles on single CTAs
-  if (bn == 256 && d.nseg != 1 && d.nseg != 2) return cudaErrorInvalidValue;
-  const int pair = bn == 256 ? 2 : 1;
+  if (d.nseg != 1 && d.nseg != 2) return cudaErrorInvalidValue;
   // rows of one B load: the CTA's share of the tile (plain) or one stacked segment
   const int b_box = d.nseg == 1 ? bn / pair : bn / d.nseg;
   if (!make_map(&a.tmA, d.A, d.M, d.K, d.lda, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B))
@@ -657,35 +918,34 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
     if (!make_map(&a.tmB[i], d.B[src], d.B_rows[src], d.K, d.ldb[src], b_box, BK,
                   CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
+    a.BL[i] = i < nmaps ? static_cast<const __nv_bfloat16*>(d.BL[i]) : nullptr;
+    a.bl_slot[i] = i < nmaps && d.BL[i] ? d.bl_slot[i] : -1;
+    a.b_rows[i] = d.B_rows[src];
   }
   bool any_ext = false;
   for (int g = 0; g < d.ngroups; ++g) any_ext |= d.ext_on[g] != 0;
+  if (any_ext != (d.n_slots > 0) || d.n_slots < 0 || d.n_slots > 3) return cudaErrorInvalidValue;
   if (any_ext) {
-    if (!d.XA || d.ldxa < kXaCols) return cudaErrorInvalidValue;
-    if (!make_map(&a.tmXA, d.XA, d.M, d.ldxa, d.ldxa, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B))
+    if (!d.XA || !d.xa_flags || (d.rank != 4 && d.rank != 8 && d.rank != 16)) return cudaErrorInvalidValue;
+    if (!make_map(&a.tmXA, d.XA, d.M, kXaCols, kXaCols, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
-    for (int i = 0; i < 3; ++i) {
-      int src = (i < nmaps && d.BX[i]) ? i : -1;
-      if (src < 0)
-        for (int j = 0; j < nmaps; ++j)
-          if (d.BX[j]) src = j;
-      if (src < 0) return cudaErrorInvalidValue;
-      if (!make_map(&a.tmBX[i], d.BX[src], d.B_rows[src], BK, BK, b_box, BK,
-                    CU_TENSOR_MAP_SWIZZLE_128B))
+    for (int j = 0; j < 3; ++j) {
+      const int src = j < d.n_slots ? j : 0;
+      if (!d.LA[src] || !make_map(&a.tmLA[j], d.LA[src], d.rank, d.K, d.K, 16, BK, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
     }
     for (int g = 0; g < d.ngroups; ++g) {
       if (!d.ext_on[g]) continue;
       // the 64-wide block must lie inside the XA row, 16-byte aligned (TMA x coordinate)
-      if (d.xa_base[g] < 0 || d.xa_base[g] % 8 != 0 || d.xa_base[g] + BK > kXaCols ||
+      if (d.xa_base[g] < 0 || d.xa_base[g] % 32 != 0 || d.xa_base[g] + BK > kXaCols ||
           d.ext_steps[g] < 1 || d.ext_steps[g] > BK / 16)
         return cudaErrorInvalidValue;
-      for (int s = 0; s < (d.ngroups == 1 ? d.nseg : 1); ++s)
-        if (!d.BX[g + s]) return cudaErrorInvalidValue;
     }
+    for (int i = 0; i < nmaps; ++i)
+      if (d.BL[i] && (d.bl_slot[i] < 0 || d.bl_slot[i] >= d.n_slots)) return cudaErrorInvalidValue;
   } else {
     a.tmXA = a.tmA;
-    for (int i = 0; i < 3; ++i) a.tmBX[i] = a.tmB[i];
+    for (int i = 0; i < 3; ++i) a.tmLA[i] = a.tmA;
   }
   a.M = d.M;
   a.K = d.K;
@@ -705,7 +965,13 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
     a.xa_base[g] = d.xa_base[g];
   }
   a.row_tiles = (d.M + BM * pair - 1) / (BM * pair);
-  a.total_tiles = a.row_tiles * a.total_n;
+  a.n_slots = any_ext ? d.n_slots : 0;
+  // two CTA halves of 16 x ceil(n_slots / 2) rows: N = 32 for one or two slots, 64 for three
+  a.down_n = 32 * ((a.n_slots + 1) / 2);
+  a.rank = d.rank;
+  a.xa = static_cast<__nv_bfloat16*>(d.XA);
+  a.xa_flags = d.xa_flags;
+  a.total_tiles = a.row_tiles * a.total_n + (a.n_slots > 0 ? a.row_tiles : 0);
   a.epi = d.epi;
   a.scale = d.scale;
   a.out = static_cast<__nv_bfloat16*>(d.out);
@@ -724,11 +990,12 @@ cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t str
   a.status = d.status;
   a.abort = d.abort;
   if (a.total_tiles == 0) return cudaSuccess;
-  if (pair == 2) return launch_impl<256, 6, 2>(a, num_sms, stream);
-  switch (bn) {
-    case 48: return launch_impl<48, 8, 1>(a, num_sms, stream);
-    case 32: return launch_impl<32, 8, 1>(a, num_sms, stream);
-    case 16: return launch_impl<16, 8, 1>(a, num_sms, stream);
+  // one kernel per epilogue: each carries only its own epilogue code, which keeps the hot loops
+  // of all its warps inside the SM's instruction cache
+  switch (d.epi) {
+    case kEpiQkv: return launch_impl<bn, 6, pair, kEpiQkv>(a, num_sms, stream);
+    case kEpiResid: return launch_impl<bn, 6, pair, kEpiResid>(a, num_sms, stream);
+    case kEpiSwiGLU: return launch_impl<bn, 6, pair, kEpiSwiGLU>(a, num_sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }

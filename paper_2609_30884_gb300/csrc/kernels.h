@@ -33,9 +33,9 @@ constexpr int kPage = 16;
 constexpr int kRankPad = 16;  // LoRA rank padded to one K=16 MMA step
 // The scaled LoRA down product is kept as a bf16 pair hi + lo (lo = bf16(v - hi)): module
 // slot j holds hi at columns [32j, 32j + 16) and lo at [32j + 16, 32j + 32) of a [rows, kXaCols]
-// buffer. The GEMM reads it as one 64-wide K block against BX = [B | B] rows (kBxCols wide).
+// buffer. A projection GEMM computes it for its rows (down tiles) and reads it back as one
+// 64-wide K block against the adapter's B rows (the up product).
 constexpr int kXaCols = 128;
-constexpr int kBxCols = 64;
 
 // Programmatic dependent launch for chains of short kernels. While a PdlScope is alive on the
 // calling thread, the launchers below that go through launch_kernel() give their kernels the
@@ -81,7 +81,6 @@ struct ReqTable {
 };
 
 enum EpiKind : int {
-  kEpiScaleBf16 = 0,  // out = hi/lo bf16 pair of acc * scale            (LoRA down product)
   kEpiQkv = 1,        // +bias, RoPE(q,k); q -> qbuf, k/v -> KV pages    (Eq. S3)
   kEpiResid = 2,      // out = bf16(resid + acc)                         (o / down projection)
   kEpiSwiGLU = 3      // out = bf16(silu(gate) * up), tile = [gate | up]  (MLP)
@@ -99,17 +98,25 @@ struct GemmDesc {
   int B_rows[3];          // rows of each B matrix
   int ldb[3];
   int group_cols[3];      // valid output columns per group (plain) / per segment (stacked)
-  // LoRA extension (one extra K block): D += XA[:, xa_base[g] .. + 64] * BX^T, where XA holds the
-  // (alpha/r)-scaled down products as hi/lo pairs and BX [B_rows, 64] the matching B rows
-  const void* XA;
-  int ldxa;
-  const void* BX[3];      // map index g + s, like B
+  // Unmerged LoRA (Eq. S3), computed inside the same launch. Down tiles (one per 256-row block)
+  // form XA[:, 32j .. 32j + 32) = hi/lo of (alpha/r) x A_j^T for the n_slots adapted modules
+  // (LA[j] = A_j, [rank, K]) and raise xa_flags[row block]; every output tile of an adapted
+  // group then adds one K block: XA[:, xa_base[g] .. + 64] against the module's B rows, placed
+  // under the K steps of its own slot (BL[i] = B of map index i, [B_rows[i], rank]; bl_slot[i]
+  // its XA slot, -1 without adapter).
+  void* XA;
+  int n_slots;
+  const void* LA[3];
+  const void* BL[3];      // map index g + s, like B
+  int bl_slot[3];
+  int rank;
+  float scale;            // alpha / r
+  int* xa_flags;          // [row blocks of 256], zero before the launch
   int ext_on[3];          // per group
   int ext_steps[3];       // K = 16 steps of the block that carry data (2 per module)
   int xa_base[3];
   // epilogue
   int epi;
-  float scale;
   void* out;
   int ldo;
   const void* resid;
@@ -126,21 +133,8 @@ struct GemmDesc {
   const int* abort;       // per-call abort word (call_aborted), or null
 };
 
-// Launch the tcgen05 GEMM. bn: 256 for projections (CTA pairs with 256-row tiles); 16/32/48 for
-// LoRA down (single CTAs).
-cudaError_t launch_gemm(const GemmDesc& d, int bn, int num_sms, cudaStream_t stream);
-
-// BX rows of up to 7 modules in one launch: out[m][r, :] = 0 except columns
-// [col_off[m], col_off[m] + 32) = [B_m[r, 0:16] | B_m[r, 0:16]] (rank padded with zeros); a null
-// B_m gives all-zero rows.
-struct BextDesc {
-  const __nv_bfloat16* B[7];
-  __nv_bfloat16* out[7];
-  int rows[7];
-  int col_off[7];
-  int n;
-};
-cudaError_t launch_lora_bext(const BextDesc& d, int rank, cudaStream_t stream);
+// Launch the tcgen05 projection GEMM (CTA pairs, 256 x 256 tiles).
+cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t stream);
 
 // ------------------------------------------------------------------ other kernels
 cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double theta,

@@ -280,30 +280,6 @@ __global__ void rope_rows_kernel(float* q, int hq, float* k, int hkv, int rows, 
   base[i + half] = x2 * cs.x + x1 * cs.y;
 }
 
-// BX rows: one thread per (row, 8-column chunk) of module blockIdx.y.
-__global__ void lora_bext_kernel(const BextDesc d, int rank) {
-  const int m = blockIdx.y;
-  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= d.rows[m] * (kBxCols / 8)) return;
-  const int r = idx / (kBxCols / 8);
-  const int c0 = (idx % (kBxCols / 8)) * 8;
-  const __nv_bfloat16* B = d.B[m];
-  const int off = d.col_off[m];
-  uint32_t w[4];
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    float v[2];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int c = c0 + 2 * j + h - off;
-      const int k = c & 15;
-      v[h] = (B && c >= 0 && c < 32 && k < rank) ? __bfloat162float(B[(size_t)r * rank + k]) : 0.f;
-    }
-    w[j] = pack_bf16(v[0], v[1]);
-  }
-  *reinterpret_cast<uint4*>(d.out[m] + (size_t)r * kBxCols + c0) = make_uint4(w[0], w[1], w[2], w[3]);
-}
-
 // m[i] = silu(g[i]) * u[i] over n elements (gate and up in separate buffers)
 __global__ void swiglu_split_f32_kernel(const float* g, const float* u, float* m, int n) {
   griddep_begin();  // gate and up come from the GEMV before
@@ -748,15 +724,6 @@ cudaError_t launch_validate_pages(const PageCheck& pc, int num_pages, int* table
   if (total == 0) return cudaSuccess;
   if (static_cast<uint32_t>(total) > (mask + 1u) / 2u) return cudaErrorInvalidValue;
   validate_pages_kernel<<<cdiv(total, 256), 256, 0, stream>>>(pc, num_pages, table, mask, abort, status);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_lora_bext(const BextDesc& d, int rank, cudaStream_t stream) {
-  int rows = 0;
-  for (int m = 0; m < d.n; ++m) rows = rows > d.rows[m] ? rows : d.rows[m];
-  if (d.n == 0 || rows == 0) return cudaSuccess;
-  if (rank < 1 || rank > kRankPad) return cudaErrorInvalidValue;
-  lora_bext_kernel<<<dim3(cdiv(rows * (kBxCols / 8), 256), d.n), 256, 0, stream>>>(d, rank);
   return cudaGetLastError();
 }
 

@@ -58,9 +58,11 @@ def test_algorithmic_work_7b_matches_hand_count():
     # base GEMMs: 2 * n * sum(in * out) over the seven projections
     h, f, qd, kvd = 3584, 18944, 3584, 512
     base = 2 * 16384 * (h * (qd + 2 * kvd) + qd * h + 2 * h * f + f * h)
-    gemm = sum(v for k, v in flops.items() if k.startswith("gemm_") and k != "gemm_lora_down")
+    gemm = sum(v for k, v in flops.items() if k.startswith("gemm_"))
+    # adapter: down products over each module's input, up products over its output
     lora_up = 2 * 16384 * 16 * (qd + 2 * kvd + h + 2 * f + h)
-    assert gemm == base + lora_up
+    lora_down = 2 * 16384 * 16 * (3 * h + qd + 2 * h + f)
+    assert gemm == base + lora_up + lora_down
     assert flops["attn_prefill_paged"] == 4 * 28 * 128 * 16384 * 16385 // 2
 
 
