@@ -167,7 +167,7 @@ struct Plan {
   int max_n = 0;
   int dec_rows = 0;   // requests asking for the first-step state
   int splits = 1;
-  size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_rope;
+  size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_bx, off_rope;
   size_t off_dx0, off_dec;  // decode: bf16 starting rows, fp32 scratch
   size_t off_abort, off_ptab;  // the call's abort word; the page-check table (ptab_slots ints)
   // the projections' XA ready words: 4 launches x ceil(M / 256) row blocks per layer, laid out
@@ -177,6 +177,17 @@ struct Plan {
   size_t dec_bytes;
   size_t total;
 };
+
+// output rows of module m (q, k, v, o, gate, up, down) and their sum
+int module_rows(const Dims& D, int m) {
+  const int r[7] = {D.qd, D.kvd, D.kvd, D.h, D.f, D.f, D.h};
+  return r[m];
+}
+int module_rows_total(const Dims& D) {
+  int t = 0;
+  for (int m = 0; m < 7; ++m) t += module_rows(D, m);
+  return t;
+}
 
 // decode attention partials: one per chunk of the longest prefix
 int dec_splits(int max_n) { return decode_attention_splits(max_n); }
@@ -215,6 +226,7 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_o = take(M * D.qd * 2);
   p.off_mlp = take(M * D.f * 2);
   p.off_xa = take(M * kXaCols * 2);
+  p.off_bx = take(static_cast<size_t>(module_rows_total(D)) * kBxCols * 2);
   p.off_rope = take(static_cast<size_t>(p.max_n) * (D.d / 2) * sizeof(float2));
   p.off_dx0 = take(static_cast<size_t>(n_req) * D.h * 2);
   long ids = 0;
@@ -299,6 +311,30 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
   // one ready word per 256-row block for each of the layer's four projection launches
   int* flags = c.xa_flags;
   const int flag_stride = (p.M + 255) / 256;
+  // BX = [B | B] rows of every module of layer l under its XA slot (up follows gate when both are
+  // adapted, so one K block carries the stacked gate|up pair), built by the RMSNorm launches:
+  // q, k, v, o with the first, gate, up, down with the second
+  __nv_bfloat16* BX[7];
+  BextDesc bext[2]{};
+  {
+    auto* bx = reinterpret_cast<__nv_bfloat16*>(ws + p.off_bx);
+    for (int m = 0; m < 7; ++m) {
+      BX[m] = bx;
+      const int rows = module_rows(D, m);
+      bx += static_cast<size_t>(rows) * kBxCols;
+      // a stacked gate|up tile reads both modules' rows: an unadapted one's are zeros
+      const bool need = adapted(c.ad, m) || ((m == CRF_MOD_GATE || m == CRF_MOD_UP) &&
+                                              (adapted(c.ad, CRF_MOD_GATE) || adapted(c.ad, CRF_MOD_UP)));
+      if (!need) continue;
+      BextDesc& d = bext[m < CRF_MOD_GATE ? 0 : 1];
+      d.B[d.n] = adapted(c.ad, m) ? static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + m]) : nullptr;
+      d.out[d.n] = BX[m];
+      d.rows[d.n] = rows;
+      d.col_off[d.n] = (m == CRF_MOD_UP && adapted(c.ad, CRF_MOD_GATE)) ? 32 : 0;
+      ++d.n;
+    }
+    bext[0].rank = bext[1].rank = c.ad->dims.rank;
+  }
   // the unmerged adapter of the listed modules, slots in list order (Eq. S3)
   auto set_lora = [&](GemmDesc& g, const int* mods, int nm, int* slot_of) {
     g.n_slots = 0;
@@ -319,7 +355,8 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
   // 1. RMSNorm before attention
   {
     ProfScope ps(c.ctx, kPNorm, c.st);
-    CRF_CUDA(launch_rmsnorm(X_in, static_cast<const __nv_bfloat16*>(w.ln1), XN, M, D.h, D.eps, c.st));
+    CRF_CUDA(launch_rmsnorm(X_in, static_cast<const __nv_bfloat16*>(w.ln1), XN, M, D.h, D.eps, c.st,
+                            bext[0].n ? &bext[0] : nullptr));
   }
 
   // 2-3. q/k/v projections (+ LoRA, bias, RoPE; K/V into the pages of layer l)
@@ -342,8 +379,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
       g.ldb[m] = D.h;
       g.group_cols[m] = rows[m];
       if (slot[m] >= 0) {
-        g.BL[m] = c.ad->B[l * 7 + m];
-        g.bl_slot[m] = slot[m];
+        g.BX[m] = BX[m];
         g.ext_on[m] = 1;
         g.ext_steps[m] = 2;
         g.xa_base[m] = 32 * slot[m];
@@ -401,8 +437,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
     int slot[1];
     set_lora(g, &m, 1, slot);
     if (slot[0] >= 0) {
-      g.BL[0] = c.ad->B[l * 7 + m];
-      g.bl_slot[0] = 0;
+      g.BX[0] = BX[m];
       g.ext_on[0] = 1;
       g.ext_steps[0] = 2;
       g.xa_base[0] = 0;
@@ -422,7 +457,8 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
   // 7. RMSNorm before the MLP
   {
     ProfScope ps(c.ctx, kPNorm, c.st);
-    CRF_CUDA(launch_rmsnorm(X1, static_cast<const __nv_bfloat16*>(w.ln2), XN, M, D.h, D.eps, c.st));
+    CRF_CUDA(launch_rmsnorm(X1, static_cast<const __nv_bfloat16*>(w.ln2), XN, M, D.h, D.eps, c.st,
+                            bext[1].n ? &bext[1] : nullptr));
   }
 
   // 8-9. gate|up projections with SwiGLU epilogue
@@ -442,10 +478,7 @@ crf_status run_layer(const LayerCtx& c, int l, const __nv_bfloat16* X_in, __nv_b
       g.B[s] = w.W[mods[s]];
       g.B_rows[s] = D.f;
       g.ldb[s] = D.h;
-      if (slot[s] >= 0) {
-        g.BL[s] = c.ad->B[l * 7 + mods[s]];
-        g.bl_slot[s] = slot[s];
-      }
+      g.BX[s] = BX[mods[s]];  // all-zero rows for a module without adapter
     }
     if (g.n_slots) {
       // one K block carries both slots; each segment's B rows sit under its own slot only

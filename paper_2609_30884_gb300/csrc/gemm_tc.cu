@@ -15,19 +15,22 @@
 // are bf16, K-major, staged with 128-byte swizzle; accumulation is fp32 in TMEM.
 //
 // The adapter term (alpha/r) (x A^T) B^T of every adapted projection (Eq. S3, W = W0 + (alpha/r)
-// B A kept unmerged) is computed in the same launch:
-//  - down tiles, one per 256-row block of A, form x A^T for the GEMM's adapted modules (N = 16
-//    per module, B operand = the LoRA A rows) and store it, scaled, as a bf16 pair [hi | lo]
-//    per module (16 + 16 columns of the XA buffer), then count themselves done in the row
-//    block's ready word;
-//  - every output tile of an adapted module adds one 64-wide K block: A side = the XA columns
-//    of its row block (loaded once the ready word shows both CTAs of the down tile done), B side
-//    = the module's B rows, written into the stage by the loading warp under the K steps of the
-//    module's own slot (zeros under the other slot), so one K block serves two stacked modules
-//    and the two halves of a pair alike.
-// Down tiles are ordered one wave ahead of the first output tiles of their row block, so those
-// rarely wait; the wait is bounded like every other. The XA rows a down tile reads in are the
-// A rows its row block's output tiles read next, so they come from L2.
+// B A kept unmerged) is computed in the same launch, on the operand tiles already staged:
+//  - the first output tile of each 256-row block (its XA tile) also accumulates x A^T for the
+//    GEMM's adapted modules (N = 16 per module, B operand = the LoRA A rows, staged beside the W
+//    rows) into the other accumulator's first columns, which the epilogue of the previous tile has
+//    drained by then. Its epilogue warps store that product, scaled, as a bf16 pair [hi | lo] per
+//    module (16 + 16 columns of the XA buffer) and count themselves done in the row block's ready
+//    word;
+//  - every output tile of an adapted module adds one 64-wide K block: A side = the XA columns of
+//    its row block (the XA tile writes them into its own stage; the others copy them once the
+//    ready word shows both CTAs done), B side = BX, the module's B rows twice over ([B | B],
+//    against [hi | lo]) under the K steps of its slot and zeros under the other slot, so one K
+//    block serves two stacked modules and the two halves of a pair alike. The RMSNorm launch
+//    before the layer's projections builds the BX rows.
+// XA tiles run first, one per unit, ahead of the other tiles of their row block, so those rarely
+// wait; the wait is bounded like every other. x is read once: the XA product needs no pass of its
+// own.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -49,7 +52,8 @@ struct GemmArgs {
   CUtensorMap tmA;
   CUtensorMap tmB[3];
   CUtensorMap tmXA;
-  CUtensorMap tmLA[3];  // LoRA A of XA slot j: the down tiles' B operand
+  CUtensorMap tmLA[3];  // LoRA A of XA slot j: the B operand of the XA product
+  CUtensorMap tmBX[3];  // BX rows of map index i: the B side of the LoRA K block
   int M, K, num_kb;
   int ngroups, nseg;
   int group_tiles[3];
@@ -58,12 +62,9 @@ struct GemmArgs {
   int ext_steps[3];   // per group: K = 16 steps of that block that carry data
   int xa_base[3];     // per group: first XA column of that block
   int row_tiles, total_n, total_tiles;
-  int n_slots;        // adapted modules (XA slots); 0: no down tiles
-  int down_n;         // N of a down tile: 16 per slot, two CTA halves of 16 x slots_per_cta
-  int down_lead;      // down tiles placed ahead of the first output tiles of their row block
-  const __nv_bfloat16* BL[3];  // adapter B of map index i, [b_rows[i], rank], or null
-  int bl_slot[3];
-  int b_rows[3];
+  int n_slots;        // adapted modules (XA slots); 0: no XA product
+  int xa_n;           // N of the XA product: 16 per slot, two CTA halves of 16 x slots_per_cta
+  int xa_lead;        // XA tiles placed before every other tile (the rest follow their row block)
   int rank;
   __nv_bfloat16* xa;
   int* xa_flags;
@@ -87,39 +88,32 @@ struct GemmArgs {
 
 struct Tile {
   int m_blk, g, n_loc;
-  bool down;  // the row block's LoRA down product
+  bool xa;  // the row block's first output tile, which also forms its XA product
 };
 
 // Output tiles run in bands of kRasterGroup column tiles over every row block (the band's B
-// rows stay in L2). With down tiles, band 0 carries them: the first `lead` down tiles, then per
-// row block m the down tile of m + lead followed by m's band-0 output tiles.
+// rows stay in L2). With an adapter, band 0 is reordered so that each row block's first tile
+// (its XA tile) runs ahead of the block's other band-0 tiles: the first `lead` XA tiles, then
+// per row block m the XA tile of m + lead followed by m's other band-0 tiles (lead = all row
+// blocks puts every XA tile first).
 __device__ __forceinline__ Tile decode_tile(int t, const GemmArgs& a) {
   Tile r;
-  r.down = false;
-  r.g = 0;
-  r.n_loc = 0;
+  r.xa = false;
   if (a.n_slots > 0) {
     const int w0 = min(kRasterGroup, a.total_n);
-    const int lead = min(a.down_lead, a.row_tiles);
+    const int lead = min(a.xa_lead, a.row_tiles);
+    const int g1 = a.row_tiles - lead;  // row blocks whose other tiles follow an XA tile
     if (t < lead) {
-      r.down = true;
-      r.m_blk = t;
-      return r;
-    }
-    int u = t - lead;
-    const int g1 = a.row_tiles - lead;  // row blocks whose band-0 tiles follow a down tile
-    if (u < g1 * (w0 + 1)) {
-      r.m_blk = u / (w0 + 1);
-      const int i = u - r.m_blk * (w0 + 1);
-      if (i == 0) {
-        r.down = true;
-        r.m_blk += lead;
-        return r;
-      }
-      t = r.m_blk * w0 + (i - 1);  // the plain order's index of output tile (m, i - 1)
-    } else {
-      t = u - g1;  // the remaining band-0 tiles, then the later bands, in plain order
-    }
+      t = t * w0;  // the plain order's index of tile (t, 0)
+    } else if (t - lead < g1 * w0) {
+      const int u = t - lead;
+      const int m = u / w0, i = u - m * w0;
+      t = i == 0 ? (m + lead) * w0 : m * w0 + i;
+    } else if (t - lead - g1 * w0 < lead * (w0 - 1)) {
+      const int v = t - lead - g1 * w0;
+      const int m = g1 + v / (w0 - 1);
+      t = m * w0 + 1 + v % (w0 - 1);
+    }  // else: the later bands keep their plain index
   }
   const int band_tiles = a.row_tiles * kRasterGroup;
   const int band = t / band_tiles;
@@ -128,6 +122,7 @@ __device__ __forceinline__ Tile decode_tile(int t, const GemmArgs& a) {
   const int width = min(kRasterGroup, a.total_n - n0);
   r.m_blk = idx / width;
   int n = n0 + (idx - r.m_blk * width);
+  r.xa = a.n_slots > 0 && n == 0;
   int g = 0;
   while (g < a.ngroups - 1 && n >= a.group_tiles[g]) {
     n -= a.group_tiles[g];
@@ -346,27 +341,6 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs& a, const Tile& tl,
   }
 }
 
-// Down tile: slot j of the accumulator (columns 16j .. 16j + 15) is x A_j^T for this thread's
-// row; stored scaled as hi = bf16(v) at XA columns 32j.. and lo = bf16(v - hi) at 32j + 16..,
-// which carry the product to about 16 mantissa bits.
-__device__ __forceinline__ void epilogue_down(const GemmArgs& a, uint32_t tacc, int row) {
-  uint32_t r0[16];
-  float v[16], w[16];
-#pragma unroll 1
-  for (int j = 0; j < a.n_slots; ++j) {
-    tmem_ld16(tacc + 16 * j, r0);
-    tmem_ld_wait();
-    if (row >= a.M) continue;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      v[i] = __uint_as_float(r0[i]) * a.scale;
-      w[i] = v[i] - __bfloat162float(__float2bfloat16_rn(v[i]));
-    }
-    store16_bf16(a.xa + (size_t)row * kXaCols + 32 * j, v);
-    store16_bf16(a.xa + (size_t)row * kXaCols + 32 * j + 16, w);
-  }
-}
-
 // Bounded wait until *flag >= target (acquire at GPU scope). Gives up like mbar_wait.
 __device__ __forceinline__ bool flag_wait(const int* flag, int target, volatile int* abort_flag, int* status) {
   unsigned long long t0 = 0;
@@ -393,42 +367,13 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-// The B side of an output tile's LoRA K block, written by the 128 epilogue threads into the
-// stage (128 rows x 128 bytes, 128-byte swizzle), one row each: row i is adapter B row y0 + i of
-// map index src, 16-byte unit c (K = 8c .. 8c + 7 of the block) holds B[row, 8 (c & 1) ..] when
-// K step c / 2 belongs to src's XA slot, zeros otherwise and past the rank or the matrix.
-__device__ __forceinline__ void load_lora_b(const GemmArgs& a, int src, int y, uint4& lo, uint4& hi) {
-  const __nv_bfloat16* B = a.BL[src];
-  const int rank = a.rank;
-  lo = make_uint4(0u, 0u, 0u, 0u);
-  hi = lo;
-  if (!B || y >= a.b_rows[src]) return;
-  const __nv_bfloat16* br = B + (size_t)y * rank;
-  if (rank >= 16) {
-    lo = reinterpret_cast<const uint4*>(br)[0];
-    hi = reinterpret_cast<const uint4*>(br)[1];
-  } else if (rank == 8) {
-    lo = reinterpret_cast<const uint4*>(br)[0];
-  } else {
-    const uint2 v = reinterpret_cast<const uint2*>(br)[0];
-    lo.x = v.x;
-    lo.y = v.y;
-  }
-}
-
-__device__ __forceinline__ void store_lora_b(const GemmArgs& a, int src, int xa_base, int steps, uint4 lo, uint4 hi,
-                                             uint8_t* sb, int i) {
-  const bool has = a.BL[src] != nullptr;
-  const int slot = a.bl_slot[src];
-  const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
-  uint8_t* row = sb + i * 128;
-#pragma unroll
-  for (int c = 0; c < 8; ++c) {
-    if (c >= 2 * steps) break;
-    const bool mine = has && xa_base / 32 + (c >> 2) == slot;
-    *reinterpret_cast<uint4*>(row + ((c ^ (i & 7)) << 4)) = mine ? ((c & 1) ? hi : lo) : zero;
-  }
-}
+// Stage layout: the A tile (this CTA's 128 rows x 64), the B tile (its 128 rows x 64) and, for XA
+// tiles, the LoRA A rows of its half of the XA product (up to 32 rows x 64); 128-byte swizzle.
+constexpr int kABytes = BM * BK * 2;
+constexpr int kBBytes = 128 * BK * 2;
+constexpr int kLaBytes = 32 * BK * 2;
+constexpr int kStageBytes = kABytes + kBBytes + kLaBytes;
+constexpr int kPair = 2;
 
 // Producer ring position (stage, phase) and whether every wait so far succeeded.
 struct Ring {
@@ -445,106 +390,210 @@ __device__ __forceinline__ void ring_next(Ring& r) {
   }
 }
 
-// Copies of a down tile: per K block the row block's x rows and the LoRA A rows of this CTA's
-// half of the tile's N (16 rows per XA slot; CTA r takes slots [r * spc, r * spc + spc)).
-template <int STAGES, int PAIR, int A_BYTES, int STAGE_BYTES>
-__device__ __noinline__ Ring load_down_tile(const GemmArgs& a, int m0, uint32_t rank, bool leader, uint8_t* smem,
-                                            uint64_t* full_bar, uint64_t* empty_bar, int* armed_parity,
-                                            volatile int* abort_flag, Ring ring) {
-  const int spc = a.down_n / (16 * PAIR);
+// B rows of an output tile staged by CTA `rank`: its share of the tile (plain) or its segment of
+// the stacked tile; with the map index of the first of them.
+template <int BN>
+__device__ __forceinline__ void tile_b_rows(const GemmArgs& a, const Tile& tl, uint32_t rank, int& g0, int& nb,
+                                            int& yb, int& b_step) {
+  const int nseg = a.nseg;
+  const int seg_rows = BN / nseg;
+  const int per = nseg / kPair;
+  g0 = nseg == 1 ? tl.g : tl.g + static_cast<int>(rank) * per;
+  nb = nseg == 1 ? 1 : per;
+  yb = nseg == 1 ? tl.n_loc * BN + static_cast<int>(rank) * (BN / kPair) : tl.n_loc * seg_rows;
+  b_step = nseg == 1 ? 0 : seg_rows * BK * 2;
+}
+
+// Copies of an XA tile: per K block the tile's x and W rows, as for any output tile, and the LoRA
+// A rows of this CTA's half of the XA product (16 rows per XA slot; CTA r takes slots
+// [r * spc, r * spc + spc)). Its LoRA stage, if it has one, gets the BX rows only: the epilogue
+// warps write the A side from the XA product.
+template <int BN, int STAGES>
+__device__ __noinline__ Ring load_xa_tile(const GemmArgs& a, const Tile& tl, int m0, uint32_t rank, bool leader,
+                                          uint8_t* smem, uint64_t* full_bar, uint64_t* empty_bar,
+                                          int* armed_parity, volatile int* abort_flag, Ring ring) {
+  int g0, nb, yb, b_step;
+  tile_b_rows<BN>(a, tl, rank, g0, nb, yb, b_step);
+  const int spc = a.xa_n / (16 * kPair);
   const int s0 = static_cast<int>(rank) * spc, s1 = min(a.n_slots, s0 + spc);
-  const uint32_t bytes = PAIR * A_BYTES + a.n_slots * 16 * BK * 2;
+  const uint32_t bytes = kPair * (kABytes + kBBytes) + a.n_slots * 16 * BK * 2;
   for (int kb = 0; kb < a.num_kb; ++kb) {
     if (!mbar_wait(&empty_bar[ring.stage], ring.phase ^ 1, abort_flag, a.status)) {
       ring.ok = 0;
       return ring;
     }
-    uint8_t* sa = smem + ring.stage * STAGE_BYTES;
-    uint8_t* sb = sa + A_BYTES;
+    uint8_t* sa = smem + ring.stage * kStageBytes;
+    uint8_t* sb = sa + kABytes;
+    uint8_t* sl = sb + kBBytes;
     if (leader) {
       mbar_arrive_expect_tx(&full_bar[ring.stage], bytes);
       armed_parity[ring.stage] = ring.phase;
     }
-    if constexpr (PAIR == 2) {
-      const uint32_t bar = mapa_shared(&full_bar[ring.stage], 0);
-      tma_load_2d_pair(sa, &a.tmA, bar, kb * BK, m0);
-      for (int j = s0; j < s1; ++j) tma_load_2d_pair(sb + (j - s0) * 16 * BK * 2, &a.tmLA[j], bar, kb * BK, 0);
-    } else {
-      tma_load_2d(sa, &a.tmA, &full_bar[ring.stage], kb * BK, m0);
-      for (int j = s0; j < s1; ++j)
-        tma_load_2d(sb + (j - s0) * 16 * BK * 2, &a.tmLA[j], &full_bar[ring.stage], kb * BK, 0);
+    const uint32_t bar = mapa_shared(&full_bar[ring.stage], 0);
+    tma_load_2d_pair(sa, &a.tmA, bar, kb * BK, m0);
+    for (int j = 0; j < nb; ++j) tma_load_2d_pair(sb + j * b_step, &a.tmB[g0 + j], bar, kb * BK, yb);
+    for (int j = s0; j < s1; ++j) tma_load_2d_pair(sl + (j - s0) * 16 * BK * 2, &a.tmLA[j], bar, kb * BK, 0);
+    ring_next<STAGES>(ring);
+  }
+  if (a.ext_on[tl.g]) {
+    if (!mbar_wait(&empty_bar[ring.stage], ring.phase ^ 1, abort_flag, a.status)) {
+      ring.ok = 0;
+      return ring;
     }
+    uint8_t* sb = smem + ring.stage * kStageBytes + kABytes;
+    if (leader) {
+      mbar_arrive_expect_tx(&full_bar[ring.stage], kPair * kBBytes);
+      armed_parity[ring.stage] = ring.phase;
+    }
+    const uint32_t bar = mapa_shared(&full_bar[ring.stage], 0);
+    for (int j = 0; j < nb; ++j) tma_load_2d_pair(sb + j * b_step, &a.tmBX[g0 + j], bar, 0, yb);
     ring_next<STAGES>(ring);
   }
   return ring;
 }
 
-// The LoRA stage of an output tile: once the stage is free, let the epilogue warps write the B
-// rows (bl_go), wait until both CTAs of the row block's down tile have stored its XA rows, and
-// copy those rows (the A side of the K block).
-template <int STAGES, int PAIR, int A_BYTES, int STAGE_BYTES>
-__device__ __noinline__ Ring load_lora_stage(const GemmArgs& a, const Tile& tl, int m0, bool leader, uint8_t* smem,
-                                             uint64_t* full_bar, uint64_t* empty_bar, uint64_t* bl_go,
+// The LoRA stage of any other output tile: once the stage is free, wait (unless seen already)
+// until both CTAs of the row block's XA tile have stored its XA rows, and copy those rows (the A
+// side of the K block) and the tile's BX rows (the B side).
+template <int BN, int STAGES>
+__device__ __noinline__ Ring load_lora_stage(const GemmArgs& a, const Tile& tl, int m0, uint32_t rank, bool xa_ready,
+                                             bool leader, uint8_t* smem, uint64_t* full_bar, uint64_t* empty_bar,
                                              int* armed_parity, volatile int* abort_flag, Ring ring) {
   if (!mbar_wait(&empty_bar[ring.stage], ring.phase ^ 1, abort_flag, a.status)) {
     ring.ok = 0;
     return ring;
   }
-  mbar_arrive(&bl_go[ring.stage]);
-  if (!flag_wait(a.xa_flags + tl.m_blk, 4 * PAIR, abort_flag, a.status)) {
+  if (!xa_ready && !flag_wait(a.xa_flags + tl.m_blk, 4 * kPair, abort_flag, a.status)) {
     ring.ok = 0;
     return ring;
   }
-  fence_proxy_async_global();  // the TMA copy below reads what the down tile's stores wrote
-  uint8_t* sa = smem + ring.stage * STAGE_BYTES;
+  fence_proxy_async_global();  // the TMA copy below reads what the XA tile's stores wrote
+  int g0, nb, yb, b_step;
+  tile_b_rows<BN>(a, tl, rank, g0, nb, yb, b_step);
+  uint8_t* sa = smem + ring.stage * kStageBytes;
   if (leader) {
-    mbar_arrive_expect_tx(&full_bar[ring.stage], PAIR * A_BYTES);
+    mbar_arrive_expect_tx(&full_bar[ring.stage], kPair * (kABytes + kBBytes));
     armed_parity[ring.stage] = ring.phase;
   }
-  if constexpr (PAIR == 2)
-    tma_load_2d_pair(sa, &a.tmXA, mapa_shared(&full_bar[ring.stage], 0), a.xa_base[tl.g], m0);
-  else
-    tma_load_2d(sa, &a.tmXA, &full_bar[ring.stage], a.xa_base[tl.g], m0);
+  const uint32_t bar = mapa_shared(&full_bar[ring.stage], 0);
+  tma_load_2d_pair(sa, &a.tmXA, bar, a.xa_base[tl.g], m0);
+  for (int j = 0; j < nb; ++j) tma_load_2d_pair(sa + kABytes + j * b_step, &a.tmBX[g0 + j], bar, 0, yb);
   ring_next<STAGES>(ring);
   return ring;
 }
 
-// Between two epilogues, the epilogue warps write an output tile's LoRA B rows (one row per
-// thread) into its LoRA stage `st` once the producer has that stage free (bl_go), and count
-// themselves on the MMA-issuing CTA's bl_bar. False when the wait gave up.
-template <int STAGES, int PAIR, int A_BYTES, int STAGE_BYTES, int BN, int CTA_ROWS>
-__device__ __noinline__ bool write_lora_stage(const GemmArgs& a, const Tile& tl, uint32_t rank, int st, int b_row,
-                                              int lane, uint8_t* smem, uint64_t* bl_go, uint64_t* bl_bar,
-                                              uint32_t* go_parity, volatile int* abort_flag) {
-  const int nseg = a.nseg;
-  const int g0 = nseg == 1 ? tl.g : tl.g + static_cast<int>(rank) * (nseg / PAIR);
-  const int yb = nseg == 1 ? tl.n_loc * BN + static_cast<int>(rank) * CTA_ROWS : tl.n_loc * (BN / nseg);
-  uint4 lo, hi;
-  load_lora_b(a, g0, yb + b_row, lo, hi);
-  bool w = true;
-  if (lane == 0) w = mbar_wait(&bl_go[st], (*go_parity >> st) & 1u, abort_flag, a.status);
-  if (!__shfl_sync(0xffffffffu, w ? 1 : 0, 0)) return false;
-  *go_parity ^= 1u << st;
-  store_lora_b(a, g0, a.xa_base[tl.g], a.ext_steps[tl.g], lo, hi, smem + st * STAGE_BYTES + A_BYTES, b_row);
-  fence_proxy_async_smem();  // the tensor core reads these stores
+// MMAs of an XA tile: per K block the tile's product into d_tmem and the XA product x A^T into
+// the other accumulator's first xa_n columns (x_tmem); then xa_full for the epilogue warps, which
+// drain the XA product (xa_done, having written it into the tile's LoRA stage) before the LoRA
+// stage, or the next tile, may use those columns.
+template <int BN, int STAGES>
+__device__ __noinline__ Ring mma_xa_tile(const GemmArgs& a, const Tile& tl, uint32_t d_tmem, uint32_t x_tmem,
+                                         uint32_t idesc, uint32_t idesc_xa, uint8_t* smem, uint64_t* full_bar,
+                                         uint64_t* empty_bar, uint64_t* xa_full, uint64_t* xa_done,
+                                         uint32_t xa_parity, volatile int* abort_flag, Ring ring) {
+  for (int kb = 0; kb < a.num_kb; ++kb) {
+    if (!mbar_wait(&full_bar[ring.stage], ring.phase, abort_flag, a.status)) {
+      ring.ok = 0;
+      return ring;
+    }
+    tc_fence_after();
+    const uint32_t sa = smem_u32(smem + ring.stage * kStageBytes);
+    const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
+    const uint64_t bd = smem_desc(sa + kABytes, 16, 1024, kSwizzle128B);
+    const uint64_t ld = smem_desc(sa + kABytes + kBBytes, 16, 1024, kSwizzle128B);
+#pragma unroll
+    for (int k = 0; k < BK / 16; ++k) {
+      const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
+      mma_bf16_ss_pair(d_tmem, ad + 2 * k, bd + 2 * k, idesc, acc);
+      mma_bf16_ss_pair(x_tmem, ad + 2 * k, ld + 2 * k, idesc_xa, acc);
+    }
+    mma_commit_pair(&empty_bar[ring.stage], 0x3);
+    ring_next<STAGES>(ring);
+  }
+  mma_commit_pair(xa_full, 0x3);
+  if (!mbar_wait<true>(xa_done, xa_parity, abort_flag, a.status)) {
+    ring.ok = 0;
+    return ring;
+  }
+  tc_fence_after();
+  if (a.ext_on[tl.g]) {
+    // BX copies landed; the A side (the XA product) came with xa_done
+    if (!mbar_wait(&full_bar[ring.stage], ring.phase, abort_flag, a.status)) {
+      ring.ok = 0;
+      return ring;
+    }
+    tc_fence_after();
+    const uint32_t sa = smem_u32(smem + ring.stage * kStageBytes);
+    const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
+    const uint64_t bd = smem_desc(sa + kABytes, 16, 1024, kSwizzle128B);
+    for (int k = 0; k < a.ext_steps[tl.g]; ++k) mma_bf16_ss_pair(d_tmem, ad + 2 * k, bd + 2 * k, idesc, 1u);
+    mma_commit_pair(&empty_bar[ring.stage], 0x3);
+    ring_next<STAGES>(ring);
+  }
+  return ring;
+}
+
+// XA tile, after its main loop: slot j of the XA product (columns 16j .. 16j + 15 of x_tmem) is
+// x A_j^T for this thread's row. Scaled by alpha / r it is stored as hi = bf16(v) at XA columns
+// 32j.. and lo = bf16(v - hi) at 32j + 16.. (the pair carries about 16 mantissa bits): to the XA
+// buffer for the row block's other tiles, and into the tile's own LoRA stage `st` (A side, the 64
+// columns from xa_base) when it has one. Then xa_done for the MMAs and the row block's ready word.
+template <int BN>
+__device__ __noinline__ bool drain_xa(const GemmArgs& a, const Tile& tl, uint32_t x_tmem, int row, int row_in_cta,
+                                      int st, int lane, uint8_t* smem, uint64_t* xa_full, uint64_t* xa_done,
+                                      uint32_t xa_parity, volatile int* abort_flag) {
+  if (!__all_sync(0xffffffffu, mbar_wait(xa_full, xa_parity, abort_flag, a.status))) return false;
+  tc_fence_after();
+  const bool ext = a.ext_on[tl.g] != 0;
+  const int xb = a.xa_base[tl.g];
+  uint8_t* arow = smem + st * kStageBytes + row_in_cta * 128;
+  uint32_t r0[16];
+  float v[16], w[16];
+#pragma unroll 1
+  for (int j = 0; j < a.n_slots; ++j) {
+    tmem_ld16(x_tmem + 16 * j, r0);
+    tmem_ld_wait();
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      v[i] = __uint_as_float(r0[i]) * a.scale;
+      w[i] = v[i] - __bfloat162float(__float2bfloat16_rn(v[i]));
+    }
+    if (row < a.M) {
+      store16_bf16(a.xa + (size_t)row * kXaCols + 32 * j, v);
+      store16_bf16(a.xa + (size_t)row * kXaCols + 32 * j + 16, w);
+    }
+    const int c0 = (32 * j - xb) / 8;  // 16-byte unit of hi within the stage's 64 columns
+    if (ext && 32 * j >= xb && 32 * j < xb + BK) {
+      uint4 q[4];
+      q[0] = make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7]));
+      q[1] = make_uint4(pack_bf16(v[8], v[9]), pack_bf16(v[10], v[11]), pack_bf16(v[12], v[13]),
+                        pack_bf16(v[14], v[15]));
+      q[2] = make_uint4(pack_bf16(w[0], w[1]), pack_bf16(w[2], w[3]), pack_bf16(w[4], w[5]), pack_bf16(w[6], w[7]));
+      q[3] = make_uint4(pack_bf16(w[8], w[9]), pack_bf16(w[10], w[11]), pack_bf16(w[12], w[13]),
+                        pack_bf16(w[14], w[15]));
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        *reinterpret_cast<uint4*>(arow + (((c0 + u) ^ (row_in_cta & 7)) << 4)) = q[u];
+    }
+  }
+  // TMEM columns read (tcgen05.wait::ld above); XA rows visible to the tensor core of this CTA
+  // (shared) and to the other tiles' copies (global, GPU scope)
+  tc_fence_before();
+  fence_proxy_async_smem();
+  __threadfence();
+  fence_proxy_async_global();
   __syncwarp();
   if (lane == 0) {
-    if constexpr (PAIR == 2)
-      mbar_arrive_cluster(mapa_shared(&bl_bar[st], 0));
-    else
-      mbar_arrive(&bl_bar[st]);
+    mbar_arrive_cluster(mapa_shared(xa_done, 0));
+    atomicAdd(a.xa_flags + tl.m_blk, 1);
   }
   return true;
 }
 
-template <int BN, int STAGES, int PAIR, int EPI>
+template <int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
-  constexpr int CTA_ROWS = BN / PAIR;  // B rows staged by this CTA
-  constexpr int A_BYTES = BM * BK * 2;
-  constexpr int B_BYTES = CTA_ROWS * BK * 2;
-  constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  constexpr uint32_t TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128
-                                                    : (2 * BN <= 256) ? 256 : 512;
+  static_assert(BN == 256 && kBBytes == (BN / kPair) * BK * 2, "CTA-pair tiles of 256 columns");
+  constexpr uint32_t TMEM_COLS = 2 * BN;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -553,8 +602,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   __shared__ __align__(8) uint64_t tfull_bar[2];
   __shared__ __align__(8) uint64_t tempty_bar[2];
   __shared__ __align__(8) uint64_t drain_bar;
-  __shared__ __align__(8) uint64_t bl_bar[STAGES];  // LoRA B rows written (each epilogue warp of both CTAs)
-  __shared__ __align__(8) uint64_t bl_go[STAGES];   // LoRA stage free for the B rows (producer)
+  __shared__ __align__(8) uint64_t xa_full;         // an XA tile's MMAs done (MMA commit)
+  __shared__ __align__(8) uint64_t xa_done;         // its XA product drained (each epilogue warp of both CTAs)
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_flag;
   // a rejected call: every CTA of every cluster sees the same word and leaves before any set-up
@@ -562,23 +611,23 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const uint32_t rank = PAIR == 2 ? cluster_ctarank() : 0u;
+  const uint32_t rank = cluster_ctarank();
   const bool leader = rank == 0;
-  const int unit = blockIdx.x / PAIR;
-  const int n_units = gridDim.x / PAIR;
+  const int unit = blockIdx.x / kPair;
+  const int n_units = gridDim.x / kPair;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
-      mbar_init(&bl_bar[s], 4 * PAIR);
-      mbar_init(&bl_go[s], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);
-      mbar_init(&tempty_bar[i], 4 * PAIR);
+      mbar_init(&tempty_bar[i], 4 * kPair);
     }
     mbar_init(&drain_bar, 1);
+    mbar_init(&xa_full, 1);
+    mbar_init(&xa_done, 4 * kPair);
     abort_flag = 0;
     fence_barrier_init();
   }
@@ -588,47 +637,44 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     if (a.n_slots > 0) {
       tma_prefetch_desc(&a.tmXA);
       for (int i = 0; i < a.n_slots; ++i) tma_prefetch_desc(&a.tmLA[i]);
+      for (int i = 0; i < 3; ++i) tma_prefetch_desc(&a.tmBX[i]);
     }
   }
   if (warp == 1) {
-    if constexpr (PAIR == 2) {
-      tmem_alloc_pair(&tmem_base_sh, TMEM_COLS);
-      tmem_relinquish_pair();
-    } else {
-      tmem_alloc(&tmem_base_sh, TMEM_COLS);
-      tmem_relinquish();
-    }
+    tmem_alloc_pair(&tmem_base_sh, TMEM_COLS);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  if constexpr (PAIR == 2) cluster_sync(); else __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = tmem_base_sh;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer (every CTA)
     // The per-stage loop of the output tiles stays minimal (one thread, on the critical path of
-    // every stage); down tiles and the LoRA stage go through out-of-line helpers.
+    // every stage); XA tiles and the LoRA stage go through out-of-line helpers.
     if (lane == 0) {
       Ring ring{0, 0u, 1};
       int armed_parity[STAGES];
       for (int s = 0; s < STAGES; ++s) armed_parity[s] = -1;
       for (int t = unit; t < a.total_tiles && ring.ok; t += n_units) {
         const Tile tl = decode_tile(t, a);
-        const int m0 = tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM;
-        if (tl.down) {
-          ring = load_down_tile<STAGES, PAIR, A_BYTES, STAGE_BYTES>(a, m0, rank, leader, smem, full_bar, empty_bar,
-                                                                   armed_parity, &abort_flag, ring);
+        const int m0 = tl.m_blk * (BM * kPair) + static_cast<int>(rank) * BM;
+        if (tl.xa) {
+          ring = load_xa_tile<BN, STAGES>(a, tl, m0, rank, leader, smem, full_bar, empty_bar, armed_parity,
+                                          &abort_flag, ring);
           continue;
         }
-        const bool ext_tile = a.ext_on[tl.g] != 0;
-        const int nseg = a.nseg;
-        const int seg_rows = BN / nseg;
-        const int per = nseg / PAIR;
-        // B rows of this CTA: the tile's CTA share (one segment) or its stacked segments
-        const int g0 = nseg == 1 ? tl.g : tl.g + static_cast<int>(rank) * per;
-        const int nb = nseg == 1 ? 1 : per;
-        const int yb = nseg == 1 ? tl.n_loc * BN + static_cast<int>(rank) * CTA_ROWS : tl.n_loc * seg_rows;
-        const int b_step = nseg == 1 ? 0 : seg_rows * BK * 2;
+        int g0, nb, yb, b_step;
+        tile_b_rows<BN>(a, tl, rank, g0, nb, yb, b_step);
+        // Whether the row block's XA rows are stored, asked (acquire) while the stages already
+        // copied still feed the MMAs; only a tile whose XA tile has not finished by then waits at
+        // its LoRA stage.
+        int xa_ready = 0;
+        if (a.ext_on[tl.g]) {
+          asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(xa_ready) : "l"(a.xa_flags + tl.m_blk) : "memory");
+          xa_ready = xa_ready >= 4 * kPair;
+        }
         int stage = ring.stage;
         uint32_t phase = ring.phase;
         for (int kb = 0; kb < a.num_kb; ++kb) {
@@ -636,22 +682,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             ring.ok = 0;
             break;
           }
-          uint8_t* sa = smem + stage * STAGE_BYTES;
-          uint8_t* sb = sa + A_BYTES;
+          uint8_t* sa = smem + stage * kStageBytes;
+          uint8_t* sb = sa + kABytes;
           // the MMA-issuing CTA's full barrier counts the bytes of both CTAs
           if (leader) {
-            mbar_arrive_expect_tx(&full_bar[stage], PAIR * STAGE_BYTES);
+            mbar_arrive_expect_tx(&full_bar[stage], kPair * (kABytes + kBBytes));
             armed_parity[stage] = phase;
           }
           const CUtensorMap* mB = &a.tmB[g0];
-          if constexpr (PAIR == 2) {
-            const uint32_t bar = mapa_shared(&full_bar[stage], 0);
-            tma_load_2d_pair(sa, &a.tmA, bar, kb * BK, m0);
-            for (int j = 0; j < nb; ++j) tma_load_2d_pair(sb + j * b_step, mB + j, bar, kb * BK, yb);
-          } else {
-            tma_load_2d(sa, &a.tmA, &full_bar[stage], kb * BK, m0);
-            for (int j = 0; j < nb; ++j) tma_load_2d(sb + j * b_step, mB + j, &full_bar[stage], kb * BK, yb);
-          }
+          const uint32_t bar = mapa_shared(&full_bar[stage], 0);
+          tma_load_2d_pair(sa, &a.tmA, bar, kb * BK, m0);
+          for (int j = 0; j < nb; ++j) tma_load_2d_pair(sb + j * b_step, mB + j, bar, kb * BK, yb);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
@@ -659,9 +700,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
         ring.stage = stage;
         ring.phase = phase;
-        if (ring.ok && ext_tile)
-          ring = load_lora_stage<STAGES, PAIR, A_BYTES, STAGE_BYTES>(a, tl, m0, leader, smem, full_bar, empty_bar, bl_go,
-                                                      armed_parity, &abort_flag, ring);
+        if (ring.ok && a.ext_on[tl.g])
+          ring = load_lora_stage<BN, STAGES>(a, tl, m0, rank, xa_ready != 0, leader, smem, full_bar, empty_bar,
+                                             armed_parity, &abort_flag, ring);
       }
       if (!ring.ok) {
         if (leader) {
@@ -682,74 +723,81 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (even CTA)
     if (lane == 0 && leader) {
-      int stage = 0;
-      uint32_t phase = 0;
+      Ring ring{0, 0u, 1};
       int it = 0;
-      bool ok = true;
       bool issued = false;
-      const uint32_t idesc_tile = idesc_bf16_f32(BM * PAIR, BN);
-      const uint32_t idesc_down = idesc_bf16_f32(BM * PAIR, a.n_slots > 0 ? a.down_n : 32);
-      uint32_t bl_parity = 0;  // bit s: phase of bl_bar[s] to wait for next
-      for (int t = unit; t < a.total_tiles && ok; t += n_units, ++it) {
+      const uint32_t idesc = idesc_bf16_f32(BM * kPair, BN);
+      const uint32_t idesc_xa = idesc_bf16_f32(BM * kPair, a.n_slots > 0 ? a.xa_n : 32);
+      uint32_t xa_it = 0;      // XA tiles so far (phase of xa_done)
+      for (int t = unit; t < a.total_tiles && ring.ok; t += n_units, ++it) {
         const Tile tl = decode_tile(t, a);
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
-        if (!mbar_wait<PAIR == 2>(&tempty_bar[acc], acc_phase ^ 1, &abort_flag, a.status)) {
-          ok = false;
+        if (!mbar_wait<true>(&tempty_bar[acc], acc_phase ^ 1, &abort_flag, a.status)) {
+          ring.ok = 0;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        const int ext_steps = !tl.down && a.ext_on[tl.g] ? a.ext_steps[tl.g] : 0;
-        const uint32_t idesc = tl.down ? idesc_down : idesc_tile;
-        auto mma = [&](uint64_t ad, uint64_t bd, uint32_t accum) {
-          if constexpr (PAIR == 2)
-            mma_bf16_ss_pair(d_tmem, ad, bd, idesc, accum);
-          else
-            mma_bf16_ss(d_tmem, ad, bd, idesc, accum);
-        };
-        auto release = [&]() {
-          if constexpr (PAIR == 2) mma_commit_pair(&empty_bar[stage], 0x3); else mma_commit(&empty_bar[stage]);
+        if (tl.xa) {
+          // the XA product takes the other accumulator's first columns: its previous tile's
+          // epilogue must have drained them
+          if (!mbar_wait<true>(&tempty_bar[acc ^ 1], (((it + 1) >> 1) & 1) ^ 1, &abort_flag, a.status)) {
+            ring.ok = 0;
+            break;
+          }
+          tc_fence_after();
+          ring = mma_xa_tile<BN, STAGES>(a, tl, d_tmem, tmem_base + (acc ^ 1) * BN, idesc, idesc_xa, smem, full_bar,
+                                         empty_bar, &xa_full, &xa_done, xa_it & 1u, &abort_flag, ring);
+          ++xa_it;
+          issued = true;
+          if (!ring.ok) break;
+          mma_commit_pair(&tfull_bar[acc], 0x3);
+          continue;
+        }
+        int stage = ring.stage;
+        uint32_t phase = ring.phase;
+        for (int kb = 0; kb < a.num_kb; ++kb) {
+          if (!mbar_wait(&full_bar[stage], phase, &abort_flag, a.status)) {
+            ring.ok = 0;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * kStageBytes);
+          const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
+          const uint64_t bd = smem_desc(sa + kABytes, 16, 1024, kSwizzle128B);
+          // K = 16 steps advance 32 bytes = 2 units of the descriptor's start-address field
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            mma_bf16_ss_pair(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          issued = true;
+          mma_commit_pair(&empty_bar[stage], 0x3);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
           }
-        };
-        for (int kb = 0; kb < a.num_kb; ++kb) {
-          if (!mbar_wait(&full_bar[stage], phase, &abort_flag, a.status)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
-          const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
-          const uint64_t bd = smem_desc(sa + A_BYTES, 16, 1024, kSwizzle128B);
-          // K = 16 steps advance 32 bytes = 2 units of the descriptor's start-address field
-#pragma unroll
-          for (int k = 0; k < BK / 16; ++k) mma(ad + 2 * k, bd + 2 * k, (kb > 0 || k > 0) ? 1u : 0u);
-          issued = true;
-          release();
         }
-        if (ok && ext_steps > 0) {
-          // the XA copies have landed and both CTAs have written their LoRA B rows
-          if (!mbar_wait(&full_bar[stage], phase, &abort_flag, a.status) ||
-              !mbar_wait<PAIR == 2>(&bl_bar[stage], (bl_parity >> stage) & 1u, &abort_flag, a.status)) {
-            ok = false;
+        ring.stage = stage;
+        ring.phase = phase;
+        if (ring.ok && a.ext_on[tl.g]) {
+          // the XA and BX copies have landed
+          if (!mbar_wait(&full_bar[ring.stage], ring.phase, &abort_flag, a.status)) {
+            ring.ok = 0;
           } else {
-            bl_parity ^= 1u << stage;
             tc_fence_after();
-            const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+            const uint32_t sa = smem_u32(smem + ring.stage * kStageBytes);
             const uint64_t ad = smem_desc(sa, 16, 1024, kSwizzle128B);
-            const uint64_t bd = smem_desc(sa + A_BYTES, 16, 1024, kSwizzle128B);
-            for (int k = 0; k < ext_steps; ++k) mma(ad + 2 * k, bd + 2 * k, 1u);
-            release();
+            const uint64_t bd = smem_desc(sa + kABytes, 16, 1024, kSwizzle128B);
+            for (int k = 0; k < a.ext_steps[tl.g]; ++k) mma_bf16_ss_pair(d_tmem, ad + 2 * k, bd + 2 * k, idesc, 1u);
+            mma_commit_pair(&empty_bar[ring.stage], 0x3);
+            ring_next<STAGES>(ring);
           }
         }
-        if (!ok) break;
-        if constexpr (PAIR == 2) mma_commit_pair(&tfull_bar[acc], 0x3); else mma_commit(&tfull_bar[acc]);
+        if (!ring.ok) break;
+        mma_commit_pair(&tfull_bar[acc], 0x3);
       }
-      if (!ok && issued) {
-        if constexpr (PAIR == 2) mma_commit_pair(&drain_bar, 0x1); else mma_commit(&drain_bar);
+      if (!ring.ok && issued) {
+        mma_commit_pair(&drain_bar, 0x1);
         volatile int never = 0;
         mbar_wait(&drain_bar, 0, &never, nullptr);
       }
@@ -758,58 +806,46 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     // ------------------------------------------------------------ epilogue (warps 2..5, every CTA)
     const int quarter = warp & 3;  // TMEM lane quarter this warp may access
     const int row_in_cta = quarter * 32 + lane;
-    const int b_row = (warp - 2) * 32 + lane;  // LoRA B row this thread writes
     uint32_t tempty_addr[2];
-    for (int i = 0; i < 2; ++i)
-      tempty_addr[i] = PAIR == 2 ? mapa_shared(&tempty_bar[i], 0) : smem_u32(&tempty_bar[i]);
+    for (int i = 0; i < 2; ++i) tempty_addr[i] = mapa_shared(&tempty_bar[i], 0);
     int pos = 0;             // producer stages used by the tiles before this one
-    uint32_t go_parity = 0;  // bit s: phase of bl_go[s] to wait for next
+    uint32_t xa_it = 0;      // XA tiles so far (phase of xa_full)
     int it = 0;
     for (int t = unit; t < a.total_tiles; t += n_units, ++it) {
       const Tile tl = decode_tile(t, a);
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
-      const bool ext_tile = !tl.down && a.ext_on[tl.g] != 0;
-      if (ext_tile &&
-          !write_lora_stage<STAGES, PAIR, A_BYTES, STAGE_BYTES, BN, CTA_ROWS>(a, tl, rank, (pos + a.num_kb) % STAGES,
-                                                                            b_row, lane, smem, bl_go, bl_bar,
-                                                                            &go_parity, &abort_flag))
-        break;
-      pos += tl.down ? a.num_kb : a.num_kb + (ext_tile ? 1 : 0);
+      const bool ext_tile = a.ext_on[tl.g] != 0;
+      const int st = (pos + a.num_kb) % STAGES;  // the tile's LoRA stage
+      const int row = tl.m_blk * (BM * kPair) + static_cast<int>(rank) * BM + row_in_cta;
+      if (tl.xa) {
+        const uint32_t x_tmem = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + (acc ^ 1) * BN;
+        if (!drain_xa<BN>(a, tl, x_tmem, row, row_in_cta, st, lane, smem, &xa_full, &xa_done, xa_it & 1u,
+                          &abort_flag))
+          break;
+        ++xa_it;
+      }
+      pos += a.num_kb + (ext_tile ? 1 : 0);
       // warp-uniform outcome: the TMEM loads of the epilogue are warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait(&tfull_bar[acc], acc_phase, &abort_flag, a.status)))
         break;
       tc_fence_after();
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      const int row = tl.m_blk * (BM * PAIR) + static_cast<int>(rank) * BM + row_in_cta;
-      if (tl.down)
-        epilogue_down(a, tacc, row);
-      else
-        epilogue_tile<BN, EPI>(a, tl, tacc, row);
+      epilogue_tile<BN, EPI>(a, tl, tacc, row);
       // the accumulator is free once this warp's TMEM loads have completed (tcgen05.wait::ld in
       // the epilogue); the tile's global stores need not be visible first, so the arrival on
       // the MMA-issuing CTA's barrier is relaxed
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        if constexpr (PAIR == 2) mbar_arrive_cluster_relaxed(tempty_addr[acc]); else mbar_arrive(&tempty_bar[acc]);
-      }
-      if (tl.down) {
-        // publish this warp's XA rows: GPU-scope fence, then count the warp in the block's word
-        // (4 warps x both CTAs); the readers load them with TMA after an acquire
-        __threadfence();
-        fence_proxy_async_global();
-        __syncwarp();
-        if (lane == 0) atomicAdd(a.xa_flags + tl.m_blk, 1);
-      }
+      if (lane == 0) mbar_arrive_cluster_relaxed(tempty_addr[acc]);
     }
   }
 
   tc_fence_before();
-  if constexpr (PAIR == 2) cluster_sync(); else __syncthreads();
+  cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    if constexpr (PAIR == 2) tmem_dealloc_pair(tmem_base, TMEM_COLS); else tmem_dealloc(tmem_base, TMEM_COLS);
+    tmem_dealloc_pair(tmem_base, TMEM_COLS);
   }
 }
 
@@ -847,10 +883,11 @@ bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int ld, int 
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, int PAIR, int EPI>
+template <int BN, int STAGES, int EPI>
 cudaError_t launch_impl(GemmArgs& args, int num_sms, cudaStream_t stream) {
-  constexpr int smem = STAGES * (BM * BK * 2 + (BN / PAIR) * BK * 2) + 1024;
-  auto kern = gemm_tc_kernel<BN, STAGES, PAIR, EPI>;
+  constexpr int PAIR = kPair;
+  constexpr int smem = STAGES * kStageBytes + 1024;
+  auto kern = gemm_tc_kernel<BN, STAGES, EPI>;
   // the attributes and the co-resident cluster count are per device
   static PerDevice once;
   static std::atomic<int> units_of[64];
@@ -881,11 +918,11 @@ cudaError_t launch_impl(GemmArgs& args, int num_sms, cudaStream_t stream) {
     once.done(dev);
   }
   // every unit of the grid is resident at once (one CTA per SM): a tile that waits for its row
-  // block's down tile never waits on a unit that has not started
+  // block's XA tile never waits on a unit that has not started
   const int units = std::max(1, std::min(max_units, args.total_tiles));
-  // down tiles one wave of units ahead of their row block's first output tiles
-  const int w0 = std::min(kRasterGroup, args.total_n);
-  args.down_lead = (units + w0) / (w0 + 1);
+  // every XA tile first: consecutive tiles go to consecutive units, so the XA products (and the
+  // extra MMAs they cost) spread over the units instead of piling on a few
+  args.xa_lead = args.row_tiles;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -918,9 +955,6 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t stream) {
     if (!make_map(&a.tmB[i], d.B[src], d.B_rows[src], d.K, d.ldb[src], b_box, BK,
                   CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
-    a.BL[i] = i < nmaps ? static_cast<const __nv_bfloat16*>(d.BL[i]) : nullptr;
-    a.bl_slot[i] = i < nmaps && d.BL[i] ? d.bl_slot[i] : -1;
-    a.b_rows[i] = d.B_rows[src];
   }
   bool any_ext = false;
   for (int g = 0; g < d.ngroups; ++g) any_ext |= d.ext_on[g] != 0;
@@ -941,11 +975,21 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t stream) {
           d.ext_steps[g] < 1 || d.ext_steps[g] > BK / 16)
         return cudaErrorInvalidValue;
     }
-    for (int i = 0; i < nmaps; ++i)
-      if (d.BL[i] && (d.bl_slot[i] < 0 || d.bl_slot[i] >= d.n_slots)) return cudaErrorInvalidValue;
+    for (int i = 0; i < 3; ++i) {
+      int src = (i < nmaps && d.BX[i]) ? i : -1;
+      if (src < 0)
+        for (int j = 0; j < nmaps; ++j)
+          if (d.BX[j]) src = j;  // unused slots alias a valid map
+      if (src < 0) return cudaErrorInvalidValue;
+      if (!make_map(&a.tmBX[i], d.BX[src], d.B_rows[src], kBxCols, kBxCols, b_box, BK, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    }
+    for (int g = 0; g < d.ngroups; ++g)
+      for (int s = 0; s < (d.ngroups == 1 ? d.nseg : 1); ++s)
+        if (d.ext_on[g] && !d.BX[g + s]) return cudaErrorInvalidValue;
   } else {
     a.tmXA = a.tmA;
-    for (int i = 0; i < 3; ++i) a.tmLA[i] = a.tmA;
+    for (int i = 0; i < 3; ++i) a.tmLA[i] = a.tmBX[i] = a.tmA;
   }
   a.M = d.M;
   a.K = d.K;
@@ -967,11 +1011,11 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t stream) {
   a.row_tiles = (d.M + BM * pair - 1) / (BM * pair);
   a.n_slots = any_ext ? d.n_slots : 0;
   // two CTA halves of 16 x ceil(n_slots / 2) rows: N = 32 for one or two slots, 64 for three
-  a.down_n = 32 * ((a.n_slots + 1) / 2);
+  a.xa_n = 32 * ((a.n_slots + 1) / 2);
   a.rank = d.rank;
   a.xa = static_cast<__nv_bfloat16*>(d.XA);
   a.xa_flags = d.xa_flags;
-  a.total_tiles = a.row_tiles * a.total_n + (a.n_slots > 0 ? a.row_tiles : 0);
+  a.total_tiles = a.row_tiles * a.total_n;
   a.epi = d.epi;
   a.scale = d.scale;
   a.out = static_cast<__nv_bfloat16*>(d.out);
@@ -993,9 +1037,9 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t stream) {
   // one kernel per epilogue: each carries only its own epilogue code, which keeps the hot loops
   // of all its warps inside the SM's instruction cache
   switch (d.epi) {
-    case kEpiQkv: return launch_impl<bn, 6, pair, kEpiQkv>(a, num_sms, stream);
-    case kEpiResid: return launch_impl<bn, 6, pair, kEpiResid>(a, num_sms, stream);
-    case kEpiSwiGLU: return launch_impl<bn, 6, pair, kEpiSwiGLU>(a, num_sms, stream);
+    case kEpiQkv: return launch_impl<bn, 6, kEpiQkv>(a, num_sms, stream);
+    case kEpiResid: return launch_impl<bn, 6, kEpiResid>(a, num_sms, stream);
+    case kEpiSwiGLU: return launch_impl<bn, 6, kEpiSwiGLU>(a, num_sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -33,9 +33,10 @@ constexpr int kPage = 16;
 constexpr int kRankPad = 16;  // LoRA rank padded to one K=16 MMA step
 // The scaled LoRA down product is kept as a bf16 pair hi + lo (lo = bf16(v - hi)): module
 // slot j holds hi at columns [32j, 32j + 16) and lo at [32j + 16, 32j + 32) of a [rows, kXaCols]
-// buffer. A projection GEMM computes it for its rows (down tiles) and reads it back as one
-// 64-wide K block against the adapter's B rows (the up product).
+// buffer. A projection GEMM computes it for its rows and reads it back as one 64-wide K block
+// against BX = [B | B] rows (kBxCols wide) of the module (the up product).
 constexpr int kXaCols = 128;
+constexpr int kBxCols = 64;
 
 // Programmatic dependent launch for chains of short kernels. While a PdlScope is alive on the
 // calling thread, the launchers below that go through launch_kernel() give their kernels the
@@ -98,17 +99,15 @@ struct GemmDesc {
   int B_rows[3];          // rows of each B matrix
   int ldb[3];
   int group_cols[3];      // valid output columns per group (plain) / per segment (stacked)
-  // Unmerged LoRA (Eq. S3), computed inside the same launch. Down tiles (one per 256-row block)
-  // form XA[:, 32j .. 32j + 32) = hi/lo of (alpha/r) x A_j^T for the n_slots adapted modules
-  // (LA[j] = A_j, [rank, K]) and raise xa_flags[row block]; every output tile of an adapted
-  // group then adds one K block: XA[:, xa_base[g] .. + 64] against the module's B rows, placed
-  // under the K steps of its own slot (BL[i] = B of map index i, [B_rows[i], rank]; bl_slot[i]
-  // its XA slot, -1 without adapter).
+  // Unmerged LoRA (Eq. S3), computed inside the same launch. The first output tile of each
+  // 256-row block also forms XA[:, 32j .. 32j + 32) = hi/lo of (alpha/r) x A_j^T for the n_slots
+  // adapted modules (LA[j] = A_j, [rank, K]) and raises xa_flags[row block]; every output tile of
+  // an adapted group then adds one K block: XA[:, xa_base[g] .. + 64] against BX[i] (the module's
+  // [B | B] rows under its slot, zeros elsewhere; [B_rows[i], kBxCols], map index i like B).
   void* XA;
   int n_slots;
   const void* LA[3];
-  const void* BL[3];      // map index g + s, like B
-  int bl_slot[3];
+  const void* BX[3];
   int rank;
   float scale;            // alpha / r
   int* xa_flags;          // [row blocks of 256], zero before the launch
@@ -139,8 +138,19 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t stream);
 // ------------------------------------------------------------------ other kernels
 cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double theta,
                               cudaStream_t stream);
+// BX rows of up to 4 modules: out[m][r, :] = 0 except columns [col_off[m], col_off[m] + 32) =
+// [B_m[r, 0:16] | B_m[r, 0:16]] (rank padded with zeros); a null B_m gives all-zero rows.
+struct BextDesc {
+  const __nv_bfloat16* B[4];
+  __nv_bfloat16* out[4];
+  int rows[4];
+  int col_off[4];
+  int n, rank;
+};
+// RMSNorm of `rows` rows; with `bx`, the same launch also builds those BX rows (extra blocks).
 cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bfloat16* y,
-                           int rows, int hidden, float eps, cudaStream_t stream);
+                           int rows, int hidden, float eps, cudaStream_t stream,
+                           const BextDesc* bx = nullptr);
 // Token ids outside [0, vocab) read row 0 and set kStatusBounds in *status.
 cudaError_t launch_embed(const __nv_bfloat16* embed, const int32_t* tokens, __nv_bfloat16* out,
                          int n, int hidden, int vocab, int* status, cudaStream_t stream);

@@ -32,11 +32,46 @@ __global__ void rope_table_kernel(float2* table, int n_pos, int half, const __gr
   table[idx] = make_float2(c, s);
 }
 
-// ------------------------------------------------------------------ RMSNorm
-// One warp per row: y = x * rsqrt(mean(x^2) + eps) * g, fp32 math, bf16 out.
+// ------------------------------------------------------------------ RMSNorm (+ BX rows)
+// One 16-byte chunk (8 columns) of a BX row per thread: the module's B row (rank values, zero
+// padded to 16) at columns col_off .. col_off + 15 and again at col_off + 16 .. col_off + 31.
+__device__ __forceinline__ void bext_chunk(const BextDesc& d, long idx) {
+  int m = 0;
+  long base = 0;
+  while (m < d.n && idx >= base + static_cast<long>(d.rows[m]) * (kBxCols / 8)) {
+    base += static_cast<long>(d.rows[m]) * (kBxCols / 8);
+    ++m;
+  }
+  if (m >= d.n) return;
+  const long k = idx - base;
+  const int r = static_cast<int>(k / (kBxCols / 8));
+  const int c0 = static_cast<int>(k % (kBxCols / 8)) * 8;
+  const __nv_bfloat16* B = d.B[m];
+  uint32_t w[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    float v[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = c0 + 2 * j + h - d.col_off[m];
+      const int q = c & 15;
+      v[h] = (B && c >= 0 && c < 32 && q < d.rank) ? __bfloat162float(B[(size_t)r * d.rank + q]) : 0.f;
+    }
+    w[j] = pack_bf16(v[0], v[1]);
+  }
+  *reinterpret_cast<uint4*>(d.out[m] + (size_t)r * kBxCols + c0) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Blocks [0, norm_blocks): one warp per row, y = x * rsqrt(mean(x^2) + eps) * g, fp32 math, bf16
+// out. The blocks after them: the BX rows of `bx`, one chunk per thread.
 __global__ void rmsnorm_kernel(const __nv_bfloat16* __restrict__ x,
                                const __nv_bfloat16* __restrict__ g, __nv_bfloat16* __restrict__ y,
-                               int rows, int hidden, float eps) {
+                               int rows, int hidden, float eps, const __grid_constant__ BextDesc bx,
+                               int norm_blocks) {
+  if (static_cast<int>(blockIdx.x) >= norm_blocks) {
+    bext_chunk(bx, static_cast<long>(blockIdx.x - norm_blocks) * blockDim.x + threadIdx.x);
+    return;
+  }
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= rows) return;
@@ -445,9 +480,18 @@ cudaError_t launch_rope_table(float2* table, int n_pos, int head_dim, double the
 }
 
 cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bfloat16* y,
-                           int rows, int hidden, float eps, cudaStream_t stream) {
-  if (rows == 0) return cudaSuccess;
-  rmsnorm_kernel<<<cdiv(rows, 8), 256, 0, stream>>>(x, g, y, rows, hidden, eps);
+                           int rows, int hidden, float eps, cudaStream_t stream, const BextDesc* bx) {
+  BextDesc d{};
+  long chunks = 0;
+  if (bx) {
+    d = *bx;
+    if (d.n < 0 || d.n > 4 || d.rank < 1 || d.rank > kRankPad) return cudaErrorInvalidValue;
+    for (int m = 0; m < d.n; ++m) chunks += static_cast<long>(d.rows[m]) * (kBxCols / 8);
+  }
+  const int norm_blocks = cdiv(rows, 8);
+  const int blocks = norm_blocks + static_cast<int>(cdiv(chunks, 256));
+  if (blocks == 0) return cudaSuccess;
+  rmsnorm_kernel<<<blocks, 256, 0, stream>>>(x, g, y, rows, hidden, eps, d, norm_blocks);
   return cudaGetLastError();
 }
 
