@@ -44,7 +44,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu --set full
 # capture of the kernel as it now stands, at the full launch size of the 7B-shape 16K workload
 # (profiles/gemm_gateup_swiglu_7b16k.md). An entry is removed whenever its kernel changes.
-NCU_TRAFFIC_BYTES = {}
+NCU_TRAFFIC_BYTES = {"gemm_gateup_swiglu": 2.921001e9 + 0.616805e9}
 
 
 def load_peaks():

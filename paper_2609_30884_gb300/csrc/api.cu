@@ -242,8 +242,8 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
   p.off_abort = take((1 + p.flag_words) * sizeof(int));
   p.off_ptab = take(static_cast<size_t>(p.ptab_slots) * sizeof(int));
   p.splits = dec_splits(p.max_n);
-  // decode scratch per row, fp32: x, xn, x1, q, k, v, o, xa (3 slots), gu, m, attention partials
-  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 3 * kRankPad + 3 * D.f) * 4 +
+  // decode scratch per row, fp32: x, xn, x1, q, k, v, o, xa (7 slots), gu, m, attention partials
+  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 7 * kRankPad + 3 * D.f) * 4 +
                          static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
   p.dec_bytes = align256(dec_row * std::max(1, p.dec_rows));
   p.off_dec = take(p.dec_rows ? p.dec_bytes : 0);
@@ -531,6 +531,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
   std::stable_sort(rows.begin(), rows.end(), [](const DecodeRow& a, const DecodeRow& b) { return a.e < b.e; });
   const int l0 = rows[0].e;
   const size_t Rs = static_cast<size_t>(R);
+  const int rank = c.ad->dims.rank;
   float* x = reinterpret_cast<float*>(c.ws + p.off_dec);
   float* xn = x + Rs * D.h;
   float* x1 = xn + Rs * D.h;
@@ -538,13 +539,22 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
   float* k = q + Rs * D.qd;
   float* v = k + Rs * D.kvd;
   float* o = v + Rs * D.kvd;
-  float* xa = o + Rs * D.qd;  // three slots of [R, rank]
-  float* gu = xa + 3 * Rs * kRankPad;
+  float* xa = o + Rs * D.qd;  // one [R, rank] slot per module: q, k, v, o, gate, up, down
+  float* gu = xa + 7 * Rs * kRankPad;
   float* m = gu + Rs * 2 * D.f;
   float* part = m + Rs * D.f;
-  const int rank = c.ad->dims.rank;
-  // kernels per layer with up to 8 rows: 2 norm + LoRA-down launches, the o/down LoRA downs,
-  // 4 GEMVs, 1 RoPE, 2 attention, 1 SwiGLU; plus a conversion in and out per row
+  auto xa_of = [&](int mod) { return xa + static_cast<size_t>(mod) * Rs * kRankPad; };
+  auto up_of = [&](int l, int mod) {
+    RowUp u{};
+    if (adapted(c.ad, mod)) {
+      u.B = static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + mod]);
+      u.xa = xa_of(mod);
+    }
+    return u;
+  };
+  // kernels per layer: 2 norms (with the pending up products), 4 GEMV passes per 8 rows, RoPE
+  // (with the q|k|v up products), 2 attention, SwiGLU (with the gate|up up products), the K/V
+  // write of a generation step; then the last layer's down up product and a conversion per row
   int launches = 0;
   for (const auto& r : rows) launches += (r.start ? 1 : 0) + (r.out ? 1 : 0);
   bool any_token = false;
@@ -553,9 +563,9 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
   for (int l = l0; l < D.N; ++l) {
     int nr = 0;
     for (const auto& r : rows) nr += r.e <= l;
-    launches += 6 + (opt.write_kv ? 1 : 0) + adapted(c.ad, CRF_MOD_O) + adapted(c.ad, CRF_MOD_DOWN) +
-                4 * ((nr + 7) / 8);
+    launches += 6 + (opt.write_kv ? 1 : 0) + 4 * ((nr + 7) / 8);
   }
+  if (l0 < D.N && adapted(c.ad, CRF_MOD_DOWN)) ++launches;
   ProfScope ps(c.ctx, kPDecode, c.st, launches);
   TokenRows tr{};
   for (int i = 0; i < R; ++i) {
@@ -572,46 +582,35 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
     CRF_CUDA(launch_embed_rows_f32(static_cast<const __nv_bfloat16*>(c.model->embed), tr, R, x, D.h, D.V,
                                    c.ctx->status_dev, c.st));
   }
-  // segments [mods] sharing the fp32 rows `raw` (optionally RMS-normalised into `in` inside the
-  // LoRA-down launch), one GEMV per group of up to 8 rows
-  auto proj = [&](int l, int nr, const int* mods, int nm, const float* raw, const void* norm_gain,
-                  float* in, int in_dim, float* const* ys, const int* outs, const float* resid,
-                  int resid_ld) -> cudaError_t {
-    if (!norm_gain) in = const_cast<float*>(raw);
-    LoraDownRows ld{};
-    for (int s = 0; s < nm; ++s)
-      if (adapted(c.ad, mods[s])) {
-        ld.A[ld.n] = static_cast<const __nv_bfloat16*>(c.ad->A[l * 7 + mods[s]]);
-        ld.xa[ld.n] = xa + s * Rs * kRankPad;
-        ++ld.n;
-      }
-    if (ld.n || norm_gain) {
-      cudaError_t e = launch_lora_down_rows(ld, rank, in_dim, raw, nr, c.scale,
-                                            static_cast<const __nv_bfloat16*>(norm_gain), D.eps,
-                                            in, c.st);
-      if (e != cudaSuccess) return e;
-    }
+  // one weight pass per group of up to 8 rows: the modules' base rows (y = W in + bias + resid)
+  // and, as segments of their own, their LoRA A rows (xa = (alpha/r) A in, Eq. S3)
+  auto proj = [&](int l, int nr, const int* mods, int nm, const float* in, int in_dim, float* const* ys,
+                  const int* outs, const float* resid, int resid_ld) -> cudaError_t {
     for (int r0 = 0; r0 < nr; r0 += 8) {
       GemvDesc g{};
       g.abort = c.abort;
-      g.nseg = nm;
       g.in_dim = in_dim;
       g.x = in + static_cast<size_t>(r0) * in_dim;
       g.rows = std::min(8, nr - r0);
-      g.rank = rank;
       for (int s = 0; s < nm; ++s) {
         const int mod = mods[s];
-        GemvSeg& sg = g.seg[s];
+        GemvSeg& sg = g.seg[g.nseg++];
         sg.W = static_cast<const __nv_bfloat16*>(c.model->layers[l].W[mod]);
         sg.out_dim = outs[s];
+        sg.scale = 1.f;
         sg.bias = (mod < 3 && D.bias) ? static_cast<const __nv_bfloat16*>(c.model->layers[l].bias[mod])
                                       : nullptr;
         sg.y = ys[s] + static_cast<size_t>(r0) * outs[s];
         sg.resid = resid ? resid + static_cast<size_t>(r0) * resid_ld : nullptr;
-        if (adapted(c.ad, mod)) {
-          sg.BL = static_cast<const __nv_bfloat16*>(c.ad->B[l * 7 + mod]);
-          sg.xa = xa + s * Rs * kRankPad + static_cast<size_t>(r0) * rank;
-        }
+      }
+      for (int s = 0; s < nm; ++s) {
+        const int mod = mods[s];
+        if (!adapted(c.ad, mod)) continue;
+        GemvSeg& sg = g.seg[g.nseg++];
+        sg.W = static_cast<const __nv_bfloat16*>(c.ad->A[l * 7 + mod]);
+        sg.out_dim = rank;
+        sg.scale = c.scale;
+        sg.y = xa_of(mod) + static_cast<size_t>(r0) * rank;
       }
       cudaError_t e = launch_gemv(g, c.ctx->num_sms, c.st, nr);
       if (e != cudaSuccess) return e;
@@ -629,6 +628,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
   float* const y_d[1] = {x};
   RowPositions rp{};
   for (int i = 0; i < R; ++i) rp.pos[i] = rows[i].pos;
+  int nr_prev = 0;  // rows that carry the previous layer's pending down up product
   {
     // the layer loop is a chain of short kernels only: each may become resident and prefetch its
     // weights while the one before it finishes
@@ -637,11 +637,15 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
       int nr = 0;
       while (nr < R && rows[nr].e <= l) ++nr;
       const crf_layer_weights& w = c.model->layers[l];
-      CRF_CUDA(proj(l, nr, m_qkv, 3, x, w.ln1, xn, D.h, y_qkv, o_qkv, nullptr, 0));
-      CRF_CUDA(launch_rope_rows(q, D.hq, k, D.hkv, nr, D.d,
-                                opt.rope_by_row ? opt.rope_by_row
-                                                : reinterpret_cast<const float2*>(c.ws + p.off_rope),
-                                rp, opt.rope_by_row != nullptr, c.st));
+      // x += the previous layer's down up product (rows active there), xn = RMSNorm(x)
+      CRF_CUDA(launch_norm_up_rows(x, D.h, nr, l > l0 ? up_of(l - 1, CRF_MOD_DOWN) : RowUp{}, nr_prev, rank,
+                                   static_cast<const __nv_bfloat16*>(w.ln1), D.eps, xn, c.st));
+      CRF_CUDA(proj(l, nr, m_qkv, 3, xn, D.h, y_qkv, o_qkv, nullptr, 0));
+      const RowUp up_qkv[3] = {up_of(l, CRF_MOD_Q), up_of(l, CRF_MOD_K), up_of(l, CRF_MOD_V)};
+      CRF_CUDA(launch_rope_up_rows(q, D.hq, k, D.hkv, v, nr, D.d, up_qkv, rank,
+                                   opt.rope_by_row ? opt.rope_by_row
+                                                   : reinterpret_cast<const float2*>(c.ws + p.off_rope),
+                                   rp, opt.rope_by_row != nullptr, c.st));
       DecodeAttnDesc a;
       std::memset(&a, 0, sizeof(a));
       a.q = q;
@@ -672,12 +676,19 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
         CRF_CUDA(launch_kv_write_rows(k, v, c.pool->k_pages[l], c.pool->v_pages[l], pg, nr, D.hkv, D.d,
                                       c.ctx->status_dev, c.abort, c.st));
       }
-      CRF_CUDA(proj(l, nr, m_o, 1, o, nullptr, nullptr, D.qd, y_o, o_o, x, D.h));
-      CRF_CUDA(proj(l, nr, m_gu, 2, x1, w.ln2, xn, D.h, y_gu, o_gu, nullptr, 0));
+      // x1 = x + o W_o^T, then x1 += the o up product and xn = RMSNorm(x1)
+      CRF_CUDA(proj(l, nr, m_o, 1, o, D.qd, y_o, o_o, x, D.h));
+      CRF_CUDA(launch_norm_up_rows(x1, D.h, nr, up_of(l, CRF_MOD_O), nr, rank,
+                                   static_cast<const __nv_bfloat16*>(w.ln2), D.eps, xn, c.st));
+      CRF_CUDA(proj(l, nr, m_gu, 2, xn, D.h, y_gu, o_gu, nullptr, 0));
       // gate rows then up rows: SwiGLU over [nr, f] with the up half Rs * f further on
-      CRF_CUDA(launch_swiglu_split_f32(gu, gu + Rs * D.f, m, nr * D.f, c.st));
-      CRF_CUDA(proj(l, nr, m_d, 1, m, nullptr, nullptr, D.f, y_d, o_d, x1, D.h));
+      CRF_CUDA(launch_swiglu_up_rows(gu, gu + Rs * D.f, m, nr, D.f, up_of(l, CRF_MOD_GATE), up_of(l, CRF_MOD_UP),
+                                     rank, c.st));
+      // x = x1 + m W_d^T; its up product is added by the next layer's norm (or below)
+      CRF_CUDA(proj(l, nr, m_d, 1, m, D.f, y_d, o_d, x1, D.h));
+      nr_prev = nr;
     }
+    if (l0 < D.N) CRF_CUDA(launch_rows_up(x, D.h, nr_prev, up_of(D.N - 1, CRF_MOD_DOWN), rank, c.st));
   }
   for (int i = 0; i < R; ++i)
     if (rows[i].out)
@@ -761,7 +772,7 @@ StepPlan make_step_plan(const Dims& D, const crf_decode_row* rows, int n) {
   p.max_n = 1;
   for (int i = 0; i < n; ++i) p.max_n = std::max(p.max_n, rows[i].pos + 1);
   p.splits = dec_splits(p.max_n);
-  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 3 * kRankPad + 3 * D.f) * 4 +
+  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 7 * kRankPad + 3 * D.f) * 4 +
                          static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
   p.dec_bytes = align256(dec_row * std::max(1, n));
   size_t o = 0;

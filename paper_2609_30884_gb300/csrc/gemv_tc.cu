@@ -1,4 +1,4 @@
-// Multi-row GEMV on the tensor cores: y[r, j] = sum_i W[j, i] x[r, i] (+ bias, LoRA up, residual)
+// Multi-row GEMV on the tensor cores: y[r, j] = scale sum_i W[j, i] x[r, i] (+ bias, residual)
 // for up to 8 fp32 rows x (the first-step rows of a window and the rows of a generation step): the
 // adapted projections of Eq. S3 for single rows (Section 3.1 hybrid rows, Section S2.1 decoding).
 //
@@ -10,7 +10,7 @@
 // columns 4c..4c+3 of both W's rows and x's row: logical {2c, 2c+1} -> 4c, 4c+1 and
 // {2c+8, 2c+9} -> 4c+2, 4c+3 (a bijection on the step's 16 columns, the same for A and B), so
 // every load is a contiguous vector. Warps of a block split K; a fixed-order shared-memory
-// reduction and the epilogue (bias, LoRA up from the rank-r down product, residual) follow.
+// reduction and the epilogue (scale, bias, residual) follow.
 // The work is bound by the weight bytes: the MMAs replace the 8 fp32 FMAs per weight element
 // and row of the scalar kernel.
 #include "common.cuh"
@@ -27,8 +27,8 @@ constexpr int kRowsMax = 8;
 
 struct GemvTcLaunch {
   GemvDesc d;
-  int ks;          // warps per 16-row tile (split K)
-  int block0[4];   // first block of each segment
+  int ks;                        // warps per 16-row tile (split K)
+  int block0[kGemvMaxSeg + 1];   // first block of each segment
 };
 
 __device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi, uint32_t& lo) {
@@ -121,10 +121,8 @@ __global__ void __launch_bounds__(kWarps * 32) gemv_tc_kernel(const __grid_const
     if (j >= sg.out_dim || r >= d.rows) continue;
     float v = 0.f;
     for (int q = 0; q < ks; ++q) v += red[tl * ks + q][jj][r];
+    v *= sg.scale;
     if (sg.bias) v += __bfloat162float(sg.bias[j]);
-    if (sg.BL)
-      for (int k = 0; k < d.rank; ++k)
-        v += __bfloat162float(sg.BL[(size_t)j * d.rank + k]) * sg.xa[(size_t)r * d.rank + k];
     if (sg.resid) v += sg.resid[(size_t)r * sg.out_dim + j];
     sg.y[(size_t)r * sg.out_dim + j] = v;
   }
@@ -133,7 +131,7 @@ __global__ void __launch_bounds__(kWarps * 32) gemv_tc_kernel(const __grid_const
 }  // namespace
 
 cudaError_t launch_gemv_tc(const GemvDesc& d, int num_sms, cudaStream_t stream) {
-  if (d.rows < 1 || d.rows > kRowsMax || d.nseg < 1 || d.nseg > 3 || d.in_dim % 16 != 0)
+  if (d.rows < 1 || d.rows > kRowsMax || d.nseg < 1 || d.nseg > kGemvMaxSeg || d.in_dim % 16 != 0)
     return cudaErrorInvalidValue;
   GemvTcLaunch L;
   L.d = d;
@@ -147,11 +145,11 @@ cudaError_t launch_gemv_tc(const GemvDesc& d, int num_sms, cudaStream_t stream) 
   while (L.ks < kWarps && tiles * L.ks < want_warps && (d.in_dim / 32) / (2 * L.ks) >= 4) L.ks *= 2;
   const int tiles_per_block = kWarps / L.ks;
   int blocks = 0;
-  for (int s = 0; s < 3; ++s) {
+  for (int s = 0; s < kGemvMaxSeg; ++s) {
     L.block0[s] = blocks;
     if (s < d.nseg) blocks += ((d.seg[s].out_dim + 15) / 16 + tiles_per_block - 1) / tiles_per_block;
   }
-  L.block0[3] = blocks;
+  L.block0[kGemvMaxSeg] = blocks;
   return launch_kernel(gemv_tc_kernel, dim3(blocks), dim3(kWarps * 32), 0, stream, L);
 }
 

@@ -175,22 +175,24 @@ cudaError_t launch_attention_tc(const AttnDesc& d, int num_pages, int total_rows
 // Small-M decode path (the last prefix row through the layers after the window).
 // Up to three row-stacked weight segments share one launch and one input x:
 // y_s[r, j] = sum_i W_s[j, i] x[r, i] (+ bias_s[j]) (+ sum_k BL_s[j, k] xa_s[r, k]) (+ resid_s[r, j])
+// y = scale * (W x) + bias + resid for each segment of weight rows sharing the input rows x: the
+// projections' base rows and, as segments of their own, the LoRA A rows (y = the scaled down
+// product xa, [rows, rank]).
 struct GemvSeg {
   const __nv_bfloat16* W;  // [out_dim, in_dim]
   int out_dim;
+  float scale;
   const __nv_bfloat16* bias;  // [out_dim] or null
-  const __nv_bfloat16* BL;    // [out_dim, rank] or null
-  const float* xa;            // [rows, rank] fp32, already scaled by alpha/r
   const float* resid;         // [rows, out_dim] fp32 or null
   float* y;                   // [rows, out_dim] fp32
 };
+constexpr int kGemvMaxSeg = 6;
 struct GemvDesc {
-  GemvSeg seg[3];
+  GemvSeg seg[kGemvMaxSeg];
   int nseg;
   int in_dim;
   const float* x;  // [rows, in_dim] fp32
   int rows;        // 1..8
-  int rank;
   int prefetch;    // set by the launcher: prefetch the block's weight rows into L2 before the wait
   const int* abort;  // per-call abort word, or null
 };
@@ -200,18 +202,19 @@ struct GemvDesc {
 // keeps equal rows equal across chunks.
 cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int total_rows = 0);
 cudaError_t launch_gemv_tc(const GemvDesc& d, int num_sms, cudaStream_t stream);
-// xa_m[r, k] = scale * sum_i A_m[k, i] x[r, i] for up to three modules m sharing x
-struct LoraDownRows {
-  const __nv_bfloat16* A[3];
-  float* xa[3];
-  int n;
-  int prefetch;  // set by the launcher: prefetch the block's A row into L2 before the wait
+// The adapter's up product for decode rows, added where the projection's output is consumed:
+// up[r, j] = sum_k B[j, k] xa[r, k] (B [out_dim, rank] bf16, xa [rows, rank] fp32 already scaled
+// by alpha / r); a null B adds nothing.
+struct RowUp {
+  const __nv_bfloat16* B;
+  const float* xa;
 };
-// With norm_gain != null, x is normalised first (rmsnorm(x) * norm_gain, eps) and the
-// normalised rows are also written to xn (so the launch replaces the separate RMSNorm).
-cudaError_t launch_lora_down_rows(const LoraDownRows& m, int rank, int in_dim, const float* x,
-                                  int rows, float scale, const __nv_bfloat16* norm_gain, float eps,
-                                  float* xn, cudaStream_t stream);
+// x[r] += up(r) for r < up_rows (the rows that carry a pending product), then for every row
+// xn[r] = rmsnorm(x[r]) * g (eps): the residual stream's update and the next RMSNorm in one launch.
+cudaError_t launch_norm_up_rows(float* x, int dim, int rows, RowUp up, int up_rows, int rank,
+                                const __nv_bfloat16* g, float eps, float* xn, cudaStream_t stream);
+// x[r] += up(r) for every row (the last projection's product, before the rows leave).
+cudaError_t launch_rows_up(float* x, int dim, int rows, RowUp up, int rank, cudaStream_t stream);
 cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y, int rows,
                                int hidden, float eps, cudaStream_t stream);
 // Single-query attention of `rows` decode rows (one per request) over pages [0, pos) plus own k/v.
@@ -238,12 +241,13 @@ int decode_attention_splits(int max_positions);
 struct RowPositions {
   int pos[kMaxReq];
 };
-// Rotate-half RoPE on the fp32 q [rows, hq, head_dim] and k [rows, hkv, head_dim] of decode
-// rows, row r at position pos.pos[r]; (cos, sin) from `table` [positions][head_dim / 2], or with
-// table_by_row from row r of a [rows][head_dim / 2] table of the rows' own positions.
-cudaError_t launch_rope_rows(float* q, int hq, float* k, int hkv, int rows, int head_dim,
-                             const float2* table, const RowPositions& pos, bool table_by_row,
-                             cudaStream_t stream);
+// q, k, v of decode rows: the up products added (up[0..2] for q, k, v), then rotate-half RoPE on
+// q [rows, hq, head_dim] and k [rows, hkv, head_dim], row r at position pos.pos[r]; (cos, sin)
+// from `table` [positions][head_dim / 2], or with table_by_row from row r of a
+// [rows][head_dim / 2] table of the rows' own positions.
+cudaError_t launch_rope_up_rows(float* q, int hq, float* k, int hkv, float* v, int rows, int head_dim,
+                                const RowUp* up, int rank, const float2* table, const RowPositions& pos,
+                                bool table_by_row, cudaStream_t stream);
 // (cos, sin) of the rows' positions: table [rows][head_dim / 2].
 cudaError_t launch_rope_table_rows(float2* table, const RowPositions& pos, int rows, int head_dim,
                                    double theta, cudaStream_t stream);
@@ -268,8 +272,9 @@ cudaError_t launch_kv_write_rows(const float* k, const float* v, void* kpages, v
 cudaError_t launch_wait_selftest(int* status, cudaStream_t stream);
 cudaError_t launch_argmax_rows(const float* logits, int rows, int vocab, int32_t* out,
                                cudaStream_t stream, const int* abort = nullptr);
-cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
-                                    cudaStream_t stream);
+// m[r, j] = silu(g[r, j] + up_g) * (u[r, j] + up_u) over [rows, f] (gate and up in separate buffers).
+cudaError_t launch_swiglu_up_rows(const float* g, const float* u, float* m, int rows, int f, RowUp up_g,
+                                  RowUp up_u, int rank, cudaStream_t stream);
 cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream,
                                const int* abort = nullptr);
 // dst[0 .. n) = src[0 .. n) (bf16), unless the call's abort word is set.

@@ -145,15 +145,15 @@ __global__ void embed_kernel(const __nv_bfloat16* __restrict__ e, const int32_t*
 // A block of 8 warps takes 8/KS groups of OPW consecutive outputs of one segment; the KS
 // warps of a group split the input dimension, each lane streaming 16-byte pieces of the
 // OPW weight rows (x read through the cache and reused across the OPW rows). Partials are
-// summed in shared memory in a fixed order (deterministic), then bias, LoRA up product and
-// residual are added.
+// summed in shared memory in a fixed order (deterministic), then scaled, and bias and residual
+// are added.
 constexpr int kGemvWarps = 8;
 constexpr int kGemvMaxRows = 8;
 
 struct GemvLaunch {
   GemvDesc d;
   int opw, ks;
-  int block0[4];  // first block of each segment
+  int block0[kGemvMaxSeg + 1];  // first block of each segment
 };
 
 template <int OPW, int NR>
@@ -222,104 +222,130 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const __grid_cons
   if (j >= sg.out_dim || r >= d.rows) return;
   float v = 0.f;
   for (int q = 0; q < ks; ++q) v += red[gl * ks + q][o][r];
+  v *= sg.scale;
   if (sg.bias) v += __bfloat162float(sg.bias[j]);
-  if (sg.BL)
-    for (int k = 0; k < d.rank; ++k)
-      v += __bfloat162float(sg.BL[(size_t)j * d.rank + k]) * sg.xa[(size_t)r * d.rank + k];
   if (sg.resid) v += sg.resid[(size_t)r * sg.out_dim + j];
   sg.y[(size_t)r * sg.out_dim + j] = v;
 }
 
-// xa_m[r, k] = scale * <A_m[k, :], x_r> for up to three modules, one block per (module, row, k).
-// With a norm gain g, x_r is first replaced by rmsnorm(x_r) * g: every block computes the row's
-// mean square, and the extra blocks (one per row) also write the normalised row to xn.
-constexpr int kLdThreads = 256;
-
-__global__ void __launch_bounds__(kLdThreads) lora_down_rows_kernel(
-    const __grid_constant__ LoraDownRows m, int rank, int in_dim, const float* __restrict__ x, int rows,
-    float scale, const __nv_bfloat16* __restrict__ g, float eps, float* __restrict__ xn) {
-  __shared__ float red[kLdThreads / 32];
-  const int b = blockIdx.x;
-  const int n_dot = m.n * rows * rank;
-  const int r = b < n_dot ? (b / rank) % rows : b - n_dot;
-  const int mi = b / (rows * rank), k = b % rank;
-  if (m.prefetch) prefetch_l2_range(b < n_dot ? m.A[mi] + (size_t)k * in_dim : g, g || b < n_dot ? in_dim * 2 : 0);
-  griddep_begin();  // x comes from the kernel before
-  const float* xr = x + (size_t)r * in_dim;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float inv = 1.f;
-  if (g) {
-    float ss = 0.f;
-#pragma unroll 4
-    for (int i = threadIdx.x * 4; i < in_dim; i += kLdThreads * 4) {
-      const float4 a = __ldg(reinterpret_cast<const float4*>(xr + i));
-      ss += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
-    }
-    ss = warp_sum(ss);
-    if (lane == 0) red[warp] = ss;
-    __syncthreads();
-    ss = 0.f;
-#pragma unroll
-    for (int w = 0; w < kLdThreads / 32; ++w) ss += red[w];
-    inv = rsqrtf(ss / in_dim + eps);
-    __syncthreads();
-  }
-  if (b >= n_dot) {  // normalised row for the GEMV that follows
-    for (int i = threadIdx.x; i < in_dim; i += kLdThreads)
-      xn[(size_t)r * in_dim + i] = xr[i] * inv * __bfloat162float(g[i]);
-    return;
-  }
-  const __nv_bfloat16* A = m.A[mi] + (size_t)k * in_dim;
+// sum_k B[j, k] xa[k] for one output j of a rank-r up product (B row: r bf16, 8-byte aligned)
+__device__ __forceinline__ float up_dot(const __nv_bfloat16* __restrict__ B, int j, const float* __restrict__ xa,
+                                        int rank) {
+  const __nv_bfloat16* br = B + (size_t)j * rank;
   float s = 0.f;
-#pragma unroll 4
-  for (int i = threadIdx.x * 8; i < in_dim; i += kLdThreads * 8) {
-    const uint4 u = __ldg(reinterpret_cast<const uint4*>(A + i));
-    const float4* xp = reinterpret_cast<const float4*>(xr + i);
-    float4 a = __ldg(xp), c = __ldg(xp + 1);
-    if (g) {
-      const uint4 gv = __ldg(reinterpret_cast<const uint4*>(g + i));
-      a.x *= inv * bf16_lo(gv.x); a.y *= inv * bf16_hi(gv.x); a.z *= inv * bf16_lo(gv.y);
-      a.w *= inv * bf16_hi(gv.y); c.x *= inv * bf16_lo(gv.z); c.y *= inv * bf16_hi(gv.z);
-      c.z *= inv * bf16_lo(gv.w); c.w *= inv * bf16_hi(gv.w);
-    }
-    s += bf16_lo(u.x) * a.x + bf16_hi(u.x) * a.y + bf16_lo(u.y) * a.z + bf16_hi(u.y) * a.w +
-         bf16_lo(u.z) * c.x + bf16_hi(u.z) * c.y + bf16_lo(u.w) * c.z + bf16_hi(u.w) * c.w;
-  }
-  s = warp_sum(s);
-  if (lane == 0) red[warp] = s;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float t = 0.f;
+  if (rank == 16) {
+    const uint4 u0 = __ldg(reinterpret_cast<const uint4*>(br)), u1 = __ldg(reinterpret_cast<const uint4*>(br) + 1);
+    const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
 #pragma unroll
-    for (int w = 0; w < kLdThreads / 32; ++w) t += red[w];
-    m.xa[mi][(size_t)r * rank + k] = t * scale;
+    for (int i = 0; i < 8; ++i) s += bf16_lo(w[i]) * xa[2 * i] + bf16_hi(w[i]) * xa[2 * i + 1];
+  } else if (rank == 8) {
+    const uint4 u0 = __ldg(reinterpret_cast<const uint4*>(br));
+    const uint32_t w[4] = {u0.x, u0.y, u0.z, u0.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) s += bf16_lo(w[i]) * xa[2 * i] + bf16_hi(w[i]) * xa[2 * i + 1];
+  } else {
+    for (int i = 0; i < rank; ++i) s += __bfloat162float(br[i]) * xa[i];
   }
+  return s;
 }
 
-// Rotate-half RoPE on the fp32 q [rows, hq, d] and k [rows, hkv, d] of decode rows, row r at
-// position pos[r], angles from the (cos, sin) table of the window pass.
-__global__ void rope_rows_kernel(float* q, int hq, float* k, int hkv, int rows, int d,
-                                 const float2* __restrict__ table, const RowPositions pos, int by_row) {
-  griddep_begin();  // q, k come from the GEMV before
+// One block per row: x[r] += up(r) when r < up_rows, then xn[r] = rmsnorm(x[r]) * g.
+constexpr int kNormThreads = 512;
+__global__ void __launch_bounds__(kNormThreads) norm_up_rows_kernel(float* __restrict__ x, int dim, RowUp up,
+                                                                    int up_rows, int rank,
+                                                                    const __nv_bfloat16* __restrict__ g, float eps,
+                                                                    float* __restrict__ xn) {
+  __shared__ float red[kNormThreads / 32];
+  __shared__ float xa_s[kRankPad];
+  const int r = blockIdx.x;
+  const bool add = up.B != nullptr && r < up_rows;
+  if (add) prefetch_l2_range(up.B, (size_t)dim * rank * 2);
+  griddep_begin();  // x and xa come from the kernels before
+  float* xr = x + (size_t)r * dim;
+  if (add && threadIdx.x < rank) xa_s[threadIdx.x] = up.xa[(size_t)r * rank + threadIdx.x];
+  __syncthreads();
+  float ss = 0.f;
+  for (int j = threadIdx.x; j < dim; j += kNormThreads) {
+    float v = xr[j];
+    if (add) {
+      v += up_dot(up.B, j, xa_s, rank);
+      xr[j] = v;
+    }
+    ss += v * v;
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  ss = 0.f;
+#pragma unroll
+  for (int w = 0; w < kNormThreads / 32; ++w) ss += red[w];
+  const float inv = rsqrtf(ss / dim + eps);
+  for (int j = threadIdx.x; j < dim; j += kNormThreads)
+    xn[(size_t)r * dim + j] = xr[j] * inv * __bfloat162float(g[j]);
+}
+
+// x[r, j] += up(r, j), one thread per element.
+__global__ void rows_up_kernel(float* __restrict__ x, int dim, int rows, RowUp up, int rank) {
+  griddep_begin();  // x and xa come from the kernels before
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * dim) return;
+  const int r = idx / dim, j = idx % dim;
+  x[idx] += up_dot(up.B, j, up.xa + (size_t)r * rank, rank);
+}
+
+struct RowUp3 {
+  RowUp m[3];  // q, k, v
+};
+
+// Threads [0, rows * (hq + hkv) * d/2): one rotation pair (i, i + d/2) of a q or k head: the up
+// products added, then rotate-half RoPE at the row's position. The rest: one v element each,
+// the up product added.
+__global__ void rope_up_rows_kernel(float* q, int hq, float* k, int hkv, float* v, int rows, int d,
+                                    const __grid_constant__ RowUp3 up, int rank,
+                                    const float2* __restrict__ table, const RowPositions pos, int by_row) {
+  griddep_begin();  // q, k, v and xa come from the GEMV before
   const int half = d / 2;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   const int heads = hq + hkv;
-  if (idx >= rows * heads * half) return;
+  const int n_pairs = rows * heads * half;
+  if (idx >= n_pairs) {
+    const int e = idx - n_pairs;
+    if (e >= rows * hkv * d) return;
+    if (up.m[2].B) {
+      const int r = e / (hkv * d), j = e % (hkv * d);
+      v[e] += up_dot(up.m[2].B, j, up.m[2].xa + (size_t)r * rank, rank);
+    }
+    return;
+  }
   const int i = idx % half;
   const int h = (idx / half) % heads;
   const int r = idx / (half * heads);
+  const bool is_q = h < hq;
+  const int hh = is_q ? h : h - hq;
+  const RowUp& u = up.m[is_q ? 0 : 1];
+  float* base = is_q ? q + ((size_t)r * hq + hh) * d : k + ((size_t)r * hkv + hh) * d;
+  float x1 = base[i], x2 = base[i + half];
+  if (u.B) {
+    const float* xa = u.xa + (size_t)r * rank;
+    x1 += up_dot(u.B, hh * d + i, xa, rank);
+    x2 += up_dot(u.B, hh * d + i + half, xa, rank);
+  }
   const float2 cs = table[(size_t)(by_row ? r : pos.pos[r]) * half + i];
-  float* base = h < hq ? q + ((size_t)r * hq + h) * d : k + ((size_t)r * hkv + (h - hq)) * d;
-  const float x1 = base[i], x2 = base[i + half];
   base[i] = x1 * cs.x - x2 * cs.y;
   base[i + half] = x2 * cs.x + x1 * cs.y;
 }
 
-// m[i] = silu(g[i]) * u[i] over n elements (gate and up in separate buffers)
-__global__ void swiglu_split_f32_kernel(const float* g, const float* u, float* m, int n) {
-  griddep_begin();  // gate and up come from the GEMV before
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < n) m[i] = g[i] / (1.f + __expf(-g[i])) * u[i];
+// m[r, j] = silu(g + up_g) * (u + up_u) over [rows, f] (gate and up in separate buffers)
+__global__ void swiglu_up_rows_kernel(const float* g, const float* u, float* m, int rows, int f, RowUp up_g,
+                                      RowUp up_u, int rank) {
+  griddep_begin();  // gate, up and xa come from the GEMV before
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * f) return;
+  const int r = idx / f, j = idx % f;
+  float gv = g[idx], uv = u[idx];
+  if (up_g.B) gv += up_dot(up_g.B, j, up_g.xa + (size_t)r * rank, rank);
+  if (up_u.B) uv += up_dot(up_u.B, j, up_u.xa + (size_t)r * rank, rank);
+  m[idx] = gv / (1.f + __expf(-gv)) * uv;
 }
 
 __global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int n, const int* abort) {
@@ -528,7 +554,7 @@ bool gemv_use_tensor(int total_rows, int in_dim) {
 
 cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int total_rows) {
   if (gemv_use_tensor(total_rows > 0 ? total_rows : d.rows, d.in_dim)) return launch_gemv_tc(d, num_sms, stream);
-  if (d.rows < 1 || d.rows > kGemvMaxRows || d.nseg < 1 || d.nseg > 3 || d.in_dim % 8 != 0)
+  if (d.rows < 1 || d.rows > kGemvMaxRows || d.nseg < 1 || d.nseg > kGemvMaxSeg || d.in_dim % 8 != 0)
     return cudaErrorInvalidValue;
   GemvLaunch L;
   L.d = d;
@@ -546,14 +572,14 @@ cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int
     L.ks *= 2;
   const int groups_per_block = kGemvWarps / L.ks;
   int blocks = 0;
-  for (int s = 0; s < 3; ++s) {
+  for (int s = 0; s < kGemvMaxSeg; ++s) {
     L.block0[s] = blocks;
     if (s < d.nseg) {
       const int groups = (d.seg[s].out_dim + L.opw - 1) / L.opw;
       blocks += (groups + groups_per_block - 1) / groups_per_block;
     }
   }
-  L.block0[3] = blocks;
+  L.block0[kGemvMaxSeg] = blocks;
   switch (L.opw) {
     case 4: return gemv_dispatch<4>(L, blocks, stream);
     case 2: return gemv_dispatch<2>(L, blocks, stream);
@@ -561,17 +587,6 @@ cudaError_t launch_gemv(const GemvDesc& d, int num_sms, cudaStream_t stream, int
   }
 }
 
-cudaError_t launch_lora_down_rows(const LoraDownRows& m, int rank, int in_dim, const float* x,
-                                  int rows, float scale, const __nv_bfloat16* norm_gain, float eps,
-                                  float* xn, cudaStream_t stream) {
-  const int blocks = m.n * rows * rank + (norm_gain ? rows : 0);
-  if (blocks == 0) return cudaSuccess;
-  if (in_dim % 8 != 0) return cudaErrorInvalidValue;
-  LoraDownRows mp = m;
-  mp.prefetch = pdl_active() ? 1 : 0;
-  return launch_kernel(lora_down_rows_kernel, dim3(blocks), dim3(kLdThreads), 0, stream, mp, rank, in_dim, x,
-                       rows, scale, norm_gain, eps, xn);
-}
 
 // Bounded-wait self-test: thread 0 waits on an mbarrier that nothing arrives on. The wait
 // gives up after the library's limit, raises the status bit and the kernel returns, so the
@@ -600,13 +615,31 @@ cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y,
   return cudaGetLastError();
 }
 
-cudaError_t launch_rope_rows(float* q, int hq, float* k, int hkv, int rows, int head_dim,
-                             const float2* table, const RowPositions& pos, bool table_by_row,
-                             cudaStream_t stream) {
-  const int n = rows * (hq + hkv) * head_dim / 2;
+cudaError_t launch_rope_up_rows(float* q, int hq, float* k, int hkv, float* v, int rows, int head_dim,
+                                const RowUp* up, int rank, const float2* table, const RowPositions& pos,
+                                bool table_by_row, cudaStream_t stream) {
+  const long n = (long)rows * (hq + hkv) * (head_dim / 2) + (long)rows * hkv * head_dim;
   if (n == 0) return cudaSuccess;
-  return launch_kernel(rope_rows_kernel, dim3(cdiv(n, 256)), dim3(256), 0, stream, q, hq, k, hkv, rows, head_dim,
-                       table, pos, table_by_row ? 1 : 0);
+  if (rank != 4 && rank != 8 && rank != 16) return cudaErrorInvalidValue;
+  RowUp3 u{};
+  for (int i = 0; i < 3; ++i) u.m[i] = up[i];
+  return launch_kernel(rope_up_rows_kernel, dim3(cdiv(n, 256)), dim3(256), 0, stream, q, hq, k, hkv, v, rows,
+                       head_dim, u, rank, table, pos, table_by_row ? 1 : 0);
+}
+
+cudaError_t launch_norm_up_rows(float* x, int dim, int rows, RowUp up, int up_rows, int rank,
+                                const __nv_bfloat16* g, float eps, float* xn, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  if (rank != 4 && rank != 8 && rank != 16) return cudaErrorInvalidValue;
+  return launch_kernel(norm_up_rows_kernel, dim3(rows), dim3(kNormThreads), 0, stream, x, dim, up, up_rows, rank,
+                       g, eps, xn);
+}
+
+cudaError_t launch_rows_up(float* x, int dim, int rows, RowUp up, int rank, cudaStream_t stream) {
+  if (rows == 0 || !up.B) return cudaSuccess;
+  if (rank != 4 && rank != 8 && rank != 16) return cudaErrorInvalidValue;
+  return launch_kernel(rows_up_kernel, dim3(cdiv((long)rows * dim, 256)), dim3(256), 0, stream, x, dim, rows, up,
+                       rank);
 }
 
 // (cos, sin) of the rows' own positions only: table[r][i] for position pos[r].
@@ -771,10 +804,12 @@ cudaError_t launch_validate_pages(const PageCheck& pc, int num_pages, int* table
   return cudaGetLastError();
 }
 
-cudaError_t launch_swiglu_split_f32(const float* g, const float* u, float* m, int n,
-                                    cudaStream_t stream) {
-  if (n == 0) return cudaSuccess;
-  return launch_kernel(swiglu_split_f32_kernel, dim3(cdiv(n, 256)), dim3(256), 0, stream, g, u, m, n);
+cudaError_t launch_swiglu_up_rows(const float* g, const float* u, float* m, int rows, int f, RowUp up_g,
+                                  RowUp up_u, int rank, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  if (rank != 4 && rank != 8 && rank != 16) return cudaErrorInvalidValue;
+  return launch_kernel(swiglu_up_rows_kernel, dim3(cdiv((long)rows * f, 256)), dim3(256), 0, stream, g, u, m, rows,
+                       f, up_g, up_u, rank);
 }
 
 cudaError_t launch_f32_to_bf16(const float* x, __nv_bfloat16* y, int n, cudaStream_t stream,
@@ -796,6 +831,7 @@ cudaError_t launch_lm_head(const __nv_bfloat16* W, const float* h, int rows, int
     d.abort = abort;
     d.seg[0].W = W;
     d.seg[0].out_dim = vocab;
+    d.seg[0].scale = 1.f;
     d.seg[0].y = logits + (size_t)r0 * vocab;
     d.nseg = 1;
     d.in_dim = hidden;
