@@ -38,7 +38,7 @@ constexpr int kDtThreads = 256;
 constexpr int kDtRows = 256;   // long-dimension rows per step: 8 warps x 2 slices x 16
 constexpr int kDtSlices = kDtRows / 128;  // 16-row slices per warp and step
 constexpr int kDtStages = 3;   // two steps in flight while one is multiplied
-constexpr int kDtCtasPerSm = 2;
+constexpr int kDtCtasPerSm = 3;
 constexpr int kDtMaxItems = 224;
 constexpr int kDtMaxSegs = 2 * kDtMaxItems;
 constexpr int kDtAStride = kDtRows * 2 + 16;  // bytes per A row in a stage (+16: no bank conflicts)
@@ -52,7 +52,9 @@ struct DriftTcArgs {
 template <int R>
 struct DtShape {
   static constexpr int RP = R < 8 ? 8 : R;                      // features per part (zero padded)
-  static constexpr int kBStride = RP == 16 ? 48 : 16;          // bytes per B row in a stage
+  // bytes per B row in a stage: 32 for RP = 16, its two 16-byte halves swapped in rows 4-7 of
+  // every 8 (b_unit), so the transposed ldmatrix of 8 consecutive rows meets 8 distinct bank groups
+  static constexpr int kBStride = RP == 16 ? 32 : 16;
   static constexpr int kBVersion = kDtRows * kBStride;          // one version of the B side
   static constexpr int kAVersion = RP * kDtAStride;             // one version of the A side
   static constexpr int kStage = 2 * (kBVersion > kAVersion ? kBVersion : kAVersion);
@@ -121,6 +123,12 @@ __device__ __forceinline__ void split_diff(uint32_t a, uint32_t b, uint32_t& hi,
   lo = bf2_sub(bf2_sub(a, av), bf2_add(b, bv));
 }
 
+// Byte offset of 16-byte unit `ch` of B row `row` in a stage (rank 16: the XOR swizzle above).
+template <int RP>
+__device__ __forceinline__ int b_unit(int row, int ch) {
+  return RP == 16 ? ((ch ^ ((row >> 2) & 1)) << 4) : (ch << 4);
+}
+
 // The item a run of steps belongs to, cached while the run stays in one segment.
 struct SegCache {
   int seg = -1, side = 0, len = 0, step0 = 0, next0 = 0;
@@ -160,7 +168,7 @@ __device__ __forceinline__ void load_step(const SegCache& sc, int x, uint32_t st
       const bool ok = row0 + row < sc.len;
       const __nv_bfloat16* src =
           (v == 0 ? sc.p1 : sc.p0) + (ok ? blk + row * R + ch * (S::kBChunkBytes / 2) : 0);
-      const uint32_t dst = stage + v * S::kBVersion + row * S::kBStride + ch * 16;
+      const uint32_t dst = stage + v * S::kBVersion + row * S::kBStride + b_unit<S::RP>(row, ch);
       if constexpr (S::kBChunkBytes == 16)
         cp_async16(dst, src, ok);
       else
@@ -193,7 +201,8 @@ __device__ __forceinline__ void mma_slice(int side, uint32_t stage, int row0,
   if (side == 0) {
     // X[o][f] rows: matrix m covers rows k0 + (m >> 1) * 8 .. and features (m & 1) * 8 ..
     if constexpr (RP == 16) {
-      const uint32_t off = (row0 + (m >> 1) * 8 + i) * S::kBStride + (m & 1) * 16;
+      const int row = row0 + (m >> 1) * 8 + i;
+      const uint32_t off = row * S::kBStride + b_unit<RP>(row, m & 1);
       ldsm_x4_t(stage + off, f1[0], f1[1], f1[2], f1[3]);
       ldsm_x4_t(stage + S::kBVersion + off, f0[0], f0[1], f0[2], f0[3]);
     } else {
