@@ -170,9 +170,10 @@ struct Plan {
   size_t off_g0, off_g1, off_x1, off_xn, off_q, off_o, off_mlp, off_xa, off_bx, off_rope;
   size_t off_dx0, off_dec;  // decode: bf16 starting rows, fp32 scratch
   size_t off_abort, off_ptab;  // the call's abort word; the page-check table (ptab_slots ints)
-  // the projections' XA ready words: 4 launches x ceil(M / 256) row blocks per layer, laid out
-  // after the abort word so one clear at the start of the call covers both
-  size_t flag_words = 0;
+  // the projections' XA ready words (4 launches x ceil(M / 256) row blocks per layer) and the
+  // decode-row norms' per-row counters (kMaxReq), laid out after the abort word so one clear at
+  // the start of the call covers them all
+  size_t flag_words = kMaxReq;
   uint32_t ptab_slots = 2;
   size_t dec_bytes;
   size_t total;
@@ -238,12 +239,13 @@ Plan make_plan(const Dims& D, const crf_request* reqs, int n_req) {
     for (int i = 0; i < n_req; ++i) any |= reqs[i].s <= l && l < reqs[i].e;
     layers += any ? 1 : 0;
   }
-  p.flag_words = static_cast<size_t>(layers) * 4 * ((p.M + 255) / 256);
+  p.flag_words = static_cast<size_t>(layers) * 4 * ((p.M + 255) / 256) + kMaxReq;
   p.off_abort = take((1 + p.flag_words) * sizeof(int));
   p.off_ptab = take(static_cast<size_t>(p.ptab_slots) * sizeof(int));
   p.splits = dec_splits(p.max_n);
-  // decode scratch per row, fp32: x, xn, x1, q, k, v, o, xa (7 slots), gu, m, attention partials
-  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 7 * kRankPad + 3 * D.f) * 4 +
+  // decode scratch per row, fp32: x, xn, x1, q, k, v, o, xa (7 slots), gu, m, norm partials,
+  // attention partials
+  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 7 * kRankPad + 3 * D.f + norm_up_slices(D.h)) * 4 +
                          static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
   p.dec_bytes = align256(dec_row * std::max(1, p.dec_rows));
   p.off_dec = take(p.dec_rows ? p.dec_bytes : 0);
@@ -542,7 +544,9 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
   float* xa = o + Rs * D.qd;  // one [R, rank] slot per module: q, k, v, o, gate, up, down
   float* gu = xa + 7 * Rs * kRankPad;
   float* m = gu + Rs * 2 * D.f;
-  float* part = m + Rs * D.f;
+  float* npart = m + Rs * D.f;  // [R, slices] partial sums of squares of the norms
+  float* part = npart + Rs * norm_up_slices(D.h);
+  int* ncount = reinterpret_cast<int*>(c.ws + p.off_abort) + 1 + (p.flag_words - kMaxReq);
   auto xa_of = [&](int mod) { return xa + static_cast<size_t>(mod) * Rs * kRankPad; };
   auto up_of = [&](int l, int mod) {
     RowUp u{};
@@ -639,7 +643,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
       const crf_layer_weights& w = c.model->layers[l];
       // x += the previous layer's down up product (rows active there), xn = RMSNorm(x)
       CRF_CUDA(launch_norm_up_rows(x, D.h, nr, l > l0 ? up_of(l - 1, CRF_MOD_DOWN) : RowUp{}, nr_prev, rank,
-                                   static_cast<const __nv_bfloat16*>(w.ln1), D.eps, xn, c.st));
+                                   static_cast<const __nv_bfloat16*>(w.ln1), D.eps, xn, npart, ncount, c.st));
       CRF_CUDA(proj(l, nr, m_qkv, 3, xn, D.h, y_qkv, o_qkv, nullptr, 0));
       const RowUp up_qkv[3] = {up_of(l, CRF_MOD_Q), up_of(l, CRF_MOD_K), up_of(l, CRF_MOD_V)};
       CRF_CUDA(launch_rope_up_rows(q, D.hq, k, D.hkv, v, nr, D.d, up_qkv, rank,
@@ -679,7 +683,7 @@ crf_status decode_rows(const LayerCtx& c, std::vector<DecodeRow> rows, const Dec
       // x1 = x + o W_o^T, then x1 += the o up product and xn = RMSNorm(x1)
       CRF_CUDA(proj(l, nr, m_o, 1, o, D.qd, y_o, o_o, x, D.h));
       CRF_CUDA(launch_norm_up_rows(x1, D.h, nr, up_of(l, CRF_MOD_O), nr, rank,
-                                   static_cast<const __nv_bfloat16*>(w.ln2), D.eps, xn, c.st));
+                                   static_cast<const __nv_bfloat16*>(w.ln2), D.eps, xn, npart, ncount, c.st));
       CRF_CUDA(proj(l, nr, m_gu, 2, xn, D.h, y_gu, o_gu, nullptr, 0));
       // gate rows then up rows: SwiGLU over [nr, f] with the up half Rs * f further on
       CRF_CUDA(launch_swiglu_up_rows(gu, gu + Rs * D.f, m, nr, D.f, up_of(l, CRF_MOD_GATE), up_of(l, CRF_MOD_UP),
@@ -772,7 +776,7 @@ StepPlan make_step_plan(const Dims& D, const crf_decode_row* rows, int n) {
   p.max_n = 1;
   for (int i = 0; i < n; ++i) p.max_n = std::max(p.max_n, rows[i].pos + 1);
   p.splits = dec_splits(p.max_n);
-  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 7 * kRankPad + 3 * D.f) * 4 +
+  const size_t dec_row = static_cast<size_t>(3 * D.h + 2 * D.qd + 2 * D.kvd + 7 * kRankPad + 3 * D.f + norm_up_slices(D.h)) * 4 +
                          static_cast<size_t>(D.hq) * p.splits * (D.d + 2) * 4;
   p.dec_bytes = align256(dec_row * std::max(1, n));
   size_t o = 0;
@@ -789,7 +793,7 @@ StepPlan make_step_plan(const Dims& D, const crf_decode_row* rows, int n) {
   long ids = 0;
   for (int i = 0; i < n; ++i) ids += rows[i].pos / kPage + 1;
   p.ptab_slots = ptab_slots_for(ids);
-  p.off_abort = take(sizeof(int));
+  p.off_abort = take((1 + p.flag_words) * sizeof(int));
   p.off_ptab = take(static_cast<size_t>(p.ptab_slots) * sizeof(int));
   sp.total = p.total = o;
   return sp;
@@ -1142,7 +1146,8 @@ crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const crf_adapt
       pc.pt[i] = rows[i].page_table;
       pc.first[i + 1] = pc.first[i] + rows[i].pos / kPage + 1;
     }
-    s = open_call(ctx, pc, pool->num_pages, ws, sp.p.off_abort, 0, sp.p.off_ptab, sp.p.ptab_slots, st);
+    s = open_call(ctx, pc, pool->num_pages, ws, sp.p.off_abort, sp.p.flag_words, sp.p.off_ptab, sp.p.ptab_slots,
+                  st);
     if (s != CRF_OK) return s;
   }
   RowPositions rp{};

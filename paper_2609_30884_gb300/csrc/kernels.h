@@ -210,9 +210,13 @@ struct RowUp {
   const float* xa;
 };
 // x[r] += up(r) for r < up_rows (the rows that carry a pending product), then for every row
-// xn[r] = rmsnorm(x[r]) * g (eps): the residual stream's update and the next RMSNorm in one launch.
+// xn[r] = rmsnorm(x[r]) * g (eps): the residual stream's update and the next RMSNorm in one launch,
+// over norm_up_slices(dim) blocks per row. part: [rows, slices] fp32 scratch; counter: [rows] ints,
+// zero before the first launch and left zero by every launch.
+int norm_up_slices(int dim);
 cudaError_t launch_norm_up_rows(float* x, int dim, int rows, RowUp up, int up_rows, int rank,
-                                const __nv_bfloat16* g, float eps, float* xn, cudaStream_t stream);
+                                const __nv_bfloat16* g, float eps, float* xn, float* part, int* counter,
+                                cudaStream_t stream);
 // x[r] += up(r) for every row (the last projection's product, before the rows leave).
 cudaError_t launch_rows_up(float* x, int dim, int rows, RowUp up, int rank, cudaStream_t stream);
 cudaError_t launch_rmsnorm_f32(const float* x, const __nv_bfloat16* g, float* y, int rows,

@@ -249,39 +249,62 @@ __device__ __forceinline__ float up_dot(const __nv_bfloat16* __restrict__ B, int
   return s;
 }
 
-// One block per row: x[r] += up(r) when r < up_rows, then xn[r] = rmsnorm(x[r]) * g.
-constexpr int kNormThreads = 512;
-__global__ void __launch_bounds__(kNormThreads) norm_up_rows_kernel(float* __restrict__ x, int dim, RowUp up,
-                                                                    int up_rows, int rank,
-                                                                    const __nv_bfloat16* __restrict__ g, float eps,
-                                                                    float* __restrict__ xn) {
-  __shared__ float red[kNormThreads / 32];
+// x[r] += up(r) when r < up_rows, then xn[r] = rmsnorm(x[r]) * g, with each row cut into slices of
+// kNormSlice elements, one block per (row, slice): the block adds its slice's up products (the
+// rank-r B rows of the slice) and writes the slice's sum of squares to part[r][slice]; the last
+// block of the row to finish (a counter per row, reset by it) sums the partials in slice order
+// and normalises the whole row. Deterministic: the same partials, summed in the same order.
+constexpr int kNormSlice = 256;
+__global__ void __launch_bounds__(kNormSlice) norm_up_rows_kernel(float* __restrict__ x, int dim, RowUp up,
+                                                                  int up_rows, int rank,
+                                                                  const __nv_bfloat16* __restrict__ g, float eps,
+                                                                  float* __restrict__ xn, float* __restrict__ part,
+                                                                  int* __restrict__ counter, int slices) {
+  __shared__ float red[kNormSlice / 32];
   __shared__ float xa_s[kRankPad];
-  const int r = blockIdx.x;
+  __shared__ int last_s;
+  const int r = blockIdx.x / slices, sl = blockIdx.x % slices;
+  const int j = sl * kNormSlice + threadIdx.x;
   const bool add = up.B != nullptr && r < up_rows;
-  if (add) prefetch_l2_range(up.B, (size_t)dim * rank * 2);
+  if (add && threadIdx.x == 0)
+    prefetch_l2_range(up.B + (size_t)sl * kNormSlice * rank, (size_t)kNormSlice * rank * 2);
   griddep_begin();  // x and xa come from the kernels before
   float* xr = x + (size_t)r * dim;
   if (add && threadIdx.x < rank) xa_s[threadIdx.x] = up.xa[(size_t)r * rank + threadIdx.x];
   __syncthreads();
   float ss = 0.f;
-  for (int j = threadIdx.x; j < dim; j += kNormThreads) {
+  if (j < dim) {
     float v = xr[j];
     if (add) {
       v += up_dot(up.B, j, xa_s, rank);
       xr[j] = v;
     }
-    ss += v * v;
+    ss = v * v;
   }
   ss = warp_sum(ss);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
-  ss = 0.f;
+  if (threadIdx.x == 0) {
+    float t = 0.f;
 #pragma unroll
-  for (int w = 0; w < kNormThreads / 32; ++w) ss += red[w];
-  const float inv = rsqrtf(ss / dim + eps);
-  for (int j = threadIdx.x; j < dim; j += kNormThreads)
-    xn[(size_t)r * dim + j] = xr[j] * inv * __bfloat162float(g[j]);
+    for (int w = 0; w < kNormSlice / 32; ++w) t += red[w];
+    part[(size_t)r * slices + sl] = t;
+    __threadfence();  // the slice's x and its partial before the count
+    last_s = atomicAdd(counter + r, 1) == slices - 1;
+  }
+  __syncthreads();
+  if (!last_s) return;
+  __threadfence();  // every slice's x and partial are visible to this block
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+    for (int q = 0; q < slices; ++q) t += __ldcg(part + (size_t)r * slices + q);
+    red[0] = rsqrtf(t / dim + eps);
+    counter[r] = 0;  // ready for the next launch
+  }
+  __syncthreads();
+  const float inv = red[0];
+  for (int i = threadIdx.x; i < dim; i += kNormSlice)
+    xn[(size_t)r * dim + i] = __ldcg(xr + i) * inv * __bfloat162float(g[i]);
 }
 
 // x[r, j] += up(r, j), one thread per element.
@@ -627,12 +650,16 @@ cudaError_t launch_rope_up_rows(float* q, int hq, float* k, int hkv, float* v, i
                        head_dim, u, rank, table, pos, table_by_row ? 1 : 0);
 }
 
+int norm_up_slices(int dim) { return cdiv(dim, kNormSlice); }
+
 cudaError_t launch_norm_up_rows(float* x, int dim, int rows, RowUp up, int up_rows, int rank,
-                                const __nv_bfloat16* g, float eps, float* xn, cudaStream_t stream) {
+                                const __nv_bfloat16* g, float eps, float* xn, float* part, int* counter,
+                                cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
   if (rank != 4 && rank != 8 && rank != 16) return cudaErrorInvalidValue;
-  return launch_kernel(norm_up_rows_kernel, dim3(rows), dim3(kNormThreads), 0, stream, x, dim, up, up_rows, rank,
-                       g, eps, xn);
+  const int slices = norm_up_slices(dim);
+  return launch_kernel(norm_up_rows_kernel, dim3(rows * slices), dim3(kNormSlice), 0, stream, x, dim, up, up_rows,
+                       rank, g, eps, xn, part, counter, slices);
 }
 
 cudaError_t launch_rows_up(float* x, int dim, int rows, RowUp up, int rank, cudaStream_t stream) {
