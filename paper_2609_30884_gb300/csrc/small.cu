@@ -303,8 +303,21 @@ __global__ void __launch_bounds__(kNormSlice) norm_up_rows_kernel(float* __restr
   }
   __syncthreads();
   const float inv = red[0];
-  for (int i = threadIdx.x; i < dim; i += kNormSlice)
-    xn[(size_t)r * dim + i] = __ldcg(xr + i) * inv * __bfloat162float(g[i]);
+  // eight elements per thread in flight: the row's other slices come from L2
+  for (int i0 = threadIdx.x; i0 < dim; i0 += 8 * kNormSlice) {
+    float xv[8], gv[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int i = i0 + u * kNormSlice;
+      xv[u] = i < dim ? __ldcg(xr + i) : 0.f;
+      gv[u] = i < dim ? __bfloat162float(g[i]) : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int i = i0 + u * kNormSlice;
+      if (i < dim) xn[(size_t)r * dim + i] = xv[u] * inv * gv[u];
+    }
+  }
 }
 
 // x[r, j] += up(r, j), one thread per element.
