@@ -347,27 +347,46 @@ __global__ void __launch_bounds__(256) drift_tc_final_kernel(const __grid_consta
   __shared__ float gb[r2][r2 + 1], ga[r2][r2 + 1];
   __shared__ double red[2][8];
   const int item = blockIdx.x;
+  // slots b_lo .. b_hi of each side's segment, summed in CTA order; every load of one slot
+  // offset (both sides, all of a thread's entries) is issued before any of them is added
+  constexpr int kPer = (S::kSlotFloats + 255) / 256;
+  int b_lo[2], n_slot[2];
   for (int side = 0; side < 2; ++side) {
     const int seg = 2 * item + side;
     const long long s0 = a.seg_step0[seg], s1 = a.seg_step0[seg + 1] - 1;
-    const int b_lo = static_cast<int>(((s0 + 1) * a.grid - 1) / a.total_steps);
-    const int b_hi = static_cast<int>(((s1 + 1) * a.grid - 1) / a.total_steps);
-    for (int e = threadIdx.x; e < S::kSlotFloats; e += 256) {
-      const float* p = slots + static_cast<size_t>(b_lo + seg) * S::kSlotFloats + e;
-      float v = 0.f;
-      int bb = b_lo;
-      for (; bb + 4 <= b_hi + 1; bb += 4, p += 4 * S::kSlotFloats) {  // four loads in flight
-        const float x0 = p[0], x1 = p[S::kSlotFloats], x2 = p[2 * S::kSlotFloats],
-                    x3 = p[3 * S::kSlotFloats];
-        v += x0;
-        v += x1;
-        v += x2;
-        v += x3;
-      }
-      for (; bb <= b_hi; ++bb, p += S::kSlotFloats) v += *p;
-      g[side][e] = v;
-    }
+    b_lo[side] = static_cast<int>(((s0 + 1) * a.grid - 1) / a.total_steps);
+    n_slot[side] = static_cast<int>(((s1 + 1) * a.grid - 1) / a.total_steps) - b_lo[side] + 1;
   }
+  float v[2][kPer];
+#pragma unroll
+  for (int side = 0; side < 2; ++side)
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) v[side][u] = 0.f;
+  const int n_max = n_slot[0] > n_slot[1] ? n_slot[0] : n_slot[1];
+  for (int k = 0; k < n_max; ++k) {
+    float x[2][kPer];
+#pragma unroll
+    for (int side = 0; side < 2; ++side) {
+      const float* p = slots + static_cast<size_t>(b_lo[side] + k + 2 * item + side) * S::kSlotFloats;
+#pragma unroll
+      for (int u = 0; u < kPer; ++u) {
+        const int e = threadIdx.x + 256 * u;
+        x[side][u] = (k < n_slot[side] && e < S::kSlotFloats) ? p[e] : 0.f;
+      }
+    }
+#pragma unroll
+    for (int side = 0; side < 2; ++side)
+#pragma unroll
+      for (int u = 0; u < kPer; ++u)
+        if (k < n_slot[side]) v[side][u] += x[side][u];
+  }
+#pragma unroll
+  for (int side = 0; side < 2; ++side)
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int e = threadIdx.x + 256 * u;
+      if (e < S::kSlotFloats) g[side][e] = v[side][u];
+    }
   __syncthreads();
   // entry (f1, f2) of a side's symmetric feature Gram from its accumulated block pairs
   auto G = [&](int side, int f1, int f2) -> float {
