@@ -160,6 +160,22 @@ def algorithmic_work(cfg, lc, n):
     return flops, byts
 
 
+def step_bytes(cfg, lc, ns, wins):
+    """Algorithmic HBM bytes of the step's bandwidth-bound parts, once per step.
+
+    drift_gram: both adapter versions' factors of every layer and module (bf16). tail_decode: per
+    request, the weights of layers e..N-1 (base rows and LoRA A and B, bf16) and the K/V of its
+    prefix at those layers. lm_head: the head's rows once (fresh and recovered rows share the pass).
+    """
+    h, f, qd, kvd, r = cfg.hidden, cfg.ffn, cfg.n_q_heads * cfg.head_dim, cfg.n_kv_heads * cfg.head_dim, lc.rank
+    dims = {"q": (h, qd), "k": (h, kvd), "v": (h, kvd), "o": (qd, h), "gate": (h, f), "up": (h, f), "down": (f, h)}
+    lora = sum(r * (i + o) * 2 for m, (i, o) in dims.items() if m in lc.modules)
+    base = sum(i * o * 2 for i, o in dims.values())
+    tail = sum((cfg.n_layers - e) * (base + lora + 2 * (n - 1) * kvd * 2) for n, (_, e) in zip(ns, wins))
+    return {"drift_gram": 2 * cfg.n_layers * lora, "tail_decode": tail,
+            "lm_head": cfg.vocab * h * 2}
+
+
 def shard_requests(loads, world):
     """Split independent requests over ranks (longest first onto the least-loaded rank).
 
@@ -900,6 +916,8 @@ def main():
             flops_step[k] = flops_step.get(k, 0) + v * (e_i - s_i)
         for k, v in by.items():
             bytes_step[k] = bytes_step.get(k, 0) + v * (e_i - s_i)
+    for k, v in step_bytes(cfg, lc, st["ns"], st["wins"]).items():
+        bytes_step[k] = bytes_step.get(k, 0) + v
     flops_layer, _ = algorithmic_work(cfg, lc, n)
     kernels = {}
     gpu_launches = 0

@@ -115,3 +115,16 @@ def test_clock_summary_reports_median_and_active_reasons():
     assert bench.ClockSampler.summarise([])["reasons"] == ["no samples"]
     na = bench.ClockSampler.summarise(["0, [N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A]\n"])
     assert na["sm_mhz"] is None and na["sm_max_mhz"] is None
+
+
+def test_step_bytes_7b_match_hand_count():
+    import synth
+    wl = synth.workload("7b-16k-w4")
+    b = bench.step_bytes(wl.model, wl.lora, wl.n_tokens, wl.windows)
+    h, f, qd, kvd, r, N = 3584, 18944, 3584, 512, 16, 28
+    per_layer_w = 2 * (h * (qd + 2 * kvd) + qd * h + 2 * h * f + f * h)
+    per_layer_lora = 2 * r * ((h + qd) + 2 * (h + kvd) + (qd + h) + 2 * (h + f) + (f + h))
+    assert b["drift_gram"] == 2 * N * per_layer_lora == 161480704
+    # window [14, 18): the row runs layers 18..27 over 16383 cached keys per layer (K and V)
+    assert b["tail_decode"] == 10 * (per_layer_w + per_layer_lora + 2 * 16383 * kvd * 2)
+    assert b["lm_head"] == 152064 * h * 2
