@@ -3,8 +3,9 @@ its own window, one shared pool with a randomly permuted page table.
 
 * Batching is invisible in the window: the batched call gives bit-identical pages and refreshed
   checkpoints to running every request alone (each row is computed the same way whatever else
-  shares its tile or launch); the first-step rows agree to bf16 rounding (their GEMV kernel
-  depends on how many rows share a weight pass).
+  shares its tile or launch); the first-step rows agree to the per-layer 1e-2 bar (their GEMV
+  kernel depends on how many rows share a weight pass, and its rounding compounds over the layers
+  after the window).
 * Against the oracle, per request, on what it computes at this size: K and V of every position of
   the request's first window layer, and that layer's output at 48 rows spread over the prefix,
   held to 1e-2 or 1.25x the distance the oracle's layer moves at the same rows when it stores its
@@ -66,6 +67,7 @@ def test_batch7b_equals_single_and_oracle(ctx):
     got_v = [t.clone() for t in pool.v_pages]
 
     # every request alone on a fresh copy of the historical pool
+    fin_err = []
     for i in range(len(reqs)):
         for l in range(cfg.n_layers):
             pool.k_pages[l].copy_(bk[l])
@@ -79,9 +81,13 @@ def test_batch7b_equals_single_and_oracle(ctx):
             assert torch.equal(request_kv_t(pool.k_pages[l], pts[i], n), request_kv_t(got_k[l], pts[i], n)), (i, l)
             assert torch.equal(request_kv_t(pool.v_pages[l], pts[i], n), request_kv_t(got_v[l], pts[i], n)), (i, l)
             assert torch.equal(keep1[i][2][l - s], keep[i][2][l - s]), (i, l)
-        # the first-step row takes the tensor-core GEMV when >= 3 rows share a weight pass and the
-        # CUDA-core one alone: both fp32-accurate, so only bf16 rounding of the output may differ
-        assert rel_frob(to_np(keep1[i][3]), to_np(keep[i][3])) <= 5e-3, i
+        # the first-step row takes the tensor-core GEMV (main and adapter-down products) when >= 3
+        # rows share a weight pass and the CUDA-core one alone: both fp32-accurate, but their
+        # rounding differs and compounds over every layer the row passes after its window (26 after a
+        # window [0, 2)), so it is held to the per-layer bar the oracle tests use
+        fin_err.append(rel_frob(to_np(keep1[i][3]), to_np(keep[i][3])))
+    print("first-step row, batched vs alone:", [f"{x:.2e}" for x in fin_err])
+    assert max(fin_err) <= REL_KVH, fin_err
 
     # untouched slots and layers, bit-exact
     free = untouched_mask(P, list(zip(pts, wl.n_tokens)))
