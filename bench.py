@@ -659,9 +659,14 @@ def run_drift_case(args):
     ctx.check()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
+    # the device sleeps while the host enqueues every timed call, so the events time the device
+    # alone (a call's host side, ctypes marshalling and two launches, can outlast its kernels)
+    torch.cuda._sleep(int(2e6) * max(1, args.steps))
     a.record()
+    h0 = time.perf_counter()
     for _ in range(args.steps):
         ctx.drift(dm.crf.dims_c, cur.crf, which, out, ws)
+    host_us = (time.perf_counter() - h0) / args.steps * 1e6
     b.record()
     torch.cuda.synchronize()
     ctx.check()
@@ -674,6 +679,7 @@ def run_drift_case(args):
     gbs = factor_bytes / (ms / 1000.0) / 1e9
     print(json.dumps({"case": "drift", "workload": f"{args.workload}: {wl.name}", "rank": lc.rank,
                       "modules": list(lc.modules), "ms_per_call": round(ms, 4),
+                      "host_us_per_call": round(host_us, 1),
                       "hbm": {"bytes": factor_bytes, "achieved_gbs": round(gbs, 1),
                               "frac": round(gbs / peaks["hbm_gbs"], 4), "peak_source": src}}))
     ctx.close()

@@ -1207,7 +1207,7 @@ crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter
   if (!cur->A || !cur->B) return fail(CRF_EINVAL, "adapter tables missing");
   const Dims D = dims_of(*dims);
   if (D.h % 8 || D.f % 8 || D.qd % 8 || D.kvd % 8)
-    return fail(CRF_EUNSUPPORTED, "drift needs every projection's input width to be a multiple of 8");
+    return fail(CRF_EUNSUPPORTED, "drift needs every projection's widths to be multiples of 8");
   std::vector<DriftItem> items;
   for (int l = 0; l < D.N; ++l) {
     const crf_adapter* an = anchors[l];
@@ -1237,11 +1237,14 @@ crf_status crf_drift(crf_ctx* ctx, const crf_model_dims* dims, const crf_adapter
     return fail(CRF_ENOMEM, "drift workspace null, misaligned or %zu < %zu bytes", ws_bytes, need);
   CRF_CUDA(cudaSetDevice(ctx->device));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  CRF_CUDA(cudaMemsetAsync(out_sq, 0, static_cast<size_t>(D.N) * 7 * 2 * sizeof(float), st));
-  if (items.empty()) return CRF_OK;
+  if (items.empty()) {
+    CRF_CUDA(cudaMemsetAsync(out_sq, 0, static_cast<size_t>(D.N) * 7 * 2 * sizeof(float), st));
+    return CRF_OK;
+  }
   ProfScope ps(ctx, kPDrift, st, drift_launches(static_cast<int>(items.size())));
-  CRF_CUDA(launch_drift(items.data(), static_cast<int>(items.size()), cur->dims.rank,
-                        static_cast<float*>(workspace), ctx->num_sms, out_sq, st));
+  CRF_CUDA(launch_drift(items.data(), static_cast<int>(items.size()), cur->dims.rank, D.N * 7,
+                        static_cast<int>(cur->dims.module_mask), workspace, ctx->num_sms, out_sq,
+                        ctx->status_dev, st));
   return CRF_OK;
 }
 

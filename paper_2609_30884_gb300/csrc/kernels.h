@@ -322,12 +322,14 @@ struct DriftItem {
   int in_dim, out_dim;
   int out_index;           // layer * 7 + module
 };
-// Tensor-core drift (mma.sync Grams over the long dimensions, fp64 combine); `slots` is device
-// scratch of drift_workspace_bytes(num_sms, rank, n_items) bytes. Launches drift_launches(n)
-// kernels.
+// Tensor-core drift (mma.sync Grams over the long dimensions, then a dependent-launched fp64
+// combine per item); `workspace` is device scratch of drift_workspace_bytes(num_sms, rank,
+// n_items) bytes (partial Grams). Launches drift_launches(n) kernels. out_sq holds n_out
+// (layer, module) pairs; the entries of modules outside `adapted_mask` are cleared. A copy wait
+// that exceeds its time limit sets kStatusTimeout in `status`.
 size_t drift_workspace_bytes(int num_sms, int rank, int n_items);
 int drift_launches(int n_items);
-cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, float* slots, int num_sms,
-                         float* out_sq, cudaStream_t stream);
+cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, int n_out, int adapted_mask,
+                         void* workspace, int num_sms, float* out_sq, int* status, cudaStream_t stream);
 
 }  // namespace crf
