@@ -74,22 +74,18 @@ struct DtShape {
   static constexpr int kPairs = RP == 16 ? 5 : 3;
   static constexpr int kSlotFloats = kPairs * 256;
   static constexpr int kRedFloats = kPairs * 8 * 32;  // one warp's accumulators
-  // the combine's scratch: both sides' summed slots, GB and GA, 2 x 8 doubles
-  static constexpr int kCombineBytes = (2 * kSlotFloats * 4 + 2 * (2 * R) * (2 * R + 1) * 4 + 7) / 8 * 8 + 128;
+  // the combine's scratch: both sides' summed slots, 2 x 8 doubles
+  static constexpr int kCombineBytes = 2 * kSlotFloats * 4 + 128;
   static constexpr int kScratch = 4 * kRedFloats * 4;  // the warp-sum tree's first round
   // stages, the tree's scratch, a full and an empty mbarrier per stage, the abort flag
   static constexpr int kSmem = kDtStages * kStage + kScratch + kDtStages * 16 + 16;
 };
 
-// (I, J) of accumulated pair p, and the pair of (I, J) (-1: not accumulated, reads as zero)
+// (I, J): the 16-feature blocks of accumulated pair p
 template <int RP>
 __host__ __device__ constexpr int pair_I(int p) { return RP == 16 ? (p < 3 ? 0 : (p == 3 ? 1 : 2)) : (p < 2 ? 0 : 1); }
 template <int RP>
 __host__ __device__ constexpr int pair_J(int p) { return RP == 16 ? (p < 3 ? p : 2) : (p < 2 ? p : 1); }
-template <int RP>
-__host__ __device__ constexpr int pair_of(int I, int J) {
-  return RP == 16 ? (I == 0 ? J : (I == 1 ? (J == 2 ? 3 : -1) : 4)) : (I == 0 ? J : 2);
-}
 
 // 1-D bulk copy global -> this CTA's shared memory, completing `bytes` on mbarrier `bar`. Both
 // addresses 16-byte aligned, `bytes` a positive multiple of 16.
@@ -220,14 +216,14 @@ __device__ __forceinline__ void issue_step(const ProdSeg& ps, int x, uint32_t st
   }
 }
 
-// This warp's 16-row slice of a staged step into its Gram accumulators.
+// This warp's fragments of one 16-row slice of a staged step, both versions:
+// {m0, m1, m2, m3} (RP = 8: m0, m2).
 template <int R, int SIDE>
-__device__ __forceinline__ void mma_slice(uint32_t st, int row0, float (&acc)[DtShape<R>::kPairs][2][4]) {
+__device__ __forceinline__ void load_frags(uint32_t st, int row0, uint32_t (&f1)[4], uint32_t (&f0)[4]) {
   using S = DtShape<R>;
   constexpr int RP = S::RP;
   const int lane = threadIdx.x & 31;
   const int m = lane >> 3, i = lane & 7;
-  uint32_t f1[4], f0[4];  // fragments of version 1 and version 0: {m0, m1, m2, m3} (RP = 8: m0, m2)
   if constexpr (SIDE == 0) {
     // X[o][f] rows: matrix m covers rows row0 + (m >> 1) * 8 .. and features (m & 1) * 8 ..
     if constexpr (RP == 16) {
@@ -255,7 +251,15 @@ __device__ __forceinline__ void mma_slice(uint32_t st, int row0, float (&acc)[Dt
       }
     }
   }
-  // base: B0 on the B side, A1 on the A side
+}
+
+// One slice's fragments into the Gram accumulators: [hi | lo | base] built in registers
+// (base: B0 on the B side, A1 on the A side), then the accumulated block pairs.
+template <int R, int SIDE>
+__device__ __forceinline__ void mma_frags(const uint32_t (&f1)[4], const uint32_t (&f0)[4],
+                                          float (&acc)[DtShape<R>::kPairs][2][4]) {
+  using S = DtShape<R>;
+  constexpr int RP = S::RP;
   uint32_t blk[S::kBlocks][4];
   if constexpr (RP == 16) {
 #pragma unroll
@@ -298,10 +302,15 @@ __device__ __forceinline__ bool run_steps(int& x, int end, int& stage, uint32_t&
   for (; x < end; ++x) {
     if (!mbar_wait(full + stage, phase, abort_flag, status)) return false;
     const uint32_t st = stage0 + stage * S::kStage;
+    // both slices' fragments into registers, then the stage goes back to the producer before
+    // they are multiplied
+    uint32_t f1[kDtSlices][4], f0[kDtSlices][4];
 #pragma unroll
-    for (int sl = 0; sl < kDtSlices; ++sl) mma_slice<R, SIDE>(st, (warp * kDtSlices + sl) * 16, acc);
+    for (int sl = 0; sl < kDtSlices; ++sl) load_frags<R, SIDE>(st, (warp * kDtSlices + sl) * 16, f1[sl], f0[sl]);
     __syncwarp();
     if ((threadIdx.x & 31) == 0) mbar_arrive(empty + stage);
+#pragma unroll
+    for (int sl = 0; sl < kDtSlices; ++sl) mma_frags<R, SIDE>(f1[sl], f0[sl], acc);
     if (++stage == kDtStages) {
       stage = 0;
       phase ^= 1u;
@@ -352,24 +361,44 @@ __device__ __forceinline__ void seg_slots(const DriftTcArgs& a, int seg, int& b_
   n_slot = static_cast<int>(((s1 + 1) * a.grid - 1) / a.total_steps) - b_lo + 1;
 }
 
-// One item, by 256 threads: both segments' slots summed in CTA order, GB and GA assembled from the [hi | lo | base] Grams (fp32: sums of at most four
-// entries; rank 4 adds the B side's two packed halves first), then tr(GB GA) and the parameter
-// distance in fp64, written to the item's out_sq pair. `buf` is shared scratch of
-// kCombineBytes. The slots come from other CTAs: read through L2.
+// Entries of one side's difference/base Grams from its accumulated block pairs `gs`
+// ([pair][16][16]): features hi_i, lo_i (d = hi + lo) and base_i.
+//   DD(i, j) = <d_i, d_j>,  DB(i, j) = <d_i, base_j>,  BB(i, j) = <base_i, base_j>.
+// RP = 16: blocks hi | lo | base, pairs (hi,hi) (hi,lo) (hi,base) (lo,base) (base,base), lo x lo
+// not accumulated. RP = 8: blocks [hi | lo] | [base | 0], pairs (0,0) (0,1) (1,1).
+template <int RP>
+struct SideGram {
+  const float* gs;
+  __device__ __forceinline__ float P(int k, int r, int c) const { return gs[k * 256 + r * 16 + c]; }
+  __device__ __forceinline__ float DD(int i, int j) const {
+    if constexpr (RP == 16) return P(0, i, j) + P(1, i, j) + P(1, j, i);
+    else return P(0, i, j) + P(0, i, 8 + j) + P(0, 8 + i, j) + P(0, 8 + i, 8 + j);
+  }
+  __device__ __forceinline__ float DB(int i, int j) const {
+    if constexpr (RP == 16) return P(2, i, j) + P(3, i, j);
+    else return P(1, i, j) + P(1, 8 + i, j);
+  }
+  __device__ __forceinline__ float BB(int i, int j) const { return RP == 16 ? P(4, i, j) : P(2, i, j); }
+};
+
+// One item, by 256 threads: both segments' slots summed in CTA order, then
+//   tr(GB GA) = sum_ij DD_B(i,j) BB_A(i,j) + BB_B(i,j) DD_A(i,j) + 2 DB_B(i,j) DB_A(j,i)
+// (GB = [[DD_B, DB_B], [DB_B^T, BB_B]] over [B1 - B0 | B0]; GA = [[BB_A, DB_A^T], [DB_A, DD_A]]
+// over [A1 ; A1 - A0]) and the parameter distance sum_i DD_B(i,i) + DD_A(i,i): one (i, j) term
+// per thread in fp64 from fp32 Gram entries, reduced in a fixed order, written to the item's
+// out_sq pair. Rank 4 adds the B side's two packed halves (fragment features i and i + 4).
+// `buf` is shared scratch of kCombineBytes. The slots come from other CTAs: read through L2.
 template <int R>
 __device__ void combine_item(const DriftTcArgs& a, int item, const float* __restrict__ slots,
                              float* __restrict__ out_sq, uint8_t* buf) {
   using S = DtShape<R>;
   constexpr int RP = S::RP;
-  constexpr int r2 = 2 * R;
   float (*g)[S::kSlotFloats] = reinterpret_cast<float (*)[S::kSlotFloats]>(buf);
-  float (*gb)[r2 + 1] = reinterpret_cast<float (*)[r2 + 1]>(buf + 2 * S::kSlotFloats * 4);
-  float (*ga)[r2 + 1] = gb + r2;
   double (*red)[8] = reinterpret_cast<double (*)[8]>(buf + S::kCombineBytes - 128);
-  // every load of two slot offsets (both sides, all of a thread's entries) is issued before any
-  // of them is added; the adds keep CTA order
+  // every load of up to eight slot offsets (both sides, all of a thread's entries) is issued
+  // before any of them is added; the adds keep CTA order
   constexpr int kPer = (S::kSlotFloats + kDtConsumers - 1) / kDtConsumers;
-  constexpr int kBatch = 2;
+  constexpr int kBatch = 8;
   int b_lo[2], n_slot[2];
   for (int side = 0; side < 2; ++side) seg_slots(a, 2 * item + side, b_lo[side], n_slot[side]);
   float v[2][kPer];
@@ -408,48 +437,20 @@ __device__ void combine_item(const DriftTcArgs& a, int item, const float* __rest
       if (e < S::kSlotFloats) g[side][e] = v[side][u];
     }
   consumers_sync();
-  // entry (f1, f2) of a side's symmetric feature Gram from its accumulated block pairs
-  auto G = [&](int side, int f1, int f2) -> float {
-    int I = f1 >> 4, J = f2 >> 4;
-    if (I > J) {
-      const int t = f1;
-      f1 = f2;
-      f2 = t;
-      I = f1 >> 4;
-      J = f2 >> 4;
-    }
-    const int p = pair_of<RP>(I, J);
-    return p < 0 ? 0.f : g[side][p * 256 + (f1 & 15) * 16 + (f2 & 15)];
-  };
-  // rank 4, B side: fragment feature i < 4 of a part is row 2j, feature i + 4 row 2j + 1
-  auto Gs = [&](int side, int f1, int f2) -> float {
-    float t = G(side, f1, f2);
-    if constexpr (R < RP) {
-      if (side == 0) t += G(side, f1 + R, f2 + R);
-    }
-    return t;
-  };
-  // <d_i, d_j>, <d_i, base_j>, <base_i, base_j> with d = hi + lo; features hi_i = i,
-  // lo_i = RP + i, base_i = 2 RP + i
-  auto dd = [&](int s, int i, int j) {
-    return Gs(s, i, j) + Gs(s, i, RP + j) + Gs(s, RP + i, j) + Gs(s, RP + i, RP + j);
-  };
-  auto db = [&](int s, int i, int j) { return Gs(s, i, 2 * RP + j) + Gs(s, RP + i, 2 * RP + j); };
-  auto bb = [&](int s, int i, int j) { return Gs(s, 2 * RP + i, 2 * RP + j); };
-  for (int idx = threadIdx.x; idx < r2 * r2; idx += kDtConsumers) {
-    const int p = idx / r2, q = idx % r2;
-    // GB over [B1 - B0 | B0]; GA over [A1 ; A1 - A0]: base first on the A side
-    gb[p][q] = p < R ? (q < R ? dd(0, p, q) : db(0, p, q - R)) : (q < R ? db(0, q, p - R) : bb(0, p - R, q - R));
-    ga[p][q] = p < R ? (q < R ? bb(1, p, q) : db(1, q - R, p)) : (q < R ? db(1, p - R, q) : dd(1, p - R, q - R));
-  }
-  consumers_sync();
+  const SideGram<RP> gB{g[0]}, gA{g[1]};
   double t = 0.0, par = 0.0;
-  for (int idx = threadIdx.x; idx < r2 * r2; idx += kDtConsumers) {
-    const int p = idx / r2, q = idx % r2;
-    t += static_cast<double>(gb[p][q]) * static_cast<double>(ga[p][q]);  // both symmetric
+  if (threadIdx.x < R * R) {
+    const int i = threadIdx.x / R, j = threadIdx.x % R;
+    float dd0 = gB.DD(i, j), db0 = gB.DB(i, j), bb0 = gB.BB(i, j);
+    if constexpr (R < RP) {
+      dd0 += gB.DD(i + R, j + R);
+      db0 += gB.DB(i + R, j + R);
+      bb0 += gB.BB(i + R, j + R);
+    }
+    const float dd1 = gA.DD(i, j), db1t = gA.DB(j, i), bb1 = gA.BB(i, j);
+    t = static_cast<double>(dd0) * bb1 + static_cast<double>(bb0) * dd1 + 2.0 * (static_cast<double>(db0) * db1t);
+    if (i == j) par = static_cast<double>(dd0) + static_cast<double>(dd1);
   }
-  if (threadIdx.x < R)
-    par = static_cast<double>(gb[threadIdx.x][threadIdx.x]) + static_cast<double>(ga[R + threadIdx.x][R + threadIdx.x]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     t += __shfl_xor_sync(0xffffffffu, t, o);
@@ -469,7 +470,6 @@ __device__ void combine_item(const DriftTcArgs& a, int item, const float* __rest
     out_sq[a.items[item].out_index * 2 + 0] = static_cast<float>(tt);
     out_sq[a.items[item].out_index * 2 + 1] = static_cast<float>(pp);
   }
-  consumers_sync();  // the scratch is free again
 }
 
 template <int R>
