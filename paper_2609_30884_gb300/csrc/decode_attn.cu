@@ -119,23 +119,28 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
 
   if (warp == 4) {
     // ---------------------------------------------------------------- producer
-    if (lane == 0) {
-      const int32_t* pt = p.page_table[r];
-      int armed[kStages];
-      for (int st = 0; st < kStages; ++st) armed[st] = -1;
-      for (int c = c_beg; c < c_end; ++c) {
-        const int i = c - c_beg, st = i % kStages;
-        if (i >= kStages && !mbar_wait(&empty[st], (i / kStages - 1) & 1, &abort_flag, a.status)) break;
-        const int t0 = c * kChunk;
-        const int pages = (min(kChunk, pos - t0) + kPage - 1) / kPage;
-        uint8_t* sK = sKV + st * 2 * TILE;
-        uint8_t* sV = sK + TILE;
-        if (pages == 0) {
-          mbar_arrive(&full[st]);  // only the row's own key here: nothing to copy
-        } else {
-          mbar_arrive_expect_tx(&full[st], 2 * pages * HALVES * kPage * 128);
-          for (int pg = 0; pg < pages; ++pg) {
-            const int page = checked_page(pt[t0 / kPage + pg], a.num_pages, a.status);
+    // Lane l reads page id l of the chunk (all of a chunk's ids in flight at once, before the
+    // wait for its stage); lane 0 takes them by shuffle and issues the copies.
+    const int32_t* pt = p.page_table[r];
+    int armed[kStages];
+    for (int st = 0; st < kStages; ++st) armed[st] = -1;
+    for (int c = c_beg; c < c_end; ++c) {
+      const int i = c - c_beg, st = i % kStages;
+      const int t0 = c * kChunk;
+      const int pages = (min(kChunk, pos - t0) + kPage - 1) / kPage;  // <= kChunk / kPage
+      const int my_page = lane < pages ? checked_page(pt[t0 / kPage + lane], a.num_pages, a.status) : 0;
+      if (i >= kStages &&
+          !__all_sync(0xffffffffu, mbar_wait(&empty[st], (i / kStages - 1) & 1, &abort_flag, a.status)))
+        break;
+      uint8_t* sK = sKV + st * 2 * TILE;
+      uint8_t* sV = sK + TILE;
+      if (pages == 0) {
+        if (lane == 0) mbar_arrive(&full[st]);  // only the row's own key here: nothing to copy
+      } else {
+        if (lane == 0) mbar_arrive_expect_tx(&full[st], 2 * pages * HALVES * kPage * 128);
+        for (int pg = 0; pg < pages; ++pg) {
+          const int page = __shfl_sync(0xffffffffu, my_page, pg);
+          if (lane == 0) {
             const int row = (page * p.n_kv_heads + g) * kPage;
             for (int h = 0; h < HALVES; ++h) {
               const int off = h * HALF + pg * (kPage * 128);
@@ -143,9 +148,11 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
               tma_load_2d(sV + off, &a.tmV, &full[st], 64 * h, row);
             }
           }
-          armed[st] = (i / kStages) & 1;
         }
+        armed[st] = (i / kStages) & 1;
       }
+    }
+    if (lane == 0) {
       // copies still in flight land before the block's shared memory is released
       volatile int never = 0;
       for (int st = 0; st < kStages; ++st)
