@@ -7,7 +7,7 @@
 // The work is memory-bound (K and V of every cached position are read once): the positions
 // are cut into chunks of 128 and streamed.
 //   decode_attn_stream  one block per SM, walking a run of consecutive chunks of one (row,
-//                       kv head) through a two-stage ring: a copy warp gathers the next
+//                       kv head) through a two- or three-stage ring: a copy warp gathers the next
 //                       chunk's K and V pages with TMA (128-byte swizzle) while four compute
 //                       warps score the current one. The group's query heads (padded to 16 rows)
 //                       meet the chunk on mma.sync m16n8k16 (each warp takes a 32-key slice),
@@ -33,7 +33,9 @@ namespace crf {
 namespace {
 
 constexpr int kChunk = 128;                     // positions per chunk
-constexpr int kStages = 2;                      // K/V ring depth (64 KB per stage at d = 128)
+// The K/V ring depth is the stream kernel's template parameter (64 KB per stage at d = 128): 3
+// for a single decode row, 2 from two rows on (measured per generation step: one row 4.39 ->
+// 4.22 ms with 3 stages, eight rows 6.5 -> 10.4 ms)
 constexpr int kThreadsStream = 160;             // four compute warps + one copy warp
 constexpr int kMaxGroup = 8;
 
@@ -63,7 +65,7 @@ struct DecodeArgs {
   int* status;
 };
 
-template <int D>
+template <int D, int kStages>
 __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __grid_constant__ DecodeArgs a) {
   constexpr int HALVES = D / 64;
   constexpr int HALF = kChunk * 128;     // bytes of one 64-column half of a K (or V) tile
@@ -119,28 +121,23 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
 
   if (warp == 4) {
     // ---------------------------------------------------------------- producer
-    // Lane l reads page id l of the chunk (all of a chunk's ids in flight at once, before the
-    // wait for its stage); lane 0 takes them by shuffle and issues the copies.
-    const int32_t* pt = p.page_table[r];
-    int armed[kStages];
-    for (int st = 0; st < kStages; ++st) armed[st] = -1;
-    for (int c = c_beg; c < c_end; ++c) {
-      const int i = c - c_beg, st = i % kStages;
-      const int t0 = c * kChunk;
-      const int pages = (min(kChunk, pos - t0) + kPage - 1) / kPage;  // <= kChunk / kPage
-      const int my_page = lane < pages ? checked_page(pt[t0 / kPage + lane], a.num_pages, a.status) : 0;
-      if (i >= kStages &&
-          !__all_sync(0xffffffffu, mbar_wait(&empty[st], (i / kStages - 1) & 1, &abort_flag, a.status)))
-        break;
-      uint8_t* sK = sKV + st * 2 * TILE;
-      uint8_t* sV = sK + TILE;
-      if (pages == 0) {
-        if (lane == 0) mbar_arrive(&full[st]);  // only the row's own key here: nothing to copy
-      } else {
-        if (lane == 0) mbar_arrive_expect_tx(&full[st], 2 * pages * HALVES * kPage * 128);
-        for (int pg = 0; pg < pages; ++pg) {
-          const int page = __shfl_sync(0xffffffffu, my_page, pg);
-          if (lane == 0) {
+    if (lane == 0) {
+      const int32_t* pt = p.page_table[r];
+      int armed[kStages];
+      for (int st = 0; st < kStages; ++st) armed[st] = -1;
+      for (int c = c_beg; c < c_end; ++c) {
+        const int i = c - c_beg, st = i % kStages;
+        if (i >= kStages && !mbar_wait(&empty[st], (i / kStages - 1) & 1, &abort_flag, a.status)) break;
+        const int t0 = c * kChunk;
+        const int pages = (min(kChunk, pos - t0) + kPage - 1) / kPage;
+        uint8_t* sK = sKV + st * 2 * TILE;
+        uint8_t* sV = sK + TILE;
+        if (pages == 0) {
+          mbar_arrive(&full[st]);  // only the row's own key here: nothing to copy
+        } else {
+          mbar_arrive_expect_tx(&full[st], 2 * pages * HALVES * kPage * 128);
+          for (int pg = 0; pg < pages; ++pg) {
+            const int page = checked_page(pt[t0 / kPage + pg], a.num_pages, a.status);
             const int row = (page * p.n_kv_heads + g) * kPage;
             for (int h = 0; h < HALVES; ++h) {
               const int off = h * HALF + pg * (kPage * 128);
@@ -148,11 +145,9 @@ __global__ void __launch_bounds__(kThreadsStream) decode_attn_stream(const __gri
               tma_load_2d(sV + off, &a.tmV, &full[st], 64 * h, row);
             }
           }
+          armed[st] = (i / kStages) & 1;
         }
-        armed[st] = (i / kStages) & 1;
       }
-    }
-    if (lane == 0) {
       // copies still in flight land before the block's shared memory is released
       volatile int never = 0;
       for (int st = 0; st < kStages; ++st)
@@ -458,18 +453,20 @@ bool pool_map(CUtensorMap* m, const void* base, long rows, int cols) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D>
+template <int D, int kStages>
 cudaError_t launch_dec(const DecodeArgs& args, int blocks, cudaStream_t stream) {
   constexpr int smem = 2 * kStages * kChunk * D * 2 + 2 * 16 * D * 2 + 1024;  // K/V stages, q hi/lo
   static PerDevice once;
   int dev = 0;
   if (once.pending(&dev)) {
-    cudaError_t e = cudaFuncSetAttribute(decode_attn_stream<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(decode_attn_stream<D, kStages>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     once.done(dev);
   }
   const DecodeAttnDesc& d = args.d;
-  cudaError_t e = launch_kernel(decode_attn_stream<D>, dim3(blocks), dim3(kThreadsStream), smem, stream, args);
+  cudaError_t e =
+      launch_kernel(decode_attn_stream<D, kStages>, dim3(blocks), dim3(kThreadsStream), smem, stream, args);
   if (e != cudaSuccess) return e;
   // d carries chunks_per_block
   return launch_kernel(decode_attn_merge<D>, dim3(d.n_q_heads, d.rows, D / 32), dim3(128), 0, stream, d);
@@ -487,7 +484,7 @@ cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int 
   int max_pos = 0;
   for (int r = 0; r < d.rows; ++r) max_pos = std::max(max_pos, d.pos[r]);
   if (max_pos / kChunk + 1 > d.splits) return cudaErrorInvalidValue;
-  // one block per SM (two 64 KB K/V stages each), each streaming a run of consecutive chunks
+  // one block per SM (two or three 64 KB K/V stages each), each streaming a run of consecutive chunks
   // of one (row, kv head): the fewest chunks per block that keeps every block in one wave
   if (num_sms < 1) return cudaErrorInvalidValue;
   long items = 0;
@@ -509,8 +506,9 @@ cudaError_t launch_decode_attention(const DecodeAttnDesc& d, int num_pages, int 
   a.d.chunks_per_block = cpb;
   a.num_pages = num_pages;
   a.status = status;
-  if (d.head_dim == 128) return launch_dec<128>(a, blocks, stream);
-  if (d.head_dim == 64) return launch_dec<64>(a, blocks, stream);
+  const bool one_row = d.rows == 1;
+  if (d.head_dim == 128) return one_row ? launch_dec<128, 3>(a, blocks, stream) : launch_dec<128, 2>(a, blocks, stream);
+  if (d.head_dim == 64) return one_row ? launch_dec<64, 3>(a, blocks, stream) : launch_dec<64, 2>(a, blocks, stream);
   return cudaErrorInvalidValue;
 }
 
