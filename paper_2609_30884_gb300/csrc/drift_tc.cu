@@ -53,7 +53,7 @@ constexpr int kDtAStride = kDtRows * 2 + 16;  // bytes per A row in a stage (+16
 struct DriftTcArgs {
   DriftItem items[kDtMaxItems];
   int seg_step0[kDtMaxSegs + 1];  // first step of segment s = 2 * item + side; [n_segs] = total
-  int n_items, n_segs, total_steps, grid, rank;
+  int n_items, n_segs, total_steps, grid;
   int n_out;      // (layer, module) entries of out_sq (pairs of floats)
   int zero_mask;  // modules whose entries CTA 0 clears (0: none)
 };
@@ -320,8 +320,9 @@ __device__ __forceinline__ bool run_steps(int& x, int end, int& stage, uint32_t&
 }
 
 // Producer warp: steps [x0, x1) into the stages in turn, each once the consumers have released
-// the stage's previous step. On a timeout (its own or the consumers') it waits, within the same
-// limit, for the copies it has issued, so none is in flight when the CTA's shared memory goes.
+// the stage's previous step; then it waits until they have released the last ones. On a timeout
+// (its own or the consumers') it waits, within the same limit, for the copies it has issued, so
+// none is in flight when the CTA's shared memory goes.
 template <int R>
 __device__ __forceinline__ void produce(const DriftTcArgs& a, int x0, int x1, uint64_t* full,
                                         uint64_t* empty, uint32_t stage0, volatile int* abort_flag,
@@ -341,7 +342,9 @@ __device__ __forceinline__ void produce(const DriftTcArgs& a, int x0, int x1, ui
     ++issued;
     if (++ls == kDtStages) ls = 0;
   }
-  if (ok && !*abort_flag) return;
+  for (int i = issued > kDtStages ? issued - kDtStages : 0; ok && i < issued; ++i)
+    ok = mbar_wait(empty + i % kDtStages, static_cast<uint32_t>((i / kDtStages) & 1), abort_flag, status);
+  if (ok) return;
   if ((threadIdx.x & 31) == 0) {
     // the last use of every stage: step issued - 1 - k sits in stage (issued - 1 - k) % S
     const unsigned long long t0 = globaltimer_ns();
@@ -521,7 +524,9 @@ __global__ void __launch_bounds__(kDtThreads, kDtCtasPerSm)
     const bool ok = (seg & 1) == 0
                         ? run_steps<R, 0>(x, end, stage, phase, full, empty, stage0, abort_flag, status, acc)
                         : run_steps<R, 1>(x, end, stage, phase, full, empty, stage0, abort_flag, status, acc);
-    if (!ok) return;  // the producer drains the copies in flight
+    // the producer drains the copies in flight; a warp that got past a wait another warp gave
+    // up on stops here too, before the flush's barriers
+    if (!ok || *abort_flag) return;
     // the warps' partial Grams summed in a fixed tree ((w0 + w4) + (w2 + w6)) + ((w1 + w5) +
     // (w3 + w7)), then written as one slot
 #pragma unroll 1
@@ -632,7 +637,6 @@ cudaError_t launch_drift(const DriftItem* items, int n_items, int rank, int n_ou
     DriftTcArgs a;
     a.n_items = n_items - base < kDtMaxItems ? n_items - base : kDtMaxItems;
     a.n_segs = 2 * a.n_items;
-    a.rank = rank;
     a.n_out = n_out;
     a.zero_mask = base == 0 ? (~adapted_mask & 0x7f) : 0;
     int steps = 0;
