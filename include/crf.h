@@ -237,6 +237,8 @@ CRF_API crf_status crf_decode_step(crf_ctx* ctx, const crf_model* model, const c
  * version that produced layer l's cache; all of the same lora dims as cur).
  * out_sq: device fp32 [n_layers][7][2]: {||B1 A1 - B0 A0||_F^2 (unscaled),
  * ||A1 - A0||_F^2 + ||B1 - B0||_F^2}, zeros for modules not in the mask.
+ * Every projection width (hidden, ffn, query and key/value widths) must be a
+ * multiple of 8 (CRF_EUNSUPPORTED otherwise); every factor 16-byte aligned.
  * `workspace` >= crf_drift_workspace_size bytes. */
 CRF_API crf_status crf_drift_workspace_size(crf_ctx* ctx, const crf_model_dims* dims,
                                     const crf_lora_dims* lora, size_t* bytes);
