@@ -92,6 +92,32 @@ def test_drift_matches_oracle(ctx, cfg, lc):
     assert np.all(got[[l for l in range(n) if which[l] == 3]] == 0)
 
 
+def test_drift_more_items_than_one_launch(ctx):
+    """240 (layer, module) items, more than one launch pair takes: the host splits them over two
+    Gram + combine launches that reuse one workspace. Every adapted entry matches the factored
+    oracle; the unadapted down entries, poisoned with NaN first, read zero."""
+    cfg = synth.replace(synth.TINY, n_layers=40)
+    lc = synth.replace(synth.LORA_TINY, rank=16, modules=("q", "k", "v", "o", "gate", "up"))
+    cur, anchor = DeviceAdapter(cfg, lc, 2), DeviceAdapter(cfg, lc, 0)
+    out = torch.full((cfg.n_layers, 7, 2), float("nan"), dtype=torch.float32, device="cuda")
+    ws = ctx.drift_workspace(_dims_c(cfg), cur.crf.dims_c)
+    ctx.drift(_dims_c(cfg), cur.crf, [anchor.crf] * cfg.n_layers, out, ws)
+    ctx.check()
+    got = to_np(out).astype(np.float64)
+    oc, oa = oracle_adapter(cur).layers, oracle_adapter(anchor).layers
+    worst = 0.0
+    for l in range(cfg.n_layers):
+        for j, m in enumerate(synth.MODULES):
+            if m not in lc.modules:
+                assert got[l, j, 0] == 0.0 and got[l, j, 1] == 0.0, (l, m)
+                continue
+            A0, B0 = oa[l].AB[m]
+            A1, B1 = oc[l].AB[m]
+            for k, ref in enumerate((odrift.factored_sq(A0, B0, A1, B1), odrift.param_sq(A0, B0, A1, B1))):
+                worst = max(worst, abs(got[l, j, k] - ref) / ref)
+    assert worst <= DRIFT_REL, f"max rel drift error {worst:.3e}"
+
+
 def _dims_c(cfg):
     from paper_2609_30884_gb300 import abi
     return abi.ModelDims(cfg.n_layers, cfg.hidden, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim,
