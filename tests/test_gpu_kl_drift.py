@@ -95,9 +95,10 @@ def test_drift_matches_oracle(ctx, cfg, lc):
 def test_drift_more_items_than_one_launch(ctx):
     """240 (layer, module) items, more than one launch pair takes: the host splits them over two
     Gram + combine launches that reuse one workspace. Every adapted entry matches the factored
-    oracle; the unadapted down entries, poisoned with NaN first, read zero."""
+    oracle (down's 688-wide input ends in a 176-column step, zero-filled past its columns); the
+    unadapted v entries, poisoned with NaN first, read zero."""
     cfg = synth.replace(synth.TINY, n_layers=40)
-    lc = synth.replace(synth.LORA_TINY, rank=16, modules=("q", "k", "v", "o", "gate", "up"))
+    lc = synth.replace(synth.LORA_TINY, rank=16, modules=("q", "k", "o", "gate", "up", "down"))
     cur, anchor = DeviceAdapter(cfg, lc, 2), DeviceAdapter(cfg, lc, 0)
     out = torch.full((cfg.n_layers, 7, 2), float("nan"), dtype=torch.float32, device="cuda")
     ws = ctx.drift_workspace(_dims_c(cfg), cur.crf.dims_c)
